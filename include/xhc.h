@@ -1,0 +1,225 @@
+/*
+ * libxhc -- the expanded-residual connection op of xHC / xHC-Flash / mHC
+ * (arXiv 2607.14530, "xHC: Expanded Hyper-Connections") as a C ABI over CUDA kernels for
+ * sm_103a (GB300).
+ *
+ * One "group" is G consecutive sublayers (slots) that share one routing decision and one
+ * full-state mapping generation:
+ *   G = 1  full xHC sublayer (Alg. 1) or mHC sublayer (Sec. 3.1, k = m = N);
+ *   G = 2  xHC-Flash block (Alg. 2, slots Attention, MLP);
+ *   G = 4  xHC-Flash-4sub group (Sec. 5.2 and App. E.2, slots A, M, A, M).
+ * Per group the caller runs, in order,
+ *   forward :  pre_fwd(0) F_0 post_fwd(0)  pre_fwd(1) F_1 post_fwd(1) ... post_fwd(G-1)
+ *   backward:  post_bwd(G-1) F_{G-1}' pre_bwd(G-1) ... post_bwd(0) F_0' pre_bwd(0)
+ * where F_t is the caller's sublayer (Attention / MLP) and F_t' its backward.
+ *
+ * Tensor layouts (row-major, contiguous):
+ *   X, dX        [T, N, C] bf16 residual state / its gradient; token t = b*S + s
+ *                (sequence-major, S = seq_len), stream i, channel c at (t*N + i)*C + c.
+ *   input        [T, C] bf16 sublayer input written by pre_fwd (Eq. dense_read).
+ *   out          [T, C] bf16 sublayer output read by post_fwd / post_bwd.
+ *   d_input      [T, C] bf16 gradient w.r.t. input (read by pre_bwd).
+ *   d_out        [T, C] bf16 gradient w.r.t. out (written by post_bwd).
+ *   parameters   fp32, shapes in xhc_params; gradients fp32 with the same shapes.
+ * bf16 values are passed as their 16-bit patterns (uint16_t).
+ *
+ * Ownership and execution: every buffer is allocated and owned by the caller (device memory
+ * unless stated).  The library allocates no device memory, never synchronises, and enqueues
+ * all work asynchronously on the caller's stream (a cudaStream_t passed as void*; NULL = the
+ * legacy default stream).  `saved` (xhc_saved_bytes) carries the group's forward state to its
+ * backward and must not be touched in between; `workspace` (xhc_workspace_bytes) is scratch that
+ * must stay the same buffer across the calls of one group's forward and across those of its
+ * backward, and may be reused by other groups between those phases.  Two groups in flight on
+ * different streams need separate saved and workspace buffers.
+ *
+ * State is updated in place: post_fwd(G-1) overwrites the k active rows of X (Eq.
+ * sparse_write, inactive rows untouched); post_bwd(G-1) restores them from `saved`, so after the
+ * backward call sequence X holds the group-entry state again.  dX is updated in place from the
+ * gradient w.r.t. the group's output state to the gradient w.r.t. its entry state.  Parameter
+ * gradients are ACCUMULATED (+=) in fp32 with a fixed reduction order (run-to-run
+ * deterministic, no float atomics).
+ *
+ * Errors: every entry point validates its arguments on the host before enqueueing anything and
+ * returns a status; no exception crosses the ABI.  Requirements: device pointers 16-byte
+ * aligned; C % 8 == 0 and 8 <= C <= 16384; 1 <= N <= 32; 1 <= k <= 8; 0 <= m <= k <= N;
+ * T % seq_len == 0.  A launch failure returns XHC_ERR_CUDA; xhc_last_error_string() gives the
+ * CUDA message of the most recent failure on the calling thread.
+ */
+#ifndef XHC_H
+#define XHC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    XHC_OK = 0,
+    XHC_ERR_INVALID_ARG = 1, /* null pointer, bad slot, T or config field out of range     */
+    XHC_ERR_UNSUPPORTED = 2, /* valid per the paper but outside the limits listed above     */
+    XHC_ERR_ALIGNMENT = 3,   /* a pointer is not 16-byte aligned                            */
+    XHC_ERR_CUDA = 4,        /* a CUDA launch or query failed                               */
+    XHC_ERR_TIMEOUT = 5      /* reserved: a bounded device-side wait gave up                */
+} xhc_status;
+
+typedef enum {
+    XHC_MHC = 0,   /* mHC (Sec. 3.1): k = m = N, no router, G = 1, single write-back signal */
+    XHC_FULL = 1,  /* full xHC sublayer (Alg. 1), G = 1                                    */
+    XHC_FLASH = 2  /* xHC-Flash group (Alg. 2, App. E.2), G = 2 or 4                        */
+} xhc_variant;
+
+#define XHC_MAX_GROUP 4
+#define XHC_MAX_CONV 3
+
+/* Immutable after xhc_create.  Hyper-parameters of Sec. 3.3 / App. A. */
+typedef struct {
+    int variant;               /* xhc_variant                                                */
+    int N;                     /* streams (expansion rate)                                   */
+    int k;                     /* active streams per sublayer                                */
+    int m;                     /* fixed streams (always active, p = 1), Eq. router_topk      */
+    int C;                     /* hidden size                                                */
+    int group;                 /* G: sublayers sharing the routing decision                  */
+    int mlp_mask;              /* bit t set: slot t is an MLP sublayer (temporal augmentation)*/
+    int n_conv;                /* r causal depthwise conv branches (0 = none), Eq. aug        */
+    int conv_k[XHC_MAX_CONV];  /* kernel sizes kappa_j (paper: 4, 8, 12), each 1..16          */
+    int gram_schmidt;          /* 1: Eq. gs on [out, g_1..g_r]; 0: raw components            */
+    int sinkhorn_iters;        /* 20 in App. A                                                */
+    float eps_norm;            /* LayerNorm / RMSNorm epsilon (1e-5)                          */
+    float eps_gs;              /* Gram-Schmidt denominator epsilon; <= 0 means 1e-6 * C        */
+    int seq_len;               /* S: the conv never crosses a sequence start; 0 means T       */
+} xhc_config;
+
+/* Device pointers to the fp32 parameters of one group (Sec. 3.3.4, Sec. 5.2).
+ *   W_r        [N*C, N]      router projection (Eq. router); NULL when m == k
+ *   W_pre[t]   [N*C, N]      pre-map projection of slot t (Eq. param_pre)
+ *   alpha_pre  [G]           gating scalars of the pre-maps;  b_pre [G, N] biases
+ *   W_post[t]  [k*C, k*K_t]  post-map projection of slot t (Eq. param_post), K_t = 1 + r for
+ *                            MLP slots with augmentation, 1 otherwise
+ *   alpha_post [G];  b_post[t] [k*K_t]
+ *   W_res      [k*C, k*k]    residual-map projection of the last slot (Eq. param_res)
+ *   alpha_res  [1];  b_res [k*k]
+ *   conv_w[t][j] [kappa_j, C] depthwise taps of branch j of MLP slot t; tap 0 = current token
+ * Row index of every W is the flattened (stream-major) state index i*C + c; mat_{a x b} of a
+ * projection is row-major (column j*b + r is entry [j][r]). */
+typedef struct {
+    const float* W_r;
+    const float* W_pre[XHC_MAX_GROUP];
+    const float* alpha_pre;
+    const float* b_pre;
+    const float* W_post[XHC_MAX_GROUP];
+    const float* alpha_post;
+    const float* b_post[XHC_MAX_GROUP];
+    const float* W_res;
+    const float* alpha_res;
+    const float* b_res;
+    const float* conv_w[XHC_MAX_GROUP][XHC_MAX_CONV];
+} xhc_params;
+
+/* Gradient buffers, same shapes as xhc_params; every field is accumulated (+=).  A NULL field
+ * is an error if the parameter exists in the configuration. */
+typedef struct {
+    float* W_r;
+    float* W_pre[XHC_MAX_GROUP];
+    float* alpha_pre;
+    float* b_pre;
+    float* W_post[XHC_MAX_GROUP];
+    float* alpha_post;
+    float* b_post[XHC_MAX_GROUP];
+    float* W_res;
+    float* alpha_res;
+    float* b_res;
+    float* conv_w[XHC_MAX_GROUP][XHC_MAX_CONV];
+} xhc_grads;
+
+typedef struct xhc_handle xhc_handle;
+
+/* Validate *cfg and create a handle (host memory only).  XHC_ERR_INVALID_ARG for values the
+ * paper's method cannot take (e.g. m > k), XHC_ERR_UNSUPPORTED for values beyond the limits
+ * above, or for a variant whose structure does not match (MHC needs k = m = N, G = 1, no MLP
+ * augmentation; FULL needs G = 1; FLASH needs G in {2, 4} with slots alternating A, M). */
+xhc_status xhc_create(const xhc_config* cfg, xhc_handle** out);
+void xhc_destroy(xhc_handle* h);
+
+/* Bytes of the caller-allocated `saved` and `workspace` buffers for T tokens. */
+xhc_status xhc_saved_bytes(const xhc_handle* h, int64_t T, size_t* bytes);
+xhc_status xhc_workspace_bytes(const xhc_handle* h, int64_t T, size_t* bytes);
+
+/* Byte offsets, inside `saved`, of the coefficients a forward pass leaves there (for inspection
+ * and tests; the content is defined once pre_fwd(slot) has run for the slot concerned):
+ *   I        int32 [T, k]        active stream indices, fixed streams first (Eq. router_topk)
+ *   p        fp32  [T, k]        routing weights (1 for fixed streams)
+ *   hpre     fp32  [T, G, N]     pre-maps of the G slots (Eq. param_pre)
+ *   hpost[t] fp32  [T, k, K_t]   post-map of slot t (Eq. param_post)
+ *   hres     fp32  [T, k, k]     clamped Sinkhorn residual map of the last slot (Eq. param_res)
+ *   xact     bf16  [G, T, k, C]  active state entering each slot */
+typedef struct {
+    size_t I;
+    size_t p;
+    size_t hpre;
+    size_t hpost[XHC_MAX_GROUP];
+    size_t hres;
+    size_t xact;
+} xhc_saved_layout;
+xhc_status xhc_saved_layout_of(const xhc_handle* h, int64_t T, xhc_saved_layout* out);
+
+/* Forward, before sublayer `slot`: writes input [T, C].
+ * slot 0 runs the group's full-state passes: norm statistics, the projections of Eq.
+ * fused_normalized_projection (router and the G pre-maps), Eq. router_topk, the dense read of
+ * Eq. dense_read, the non-active base readouts of Eq. app_four_sub_base and the gather of the
+ * active streams; slot t > 0 forms input = base_t + sum_j H_pre_t[I_j] x_act_j (Eq.
+ * app_active_state_correction).  Every slot then generates its post-map (and, for the last
+ * slot, the Sinkhorn residual map with the App. A row clamp) from the current active state
+ * (Eq. param_post, Eq. param_res). */
+xhc_status xhc_pre_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
+                       const uint16_t* X, uint16_t* input, void* saved, void* workspace,
+                       void* stream);
+
+/* Forward, after sublayer `slot`: sparse write-back of out (Eq. sparse_write_delta,
+ * Eq. sparse_write; temporal augmentation Eq. aug + Eq. gs on MLP slots).  Slots before the
+ * last update the saved active state only (no mixing, Eq. flash_attn_update); the last slot
+ * applies H_res and scatters the k active rows into X in place. */
+xhc_status xhc_post_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
+                        uint16_t* X, const uint16_t* out, void* saved, void* workspace,
+                        void* stream);
+
+/* Backward of post_fwd(slot).  Reads dX (slot G-1: the gradient w.r.t. the group output) or the
+ * workspace-held active gradient, writes d_out [T, C] (= dL/d out, including the paths through
+ * later sublayer inputs), accumulates the post/res/conv parameter gradients.  slot G-1 also
+ * restores the active rows of X to the group-entry state. */
+xhc_status xhc_post_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
+                        uint16_t* X, uint16_t* dX, const uint16_t* out, uint16_t* d_out,
+                        const xhc_grads* grads, void* saved, void* workspace, void* stream);
+
+/* Backward of pre_fwd(slot).  Adds the dense-read gradient of d_input to the active gradient;
+ * slot 0 finishes the group: dX becomes the gradient w.r.t. the entry state (dense reads,
+ * norm statistics, router through the selected routed scores only) and the W_r / W_pre /
+ * alpha_pre / b_pre gradients are accumulated. */
+xhc_status xhc_pre_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
+                       const uint16_t* X, const uint16_t* d_input, uint16_t* dX,
+                       const xhc_grads* grads, void* saved, void* workspace, void* stream);
+
+/* Tracing, a host-side profiling aid: while enabled, every kernel launch of the library is
+ * bracketed by two CUDA events recorded on the caller's stream.  xhc_trace_enable(1) drops the
+ * previous records and starts recording; xhc_trace_enable(0) stops.  xhc_trace_record gives the
+ * launch's name and device duration in ms; the caller must have synchronised the stream first
+ * (otherwise XHC_ERR_CUDA, "not ready").  Not for concurrent use from several host threads. */
+xhc_status xhc_trace_enable(int on);
+int xhc_trace_count(void);
+xhc_status xhc_trace_record(int i, const char** name, float* ms);
+
+/* Number of kernels the library has launched since it was loaded. */
+uint64_t xhc_launch_count(void);
+
+/* Short static description of a status; message of the last CUDA failure on this thread. */
+const char* xhc_status_string(xhc_status s);
+const char* xhc_last_error_string(void);
+
+/* Library version as major*10000 + minor*100 + patch. */
+int xhc_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* XHC_H */
