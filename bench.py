@@ -1,0 +1,497 @@
+#!/usr/bin/env python
+"""Benchmark of libxhc: connection-op tokens/s, forward + backward, on one GB300 per rank.
+
+One step = the whole hot path over one batch: pre_fwd/post_fwd of every slot of one connection
+op group, then post_bwd/pre_bwd of every slot in reverse, on synthetic inputs already resident in
+HBM (the state alone is larger than L2, so no L2 flush is needed between steps).  The default
+workload is the xHC-Flash-4sub group (slots Attention, MLP, Attention, MLP) with N=16 streams,
+k=4 active, m=2 fixed, C=4096, T=32768 tokens (8 sequences of 4096).
+
+Prints one JSON line (rank 0).  ``--impl reference`` times the fp64 CPU oracle instead, on a
+bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import glob
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "connection-op tokens/s fwd+bwd at N=16,k=4; achieved HBM GB/s vs peak"
+
+
+def workloads():
+    from paper_2607_14530_gb300.xhc import Config
+    return {
+        "flash4": ("xHC-Flash-4sub group (A,M,A,M) N=16 k=4 m=2 C=4096 T=32768 (8 x 4096), fwd+bwd",
+                   Config.flash(16, 4, 2, 4096, 4, seq_len=4096), 32768),
+        "mhc": ("mHC N=4 C=2048 T=8192, fwd+bwd", Config.mhc(4, 2048, seq_len=8192), 8192),
+        "fullM": ("full xHC MLP sublayer N=16 k=4 m=2 C=2048 T=16384 (2 x 8192) with TFA, fwd+bwd",
+                  Config.full(16, 4, 2, 2048, True, seq_len=8192), 16384),
+        "flash4_N4": ("xHC-Flash-4sub N=4 k=4 m=2 C=4096 T=16384, fwd+bwd",
+                      Config.flash(4, 4, 2, 4096, 4, seq_len=8192), 16384),
+        "flash4_N8": ("xHC-Flash-4sub N=8 k=4 m=2 C=4096 T=16384, fwd+bwd",
+                      Config.flash(8, 4, 2, 4096, 4, seq_len=8192), 16384),
+        "flash4_N16": ("xHC-Flash-4sub N=16 k=4 m=2 C=4096 T=16384, fwd+bwd",
+                       Config.flash(16, 4, 2, 4096, 4, seq_len=8192), 16384),
+        "flash4_N32": ("xHC-Flash-4sub N=32 k=4 m=2 C=4096 T=16384, fwd+bwd",
+                       Config.flash(32, 4, 2, 4096, 4, seq_len=8192), 16384),
+    }
+
+
+# ---------------------------------------------------------------------------------------------
+# algorithmic work of every library launch of one step (bytes each kernel must move at least:
+# every input read once, every output written once; flops of the contractions)
+
+
+def kernel_model(cfg, T):
+    N, k, C, G = cfg.N, cfg.k, cfg.C, cfg.G
+    hr = cfg.m < cfg.k
+    nfull = (N if hr else 0) + G * N
+    Ks = [cfg.K(t) for t in range(G)]
+    nact = [k * Ks[t] + (k * k if t == G - 1 else 0) for t in range(G)]
+    S = cfg.seq_len if cfg.seq_len > 0 else T
+    gs = cfg.gram_schmidt
+    b16, f32 = 2, 4
+    m = {}
+
+    def add(name, bytes_=0.0, flops=0.0, bound="hbm"):
+        e = m.setdefault(name, dict(launches=0, bytes=0.0, flops=0.0, bound=bound))
+        e["launches"] += 1
+        e["bytes"] += bytes_
+        e["flops"] += flops
+
+    X = T * N * C * b16
+    xa = T * k * C * b16
+    row = T * C * b16
+    # forward
+    if hr:
+        add("colsum", N * C * N * f32)
+    add("rowproj_full", X + N * C * nfull * f32 + T * nfull * f32, 2.0 * T * N * C * nfull, "alu")
+    add("coef_full", T * nfull * f32 + T * (G * N + 2 * k) * f32)
+    add("read", X + row + (G - 1) * T * C * f32 + xa)
+    for t in range(G):
+        if t > 0:
+            add("input", T * C * f32 + xa + row)
+        add("rowproj_active", xa + k * C * nact[t] * f32 + T * nact[t] * f32, 2.0 * T * k * C * nact[t], "alu")
+        add("coef_act", T * nact[t] * f32 * 2)
+        if Ks[t] > 1 and gs:
+            add("aug_gram", row)
+        add("post_apply", xa + row + xa)
+    # backward
+    for t in reversed(range(G)):
+        last = t == G - 1
+        dxn = xa if last else T * k * C * f32
+        if last:
+            add("restore", 2 * xa)
+        add("bwd_reduce", dxn + (xa if last else 0) + row)
+        add("bwd_coef", T * nact[t] * f32 * 2)
+        add("bwd_apply", dxn + xa + row + T * k * C * f32 + (T * Ks[t] * C * f32 if Ks[t] > 1 else row))
+        add("gemm_dzw", T * nact[t] * f32 + 2 * T * k * C * f32, 2.0 * T * k * C * nact[t], "alu")
+        add("wgrad_active", xa + T * nact[t] * f32, 2.0 * T * k * C * nact[t], "alu")
+        for _ in range(4 if last else 2):
+            add("colsum", T * 16 * f32)
+        if Ks[t] > 1:
+            add("bwd_conv", T * Ks[t] * C * f32 + 2 * row)
+            add("conv_wgrad_reduce", sum(cfg.conv_k) * C * f32 * 2)
+        add("dinput_act", row + xa + 2 * T * k * C * f32 + row)
+    if hr:
+        add("colsum", N * C * N * f32)
+    add("full_dots", T * (N - k) * C * b16 + G * row)
+    add("full_coef", T * (nfull + G * N) * f32)
+    add("full_dx", X + T * (N - k) * C * b16 + T * k * C * f32 + G * row + X, 2.0 * T * N * C * nfull, "alu")
+    add("wgrad_full", X + T * nfull * f32, 2.0 * T * N * C * nfull, "alu")
+    add("colsum", T * G * N * f32)
+    add("colsum", T * G * f32)
+    if hr:
+        add("colsum", T * N * f32)
+        add("sub_rows", 2 * N * C * N * f32)
+    return m
+
+
+def paper_forward_bytes_per_token(cfg):
+    """Forward traffic of Table overhead_analysis for this group, bytes per token."""
+    from paper_2607_14530_gb300 import traffic
+    N, k = cfg.N, cfg.k
+    if cfg.variant == 0:
+        r, w = traffic.paper_model("mhc", N)
+        per_group_C = (r + w)
+    elif cfg.G == 4:
+        r, w = traffic.paper_model("flash4", N, k)
+        per_group_C = 4 * (r + w)
+    elif cfg.G == 2:
+        r, w = traffic.paper_model("flash2", N, k)
+        per_group_C = 2 * (r + w)
+    else:
+        r, w = traffic.paper_model("xhc", N, k)
+        per_group_C = r + w
+    return per_group_C * cfg.C * 2
+
+
+# ---------------------------------------------------------------------------------------------
+# clocks during the timed region
+
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, dev: int):
+        self.dev = dev
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-i", str(self.dev)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.t.join(timeout=2)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            p = [x.strip() for x in ln.split(",")]
+            if len(p) < 8:
+                continue
+            try:
+                sm.append(float(p[0]))
+                mx.append(float(p[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, p[4:8]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# ---------------------------------------------------------------------------------------------
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "sm_max_mhz": 2070.0}, "fallback"
+
+
+def csrc_hash():
+    h = hashlib.sha256()
+    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2607_14530_gb300", "csrc", "*"))):
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(kernel, workload):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on the current
+    kernel sources and this workload; else None."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    e = d.get(workload, {}).get(kernel)
+    if not e or e.get("csrc_sha") != csrc_hash():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+def oracle_step(cfg, X, outs, dX, dins, P):
+    """One fp64 oracle fwd+bwd on CPU tensors (the oracle as it stands)."""
+    import torch
+    from oracle import xhc_oracle as O
+    ocfg = O.Config(N=cfg.N, k=cfg.k, m=cfg.m, C=cfg.C, G=cfg.G,
+                    mlp=tuple(bool((cfg.mlp_mask >> t) & 1) for t in range(cfg.G)),
+                    conv_k=tuple(cfg.conv_k), gram_schmidt=cfg.gram_schmidt,
+                    sinkhorn_iters=cfg.sinkhorn_iters, eps_norm=cfg.eps_norm,
+                    eps_gs=(cfg.eps_gs if cfg.eps_gs > 0 else None), seq_len=cfg.seq_len)
+    f64 = torch.float64
+    P64 = {n: v.to(f64) for n, v in P.items()}
+    O.backward(ocfg, P64, X.to(f64), [o.to(f64) for o in outs], dX.to(f64), [d.to(f64) for d in dins])
+
+
+def cpu_sample(cfg, T_s, seed):
+    import torch
+    from paper_2607_14530_gb300 import synth
+    d = synth.group_inputs(T_s, cfg.N, cfg.C, cfg.G, seed)
+    g = synth.group_grads(T_s, cfg.N, cfg.C, cfg.G, seed)
+    P = synth.params(cfg.param_shapes(), seed)
+    return d["X"], d["outs"], g["dX"], g["d_inputs"], P
+
+
+def run_reference(args, wl_name):
+    import torch
+    desc, cfg, T = workloads()[wl_name]
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    T_s = args.ref_tokens
+    X, outs, dX, dins, P = cpu_sample(cfg, T_s, 0)
+    for _ in range(args.warmup):
+        oracle_step(cfg, X, outs, dX, dins, P)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle_step(cfg, X, outs, dX, dins, P)
+    dt = time.perf_counter() - t0
+    value = T_s * args.steps / dt
+    cores = torch.get_num_threads()
+    sample = f"first {T_s} tokens of sequence 0 of the workload per step (fp64 oracle, fwd+bwd)"
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1000.0 * dt / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": desc, "tokens_per_step": T_s},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_xhc(args, wl_name):
+    import torch
+    import torch.distributed as dist
+    from paper_2607_14530_gb300 import build, synth, xhc
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    if rank == 0:
+        build.build()
+    if world > 1:
+        dist.barrier()
+    xhc.lib()
+
+    desc, cfg, T = workloads()[wl_name]
+    if args.tokens:
+        T = args.tokens
+    g = xhc.Group(cfg)
+    seed = 1234 + rank
+    X = synth.normal_bf16_on((T, cfg.N, cfg.C), seed, dev)
+    outs = [synth.normal_bf16_on((T, cfg.C), seed + 101 + t, dev) for t in range(cfg.G)]
+    dX0 = synth.normal_bf16_on((T, cfg.N, cfg.C), seed + 7, dev)
+    dins = [synth.normal_bf16_on((T, cfg.C), seed + 211 + t, dev) for t in range(cfg.G)]
+    P = {n: v.to(dev) for n, v in synth.params(cfg.param_shapes(), seed).items()}
+    G_ = {n: torch.zeros_like(v) for n, v in P.items()}
+    saved, ws = g.alloc(T, device=dev)
+    inputs = [torch.empty(T, cfg.C, dtype=torch.bfloat16, device=dev) for _ in range(cfg.G)]
+    d_outs = [torch.empty(T, cfg.C, dtype=torch.bfloat16, device=dev) for _ in range(cfg.G)]
+    dX = dX0.clone()
+    stream = torch.cuda.current_stream()
+
+    def step():
+        g.forward(P, X, outs, saved, ws, inputs=inputs)
+        g.backward(P, X, dX, outs, dins, G_, saved, ws, d_outs=d_outs)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    xhc.trace_enable(True)
+    n0 = xhc.launch_count()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    launches = xhc.launch_count() - n0
+    xhc.trace_enable(False)
+    ck = clocks.stop()
+    ms = e0.elapsed_time(e1)
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_step = ms / args.steps
+    value = world * T * args.steps / (ms / 1000.0)
+
+    # per-kernel device time over the timed region
+    recs = xhc.trace_records()
+    per = {}
+    for name, t_ms in recs:
+        e = per.setdefault(name, [0, 0.0])
+        e[0] += 1
+        e[1] += t_ms
+    model = kernel_model(cfg, T)
+    peaks, peak_src = measured_peaks()
+    hbm_peak = float(peaks["hbm_gbs"])
+    sm_mhz = float(peaks.get("sm_max_mhz", 2070.0))
+    alu_peak = 152 * 128 * 2 * sm_mhz * 1e6 / 1e12  # fp32 FMA lanes x 2 flop x max clock, TFLOP/s
+    kernels = {}
+    for name, (cnt, tot) in per.items():
+        mm = model.get(name)
+        ent = {"launches": cnt // args.steps, "ms_per_step": tot / args.steps,
+               "share": tot / max(1e-9, sum(v[1] for v in per.values()))}
+        if mm:
+            secs = tot / args.steps / 1000.0
+            ent["gbs"] = mm["bytes"] / secs / 1e9
+            if mm["flops"]:
+                ent["tflops"] = mm["flops"] / secs / 1e12
+            ent["bound"] = mm["bound"]
+        kernels[name] = ent
+    dom = max(per, key=lambda n: per[n][1])
+    mm = model[dom]
+    cnt, tot = per[dom]
+    secs = tot / cnt / 1000.0
+    launches_per_step = mm["launches"]
+    if mm["bound"] == "alu":
+        achieved = mm["flops"] / launches_per_step / secs / 1e12
+        roof = {"kernel": dom, "bound": "alu", "achieved": achieved, "peak": alu_peak,
+                "unit": "TFLOP/s", "frac": achieved / alu_peak,
+                "peak_source": "derived: 152 SMs x 128 fp32 lanes x 2 flop x max SM clock"}
+    else:
+        achieved = mm["bytes"] / launches_per_step / secs / 1e9
+        roof = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": hbm_peak,
+                "unit": "GB/s", "frac": achieved / hbm_peak, "peak_source": f"{peak_src} hbm_gbs"}
+    roof["traffic"] = ncu_traffic(dom, wl_name)
+
+    step_bytes = sum(v["bytes"] for v in model.values())
+    hbm = {"model_bytes_per_step": step_bytes, "achieved_gbs": step_bytes / (ms_step / 1000.0) / 1e9,
+           "frac_of_measured_peak": step_bytes / (ms_step / 1000.0) / 1e9 / hbm_peak,
+           "paper_fwd_bytes_per_token": paper_forward_bytes_per_token(cfg)}
+
+    line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic",
+            "config": {"workload": desc, "tokens": T, "storage": "bf16 state, fp32 params/coefficients",
+                       "l2": "inputs larger than L2 (state alone is %.1f GiB), no flush" % (T * cfg.N * cfg.C * 2 / 2**30),
+                       "parallelism": "replicas" if world > 1 else "1 GPU"},
+            "roofline": roof, "hbm": hbm, "gpu_launches": launches, "clocks": ck}
+
+    if args.kernels_out and rank == 0:
+        with open(args.kernels_out, "w") as f:
+            json.dump({"workload": wl_name, "kernels": kernels, "model": model}, f, indent=1)
+
+    # end to end through the public API with host buffers: H2D of the step's inputs from pinned
+    # memory, the step, D2H of its results
+    if not args.no_e2e:
+        pin = lambda t: torch.empty(t.shape, dtype=t.dtype, pin_memory=True)  # noqa: E731
+        hX, hdX = pin(X), pin(dX)
+        hX.copy_(X)
+        hdX.copy_(dX0)
+        houts = [pin(o) for o in outs]
+        hdins = [pin(d) for d in dins]
+        for h, d in zip(houts + hdins, outs + dins):
+            h.copy_(d)
+        rdX = pin(dX)
+        rins = [pin(i) for i in inputs]
+        rdouts = [pin(o) for o in d_outs]
+        h2d = sum(t.numel() * t.element_size() for t in [hX, hdX] + houts + hdins)
+        d2h = sum(t.numel() * t.element_size() for t in [rdX] + rins + rdouts)
+
+        def e2e_step():
+            X.copy_(hX, non_blocking=True)
+            dX.copy_(hdX, non_blocking=True)
+            for d, h in zip(outs + dins, houts + hdins):
+                d.copy_(h, non_blocking=True)
+            step()
+            rdX.copy_(dX, non_blocking=True)
+            for h, d in zip(rins + rdouts, inputs + d_outs):
+                h.copy_(d, non_blocking=True)
+
+        ksteps = max(2, min(args.steps, 5))
+        e2e_step()
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(ksteps):
+            e2e_step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        ems = a.elapsed_time(b)
+        if world > 1:
+            t = torch.tensor([ems], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ems = float(t.item())
+        line["e2e"] = {"value": world * T * ksteps / (ems / 1000.0), "unit": "tokens/s",
+                       "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": ksteps}
+
+    if rank == 0 and not args.no_cpu_baseline:
+        T_s = args.cpu_tokens
+        Xs, os_, dXs, dis, Ps = cpu_sample(cfg, T_s, 0)
+        t0 = time.perf_counter()
+        oracle_step(cfg, Xs, os_, dXs, dis, Ps)
+        dt = time.perf_counter() - t0
+        line["cpu_baseline"] = {"value": T_s / dt, "unit": "tokens/s", "cores": torch.get_num_threads(),
+                                "kind": "oracle",
+                                "sample": f"first {T_s} tokens of one sequence of the workload, fp64 "
+                                          f"oracle fwd+bwd, one run of {dt:.1f} s"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="xhc", choices=["xhc", "reference"])
+    ap.add_argument("--workload", default="flash4")
+    ap.add_argument("--tokens", type=int, default=0, help="override T (development only)")
+    ap.add_argument("--cpu-tokens", type=int, default=3072)
+    ap.add_argument("--ref-tokens", type=int, default=64)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--kernels-out", default="")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "xhc":
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args, args.workload)
+    else:
+        run_xhc(args, args.workload)
+
+
+if __name__ == "__main__":
+    main()

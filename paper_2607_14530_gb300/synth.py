@@ -21,6 +21,19 @@ def normal_bf16(shape, seed: int, std: float = 1.0) -> torch.Tensor:
     return (torch.randn(*shape, generator=_gen(seed), dtype=torch.float32) * std).to(torch.bfloat16)
 
 
+def normal_bf16_on(shape, seed: int, device, std: float = 1.0) -> torch.Tensor:
+    """~N(0, std^2) drawn in fp32 by a seeded generator on `device` (large inputs), as bf16."""
+    g = torch.Generator(device=device)
+    g.manual_seed(int(seed))
+    out = torch.empty(*shape, dtype=torch.bfloat16, device=device)
+    flat = out.view(-1)
+    step = 1 << 26
+    for i in range(0, flat.numel(), step):
+        n = min(step, flat.numel() - i)
+        flat[i:i + n] = (torch.randn(n, generator=g, dtype=torch.float32, device=device) * std).to(torch.bfloat16)
+    return out
+
+
 def params(shapes: dict, seed: int, alpha: float = 0.01, w_std: float = 0.02) -> dict:
     """fp32 CPU parameters for the given ``{name: shape}`` layout.
 

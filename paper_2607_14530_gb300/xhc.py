@@ -76,6 +76,11 @@ def lib() -> ctypes.CDLL:
         L.xhc_post_bwd.argtypes = [vp, ctypes.c_int, i64, P, vp, vp, vp, vp, P, vp, vp, vp]
         L.xhc_pre_bwd.argtypes = [vp, ctypes.c_int, i64, P, vp, vp, vp, P, vp, vp, vp]
         L.xhc_saved_layout_of.argtypes = [vp, i64, ctypes.POINTER(_SavedLayout)]
+        L.xhc_trace_enable.argtypes = [ctypes.c_int]
+        L.xhc_trace_count.restype = ctypes.c_int
+        L.xhc_trace_record.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_char_p),
+                                       ctypes.POINTER(ctypes.c_float)]
+        L.xhc_launch_count.restype = ctypes.c_uint64
         L.xhc_status_string.argtypes = [ctypes.c_int]
         L.xhc_status_string.restype = ctypes.c_char_p
         L.xhc_last_error_string.restype = ctypes.c_char_p
@@ -90,6 +95,27 @@ def _check(status: int, what: str):
         if status == 4:
             msg += ": " + lib().xhc_last_error_string().decode()
         raise XhcError(f"{what} failed: {msg}")
+
+
+def trace_enable(on: bool) -> None:
+    """Start (clearing old records) or stop recording per-launch CUDA events in the library."""
+    _check(lib().xhc_trace_enable(1 if on else 0), "xhc_trace_enable")
+
+
+def trace_records() -> list:
+    """[(kernel name, device ms)] of the recorded launches; synchronise the stream first."""
+    L = lib()
+    out = []
+    for i in range(L.xhc_trace_count()):
+        name, ms = ctypes.c_char_p(), ctypes.c_float()
+        _check(L.xhc_trace_record(i, ctypes.byref(name), ctypes.byref(ms)), "xhc_trace_record")
+        out.append((name.value.decode(), float(ms.value)))
+    return out
+
+
+def launch_count() -> int:
+    """Kernels launched by the library since it was loaded."""
+    return int(lib().xhc_launch_count())
 
 
 @dataclass(frozen=True)
