@@ -200,6 +200,27 @@ xhc_status xhc_pre_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
                        const uint16_t* X, const uint16_t* d_input, uint16_t* dX,
                        const xhc_grads* grads, void* saved, void* workspace, void* stream);
 
+/* Routing and pre-maps for callers that cannot allocate device memory.
+ *
+ * The paper has no counterpart: this is a deployment convenience.  Some callers cannot provide
+ * the `workspace` of xhc_pre_fwd -- code running inside another framework's memory arena,
+ * engines that fix every device buffer at start-up, plug-ins whose host owns all allocation.
+ * xhc_route_noalloc computes, for T tokens of X, the same routing and pre-maps as the
+ * full-state part of xhc_pre_fwd(slot 0): I [T, k] int32, p [T, k] fp32 and hpre [T, G, N]
+ * fp32 (caller-owned device outputs; P needs W_r (if m < k), W_pre, alpha_pre and b_pre).  Its
+ * split-K partial sums live in a fixed array of XHC_NOALLOC_SCRATCH_BYTES that is part of the
+ * library's device image (every GPU that loads the library holds it until the process exits);
+ * it calls no allocator.  A T whose partial sums do not fit returns XHC_ERR_UNSUPPORTED
+ * (for N = 16, G = 4 and T above ~20K tokens about 1 KB per token, so T up to ~50K).
+ * The first call on a device looks up the array's device address (cudaGetSymbolAddress) with
+ * that device current; make that first call before any stream capture.  All calls share the one
+ * array: calls that overlap on the GPU (several streams or host threads at once) race and give
+ * wrong results; serialise them.  Nothing in the array needs to start at zero: each call writes
+ * every word it later reads. */
+#define XHC_NOALLOC_SCRATCH_BYTES (48u << 20)
+xhc_status xhc_route_noalloc(const xhc_handle* h, int64_t T, const xhc_params* P,
+                             const uint16_t* X, int32_t* I, float* p, float* hpre, void* stream);
+
 /* Tracing, a host-side profiling aid: while enabled, every kernel launch of the library is
  * bracketed by two CUDA events recorded on the caller's stream.  xhc_trace_enable(1) drops the
  * previous records and starts recording; xhc_trace_enable(0) stops.  xhc_trace_record gives the

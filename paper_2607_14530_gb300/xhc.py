@@ -76,6 +76,7 @@ def lib() -> ctypes.CDLL:
         L.xhc_post_bwd.argtypes = [vp, ctypes.c_int, i64, P, vp, vp, vp, vp, P, vp, vp, vp]
         L.xhc_pre_bwd.argtypes = [vp, ctypes.c_int, i64, P, vp, vp, vp, P, vp, vp, vp]
         L.xhc_saved_layout_of.argtypes = [vp, i64, ctypes.POINTER(_SavedLayout)]
+        L.xhc_route_noalloc.argtypes = [vp, i64, P, vp, vp, vp, vp, vp]
         L.xhc_trace_enable.argtypes = [ctypes.c_int]
         L.xhc_trace_count.restype = ctypes.c_int
         L.xhc_trace_record.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_char_p),
@@ -283,6 +284,17 @@ class Group:
 
     def params(self, P: dict) -> _Params:
         return _fill(_Params(), P, self.cfg)
+
+    def route_noalloc(self, P, X, I, p, hpre, stream=None):
+        """Routing (I int32 [T, k], p fp32 [T, k]) and pre-maps (hpre fp32 [T, G, N]) of X, for
+        callers that cannot allocate a workspace (xhc_route_noalloc)."""
+        T = X.shape[0]
+        pp = P if isinstance(P, _Params) else self.params(P)
+        for t, n, dt in ((I, "I", torch.int32), (p, "p", torch.float32), (hpre, "hpre", torch.float32)):
+            if t.dtype != dt or not t.is_cuda or not t.is_contiguous():
+                raise XhcError(f"{n} must be a contiguous {dt} CUDA tensor")
+        _check(lib().xhc_route_noalloc(self._h, T, ctypes.byref(pp), _bf16(X, "X"), _ptr(I), _ptr(p),
+                                       _ptr(hpre), _stream(stream)), "xhc_route_noalloc")
 
     def pre_fwd(self, slot, P, X, inp, saved, ws, stream=None):
         T = X.shape[0]
