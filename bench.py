@@ -76,7 +76,10 @@ def kernel_model(cfg, T):
     # forward
     if hr:
         add("colsum", N * C * N * f32)
-    add("rowproj_full", X + N * C * nfull * f32 + T * nfull * f32, 2.0 * T * N * C * nfull, "alu")
+    nb = 2 * nfull  # hi + lo bf16 rows of the packed weight
+    add("pack_w", N * C * nfull * f32 + nb * N * C * b16)
+    # tensor-core projection: X read once; the packed weight streams from L2
+    add("proj_tc", X + T * nfull * f32, 2.0 * T * N * C * nb, "hbm")
     add("coef_full", T * nfull * f32 + T * (G * N + 2 * k) * f32)
     add("read", X + row + (G - 1) * T * C * f32 + xa)
     for t in range(G):

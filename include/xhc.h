@@ -153,7 +153,10 @@ xhc_status xhc_workspace_bytes(const xhc_handle* h, int64_t T, size_t* bytes);
  *   hpre     fp32  [T, G, N]     pre-maps of the G slots (Eq. param_pre)
  *   hpost[t] fp32  [T, k, K_t]   post-map of slot t (Eq. param_post)
  *   hres     fp32  [T, k, k]     clamped Sinkhorn residual map of the last slot (Eq. param_res)
- *   xact     bf16  [G, T, k, C]  active state entering each slot */
+ *   xact     bf16  [G, T, k, C]  active state entering each slot
+ *   zfull    fp32  [T, nfull]     raw full-state projections x W, columns [router N | pre-map
+ *                                 N of each slot] (router columns only when m < k)
+ *   stats    fp32  [T, 2]         mean and mean square of the flattened entry state */
 typedef struct {
     size_t I;
     size_t p;
@@ -161,6 +164,8 @@ typedef struct {
     size_t hpost[XHC_MAX_GROUP];
     size_t hres;
     size_t xact;
+    size_t zfull;
+    size_t stats;
 } xhc_saved_layout;
 xhc_status xhc_saved_layout_of(const xhc_handle* h, int64_t T, xhc_saved_layout* out);
 
@@ -229,6 +234,12 @@ xhc_status xhc_route_noalloc(const xhc_handle* h, int64_t T, const xhc_params* P
 xhc_status xhc_trace_enable(int on);
 int xhc_trace_count(void);
 xhc_status xhc_trace_record(int i, const char** name, float* ms);
+
+/* Device error word of a workspace: kernels with bounded waits (the tensor-core projection) set
+ * it to a nonzero code instead of waiting forever, and return.  Synchronous (a device-to-host
+ * copy).  *code receives the word; returns XHC_ERR_TIMEOUT if it is nonzero; clear != 0 resets
+ * it.  A fresh workspace must be zeroed once before first use (e.g. cudaMemset). */
+xhc_status xhc_workspace_error(const void* workspace, int* code, int clear);
 
 /* Number of kernels the library has launched since it was loaded. */
 uint64_t xhc_launch_count(void);

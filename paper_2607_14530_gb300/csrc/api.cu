@@ -148,7 +148,8 @@ Layout make_layout(const Dims& d, int64_t T) {
     L.saved_total = o;
 
     const int rowblocks = (int)((T + 63) / 64);
-    L.splits_full = pick_splits(rowblocks, d.N * d.C);
+    L.tc = plan_proj_tc((int)T, d.N * d.C, d.nfull, device_sms());
+    L.splits_full = L.tc.nseg;
     L.splits_act = pick_splits(rowblocks, d.k * d.C);
     L.nslice = (d.C + 255) / 256;
     const int ts_full = pick_tsplits(d.N * d.C, (int)T);
@@ -156,6 +157,8 @@ Layout make_layout(const Dims& d, int64_t T) {
     L.tsplits = std::max(ts_full, ts_act);
     L.ntiles = (int)((T + 127) / 128);
     o = 0;
+    L.err = o; o = al(o + 256);
+    L.wpack = o; o = al(o + (size_t)L.tc.NB * d.N * d.C * 2);
     L.part = o;
     o = al(o + std::max((size_t)L.splits_full * d.nfull, (size_t)L.splits_act * nact_max) * t * 4);
     L.pstats = o; o = al(o + (size_t)std::max(L.splits_full, L.splits_act) * t * 2 * 4);
@@ -221,6 +224,17 @@ xhc_status xhc_trace_record(int i, const char** name, float* ms) {
 }
 
 uint64_t xhc_launch_count(void) { return (uint64_t)g_launches.load(); }
+
+xhc_status xhc_workspace_error(const void* workspace, int* code, int clear) {
+    if (!workspace || !code) return XHC_ERR_INVALID_ARG;
+    cudaError_t e = cudaMemcpy(code, workspace, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, __LINE__);
+    if (clear) {
+        e = cudaMemset(const_cast<void*>(workspace), 0, sizeof(int));
+        if (e != cudaSuccess) return cuda_fail(e, __LINE__);
+    }
+    return *code ? XHC_ERR_TIMEOUT : XHC_OK;
+}
 
 const char* xhc_status_string(xhc_status s) {
     switch (s) {
@@ -300,6 +314,8 @@ xhc_status xhc_saved_layout_of(const xhc_handle* h, int64_t T, xhc_saved_layout*
     for (int q = 0; q < h->h.d.G; ++q) out->hpost[q] = L.hpost[q];
     out->hres = L.hres;
     out->xact = L.xact;
+    out->zfull = L.zfull;
+    out->stats = L.stats;
     return XHC_OK;
 }
 
@@ -465,8 +481,18 @@ xhc_status xhc_pre_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
             XHC_K("colsum", c.st, launch_colsum(P->W_r, d.N * d.C, d.N, d.N, c.W<float>(c.L.wsum), 0,
                                    c.W<float>(c.L.colscr), c.st));
         const WSegs wf = full_segs(d, P);
-        XHC_K("rowproj_full", c.st, launch_rowproj(X, (int64_t)d.N * d.C, d.N * d.C, c.T, wf, d.nfull,
-                                c.L.splits_full, c.W<float>(c.L.part), c.W<float>(c.L.pstats), c.st));
+        if (c.T < 128 || d.N * d.C < 64) {
+            // smaller than one tensor-core tile: fp32 CUDA-core projection
+            XHC_K("rowproj_full", c.st, launch_rowproj(X, (int64_t)d.N * d.C, d.N * d.C, c.T, wf,
+                                                       d.nfull, c.L.splits_full, c.W<float>(c.L.part),
+                                                       c.W<float>(c.L.pstats), c.st));
+        } else {
+        XHC_K("pack_w", c.st, launch_pack_w(wf, d.nfull, c.L.tc.NB, d.N * d.C,
+                                            c.W<uint16_t>(c.L.wpack), c.st));
+        XHC_K("proj_tc", c.st, launch_proj_tc(X, c.T, d.N * d.C, c.W<uint16_t>(c.L.wpack), d.nfull,
+                                              c.L.tc, c.W<float>(c.L.part), c.W<float>(c.L.pstats),
+                                              c.W<int>(c.L.err), c.st));
+        }
         XHC_K("coef_full", c.st, launch_coef_full(d, c.T, c.W<float>(c.L.part), c.W<float>(c.L.pstats),
                                   c.L.splits_full, c.W<float>(c.L.wsum), P->alpha_pre, P->b_pre,
                                   c.S<float>(c.L.zfull), c.S<float>(c.L.stats),

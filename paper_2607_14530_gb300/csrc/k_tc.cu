@@ -1,0 +1,455 @@
+// Full-state projection of Eq. fused_normalized_projection on the 5th-generation tensor cores:
+//   part[j][t][o] = sum over the k-blocks of segment j of x[t][e] * W[e][o]   (o < nfull)
+//   pstats[j][t]  = (sum x, sum x^2) over the same k-blocks
+// X [T, NC] bf16 is the A operand (K-major), W is pre-packed as bf16 hi and lo rows
+// Wpack[2*nfull(+pad)][NC] (B operand, K-major): one MMA of N = 2*nfull gives x*W_hi and x*W_lo,
+// summed in the epilogue, i.e. the fp32 weights to ~2^-17 relative.  Tiles of 128 tokens x 64
+// k-elements arrive by TMA (128-byte swizzle) into a 5-stage ring; one thread issues
+// tcgen05.mma into a TMEM accumulator; four warps compute the row statistics from the staged
+// tiles and, at the end of each segment, read the accumulator back with tcgen05.ld.
+// Work split (stream-K): the T/128 x NC/64 k-blocks are cut into equal contiguous ranges, one per
+// persistent CTA; a tile cut across CTAs gives several segments, summed later in a fixed order.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <string.h>
+
+#include "xhc_internal.cuh"
+
+namespace xhc {
+
+namespace {
+
+constexpr int BM = 128;        // tokens per tile (MMA M)
+constexpr int BK = 64;         // k-elements per stage (128 bytes of bf16 = one swizzle row)
+constexpr int MAXSTAGES = 8;
+constexpr int NTHREADS = 192;  // warp 0 TMA, warp 1 MMA + TMEM, warps 2..5 statistics + epilogue
+constexpr uint64_t WAIT_NS = 4000000000ull;  // give up a wait after ~4 s
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t a, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t a, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(a), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t a) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(a) : "memory");
+}
+// Bounded wait on a phase of an mbarrier: false once ~4 s (global timer) have passed.
+__device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity) {
+    uint64_t t0 = 0;
+    for (uint32_t it = 0;; ++it) {
+        uint32_t ok;
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+            " selp.u32 %0, 1, 0, p;\n}\n"
+            : "=r"(ok) : "r"(a), "r"(parity) : "memory");
+        if (ok) return true;
+        if ((it & 255u) == 255u) {
+            uint64_t now;
+            asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(now));
+            if (t0 == 0) t0 = now;
+            else if (now - t0 > WAIT_NS) return false;
+        }
+    }
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
+                                            uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst), "l"((uint64_t)map), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row groups 1024 B apart.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t addr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((addr & 0x3FFFFu) >> 4);        // start address
+    d |= (uint64_t)(16u >> 4) << 16;                 // leading byte offset (unused for SW128 K-major)
+    d |= (uint64_t)(1024u >> 4) << 32;               // stride byte offset: 8 rows x 128 B
+    d |= (uint64_t)1 << 46;                          // descriptor version for tcgen05
+    d |= (uint64_t)2 << 61;                          // swizzle: 128 B
+    return d;
+}
+
+// Instruction descriptor, kind::f16: bf16 A and B, fp32 accumulator, both K-major, M x N.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                         uint32_t accum) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"(accum)
+        : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+                 : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+struct ProjTcArgs {
+    int T, KB;          // tokens, k-blocks per tile
+    int MT;             // M tiles
+    long long W;        // total k-blocks
+    int P;              // persistent CTAs
+    int nfull;          // outputs per token (hi rows), lo rows follow
+    int NB;             // B rows = MMA N total (multiple of 16)
+    int nchunk;         // MMA instructions per k-step (N split in chunks of NB / nchunk <= 256)
+    int nseg;           // partial slots per tile
+    int stages;         // smem ring depth
+    float* part;        // [nseg][T][nfull]
+    float* pstats;      // [nseg][T][2]
+    int* err;           // set to a nonzero code when a wait gives up
+};
+
+__device__ __forceinline__ long long range_start(long long W, int P, int c) {
+    return (W * c) / P;
+}
+
+__global__ void __launch_bounds__(NTHREADS, 1)
+k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+          ProjTcArgs a) {
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    const int STAGES = a.stages;
+    unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    const uint32_t A_BYTES = BM * BK * 2;
+    const uint32_t B_BYTES = (uint32_t)a.NB * BK * 2;
+    const uint32_t STAGE = A_BYTES + B_BYTES;  // both multiples of 1024
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE);
+    // bars[0..S) full, [S..2S) empty, [2S] acc full, [2S+1] acc empty
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 2);
+    __shared__ int s_abort;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int c = blockIdx.x;
+    const long long g0 = range_start(a.W, a.P, c), g1 = range_start(a.W, a.P, c + 1);
+    const uint32_t ncols = (a.NB <= 256) ? 256u : 512u;
+
+    if (threadIdx.x == 0) {
+        s_abort = 0;
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(smem_u32(&bars[s]), 1);
+            mbar_init(smem_u32(&bars[STAGES + s]), 1 + 4);
+        }
+        mbar_init(smem_u32(&bars[2 * STAGES]), 1);
+        mbar_init(smem_u32(&bars[2 * STAGES + 1]), 4);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(tmem_slot)),
+                     "r"(ncols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        // ---------------- TMA producer ----------------
+        if (lane == 0) {
+            long long it = 0;
+            for (long long g = g0; g < g1; ++g, ++it) {
+                const int s = (int)(it % STAGES);
+                const uint32_t ph = (uint32_t)((it / STAGES) & 1);
+                if (it >= STAGES && !mbar_wait(smem_u32(&bars[STAGES + s]), ph ^ 1)) {
+                    atomicExch(a.err, 1);
+                    s_abort = 1;
+                    break;
+                }
+                if (*(volatile int*)&s_abort) break;
+                const int m = (int)(g / a.KB), kb = (int)(g % a.KB);
+                const uint32_t full = smem_u32(&bars[s]);
+                mbar_expect_tx(full, STAGE);
+                unsigned char* st = smem + (size_t)s * STAGE;
+                tma_load_2d(smem_u32(st), &tmA, kb * BK, m * BM, full);
+                const int nb_box = a.NB / a.nchunk;
+                for (int q = 0; q < a.nchunk; ++q)
+                    tma_load_2d(smem_u32(st + A_BYTES + (size_t)q * nb_box * 128), &tmB, kb * BK,
+                                q * nb_box, full);
+            }
+        }
+    } else if (warp == 1) {
+        // ---------------- MMA issuer ----------------
+        if (lane == 0) {
+            const int nb_chunk = a.NB / a.nchunk;
+            const uint32_t idesc = idesc_bf16(BM, nb_chunk);
+            long long it = 0;
+            int seg = 0;
+            long long g = g0;
+            while (g < g1) {
+                const int m = (int)(g / a.KB);
+                const long long gend = min(g1, (long long)(m + 1) * a.KB);
+                if (seg > 0 && !mbar_wait(smem_u32(&bars[2 * STAGES + 1]), (uint32_t)((seg - 1) & 1))) {
+                    atomicExch(a.err, 2);
+                    s_abort = 1;
+                    break;
+                }
+                tc_fence_after();
+                bool first = true;
+                for (; g < gend; ++g, ++it) {
+                    const int s = (int)(it % STAGES);
+                    const uint32_t ph = (uint32_t)((it / STAGES) & 1);
+                    if (!mbar_wait(smem_u32(&bars[s]), ph)) {
+                        atomicExch(a.err, 3);
+                        s_abort = 1;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t abase = smem_u32(smem + (size_t)s * STAGE);
+                    const uint32_t bbase = abase + A_BYTES;
+#pragma unroll
+                    for (int kk = 0; kk < BK / 16; ++kk) {
+                        const uint64_t ad = sw128_desc(abase + kk * 32);
+                        for (int q = 0; q < a.nchunk; ++q) {
+                            const uint64_t bd = sw128_desc(bbase + q * nb_chunk * 128 + kk * 32);
+                            mma_bf16(tmem + (uint32_t)(q * nb_chunk), ad, bd, idesc,
+                                     (first && kk == 0) ? 0u : 1u);
+                        }
+                    }
+                    first = false;
+                    mma_commit(smem_u32(&bars[STAGES + s]));  // stage free once these MMAs finish
+                }
+                if (*(volatile int*)&s_abort) break;
+                mma_commit(smem_u32(&bars[2 * STAGES]));     // accumulator ready
+                ++seg;
+            }
+        }
+    } else {
+        // ---------------- statistics + epilogue (warps 2..5) ----------------
+        const int quarter = warp & 3;           // TMEM lanes this warp may access
+        const int r = quarter * 32 + lane;      // tile row = token within the tile
+        long long it = 0;
+        int seg = 0;
+        long long g = g0;
+        bool ok = true;
+        while (g < g1 && ok) {
+            const int m = (int)(g / a.KB);
+            const long long gend = min(g1, (long long)(m + 1) * a.KB);
+            float s1 = 0.f, s2 = 0.f;
+            for (; g < gend; ++g, ++it) {
+                const int s = (int)(it % STAGES);
+                const uint32_t ph = (uint32_t)((it / STAGES) & 1);
+                if (!mbar_wait(smem_u32(&bars[s]), ph)) {
+                    atomicExch(a.err, 4);
+                    ok = false;
+                    break;
+                }
+                // row r of the A tile: 128 bytes, 16-byte chunks permuted by the swizzle (the
+                // sum over the row does not depend on the order)
+                const uint4* row = reinterpret_cast<const uint4*>(smem + (size_t)s * STAGE + r * 128);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    float f[8];
+                    unpack8(row[q], f);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        s1 += f[e];
+                        s2 = fmaf(f[e], f[e], s2);
+                    }
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&bars[STAGES + s]));
+            }
+            if (!ok) break;
+            // the segment's slot: index of this CTA among those covering tile m
+            int c0 = (int)(((long long)m * a.KB * a.P) / a.W);
+            while (c0 > 0 && range_start(a.W, a.P, c0) > (long long)m * a.KB) --c0;
+            while (range_start(a.W, a.P, c0 + 1) <= (long long)m * a.KB) ++c0;
+            const int j = c - c0;
+            if (!mbar_wait(smem_u32(&bars[2 * STAGES]), (uint32_t)(seg & 1))) {
+                atomicExch(a.err, 5);
+                break;
+            }
+            tc_fence_after();
+            const int t = m * BM + r;
+            float* dst = a.part + ((long long)j * a.T + t) * a.nfull;
+            const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
+            // hi columns [0, nfull), lo columns [nfull, 2 nfull)
+            for (int o0 = 0; o0 < a.nfull; o0 += 16) {
+                float hi[16], lo[16];
+                tmem_ld16(tl + (uint32_t)o0, hi);
+                tmem_ld16(tl + (uint32_t)(a.nfull + o0), lo);
+                if (t < a.T) {
+                    const int n = min(16, a.nfull - o0);
+                    for (int q = 0; q < n; ++q) dst[o0 + q] = hi[q] + lo[q];
+                }
+            }
+            if (t < a.T) {
+                a.pstats[((long long)j * a.T + t) * 2 + 0] = s1;
+                a.pstats[((long long)j * a.T + t) * 2 + 1] = s2;
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&bars[2 * STAGES + 1]));
+            ++seg;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(ncols)
+                     : "memory");
+    }
+}
+
+// ---------------------------------------------------------------------------------------------
+// Wpack[r][e] = hi / lo bf16 parts of W[e][o] (r = o for hi, r = nfull + o for lo; 0 for pad)
+
+__global__ void k_pack_w(WSegs W, int nfull, int NB, int K, uint16_t* __restrict__ Wpack) {
+    const int e = blockIdx.x * blockDim.x + threadIdx.x;
+    if (e >= K) return;
+    for (int o = 0; o < nfull; ++o) {
+        const int s = seg_of(W, o);
+        const float w = W.ptr[s][(int64_t)e * W.width[s] + (o - W.off[s])];
+        const __nv_bfloat16 h = __float2bfloat16_rn(w);
+        const float rem = w - __bfloat162float(h);
+        Wpack[(int64_t)o * K + e] = __bfloat16_as_ushort(h);
+        Wpack[(int64_t)(nfull + o) * K + e] = __bfloat16_as_ushort(__float2bfloat16_rn(rem));
+    }
+    for (int r = 2 * nfull; r < NB; ++r) Wpack[(int64_t)r * K + e] = 0;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        cudaDriverEntryPointQueryResult q;
+        void* p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (PFN_cuTensorMapEncodeTiled_v12000)p;
+    }
+    return fn;
+}
+
+bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows) {
+    auto enc = get_encode();
+    if (!enc) return false;
+    cuuint64_t gdim[2] = {inner, rows};
+    cuuint64_t gstride[1] = {inner * 2};
+    cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+    cuuint32_t es[2] = {1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), gdim, gstride,
+                     box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+int num_sms() {
+    static int n = 0;
+    if (!n) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        if (n <= 0) n = 148;
+    }
+    return n;
+}
+
+}  // namespace
+
+int proj_tc_nb(int nfull) {
+    int nb = (2 * nfull + 15) / 16 * 16;
+    if (nb > 256) nb = (nb + 31) / 32 * 32;  // two equal chunks, each a multiple of 16
+    return nb;
+}
+
+ProjTcPlan plan_proj_tc(int T, int K, int nfull, int nsm) {
+    ProjTcPlan p;
+    p.KB = (K + BK - 1) / BK;
+    p.MT = (T + BM - 1) / BM;
+    p.W = (long long)p.KB * p.MT;
+    const int sms = nsm > 0 ? nsm : 148;
+    long long P = std::min<long long>(sms, std::max<long long>(1, p.W / 4));
+    p.P = (int)P;
+    const long long per = p.W / p.P;  // >= 4
+    p.nseg = (int)((p.KB + per - 1) / per) + 1;
+    if (p.nseg > p.P) p.nseg = p.P;
+    p.NB = proj_tc_nb(nfull);
+    p.nchunk = p.NB > 256 ? 2 : 1;
+    return p;
+}
+
+int proj_tc_stages(int NB) {
+    const size_t stage = (size_t)BM * BK * 2 + (size_t)NB * BK * 2;
+    int s = (int)((220 * 1024 - 2048) / stage);
+    return s > MAXSTAGES ? MAXSTAGES : s;
+}
+
+size_t proj_tc_smem(int NB) {
+    const int S = proj_tc_stages(NB);
+    return (size_t)S * (BM * BK * 2 + (size_t)NB * BK * 2) + (2 * S + 2) * 8 + 16 + 1024;
+}
+
+cudaError_t launch_pack_w(const WSegs& W, int nfull, int NB, int K, uint16_t* Wpack, cudaStream_t st) {
+    k_pack_w<<<(K + 255) / 256, 256, 0, st>>>(W, nfull, NB, K, Wpack); note_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_proj_tc(const uint16_t* X, int T, int K, const uint16_t* Wpack, int nfull,
+                           const ProjTcPlan& p, float* part, float* pstats, int* err,
+                           cudaStream_t st) {
+    CUtensorMap ma, mb;
+    if (!make_map(&ma, X, (uint64_t)K, (uint64_t)T, BM)) return cudaErrorInvalidValue;
+    if (!make_map(&mb, Wpack, (uint64_t)K, (uint64_t)p.NB, (uint32_t)(p.NB / p.nchunk)))
+        return cudaErrorInvalidValue;
+    cudaError_t e = cudaMemsetAsync(part, 0, (size_t)p.nseg * T * nfull * sizeof(float), st);
+    if (e != cudaSuccess) return e;
+    e = cudaMemsetAsync(pstats, 0, (size_t)p.nseg * T * 2 * sizeof(float), st);
+    if (e != cudaSuccess) return e;
+    const size_t sm = proj_tc_smem(p.NB);
+    e = cudaFuncSetAttribute((const void*)k_proj_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+    ProjTcArgs a;
+    a.T = T;
+    a.KB = p.KB;
+    a.MT = p.MT;
+    a.W = p.W;
+    a.P = p.P;
+    a.nfull = nfull;
+    a.NB = p.NB;
+    a.nchunk = p.nchunk;
+    a.nseg = p.nseg;
+    a.stages = proj_tc_stages(p.NB);
+    if (a.stages < 2) return cudaErrorInvalidValue;
+    a.part = part;
+    a.pstats = pstats;
+    a.err = err;
+    k_proj_tc<<<p.P, NTHREADS, sm, st>>>(ma, mb, a); note_launch();
+    return cudaGetLastError();
+}
+
+int device_sms() { return num_sms(); }
+
+}  // namespace xhc

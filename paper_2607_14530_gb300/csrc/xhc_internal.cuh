@@ -49,6 +49,18 @@ struct WSegsOut {
     int n;
 };
 
+// Stream-K plan of the tensor-core full-state projection.
+struct ProjTcPlan {
+    int KB, MT;      // k-blocks per tile, token tiles
+    long long W;     // total k-blocks
+    int P;           // persistent CTAs
+    int nseg;        // partial slots per tile
+    int NB;          // B rows (hi + lo + pad)
+    int nchunk;      // MMA instructions per k-step
+};
+ProjTcPlan plan_proj_tc(int T, int K, int nfull, int nsm);
+int device_sms();
+
 // Byte offsets of the per-group buffers for a given T (all 256-byte aligned).
 struct Layout {
     // saved
@@ -64,6 +76,8 @@ struct Layout {
     size_t hres;            // f32 [T][k*k]
     size_t saved_total;
     // workspace
+    size_t err;             // int: device error word (first 256 bytes of the workspace)
+    size_t wpack;           // bf16 [NB][N*C]: hi / lo rows of the full-state projection weight
     size_t part;            // f32 [splits][T][nmax] projection split-K partials
     size_t pstats;          // f32 [splits][T][2]
     size_t wsum;            // f32 [N]: column sums of W_r
@@ -83,6 +97,7 @@ struct Layout {
     size_t colscr;          // f32 [64][256]: column-sum scratch
     size_t ws_total;
     int splits_full, splits_act, nslice, tsplits, ntiles;
+    ProjTcPlan tc;
 };
 
 constexpr int NRED = 112;    // per-token reduction slots (>= k*K + k*k + K*K)
@@ -214,6 +229,10 @@ void note_launch();  // counts every kernel launch of the library
 
 cudaError_t launch_rowproj(const uint16_t* A, int64_t lda, int K, int T, const WSegs& W, int n,
                            int splits, float* part, float* pstats, cudaStream_t st);
+cudaError_t launch_pack_w(const WSegs& W, int nfull, int NB, int K, uint16_t* Wpack, cudaStream_t st);
+cudaError_t launch_proj_tc(const uint16_t* X, int T, int K, const uint16_t* Wpack, int nfull,
+                           const ProjTcPlan& p, float* part, float* pstats, int* err,
+                           cudaStream_t st);
 cudaError_t launch_colsum(const float* in, int rows, int ld, int n, float* out, int accumulate,
                           float* scratch, cudaStream_t st);
 cudaError_t launch_sub_rows(float* G, int rows, int n, const float* v, cudaStream_t st);

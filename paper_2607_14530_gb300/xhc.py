@@ -46,7 +46,7 @@ _Grads = _Params  # same layout (float* instead of const float*)
 class _SavedLayout(ctypes.Structure):
     _fields_ = [("I", ctypes.c_size_t), ("p", ctypes.c_size_t), ("hpre", ctypes.c_size_t),
                 ("hpost", ctypes.c_size_t * MAX_GROUP), ("hres", ctypes.c_size_t),
-                ("xact", ctypes.c_size_t)]
+                ("xact", ctypes.c_size_t), ("zfull", ctypes.c_size_t), ("stats", ctypes.c_size_t)]
 
 
 class XhcError(RuntimeError):
@@ -77,6 +77,7 @@ def lib() -> ctypes.CDLL:
         L.xhc_pre_bwd.argtypes = [vp, ctypes.c_int, i64, P, vp, vp, vp, P, vp, vp, vp]
         L.xhc_saved_layout_of.argtypes = [vp, i64, ctypes.POINTER(_SavedLayout)]
         L.xhc_route_noalloc.argtypes = [vp, i64, P, vp, vp, vp, vp, vp]
+        L.xhc_workspace_error.argtypes = [vp, ctypes.POINTER(ctypes.c_int), ctypes.c_int]
         L.xhc_trace_enable.argtypes = [ctypes.c_int]
         L.xhc_trace_count.restype = ctypes.c_int
         L.xhc_trace_record.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_char_p),
@@ -273,14 +274,24 @@ class Group:
                    hpre=view(L.hpre, T * G * N, torch.float32).view(T, G, N),
                    hres=view(L.hres, T * k * k, torch.float32).view(T, k, k),
                    xact=view(L.xact, G * T * k * cfg.C, torch.bfloat16).view(G, T, k, cfg.C))
+        nfull = (N if cfg.has_router else 0) + G * N
+        out["zfull"] = view(L.zfull, T * nfull, torch.float32).view(T, nfull)
+        out["stats"] = view(L.stats, T * 2, torch.float32).view(T, 2)
         out["hpost"] = [view(L.hpost[t], T * k * cfg.K(t), torch.float32).view(T, k, cfg.K(t))
                         for t in range(G)]
         return out
 
     def alloc(self, T: int, device="cuda"):
         """(saved, workspace) uint8 CUDA tensors of the sizes the library asks for."""
-        return (torch.empty(self.saved_bytes(T), dtype=torch.uint8, device=device),
-                torch.empty(self.workspace_bytes(T), dtype=torch.uint8, device=device))
+        ws = torch.empty(self.workspace_bytes(T), dtype=torch.uint8, device=device)
+        ws[:256].zero_()  # device error word
+        return (torch.empty(self.saved_bytes(T), dtype=torch.uint8, device=device), ws)
+
+    def device_error(self, ws, clear: bool = False) -> int:
+        """The workspace's device error word (nonzero: a bounded wait gave up).  Synchronous."""
+        code = ctypes.c_int()
+        lib().xhc_workspace_error(_ptr(ws), ctypes.byref(code), 1 if clear else 0)
+        return code.value
 
     def params(self, P: dict) -> _Params:
         return _fill(_Params(), P, self.cfg)

@@ -61,6 +61,39 @@ def run_oracle(cfg: Config, inp, P, grads=None):
     return res
 
 
+def alpha_term_scales(cfg: Config, inp, P, grads):
+    """For each gating scalar alpha, the sum over tokens and map entries of |d L / d alpha| taken
+    term by term (the oracle's forward broadcasts alpha, so passing it per entry gives the
+    per-term contributions).  A scalar gradient is a sum of T * (map size) such terms with
+    cancellation; its floating-point error scale is this sum of magnitudes, not |sum|."""
+    ocfg = oracle_cfg(cfg)
+    T = inp["X"].shape[0]
+    P64 = {n: v.to(F64) for n, v in P.items()}
+    X = inp["X"].to(F64)
+    outs = [o.to(F64) for o in inp["outs"]]
+    k, N, G = cfg.k, cfg.N, cfg.G
+    a_pre = [torch.full((T, N), float(P64["alpha_pre"][t]), dtype=F64, requires_grad=True) for t in range(G)]
+    a_post = [torch.full((T, k, cfg.K(t)), float(P64["alpha_post"][t]), dtype=F64, requires_grad=True)
+              for t in range(G)]
+    a_res = torch.full((1, T, k, k), float(P64["alpha_res"][0]), dtype=F64, requires_grad=True)
+    Pp = dict(P64)
+    Pp["alpha_pre"], Pp["alpha_post"], Pp["alpha_res"] = a_pre, a_post, a_res
+    Xo, ins, _ = O.forward(ocfg, Pp, X, outs)
+    L = (Xo * grads["dX"].to(F64)).sum() + sum((a * d.to(F64)).sum() for a, d in zip(ins, grads["d_inputs"]))
+    g = torch.autograd.grad(L, a_pre + a_post + [a_res])
+    return dict(alpha_pre=torch.stack([x.abs().sum() for x in g[:G]]),
+                alpha_post=torch.stack([x.abs().sum() for x in g[G:2 * G]]),
+                alpha_res=g[-1].abs().sum().reshape(1))
+
+
+def assert_alpha_close(gpu, ref, scale, name, tol=F32_REL):
+    g = gpu.detach().to("cpu", F64)
+    r = ref.detach().to("cpu", F64)
+    err = (g - r).abs()
+    bad = err > tol * scale
+    assert not bool(bad.any()), f"{name}: error {err.tolist()} vs {tol} x term scale {scale.tolist()}"
+
+
 def assert_bf16_close(gpu, ref, name):
     g = gpu.detach().to("cpu", F64)
     r = ref.detach().to("cpu", F64)
