@@ -148,9 +148,13 @@ Layout make_layout(const Dims& d, int64_t T) {
     L.saved_total = o;
 
     const int rowblocks = (int)((T + 63) / 64);
-    L.tc = plan_proj_tc((int)T, d.N * d.C, d.nfull, device_sms());
-    L.splits_full = L.tc.nseg;
-    L.splits_act = pick_splits(rowblocks, d.k * d.C);
+    const int sms = device_sms();
+    L.tc = plan_proj_tc((int)T, d.N * d.C, d.nfull, sms);
+    L.tca = plan_proj_tc((int)T, d.k * d.C, nact_max, sms);
+    L.twf = plan_proj_tc(d.N * d.C, (int)T, d.nfull, sms);
+    L.twa = plan_proj_tc(d.k * d.C, (int)T, nact_max, sms);
+    L.splits_full = std::max(L.tc.nseg, pick_splits(rowblocks, d.N * d.C));
+    L.splits_act = std::max(L.tca.nseg, pick_splits(rowblocks, d.k * d.C));
     L.nslice = (d.C + 255) / 256;
     const int ts_full = pick_tsplits(d.N * d.C, (int)T);
     const int ts_act = pick_tsplits(d.k * d.C, (int)T);
@@ -158,7 +162,9 @@ Layout make_layout(const Dims& d, int64_t T) {
     L.ntiles = (int)((T + 127) / 128);
     o = 0;
     L.err = o; o = al(o + 256);
-    L.wpack = o; o = al(o + (size_t)L.tc.NB * d.N * d.C * 2);
+    L.wpack = o;
+    o = al(o + std::max((size_t)L.tc.NB * d.N * d.C, (size_t)L.tca.NB * d.k * d.C) * 2);
+    L.dzpack = o; o = al(o + (size_t)std::max(L.twf.NB, L.twa.NB) * ((t + 7) / 8 * 8) * 2);
     L.part = o;
     o = al(o + std::max((size_t)L.splits_full * d.nfull, (size_t)L.splits_act * nact_max) * t * 4);
     L.pstats = o; o = al(o + (size_t)std::max(L.splits_full, L.splits_act) * t * 2 * 4);
@@ -175,7 +181,11 @@ Layout make_layout(const Dims& d, int64_t T) {
     L.du = o; o = al(o + (Kmax > 1 ? t * Kmax * d.C * 4 : 0));
     L.tokgrad = o; o = al(o + t * NTG * 4);
     L.wpart = o;
-    o = al(o + std::max((size_t)ts_full * d.N * d.C * d.nfull, (size_t)ts_act * d.k * d.C * nact_max) * 4);
+    {
+        size_t w1 = std::max((size_t)ts_full * d.N * d.C * d.nfull, (size_t)ts_act * d.k * d.C * nact_max);
+        size_t w2 = std::max((size_t)L.twf.nseg * d.N * d.C * d.nfull, (size_t)L.twa.nseg * d.k * d.C * nact_max);
+        o = al(o + std::max(w1, w2) * 4);
+    }
     L.cpart = o; o = al(o + (size_t)L.ntiles * d.kapsum * d.C * 4);
     L.colscr = o; o = al(o + (size_t)64 * 256 * 4);
     L.ws_total = o;
@@ -454,10 +464,22 @@ ConvPtrs conv_of(const Dims& d, const xhc_params* P, int slot) {
 xhc_status active_maps(const Ctx& c, int slot, const xhc_params* P) {
     const Dims& d = c.d;
     const WSegs wa = act_segs(d, P, slot);
-    XHC_K("rowproj_active", c.st, launch_rowproj(c.xact(slot), (int64_t)d.k * d.C, d.k * d.C, c.T, wa, d.nact[slot],
-                            c.L.splits_act, c.W<float>(c.L.part), c.W<float>(c.L.pstats), c.st));
+    int splits = c.L.splits_act;
+    if (c.T < 128 || d.k * d.C < 64) {
+        XHC_K("rowproj_active", c.st, launch_rowproj(c.xact(slot), (int64_t)d.k * d.C, d.k * d.C, c.T, wa,
+                                                     d.nact[slot], c.L.splits_act, c.W<float>(c.L.part),
+                                                     c.W<float>(c.L.pstats), c.st));
+    } else {
+        ProjTcPlan pl = plan_proj_tc(c.T, d.k * d.C, d.nact[slot], device_sms());
+        splits = pl.nseg;
+        XHC_K("pack_w", c.st, launch_pack_w(wa, d.nact[slot], pl.NB, d.k * d.C,
+                                            c.W<uint16_t>(c.L.wpack), c.st));
+        XHC_K("proj_tc_active", c.st, launch_proj_tc(c.xact(slot), c.T, d.k * d.C, c.W<uint16_t>(c.L.wpack),
+                                                     d.nact[slot], pl, c.W<float>(c.L.part),
+                                                     c.W<float>(c.L.pstats), c.W<int>(c.L.err), c.st));
+    }
     XHC_K("coef_act", c.st, launch_coef_act(d, slot, c.T, c.W<float>(c.L.part), c.W<float>(c.L.pstats),
-                             c.L.splits_act, P->alpha_post, P->b_post[slot], P->alpha_res, P->b_res,
+                             splits, P->alpha_post, P->b_post[slot], P->alpha_res, P->b_res,
                              c.S<float>(c.L.zact[slot]), c.S<float>(c.L.rs[slot]),
                              c.S<float>(c.L.hpost[slot]), c.S<float>(c.L.hres), c.st));
     return XHC_OK;
@@ -558,9 +580,19 @@ xhc_status xhc_post_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
                               c.W<float>(c.L.tokmat), dxact, c.W<float>(c.L.du), d_out, c.st));
     const WSegs wa = act_segs(d, P, slot);
     XHC_K("gemm_dzw", c.st, launch_gemm_dzw(d, T32, c.W<float>(c.L.dz), n, n, wa, d.k * d.C, dxact, c.st));
-    const int ts = std::min(c.L.tsplits, pick_tsplits(d.k * d.C, T32));
-    XHC_K("wgrad_active", c.st, launch_wgrad(c.xact(slot), (int64_t)d.k * d.C, d.k * d.C, T32, c.W<float>(c.L.dz), n,
-                          n, ts, c.W<float>(c.L.wpart), act_segs_g(d, g, slot), c.st));
+    if (T32 < 64 || d.k * d.C < 128) {
+        const int ts = std::min(c.L.tsplits, pick_tsplits(d.k * d.C, T32));
+        XHC_K("wgrad_active", c.st, launch_wgrad(c.xact(slot), (int64_t)d.k * d.C, d.k * d.C, T32,
+                                                 c.W<float>(c.L.dz), n, n, ts, c.W<float>(c.L.wpart),
+                                                 act_segs_g(d, g, slot), c.st));
+    } else {
+        ProjTcPlan pl = plan_proj_tc(d.k * d.C, T32, n, device_sms());
+        XHC_K("wgrad_tc_active", c.st, launch_wgrad_tc(c.xact(slot), T32, d.k * d.C, c.W<float>(c.L.dz), n, n,
+                                                       c.W<uint16_t>(c.L.dzpack), pl, c.W<float>(c.L.wpart),
+                                                       c.W<int>(c.L.err), c.st));
+        XHC_K("wgrad_reduce", c.st, launch_wgrad_reduce(c.W<float>(c.L.wpart), pl.nseg, d.k * d.C, n,
+                                                        act_segs_g(d, g, slot), c.st));
+    }
     float* tg = c.W<float>(c.L.tokgrad);
     float* scr = c.W<float>(c.L.colscr);
     XHC_K("colsum", c.st, launch_colsum(tg, T32, NTG, d.k * K, g->b_post[slot], 1, scr, c.st));
@@ -608,9 +640,19 @@ xhc_status xhc_pre_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
     XHC_K("full_dx", c.st, launch_full_dx(d, T32, c.W<float>(c.L.dz), wf, X, dinput, c.S<float>(c.L.hpre),
                             c.S<int>(c.L.I), c.W<float>(c.L.dxact), c.W<float>(c.L.tokgrad), dX,
                             c.st));
-    const int ts = std::min(c.L.tsplits, pick_tsplits(d.N * d.C, T32));
-    XHC_K("wgrad_full", c.st, launch_wgrad(X, (int64_t)d.N * d.C, d.N * d.C, T32, c.W<float>(c.L.dz), d.nfull,
-                          d.nfull, ts, c.W<float>(c.L.wpart), full_segs_g(d, g), c.st));
+    if (T32 < 64 || d.N * d.C < 128) {
+        const int ts = std::min(c.L.tsplits, pick_tsplits(d.N * d.C, T32));
+        XHC_K("wgrad_full", c.st, launch_wgrad(X, (int64_t)d.N * d.C, d.N * d.C, T32, c.W<float>(c.L.dz),
+                                               d.nfull, d.nfull, ts, c.W<float>(c.L.wpart),
+                                               full_segs_g(d, g), c.st));
+    } else {
+        const ProjTcPlan& pl = c.L.twf;
+        XHC_K("wgrad_tc_full", c.st, launch_wgrad_tc(X, T32, d.N * d.C, c.W<float>(c.L.dz), d.nfull, d.nfull,
+                                                     c.W<uint16_t>(c.L.dzpack), pl, c.W<float>(c.L.wpart),
+                                                     c.W<int>(c.L.err), c.st));
+        XHC_K("wgrad_reduce", c.st, launch_wgrad_reduce(c.W<float>(c.L.wpart), pl.nseg, d.N * d.C, d.nfull,
+                                                        full_segs_g(d, g), c.st));
+    }
     float* tg = c.W<float>(c.L.tokgrad);
     float* scr = c.W<float>(c.L.colscr);
     XHC_K("colsum", c.st, launch_colsum(tg + 2, T32, NTG, d.G * d.N, g->b_pre, 1, scr, c.st));

@@ -419,6 +419,13 @@ __global__ void k_wgrad_reduce(const float* __restrict__ wpart, int splits, int 
     *dst += s;
 }
 
+cudaError_t launch_wgrad_reduce(const float* wpart, int splits, int E, int n, const WSegsOut& G,
+                                cudaStream_t st) {
+    const int64_t tot = (int64_t)E * n;
+    k_wgrad_reduce<<<(unsigned)((tot + 255) / 256), 256, 0, st>>>(wpart, splits, E, n, G); note_launch();
+    return cudaGetLastError();
+}
+
 template <int NT>
 static cudaError_t wgrad_nt(const uint16_t* A, int64_t lda, int E, int T, const float* dz, int ldz,
                             int n, int tsplits, float* wpart, const WSegsOut& G, cudaStream_t st) {

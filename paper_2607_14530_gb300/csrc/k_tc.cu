@@ -76,9 +76,23 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t addr) {
     return d;
 }
 
+// Shared-memory matrix descriptor: MN-major operand, 128-byte swizzle.  The tile is stored as
+// blocks of 64 MN-contiguous elements (one 128-byte row per K index, 8-row groups 1024 B apart);
+// consecutive 64-element MN blocks are `lbo` bytes apart.
+__device__ __forceinline__ uint64_t sw128_desc_mn(uint32_t addr, uint32_t lbo) {
+    uint64_t d = 0;
+    d |= (uint64_t)((addr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;     // leading byte offset: between MN blocks
+    d |= (uint64_t)(1024u >> 4) << 32;               // stride byte offset: between 8-row K groups
+    d |= (uint64_t)1 << 46;
+    d |= (uint64_t)2 << 61;
+    return d;
+}
+
 // Instruction descriptor, kind::f16: bf16 A and B, fp32 accumulator, both K-major, M x N.
-__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
-    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool a_mn = false) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn ? 1u : 0u) << 15) |
+           ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
 __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
@@ -132,6 +146,10 @@ __device__ __forceinline__ long long range_start(long long W, int P, int c) {
     return (W * c) / P;
 }
 
+// A_MN = false: rows of A are tokens, A tile = X[m*128.., kb*64..] (K-major); row statistics on.
+// A_MN = true : rows of A are state elements e, K = tokens; the A tile is X[t0.., e0..] as stored
+//               (two 64-wide e blocks, MN-major); no statistics (weight gradients).
+template <bool A_MN>
 __global__ void __launch_bounds__(NTHREADS, 1)
 k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
           ProjTcArgs a) {
@@ -191,7 +209,12 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                 const uint32_t full = smem_u32(&bars[s]);
                 mbar_expect_tx(full, STAGE);
                 unsigned char* st = smem + (size_t)s * STAGE;
-                tma_load_2d(smem_u32(st), &tmA, kb * BK, m * BM, full);
+                if (A_MN) {
+                    tma_load_2d(smem_u32(st), &tmA, m * BM, kb * BK, full);
+                    tma_load_2d(smem_u32(st + A_BYTES / 2), &tmA, m * BM + 64, kb * BK, full);
+                } else {
+                    tma_load_2d(smem_u32(st), &tmA, kb * BK, m * BM, full);
+                }
                 const int nb_box = a.NB / a.nchunk;
                 for (int q = 0; q < a.nchunk; ++q)
                     tma_load_2d(smem_u32(st + A_BYTES + (size_t)q * nb_box * 128), &tmB, kb * BK,
@@ -202,7 +225,7 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
         // ---------------- MMA issuer ----------------
         if (lane == 0) {
             const int nb_chunk = a.NB / a.nchunk;
-            const uint32_t idesc = idesc_bf16(BM, nb_chunk);
+            const uint32_t idesc = idesc_bf16(BM, nb_chunk, A_MN);
             long long it = 0;
             int seg = 0;
             long long g = g0;
@@ -229,7 +252,10 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                     const uint32_t bbase = abase + A_BYTES;
 #pragma unroll
                     for (int kk = 0; kk < BK / 16; ++kk) {
-                        const uint64_t ad = sw128_desc(abase + kk * 32);
+                        // K-major: +32 B per 16 k-elements inside the swizzled row; MN-major:
+                        // +16 K-rows of 128 B
+                        const uint64_t ad = A_MN ? sw128_desc_mn(abase + kk * 2048, A_BYTES / 2)
+                                                 : sw128_desc(abase + kk * 32);
                         for (int q = 0; q < a.nchunk; ++q) {
                             const uint64_t bd = sw128_desc(bbase + q * nb_chunk * 128 + kk * 32);
                             mma_bf16(tmem + (uint32_t)(q * nb_chunk), ad, bd, idesc,
@@ -264,17 +290,19 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                     ok = false;
                     break;
                 }
-                // row r of the A tile: 128 bytes, 16-byte chunks permuted by the swizzle (the
-                // sum over the row does not depend on the order)
-                const uint4* row = reinterpret_cast<const uint4*>(smem + (size_t)s * STAGE + r * 128);
+                if (!A_MN) {
+                    // row r of the A tile: 128 bytes, 16-byte chunks permuted by the swizzle (the
+                    // sum over the row does not depend on the order)
+                    const uint4* row = reinterpret_cast<const uint4*>(smem + (size_t)s * STAGE + r * 128);
 #pragma unroll
-                for (int q = 0; q < 8; ++q) {
-                    float f[8];
-                    unpack8(row[q], f);
+                    for (int q = 0; q < 8; ++q) {
+                        float f[8];
+                        unpack8(row[q], f);
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        s1 += f[e];
-                        s2 = fmaf(f[e], f[e], s2);
+                        for (int e = 0; e < 8; ++e) {
+                            s1 += f[e];
+                            s2 = fmaf(f[e], f[e], s2);
+                        }
                     }
                 }
                 __syncwarp();
@@ -304,7 +332,7 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                     for (int q = 0; q < n; ++q) dst[o0 + q] = hi[q] + lo[q];
                 }
             }
-            if (t < a.T) {
+            if (!A_MN && t < a.T) {
                 a.pstats[((long long)j * a.T + t) * 2 + 0] = s1;
                 a.pstats[((long long)j * a.T + t) * 2 + 1] = s2;
             }
@@ -353,17 +381,22 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
     return fn;
 }
 
-bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows) {
+bool make_map_box(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows,
+                  uint32_t box_inner, uint32_t box_rows, uint64_t row_bytes = 0) {
     auto enc = get_encode();
     if (!enc) return false;
     cuuint64_t gdim[2] = {inner, rows};
-    cuuint64_t gstride[1] = {inner * 2};
-    cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+    cuuint64_t gstride[1] = {row_bytes ? row_bytes : inner * 2};
+    cuuint32_t box[2] = {box_inner, box_rows};
     cuuint32_t es[2] = {1, 1};
     CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), gdim, gstride,
                      box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
+}
+
+bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows) {
+    return make_map_box(m, base, inner, rows, (uint32_t)BK, box_rows);
 }
 
 int num_sms() {
@@ -429,7 +462,7 @@ cudaError_t launch_proj_tc(const uint16_t* X, int T, int K, const uint16_t* Wpac
     e = cudaMemsetAsync(pstats, 0, (size_t)p.nseg * T * 2 * sizeof(float), st);
     if (e != cudaSuccess) return e;
     const size_t sm = proj_tc_smem(p.NB);
-    e = cudaFuncSetAttribute((const void*)k_proj_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    e = cudaFuncSetAttribute((const void*)k_proj_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
     ProjTcArgs a;
     a.T = T;
@@ -446,7 +479,61 @@ cudaError_t launch_proj_tc(const uint16_t* X, int T, int K, const uint16_t* Wpac
     a.part = part;
     a.pstats = pstats;
     a.err = err;
-    k_proj_tc<<<p.P, NTHREADS, sm, st>>>(ma, mb, a); note_launch();
+    k_proj_tc<false><<<p.P, NTHREADS, sm, st>>>(ma, mb, a); note_launch();
+    return cudaGetLastError();
+}
+
+// dZpack[r][t]: hi / lo bf16 parts of dz[t][o] (r = o for hi, r = n + o for lo, 0 for pad), the
+// K-major B operand of the weight gradient.
+__global__ void k_pack_dz(const float* __restrict__ dz, int ldz, int n, int NB, int T, int Tp,
+                          uint16_t* __restrict__ dzp) {
+    const int t = blockIdx.x * blockDim.x + threadIdx.x;
+    if (t >= T) return;
+    for (int o = 0; o < n; ++o) {
+        const float w = dz[(int64_t)t * ldz + o];
+        const __nv_bfloat16 h = __float2bfloat16_rn(w);
+        dzp[(int64_t)o * Tp + t] = __bfloat16_as_ushort(h);
+        dzp[(int64_t)(n + o) * Tp + t] = __bfloat16_as_ushort(__float2bfloat16_rn(w - __bfloat162float(h)));
+    }
+    for (int r = 2 * n; r < NB; ++r) dzp[(int64_t)r * Tp + t] = 0;
+}
+
+// Weight gradient on the tensor cores: part[j][e][o] = sum over the segment's tokens of
+// A[t][e] dz[t][o] (A = X or the active state, [T, E] bf16), with dz split into bf16 hi/lo.
+cudaError_t launch_wgrad_tc(const uint16_t* A, int T, int E, const float* dz, int ldz, int n,
+                            uint16_t* dzpack, const ProjTcPlan& p, float* part, int* err,
+                            cudaStream_t st) {
+    const int Tp = (T + 7) / 8 * 8;  // 16-byte row stride for the tensor map
+    k_pack_dz<<<(T + 255) / 256, 256, 0, st>>>(dz, ldz, n, p.NB, T, Tp, dzpack); note_launch();
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    CUtensorMap ma, mb;
+    // A: [T rows, E inner], box {64 e, 64 tokens}; B: [NB rows, T inner], box {64 tokens, NB}
+    if (!make_map_box(&ma, A, (uint64_t)E, (uint64_t)T, 64, BK)) return cudaErrorInvalidValue;
+    if (!make_map_box(&mb, dzpack, (uint64_t)T, (uint64_t)p.NB, BK, (uint32_t)(p.NB / p.nchunk),
+                      (uint64_t)Tp * 2))
+        return cudaErrorInvalidValue;
+    e = cudaMemsetAsync(part, 0, (size_t)p.nseg * E * n * sizeof(float), st);
+    if (e != cudaSuccess) return e;
+    const size_t sm = proj_tc_smem(p.NB);
+    e = cudaFuncSetAttribute((const void*)k_proj_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+    ProjTcArgs a;
+    a.T = E;  // rows of the output
+    a.KB = p.KB;
+    a.MT = p.MT;
+    a.W = p.W;
+    a.P = p.P;
+    a.nfull = n;
+    a.NB = p.NB;
+    a.nchunk = p.nchunk;
+    a.nseg = p.nseg;
+    a.stages = proj_tc_stages(p.NB);
+    if (a.stages < 2) return cudaErrorInvalidValue;
+    a.part = part;
+    a.pstats = nullptr;
+    a.err = err;
+    k_proj_tc<true><<<p.P, NTHREADS, sm, st>>>(ma, mb, a); note_launch();
     return cudaGetLastError();
 }
 

@@ -97,7 +97,11 @@ struct Layout {
     size_t colscr;          // f32 [64][256]: column-sum scratch
     size_t ws_total;
     int splits_full, splits_act, nslice, tsplits, ntiles;
-    ProjTcPlan tc;
+    ProjTcPlan tc;          // full-state projection: rows T, K = N*C
+    ProjTcPlan tca;         // active projection: rows T, K = k*C
+    ProjTcPlan twf;         // full weight gradient: rows N*C, K = T
+    ProjTcPlan twa;         // active weight gradient: rows k*C, K = T
+    size_t dzpack;          // bf16 [NB][T]: hi / lo rows of the projection-output gradient
 };
 
 constexpr int NRED = 112;    // per-token reduction slots (>= k*K + k*k + K*K)
@@ -233,6 +237,11 @@ cudaError_t launch_pack_w(const WSegs& W, int nfull, int NB, int K, uint16_t* Wp
 cudaError_t launch_proj_tc(const uint16_t* X, int T, int K, const uint16_t* Wpack, int nfull,
                            const ProjTcPlan& p, float* part, float* pstats, int* err,
                            cudaStream_t st);
+cudaError_t launch_wgrad_tc(const uint16_t* A, int T, int E, const float* dz, int ldz, int n,
+                            uint16_t* dzpack, const ProjTcPlan& p, float* part, int* err,
+                            cudaStream_t st);
+cudaError_t launch_wgrad_reduce(const float* wpart, int splits, int E, int n, const WSegsOut& G,
+                                cudaStream_t st);
 cudaError_t launch_colsum(const float* in, int rows, int ld, int n, float* out, int accumulate,
                           float* scratch, cudaStream_t st);
 cudaError_t launch_sub_rows(float* G, int rows, int n, const float* v, cudaStream_t st);
