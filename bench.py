@@ -85,7 +85,8 @@ def kernel_model(cfg, T):
     for t in range(G):
         if t > 0:
             add("input", T * C * f32 + xa + row)
-        add("rowproj_active", xa + k * C * nact[t] * f32 + T * nact[t] * f32, 2.0 * T * k * C * nact[t], "alu")
+        add("pack_w", k * C * nact[t] * f32 + 2 * nact[t] * k * C * b16)
+        add("proj_tc_active", xa + T * nact[t] * f32, 2.0 * T * k * C * 2 * nact[t], "hbm")
         add("coef_act", T * nact[t] * f32 * 2)
         if Ks[t] > 1 and gs:
             add("aug_gram", row)
@@ -100,7 +101,9 @@ def kernel_model(cfg, T):
         add("bwd_coef", T * nact[t] * f32 * 2)
         add("bwd_apply", dxn + xa + row + T * k * C * f32 + (T * Ks[t] * C * f32 if Ks[t] > 1 else row))
         add("gemm_dzw", T * nact[t] * f32 + 2 * T * k * C * f32, 2.0 * T * k * C * nact[t], "alu")
-        add("wgrad_active", xa + T * nact[t] * f32, 2.0 * T * k * C * nact[t], "alu")
+        add("wgrad_tc_active", xa + T * nact[t] * f32 + 2 * T * nact[t] * b16 + k * C * nact[t] * f32,
+            2.0 * T * k * C * 2 * nact[t], "hbm")
+        add("wgrad_reduce", 2 * k * C * nact[t] * f32)
         for _ in range(4 if last else 2):
             add("colsum", T * 16 * f32)
         if Ks[t] > 1:
@@ -111,8 +114,12 @@ def kernel_model(cfg, T):
         add("colsum", N * C * N * f32)
     add("full_dots", T * (N - k) * C * b16 + G * row)
     add("full_coef", T * (nfull + G * N) * f32)
-    add("full_dx", X + T * (N - k) * C * b16 + T * k * C * f32 + G * row + X, 2.0 * T * N * C * nfull, "alu")
-    add("wgrad_full", X + T * nfull * f32, 2.0 * T * N * C * nfull, "alu")
+    # tensor-core dX: X read, inactive dX rows read, active-row gradient read, d_input (once per
+    # token block), dX written
+    add("dx_tc", X + T * (N - k) * C * b16 + T * k * C * f32 + G * row + X, 2.0 * T * N * C * nfull, "hbm")
+    add("wgrad_tc_full", X + T * nfull * f32 + 2 * T * nfull * b16 + N * C * nfull * f32,
+        2.0 * T * N * C * 2 * nfull, "hbm")
+    add("wgrad_reduce", 2 * N * C * nfull * f32)
     add("colsum", T * G * N * f32)
     add("colsum", T * G * f32)
     if hr:
@@ -378,7 +385,7 @@ def run_xhc(args, wl_name):
                 ent["tflops"] = mm["flops"] / secs / 1e12
             ent["bound"] = mm["bound"]
         kernels[name] = ent
-    dom = max(per, key=lambda n: per[n][1])
+    dom = max((n for n in per if n in model), key=lambda n: per[n][1])
     mm = model[dom]
     cnt, tot = per[dom]
     secs = tot / cnt / 1000.0

@@ -165,6 +165,11 @@ Layout make_layout(const Dims& d, int64_t T) {
     L.wpack = o;
     o = al(o + std::max((size_t)L.tc.NB * d.N * d.C, (size_t)L.tca.NB * d.k * d.C) * 2);
     L.dzpack = o; o = al(o + (size_t)std::max(L.twf.NB, L.twa.NB) * ((t + 7) / 8 * 8) * 2);
+    {
+        const size_t ld = (size_t)(d.nfull + 7) / 8 * 8;
+        L.dz16 = o; o = al(o + t * ld * 2);
+        L.w16 = o; o = al(o + (size_t)d.N * d.C * ld * 2);
+    }
     L.part = o;
     o = al(o + std::max((size_t)L.splits_full * d.nfull, (size_t)L.splits_act * nact_max) * t * 4);
     L.pstats = o; o = al(o + (size_t)std::max(L.splits_full, L.splits_act) * t * 2 * 4);
@@ -637,9 +642,16 @@ xhc_status xhc_pre_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
                               c.S<int>(c.L.I), c.W<float>(c.L.dp), P->alpha_pre,
                               c.W<float>(c.L.dz), c.W<float>(c.L.tokgrad), c.st));
     const WSegs wf = full_segs(d, P);
-    XHC_K("full_dx", c.st, launch_full_dx(d, T32, c.W<float>(c.L.dz), wf, X, dinput, c.S<float>(c.L.hpre),
-                            c.S<int>(c.L.I), c.W<float>(c.L.dxact), c.W<float>(c.L.tokgrad), dX,
-                            c.st));
+    if (dx_tc_ok(T32, d.N, d.C, d.nfull)) {
+        XHC_K("dx_tc", c.st, launch_dx_tc(d, T32, c.W<float>(c.L.dz), wf, c.W<uint16_t>(c.L.dz16),
+                                          c.W<uint16_t>(c.L.w16), X, dinput, c.S<float>(c.L.hpre),
+                                          c.S<int>(c.L.I), c.W<float>(c.L.dxact), c.W<float>(c.L.tokgrad),
+                                          NTG, dX, c.W<int>(c.L.err), c.st));
+    } else {
+        XHC_K("full_dx", c.st, launch_full_dx(d, T32, c.W<float>(c.L.dz), wf, X, dinput, c.S<float>(c.L.hpre),
+                                              c.S<int>(c.L.I), c.W<float>(c.L.dxact),
+                                              c.W<float>(c.L.tokgrad), dX, c.st));
+    }
     if (T32 < 64 || d.N * d.C < 128) {
         const int ts = std::min(c.L.tsplits, pick_tsplits(d.N * d.C, T32));
         XHC_K("wgrad_full", c.st, launch_wgrad(X, (int64_t)d.N * d.C, d.N * d.C, T32, c.W<float>(c.L.dz),

@@ -539,4 +539,242 @@ cudaError_t launch_wgrad_tc(const uint16_t* A, int T, int E, const float* dz, in
 
 int device_sms() { return num_sms(); }
 
+// ---------------------------------------------------------------------------------------------
+// Full-state input gradient on the tensor cores (backward of the full-state projection, of the
+// norm statistics and of the dense reads):
+//   dX[t][i*C + c] = base + sum_o dZ[t][o] W[i*C + c][o] + a_t + b_t x[t][i*C + c]
+//   base = dX_act[t][j][c]                                  if stream i is active slot j
+//        = dX[t][i*C + c] + sum_q H_pre[t][q][i] d_input_q[t][c]   otherwise
+// Tiles of 128 tokens x 128 channels of one stream; MMA K = nfull (dZ and W in bf16: this term
+// is a small share of dX, whose storage is bf16).  Persistent CTAs take tiles with stride P, the
+// stream index fastest, so the d_input tile of a (token, channel) block is reused from L2.
+
+namespace {
+
+constexpr int DX_BN = 128;
+
+struct DxArgs {
+    int T, C, N, k, G;
+    int nkb, ksteps;      // k-blocks of 64, MMA k-steps of 16
+    int TT, CT;           // token tiles, channel tiles per stream
+    long long ntiles;
+    int P;
+    const uint16_t* X;
+    uint16_t* dX;
+    const uint16_t* dinput;
+    const float* hpre;
+    const int* I;
+    const float* dxact;
+    const float* scal;
+    int scal_ld;
+    int* err;
+};
+
+__global__ void __launch_bounds__(NTHREADS, 1)
+k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, DxArgs a) {
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    const uint32_t A_BYTES = (uint32_t)a.nkb * BM * BK * 2;
+    const uint32_t B_BYTES = (uint32_t)a.nkb * DX_BN * BK * 2;
+    const uint32_t STAGE = A_BYTES + B_BYTES;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 2 * STAGE);
+    // [0,2) full, [2,4) empty, [4,6) tmem full, [6,8) tmem empty
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 8);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(smem_u32(&bars[s]), 1);
+            mbar_init(smem_u32(&bars[2 + s]), 1);
+            mbar_init(smem_u32(&bars[4 + s]), 1);
+            mbar_init(smem_u32(&bars[6 + s]), 4);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(tmem_slot)), "r"(256u) : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const long long nloc = (a.ntiles > blockIdx.x) ? (a.ntiles - 1 - blockIdx.x) / a.P + 1 : 0;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            for (long long n = 0; n < nloc; ++n) {
+                const long long tile = blockIdx.x + n * a.P;
+                const int i = (int)(tile % a.N);
+                const long long rest = tile / a.N;
+                const int ct = (int)(rest % a.CT), tt = (int)(rest / a.CT);
+                const int s = (int)(n & 1);
+                if (n >= 2 && !mbar_wait(smem_u32(&bars[2 + s]), (uint32_t)(((n >> 1) - 1) & 1))) {
+                    atomicExch(a.err, 11);
+                    break;
+                }
+                const uint32_t full = smem_u32(&bars[s]);
+                mbar_expect_tx(full, STAGE);
+                unsigned char* st = smem + (size_t)s * STAGE;
+                for (int kb = 0; kb < a.nkb; ++kb) {
+                    tma_load_2d(smem_u32(st + kb * BM * BK * 2), &tmA, kb * BK, tt * BM, full);
+                    tma_load_2d(smem_u32(st + A_BYTES + kb * DX_BN * BK * 2), &tmB, kb * BK,
+                                i * a.C + ct * DX_BN, full);
+                }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16(BM, DX_BN);
+            for (long long n = 0; n < nloc; ++n) {
+                const int s = (int)(n & 1);
+                if (!mbar_wait(smem_u32(&bars[s]), (uint32_t)((n >> 1) & 1))) {
+                    atomicExch(a.err, 12);
+                    break;
+                }
+                if (n >= 2 && !mbar_wait(smem_u32(&bars[6 + s]), (uint32_t)(((n >> 1) - 1) & 1))) {
+                    atomicExch(a.err, 13);
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t abase = smem_u32(smem + (size_t)s * STAGE);
+                const uint32_t bbase = abase + A_BYTES;
+                for (int ks = 0; ks < a.ksteps; ++ks) {
+                    const int kb = ks >> 2, kk = ks & 3;
+                    mma_bf16(tmem + (uint32_t)(s * DX_BN), sw128_desc(abase + kb * BM * BK * 2 + kk * 32),
+                             sw128_desc(bbase + kb * DX_BN * BK * 2 + kk * 32), idesc, ks > 0 ? 1u : 0u);
+                }
+                mma_commit(smem_u32(&bars[2 + s]));  // operands consumed
+                mma_commit(smem_u32(&bars[4 + s]));  // accumulator ready
+            }
+        }
+    } else {
+        const int quarter = warp & 3;
+        const int r = quarter * 32 + lane;
+        for (long long n = 0; n < nloc; ++n) {
+            const long long tile = blockIdx.x + n * a.P;
+            const int i = (int)(tile % a.N);
+            const long long rest = tile / a.N;
+            const int ct = (int)(rest % a.CT), tt = (int)(rest / a.CT);
+            const int s = (int)(n & 1);
+            if (!mbar_wait(smem_u32(&bars[4 + s]), (uint32_t)((n >> 1) & 1))) {
+                atomicExch(a.err, 14);
+                break;
+            }
+            tc_fence_after();
+            const int t = tt * BM + r;
+            const uint32_t tl = tmem + (uint32_t)(s * DX_BN) + ((uint32_t)(quarter * 32) << 16);
+            int j = -1;
+            float h[4] = {0.f, 0.f, 0.f, 0.f};
+            float sa = 0.f, sb = 0.f;
+            if (t < a.T) {
+                for (int q = 0; q < a.k; ++q)
+                    if (a.I[(long long)t * a.k + q] == i) j = q;
+                for (int q = 0; q < a.G; ++q) h[q] = a.hpre[((long long)t * a.G + q) * a.N + i];
+                sa = a.scal[(long long)t * a.scal_ld + 0];
+                sb = a.scal[(long long)t * a.scal_ld + 1];
+            }
+            const long long rowoff = ((long long)t * a.N + i) * a.C + ct * DX_BN;
+            for (int c0 = 0; c0 < DX_BN; c0 += 16) {
+                float acc[16];
+                tmem_ld16(tl + (uint32_t)c0, acc);
+                if (t >= a.T) continue;
+                float x[16], v[16];
+                unpack8(*reinterpret_cast<const uint4*>(a.X + rowoff + c0), x);
+                unpack8(*reinterpret_cast<const uint4*>(a.X + rowoff + c0 + 8), x + 8);
+                const int c = ct * DX_BN + c0;
+                if (j >= 0) {
+                    const float4* b = reinterpret_cast<const float4*>(a.dxact + ((long long)t * a.k + j) * a.C + c);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const float4 f = b[q];
+                        v[4 * q] = f.x; v[4 * q + 1] = f.y; v[4 * q + 2] = f.z; v[4 * q + 3] = f.w;
+                    }
+                } else {
+                    unpack8(*reinterpret_cast<const uint4*>(a.dX + rowoff + c0), v);
+                    unpack8(*reinterpret_cast<const uint4*>(a.dX + rowoff + c0 + 8), v + 8);
+                    for (int q = 0; q < a.G; ++q) {
+                        float g[16];
+                        const uint16_t* dp = a.dinput + ((long long)q * a.T + t) * a.C + c;
+                        unpack8(*reinterpret_cast<const uint4*>(dp), g);
+                        unpack8(*reinterpret_cast<const uint4*>(dp + 8), g + 8);
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) v[e] = fmaf(h[q], g[e], v[e]);
+                    }
+                }
+                float o[16];
+#pragma unroll
+                for (int e = 0; e < 16; ++e) o[e] = v[e] + acc[e] + sa + sb * x[e];
+                *reinterpret_cast<uint4*>(a.dX + rowoff + c0) = pack8(o);
+                *reinterpret_cast<uint4*>(a.dX + rowoff + c0 + 8) = pack8(o + 8);
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&bars[6 + s]));
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(256u)
+                     : "memory");
+    }
+}
+
+// bf16 copies with a padded row stride: dst[r][o] = src[r][o] (o < n), 0 for n <= o < ld
+__global__ void k_pack_rows(WSegs W, int n, int rows, int ld, uint16_t* __restrict__ dst) {
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)rows * ld) return;
+    const int r = (int)(idx / ld), o = (int)(idx - (long long)r * ld);
+    float v = 0.f;
+    if (o < n) {
+        const int s = seg_of(W, o);
+        v = W.ptr[s][(long long)r * W.width[s] + (o - W.off[s])];
+    }
+    dst[idx] = __bfloat16_as_ushort(__float2bfloat16_rn(v));
+}
+
+}  // namespace
+
+bool dx_tc_ok(int T, int N, int C, int nfull) {
+    return T >= BM && C % DX_BN == 0 && nfull <= 3 * BK;
+}
+
+cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, uint16_t* dz16,
+                         uint16_t* w16, const uint16_t* X, const uint16_t* dinput, const float* hpre,
+                         const int* I, const float* dxact, const float* scal, int scal_ld,
+                         uint16_t* dX, int* err, cudaStream_t st) {
+    const int n = d.nfull, NC = d.N * d.C;
+    const int ld = (n + 7) / 8 * 8;
+    WSegs dzs;
+    memset(&dzs, 0, sizeof(dzs));
+    dzs.ptr[0] = dz; dzs.width[0] = n; dzs.off[0] = 0; dzs.off[1] = n; dzs.n = 1;
+    long long tot = (long long)T * ld;
+    k_pack_rows<<<(unsigned)((tot + 255) / 256), 256, 0, st>>>(dzs, n, T, ld, dz16); note_launch();
+    tot = (long long)NC * ld;
+    k_pack_rows<<<(unsigned)((tot + 255) / 256), 256, 0, st>>>(W, n, NC, ld, w16); note_launch();
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    CUtensorMap ma, mb;
+    if (!make_map_box(&ma, dz16, (uint64_t)n, (uint64_t)T, BK, BM, (uint64_t)ld * 2)) return cudaErrorInvalidValue;
+    if (!make_map_box(&mb, w16, (uint64_t)n, (uint64_t)NC, BK, DX_BN, (uint64_t)ld * 2)) return cudaErrorInvalidValue;
+    DxArgs a;
+    a.T = T; a.C = d.C; a.N = d.N; a.k = d.k; a.G = d.G;
+    a.nkb = (n + BK - 1) / BK;
+    a.ksteps = (n + 15) / 16;
+    a.TT = (T + BM - 1) / BM;
+    a.CT = d.C / DX_BN;
+    a.ntiles = (long long)a.TT * a.CT * d.N;
+    a.P = (int)std::min<long long>(num_sms(), a.ntiles);
+    a.X = X; a.dX = dX; a.dinput = dinput; a.hpre = hpre; a.I = I; a.dxact = dxact;
+    a.scal = scal; a.scal_ld = scal_ld; a.err = err;
+    const size_t sm = 2 * (size_t)a.nkb * (BM + DX_BN) * BK * 2 + 8 * 8 + 16 + 1024;
+    e = cudaFuncSetAttribute((const void*)k_dx_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+    k_dx_tc<<<a.P, NTHREADS, sm, st>>>(ma, mb, a); note_launch();
+    return cudaGetLastError();
+}
+
 }  // namespace xhc

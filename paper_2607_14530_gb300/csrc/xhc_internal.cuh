@@ -102,6 +102,8 @@ struct Layout {
     ProjTcPlan twf;         // full weight gradient: rows N*C, K = T
     ProjTcPlan twa;         // active weight gradient: rows k*C, K = T
     size_t dzpack;          // bf16 [NB][T]: hi / lo rows of the projection-output gradient
+    size_t dz16;            // bf16 [T][ld]: projection-output gradient (full-state dX GEMM)
+    size_t w16;             // bf16 [N*C][ld]: full-state projection weight rows
 };
 
 constexpr int NRED = 112;    // per-token reduction slots (>= k*K + k*k + K*K)
@@ -240,6 +242,11 @@ cudaError_t launch_proj_tc(const uint16_t* X, int T, int K, const uint16_t* Wpac
 cudaError_t launch_wgrad_tc(const uint16_t* A, int T, int E, const float* dz, int ldz, int n,
                             uint16_t* dzpack, const ProjTcPlan& p, float* part, int* err,
                             cudaStream_t st);
+bool dx_tc_ok(int T, int N, int C, int nfull);
+cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, uint16_t* dz16,
+                         uint16_t* w16, const uint16_t* X, const uint16_t* dinput, const float* hpre,
+                         const int* I, const float* dxact, const float* scal, int scal_ld,
+                         uint16_t* dX, int* err, cudaStream_t st);
 cudaError_t launch_wgrad_reduce(const float* wpart, int splits, int E, int n, const WSegsOut& G,
                                 cudaStream_t st);
 cudaError_t launch_colsum(const float* in, int rows, int ld, int n, float* out, int accumulate,
