@@ -58,6 +58,7 @@ struct TraceScope {
 static thread_local char g_last_error[256] = "";
 
 static xhc_status cuda_fail(cudaError_t e, int line) {
+    (void)cudaGetLastError();  // do not leave a launch-configuration error for the caller's next call
     snprintf(g_last_error, sizeof(g_last_error), "api.cu:%d: %s", line, cudaGetErrorString(e));
     return XHC_ERR_CUDA;
 }
@@ -155,11 +156,14 @@ Layout make_layout(const Dims& d, int64_t T) {
     L.twa = plan_proj_tc(d.k * d.C, (int)T, nact_max, sms);
     L.splits_full = std::max(L.tc.nseg, pick_splits(rowblocks, d.N * d.C));
     L.splits_act = std::max(L.tca.nseg, pick_splits(rowblocks, d.k * d.C));
-    L.nslice = (d.C + 255) / 256;
+    L.nslice = wb_nslice(d.C);
     const int ts_full = pick_tsplits(d.N * d.C, (int)T);
     const int ts_act = pick_tsplits(d.k * d.C, (int)T);
     L.tsplits = std::max(ts_full, ts_act);
-    L.ntiles = (int)((T + 127) / 128);
+    {
+        const int run = d.nconv > 0 ? wb_dw_run(d) : 128;
+        L.ntiles = (int)((T + run - 1) / run);
+    }
     o = 0;
     L.err = o; o = al(o + 256);
     L.wpack = o;
@@ -544,11 +548,12 @@ xhc_status xhc_post_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
     const Dims& d = c.d;
     const ConvPtrs cw = conv_of(d, P, slot);
     if (d.K[slot] > 1 && d.gs)
-        XHC_K("aug_gram", c.st, launch_aug_gram(d, slot, c.T, out, cw, c.L.nslice, c.W<float>(c.L.red), c.st));
+        XHC_K("wb_gram", c.st, launch_wb_gram(d, slot, c.T, out, cw, c.L.nslice, c.W<float>(c.L.red), c.st));
     const bool last = (slot == d.G - 1);
-    XHC_K("post_apply", c.st, launch_post_apply(d, slot, c.T, out, cw, c.W<float>(c.L.red), c.L.nslice, c.xact(slot),
+    XHC_K("wb_fwd", c.st, launch_wb_fwd(d, slot, c.T, out, cw, c.W<float>(c.L.red), c.L.nslice, c.xact(slot),
                                c.S<int>(c.L.I), c.S<float>(c.L.p), c.S<float>(c.L.hpost[slot]),
-                               c.S<float>(c.L.hres), last ? nullptr : c.xact(slot + 1), X, c.st));
+                               c.S<float>(c.L.hres), last ? nullptr : c.xact(slot + 1), X,
+                               c.W<int>(c.L.err), c.st));
     return XHC_OK;
 }
 
@@ -574,15 +579,16 @@ xhc_status xhc_post_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
         XHC_CUDA(cudaMemsetAsync(c.W<float>(c.L.dp), 0, (size_t)T32 * d.k * 4, c.st));
         XHC_K("restore", c.st, launch_restore(d, T32, c.xact(0), c.S<int>(c.L.I), X, c.st));
     }
-    XHC_K("bwd_reduce", c.st, launch_bwd_reduce(d, slot, T32, out, cw, dX, c.S<int>(c.L.I), dxact, c.xact(slot),
-                               c.L.nslice, red, c.st));
+    XHC_K("wb_bred", c.st, launch_wb_bred(d, slot, T32, out, cw, dX, c.S<int>(c.L.I), dxact, c.xact(slot),
+                                          c.L.nslice, red, c.W<int>(c.L.err), c.st));
     XHC_K("bwd_coef", c.st, launch_bwd_coef(d, slot, T32, red, c.L.nslice, c.S<float>(c.L.zact[slot]),
                              c.S<float>(c.L.rs[slot]), c.S<float>(c.L.p),
                              c.S<float>(c.L.hpost[slot]), P->alpha_post, P->b_post[slot],
                              P->alpha_res, P->b_res, c.W<float>(c.L.tokmat), c.W<float>(c.L.dz),
                              c.W<float>(c.L.dp), c.W<float>(c.L.tokgrad), c.st));
-    XHC_K("bwd_apply", c.st, launch_bwd_apply(d, slot, T32, out, cw, dX, c.S<int>(c.L.I), c.xact(slot),
-                              c.W<float>(c.L.tokmat), dxact, c.W<float>(c.L.du), d_out, c.st));
+    XHC_K("wb_bapp", c.st, launch_wb_bapp(d, slot, T32, out, cw, dX, c.S<int>(c.L.I), c.xact(slot),
+                                          c.W<float>(c.L.tokmat), dxact, c.W<float>(c.L.du), d_out,
+                                          c.W<int>(c.L.err), c.st));
     const WSegs wa = act_segs(d, P, slot);
     XHC_K("gemm_dzw", c.st, launch_gemm_dzw(d, T32, c.W<float>(c.L.dz), n, n, wa, d.k * d.C, dxact, c.st));
     if (T32 < 64 || d.k * d.C < 128) {
@@ -607,8 +613,8 @@ xhc_status xhc_post_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
         XHC_K("colsum", c.st, launch_colsum(tg + d.k * K + 1 + d.k * d.k, T32, NTG, 1, g->alpha_res, 1, scr, c.st));
     }
     if (K > 1) {
-        XHC_K("bwd_conv", c.st, launch_bwd_conv(d, slot, T32, out, cw, c.W<float>(c.L.du), d_out,
-                                 c.W<float>(c.L.cpart), c.L.ntiles, c.st));
+        XHC_K("wb_dout", c.st, launch_wb_dout(d, slot, T32, out, cw, c.W<float>(c.L.du), d_out,
+                                              c.W<float>(c.L.cpart), c.st));
         ConvGradPtrs gc;
         for (int j = 0; j < 3; ++j) gc.w[j] = (j < d.nconv) ? g->conv_w[slot][j] : nullptr;
         XHC_K("conv_wgrad_reduce", c.st, launch_conv_wgrad_reduce(d, slot, c.W<float>(c.L.cpart), c.L.ntiles, gc, c.st));

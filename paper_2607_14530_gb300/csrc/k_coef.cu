@@ -306,7 +306,9 @@ __global__ void k_bwd_coef(Dims d, int slot, int T, const float* __restrict__ re
     const int k = d.k, K = d.K[slot], n = d.nact[slot];
     const bool last = (slot == d.G - 1);
     const bool gs = (K > 1) && d.gs;
-    const int offQ = k * K, offG = k * K + (last ? k * k : 0);
+    // reduction slots per token (see wb_bred): P at j*4 + a, Q at KM*4 + j*KM + i, Gram at
+    // KM*4 + KM*KM (lower triangle packed)
+    const int offQ = KM * 4, offG = KM * 4 + KM * KM;
     float Pm[KM][MAXCOMP], Q[KM][KM];
     double Gm[MAXCOMP][MAXCOMP];
 #pragma unroll
@@ -324,13 +326,13 @@ __global__ void k_bwd_coef(Dims d, int slot, int T, const float* __restrict__ re
         for (int j = 0; j < KM; ++j)
 #pragma unroll
             for (int a = 0; a < MAXCOMP; ++a)
-                if (j < k && a < K) Pm[j][a] += rp[j * K + a];
+                if (j < k && a < K) Pm[j][a] += rp[j * 4 + a];
         if (last) {
 #pragma unroll
             for (int j = 0; j < KM; ++j)
 #pragma unroll
                 for (int i = 0; i < KM; ++i)
-                    if (j < k && i < k) Q[j][i] += rp[offQ + j * k + i];
+                    if (j < k && i < k) Q[j][i] += rp[offQ + j * KM + i];
         }
         if (gs) {
             int q = 0;

@@ -114,15 +114,18 @@ __device__ __forceinline__ void tc_fence_after() {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
+// TMEM -> registers (32 lanes x 16 columns); the wait is in the same statement so the outputs are
+// valid on exit, and there is no memory clobber so unrelated global loads can be scheduled
+// around it.
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
     uint32_t r[16];
     asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n"
+        "tcgen05.wait::ld.sync.aligned;"
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
           "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
           "=r"(r[14]), "=r"(r[15])
         : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
     for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
@@ -552,6 +555,8 @@ int device_sms() { return num_sms(); }
 namespace {
 
 constexpr int DX_BN = 128;
+constexpr int DX_EW = 16;                       // epilogue warps: 4 per TMEM lane quarter
+constexpr int DX_THREADS = (2 + DX_EW) * 32;    // + TMA warp + MMA warp
 
 struct DxArgs {
     int T, C, N, k, G;
@@ -570,7 +575,7 @@ struct DxArgs {
     int* err;
 };
 
-__global__ void __launch_bounds__(NTHREADS, 1)
+__global__ void __launch_bounds__(DX_THREADS, 1)
 k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, DxArgs a) {
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -586,7 +591,7 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
             mbar_init(smem_u32(&bars[s]), 1);
             mbar_init(smem_u32(&bars[2 + s]), 1);
             mbar_init(smem_u32(&bars[4 + s]), 1);
-            mbar_init(smem_u32(&bars[6 + s]), 4);
+            mbar_init(smem_u32(&bars[6 + s]), DX_EW);
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -652,6 +657,7 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
     } else {
         const int quarter = warp & 3;
         const int r = quarter * 32 + lane;
+        const int cg = (warp - 2) >> 2;            // column group of 32
         for (long long n = 0; n < nloc; ++n) {
             const long long tile = blockIdx.x + n * a.P;
             const int i = (int)(tile % a.N);
@@ -676,33 +682,39 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
                 sb = a.scal[(long long)t * a.scal_ld + 1];
             }
             const long long rowoff = ((long long)t * a.N + i) * a.C + ct * DX_BN;
-            for (int c0 = 0; c0 < DX_BN; c0 += 16) {
-                float acc[16];
-                tmem_ld16(tl + (uint32_t)c0, acc);
-                if (t >= a.T) continue;
+            for (int c0 = cg * (DX_BN / 4); c0 < (cg + 1) * (DX_BN / 4); c0 += 16) {
+                // global operands first (independent of the accumulator), then the TMEM read
                 float x[16], v[16];
-                unpack8(*reinterpret_cast<const uint4*>(a.X + rowoff + c0), x);
-                unpack8(*reinterpret_cast<const uint4*>(a.X + rowoff + c0 + 8), x + 8);
                 const int c = ct * DX_BN + c0;
-                if (j >= 0) {
-                    const float4* b = reinterpret_cast<const float4*>(a.dxact + ((long long)t * a.k + j) * a.C + c);
+                const bool tv = t < a.T;
+                if (tv) {
+                    unpack8(__ldg(reinterpret_cast<const uint4*>(a.X + rowoff + c0)), x);
+                    unpack8(__ldg(reinterpret_cast<const uint4*>(a.X + rowoff + c0 + 8)), x + 8);
+                    if (j >= 0) {
+                        const float4* b = reinterpret_cast<const float4*>(a.dxact + ((long long)t * a.k + j) * a.C + c);
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const float4 f = b[q];
-                        v[4 * q] = f.x; v[4 * q + 1] = f.y; v[4 * q + 2] = f.z; v[4 * q + 3] = f.w;
-                    }
-                } else {
-                    unpack8(*reinterpret_cast<const uint4*>(a.dX + rowoff + c0), v);
-                    unpack8(*reinterpret_cast<const uint4*>(a.dX + rowoff + c0 + 8), v + 8);
-                    for (int q = 0; q < a.G; ++q) {
-                        float g[16];
-                        const uint16_t* dp = a.dinput + ((long long)q * a.T + t) * a.C + c;
-                        unpack8(*reinterpret_cast<const uint4*>(dp), g);
-                        unpack8(*reinterpret_cast<const uint4*>(dp + 8), g + 8);
+                        for (int q = 0; q < 4; ++q) {
+                            const float4 f = b[q];
+                            v[4 * q] = f.x; v[4 * q + 1] = f.y; v[4 * q + 2] = f.z; v[4 * q + 3] = f.w;
+                        }
+                    } else {
+                        unpack8(*reinterpret_cast<const uint4*>(a.dX + rowoff + c0), v);
+                        unpack8(*reinterpret_cast<const uint4*>(a.dX + rowoff + c0 + 8), v + 8);
 #pragma unroll
-                        for (int e = 0; e < 16; ++e) v[e] = fmaf(h[q], g[e], v[e]);
+                        for (int q = 0; q < 4; ++q) {
+                            if (q >= a.G) continue;
+                            float g[16];
+                            const uint16_t* dp = a.dinput + ((long long)q * a.T + t) * a.C + c;
+                            unpack8(__ldg(reinterpret_cast<const uint4*>(dp)), g);
+                            unpack8(__ldg(reinterpret_cast<const uint4*>(dp + 8)), g + 8);
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) v[e] = fmaf(h[q], g[e], v[e]);
+                        }
                     }
                 }
+                float acc[16];
+                tmem_ld16(tl + (uint32_t)c0, acc);
+                if (!tv) continue;
                 float o[16];
 #pragma unroll
                 for (int e = 0; e < 16; ++e) o[e] = v[e] + acc[e] + sa + sb * x[e];
@@ -773,7 +785,7 @@ cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, 
     const size_t sm = 2 * (size_t)a.nkb * (BM + DX_BN) * BK * 2 + 8 * 8 + 16 + 1024;
     e = cudaFuncSetAttribute((const void*)k_dx_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
-    k_dx_tc<<<a.P, NTHREADS, sm, st>>>(ma, mb, a); note_launch();
+    k_dx_tc<<<a.P, DX_THREADS, sm, st>>>(ma, mb, a); note_launch();
     return cudaGetLastError();
 }
 

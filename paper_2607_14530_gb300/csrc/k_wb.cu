@@ -1,0 +1,842 @@
+// Write-back kernels of the connection op with the causal conv held in registers.
+//
+// Every kernel here walks a run of consecutive tokens for one pair of channels per thread.  The
+// conv taps of the pair (zero past kappa_j) and a ring of the last KW values of `out` stay in
+// registers; the token loop is unrolled by KW so the ring positions are compile-time constants,
+// and each out value is loaded once per run instead of once per tap.  Per-token reductions over
+// the channels (Gram matrix, write-back gradients) use a reduce-scatter butterfly inside the warp
+// (about V shuffles for V values instead of 5 V), then shared memory across warps.
+//   wb_gram   Gram matrix of u = [out, g_1..g_r] (Eq. aug, Eq. gs), partial per channel slice
+//   wb_fwd    X_act_new = (H_res) X_act + p (H_post out_aug) (Eq. sparse_write_delta,
+//             Eq. sparse_write), scatter into X on the last slot
+//   wb_bred   backward reductions <dXn_j, u_a>, <dXn_j, x_i>, <u_a, u_b>
+//   wb_bapp   component gradients du_a and the active-state gradient
+//   wb_dout   d_out = du_0 + conv^T(du_1..r) (anti-causal, computed with a lag of KW - 1 tokens)
+//   wb_dw     conv weight-gradient partials sum_t du_{1+j}[t] out[t - i]
+#include "xhc_internal.cuh"
+
+namespace xhc {
+namespace {
+
+constexpr int WT = 128;        // threads per CTA
+constexpr int WSL = 2 * WT;    // channels per CTA slice
+constexpr unsigned FULLM = 0xffffffffu;
+
+__device__ __forceinline__ float2 ld2(const uint16_t* p) {
+    const uint32_t u = *reinterpret_cast<const uint32_t*>(p);
+    return make_float2(__uint_as_float(u << 16), __uint_as_float(u & 0xffff0000u));
+}
+__device__ __forceinline__ void st2(uint16_t* p, float2 v) {
+    *reinterpret_cast<uint32_t*>(p) = pack2(v.x, v.y);
+}
+__device__ __forceinline__ float dot2(float2 a, float2 b) { return fmaf(a.x, b.x, a.y * b.y); }
+__device__ __forceinline__ float2 fma2(float s, float2 a, float2 acc) {
+    return make_float2(fmaf(s, a.x, acc.x), fmaf(s, a.y, acc.y));
+}
+__device__ __forceinline__ float2 f2z() { return make_float2(0.f, 0.f); }
+
+__device__ __forceinline__ uint32_t s_u32(const void* p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void bar_init(uint64_t* b, uint32_t n) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(s_u32(b)), "r"(n) : "memory");
+}
+__device__ __forceinline__ void bar_expect(uint64_t* b, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(s_u32(b)), "r"(bytes) : "memory");
+}
+// bounded wait (~4 s of global time); false when it gives up
+__device__ __forceinline__ bool bar_wait(uint64_t* b, uint32_t parity) {
+    uint64_t t0 = 0;
+    for (uint32_t it = 0;; ++it) {
+        uint32_t ok;
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+            " selp.u32 %0, 1, 0, p;\n}\n"
+            : "=r"(ok) : "r"(s_u32(b)), "r"(parity) : "memory");
+        if (ok) return true;
+        if ((it & 255u) == 255u) {
+            uint64_t now;
+            asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(now));
+            if (t0 == 0) t0 = now;
+            else if (now - t0 > 4000000000ull) return false;
+        }
+    }
+}
+// 1-D bulk copy global -> shared completing on an mbarrier (16-byte aligned, size % 16 == 0)
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            s_u32(dst)), "l"(src), "r"(bytes), "r"(s_u32(bar))
+        : "memory");
+}
+
+// Row staging of a run of tokens: per token, `nrow` rows of this CTA's channel slice are copied
+// into a shared-memory stage (two stages, batches of B tokens).  row_src(t, r) gives the global
+// address of row r of token t and its element size.
+struct StageGeom {
+    int B;          // tokens per batch
+    int nrow;       // rows per token
+    int rowb;       // bytes reserved per row in shared memory
+    int tokb;       // bytes per token = nrow * rowb
+};
+
+template <int KW>
+__device__ __forceinline__ void taps_reg(const Dims& d, const ConvPtrs& cw, int c, bool act,
+                                         float2 (&tw)[3][KW]) {
+#pragma unroll
+    for (int j = 0; j < 3; ++j)
+#pragma unroll
+        for (int i = 0; i < KW; ++i) {
+            float2 v = f2z();
+            if (act && j < d.nconv && i < d.kap[j])
+                v = make_float2(cw.w[j][(size_t)i * d.C + c], cw.w[j][(size_t)i * d.C + c + 1]);
+            tw[j][i] = v;
+        }
+}
+
+// ring w[s] = out[t] for t = s (mod KW); prepare the run starting at t0 (t0 % KW == 0)
+template <int KW>
+__device__ __forceinline__ void ring_init(const uint16_t* out, int C, int c, bool act, long long t0,
+                                          float2 (&w)[KW]) {
+    w[0] = f2z();
+#pragma unroll
+    for (int i = 1; i < KW; ++i) {
+        const long long t = t0 - i;
+        w[KW - i] = (act && t >= 0) ? ld2(out + t * C + c) : f2z();
+    }
+}
+
+// g_j = sum_{i <= pos} tw[j][i] out[t - i], with out[t - i] at ring slot (U - i) mod KW
+template <int KW>
+__device__ __forceinline__ void conv_ring(const float2 (&tw)[3][KW], const float2 (&w)[KW], int U,
+                                          int pos, float2 (&g)[3]) {
+#pragma unroll
+    for (int j = 0; j < 3; ++j) g[j] = f2z();
+#pragma unroll
+    for (int i = 0; i < KW; ++i) {
+        if (i <= pos) {
+            const float2 o = w[(U - i + KW) % KW];
+#pragma unroll
+            for (int j = 0; j < 3; ++j) {
+                g[j].x = fmaf(tw[j][i].x, o.x, g[j].x);
+                g[j].y = fmaf(tw[j][i].y, o.y, g[j].y);
+            }
+        }
+    }
+}
+
+// Reduce-scatter of V values (power of two, <= 32) over the warp: every lane returns the total
+// of value index lane >> (5 - log2 V).
+template <int V, int O>
+struct WRed {
+    static __device__ __forceinline__ float run(float* v, int lane) {
+        if constexpr (V > 1) {
+            constexpr int H = V / 2;
+            const bool up = (lane & O) != 0;
+#pragma unroll
+            for (int q = 0; q < H; ++q) {
+                const float send = up ? v[q] : v[q + H];
+                const float keep = up ? v[q + H] : v[q];
+                v[q] = keep + __shfl_xor_sync(FULLM, send, O);
+            }
+            if constexpr (O > 1) return WRed<H, O / 2>::run(v, lane);
+            else return v[0];
+        } else {
+            float x = v[0];
+#pragma unroll
+            for (int o = O; o >= 1; o >>= 1) x += __shfl_xor_sync(FULLM, x, o);
+            return x;
+        }
+    }
+};
+
+// reduce NB blocks of 32 values; lane l receives the totals of values b*32 + l
+template <int NB>
+__device__ __forceinline__ void wred32(float (&v)[NB * 32], int lane, float (&tot)[NB]) {
+#pragma unroll
+    for (int b = 0; b < NB; ++b) tot[b] = WRed<32, 16>::run(v + 32 * b, lane);
+}
+
+// ---------------------------------------------------------------------------------------------
+// wb_gram
+
+template <int KW>
+__global__ void __launch_bounds__(WT) k_wb_gram(Dims d, int slot, int T, int TB,
+                                                const uint16_t* __restrict__ out, ConvPtrs cw,
+                                                int nslice, float* __restrict__ red) {
+    extern __shared__ float wsh[];  // [TB][WT/32][16]
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int slice = blockIdx.x, C = d.C;
+    const int c = slice * WSL + 2 * threadIdx.x;
+    const bool act = c < C;
+    const long long t0 = (long long)blockIdx.y * TB;
+    const long long t1 = min((long long)T, t0 + TB);
+    const int K = d.K[slot];
+    const int nq = K * (K + 1) / 2;
+    float2 tw[3][KW], w[KW];
+    taps_reg<KW>(d, cw, c, act, tw);
+    ring_init<KW>(out, C, c, act, t0, w);
+    for (long long tb = t0; tb < t1; tb += KW) {
+#pragma unroll
+        for (int u = 0; u < KW; ++u) {
+            const long long t = tb + u;
+            if (t < t1) {
+                const float2 o = act ? ld2(out + t * C + c) : f2z();
+                w[u] = o;
+                float2 g[3];
+                conv_ring<KW>(tw, w, u, (int)(t % d.S), g);
+                const float2 uu[4] = {o, g[0], g[1], g[2]};
+                float v[16];
+                int q = 0;
+#pragma unroll
+                for (int a = 0; a < 4; ++a)
+#pragma unroll
+                    for (int b = 0; b <= a; ++b) v[q++] = (a < K) ? dot2(uu[a], uu[b]) : 0.f;
+#pragma unroll
+                for (int r = 10; r < 16; ++r) v[r] = 0.f;
+                const float tot = WRed<16, 16>::run(v, lane);
+                if ((lane & 1) == 0) wsh[((t - t0) * (WT / 32) + warp) * 16 + (lane >> 1)] = tot;
+            }
+        }
+    }
+    __syncthreads();
+    const int ntok = (int)(t1 - t0);
+    for (int idx = threadIdx.x; idx < ntok * nq; idx += WT) {
+        const int tt = idx / nq, q = idx - tt * nq;
+        float s = 0.f;
+#pragma unroll
+        for (int ww = 0; ww < WT / 32; ++ww) s += wsh[(tt * (WT / 32) + ww) * 16 + q];
+        red[((t0 + tt) * nslice + slice) * NRED + q] = s;
+    }
+}
+
+// ---------------------------------------------------------------------------------------------
+// wb_fwd: per-token coefficients E[j][a] (Gram-Schmidt folded in), H_res, I in shared memory;
+// the out row and the k active rows of every token are staged by bulk copies.
+
+template <int KM, int KW>
+__global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
+                                               const uint16_t* __restrict__ out, ConvPtrs cw,
+                                               const float* __restrict__ red, int nslice,
+                                               const uint16_t* __restrict__ xact,
+                                               const int* __restrict__ I,
+                                               const float* __restrict__ p,
+                                               const float* __restrict__ hpost,
+                                               const float* __restrict__ hres,
+                                               uint16_t* __restrict__ xact_next,
+                                               uint16_t* __restrict__ X, int* __restrict__ err) {
+    constexpr int BT = KW > 0 ? KW : 8;      // tokens per staged batch
+    extern __shared__ __align__(128) unsigned char smu[];
+    const int k = d.k, K = d.K[slot], C = d.C;
+    const bool last = (slot == d.G - 1);
+    const bool gs = (K > 1) && d.gs;
+    const int c0 = blockIdx.x * WSL;
+    const int cs = min(WSL, C - c0);                 // channels of this slice
+    const uint32_t rowb = (uint32_t)cs * 2;
+    const int tokb = (1 + k) * WSL * 2;              // out row + k active rows
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smu);
+    float* Esh = reinterpret_cast<float*>(smu + 64);           // [TB][KM][4]
+    float* Hsh = Esh + TB * KM * 4;                           // [TB][KM][KM]
+    int* Ish = reinterpret_cast<int*>(Hsh + TB * KM * KM);     // [TB][KM]
+    unsigned char* stg = smu + 64 + (size_t)TB * (KM * 4 + KM * KM + KM) * 4;
+    stg = (unsigned char*)(((uintptr_t)stg + 127) & ~(uintptr_t)127);
+    const long long t0 = (long long)blockIdx.y * TB;
+    const long long t1 = min((long long)T, t0 + TB);
+    const int ntok = (int)(t1 - t0);
+    const int nb = (ntok + BT - 1) / BT;
+    if (threadIdx.x == 0) {
+        bar_init(&bars[0], 1);
+        bar_init(&bars[1], 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+    auto issue = [&](int b) {  // warp 0
+        const int s = b & 1;
+        const int tb0 = b * BT, nt = min(BT, ntok - tb0);
+        if (threadIdx.x == 0) bar_expect(&bars[s], (uint32_t)(nt * (1 + k)) * rowb);
+        __syncwarp();
+        for (int q = threadIdx.x; q < nt * (1 + k); q += 32) {
+            const int tt = q / (1 + k), r = q - tt * (1 + k);
+            const long long t = t0 + tb0 + tt;
+            const uint16_t* src = (r == 0) ? out + t * C + c0 : xact + (t * k + (r - 1)) * C + c0;
+            bulk_g2s(stg + (size_t)s * BT * tokb + (size_t)tt * tokb + (size_t)r * WSL * 2, src, rowb, &bars[s]);
+        }
+    };
+    if (threadIdx.x < 32) {
+        issue(0);
+        if (nb > 1) issue(1);
+    }
+    for (int tt = threadIdx.x; tt < ntok; tt += WT) {
+        const long long t = t0 + tt;
+        double B[MAXCOMP][MAXCOMP];
+        for (int a = 0; a < MAXCOMP; ++a)
+            for (int b = 0; b < MAXCOMP; ++b) B[a][b] = (a == b) ? 1.0 : 0.0;
+        if (gs) {
+            double Gm[MAXCOMP][MAXCOMP], cc[MAXCOMP][MAXCOMP], vv[MAXCOMP];
+            for (int a = 0; a < MAXCOMP; ++a)
+                for (int b = 0; b < MAXCOMP; ++b) Gm[a][b] = 0.0;
+            for (int sl = 0; sl < nslice; ++sl) {
+                const float* rp = red + (t * nslice + sl) * NRED;
+                int q = 0;
+                for (int a = 0; a < K; ++a)
+                    for (int b = 0; b <= a; ++b) Gm[a][b] += (double)rp[q++];
+            }
+            for (int a = 0; a < K; ++a)
+                for (int b = a + 1; b < K; ++b) Gm[a][b] = Gm[b][a];
+            gs_coef(Gm, K, (double)d.eps_gs, B, cc, vv);
+        }
+        for (int j = 0; j < KM; ++j) {
+            const bool jv = j < k;
+            const float pj = jv ? p[t * k + j] : 0.f;
+            for (int a = 0; a < 4; ++a) {
+                float e = 0.f;
+                if (jv && a < K)
+                    for (int q = 0; q < K; ++q) e += hpost[(t * k + j) * K + q] * (float)B[q][a];
+                Esh[(tt * KM + j) * 4 + a] = pj * e;
+            }
+            Ish[tt * KM + j] = jv ? I[t * k + j] : 0;
+            for (int i = 0; i < KM; ++i)
+                Hsh[(tt * KM + j) * KM + i] = (last && jv && i < k) ? hres[t * k * k + j * k + i] : 0.f;
+        }
+    }
+    const int cl = 2 * threadIdx.x;                 // channel pair within the slice
+    const int c = c0 + cl;
+    const bool act = cl < cs;
+    float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
+    if constexpr (KW > 0) {
+        taps_reg<KW>(d, cw, c, act, tw);
+        ring_init<KW>(out, C, c, act, t0, w);
+    }
+    __syncthreads();
+    for (int b = 0; b < nb; ++b) {
+        const int s = b & 1;
+        if (!bar_wait(&bars[s], (uint32_t)((b >> 1) & 1))) {
+            if (threadIdx.x == 0) atomicExch(err, 21);
+            break;
+        }
+        const unsigned char* sb = stg + (size_t)s * BT * tokb;
+#pragma unroll
+        for (int u = 0; u < BT; ++u) {
+            const int tt = b * BT + u;
+            if (tt < ntok && act) {
+                const long long t = t0 + tt;
+                const unsigned char* tk = sb + (size_t)u * tokb;
+                const float2 o = ld2(reinterpret_cast<const uint16_t*>(tk) + cl);
+                float2 uu[4] = {o, f2z(), f2z(), f2z()};
+                if constexpr (KW > 0) {
+                    w[u] = o;
+                    float2 g[3];
+                    conv_ring<KW>(tw, w, u, (int)(t % d.S), g);
+                    uu[1] = g[0];
+                    uu[2] = g[1];
+                    uu[3] = g[2];
+                }
+                float2 x[KM];
+#pragma unroll
+                for (int j = 0; j < KM; ++j)
+                    x[j] = (j < k) ? ld2(reinterpret_cast<const uint16_t*>(tk + (size_t)(1 + j) * WSL * 2) + cl) : f2z();
+#pragma unroll
+                for (int j = 0; j < KM; ++j) {
+                    if (j >= k) continue;
+                    float2 v;
+                    if (last) {
+                        v = f2z();
+#pragma unroll
+                        for (int i = 0; i < KM; ++i) v = fma2(Hsh[(tt * KM + j) * KM + i], x[i], v);
+                    } else {
+                        v = x[j];
+                    }
+#pragma unroll
+                    for (int a = 0; a < 4; ++a) v = fma2(Esh[(tt * KM + j) * 4 + a], uu[a], v);
+                    if (last)
+                        st2(X + (t * d.N + Ish[tt * KM + j]) * C + c, v);
+                    else
+                        st2(xact_next + (t * k + j) * C + c, v);
+                }
+            } else if constexpr (KW > 0) {
+                if (tt < ntok) w[u] = f2z();
+            }
+        }
+        __syncthreads();
+        if (threadIdx.x < 32 && b + 2 < nb) issue(b + 2);
+    }
+}
+
+// ---------------------------------------------------------------------------------------------
+// wb_bred: backward reductions, fixed slots per token (zeros where a term does not apply):
+//   [j*4 + a]              P[j][a] = <dXn_j, u_a>
+//   [KM*4 + j*KM + i]      Q[j][i] = <dXn_j, x_i>          (last slot)
+//   [KM*4 + KM*KM + q]     Gram of u, lower triangle packed (Gram-Schmidt on)
+
+template <int KM, int KW, int NB>
+__global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
+                                                const uint16_t* __restrict__ out, ConvPtrs cw,
+                                                const uint16_t* __restrict__ dX,
+                                                const int* __restrict__ I,
+                                                const float* __restrict__ dxact,
+                                                const uint16_t* __restrict__ xact, int nslice,
+                                                float* __restrict__ red) {
+    extern __shared__ float wsh[];  // [TB][WT/32][NB*32]
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int slice = blockIdx.x, C = d.C, k = d.k;
+    const int K = d.K[slot];
+    const bool last = (slot == d.G - 1);
+    const bool gs = (K > 1) && d.gs;
+    const int nv = KM * 4 + KM * KM + 10;
+    const int c = slice * WSL + 2 * threadIdx.x;
+    const bool act = c < C;
+    const long long t0 = (long long)blockIdx.y * TB;
+    const long long t1 = min((long long)T, t0 + TB);
+    float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
+    if constexpr (KW > 0) {
+        taps_reg<KW>(d, cw, c, act, tw);
+        ring_init<KW>(out, C, c, act, t0, w);
+    }
+    const int RU = KW > 0 ? KW : 4;
+    for (long long tb = t0; tb < t1; tb += RU) {
+#pragma unroll
+        for (int u = 0; u < RU; ++u) {
+            const long long t = tb + u;
+            if (t < t1) {
+                float2 uu[4] = {f2z(), f2z(), f2z(), f2z()};
+                float2 dn[KM], x[KM];
+#pragma unroll
+                for (int j = 0; j < KM; ++j) {
+                    dn[j] = f2z();
+                    x[j] = f2z();
+                }
+                if (act) {
+                    const float2 o = ld2(out + t * C + c);
+                    uu[0] = o;
+                    if constexpr (KW > 0) {
+                        w[u] = o;
+                        float2 g[3];
+                        conv_ring<KW>(tw, w, u, (int)(t % d.S), g);
+                        uu[1] = g[0];
+                        uu[2] = g[1];
+                        uu[3] = g[2];
+                    }
+#pragma unroll
+                    for (int j = 0; j < KM; ++j) {
+                        if (j >= k) continue;
+                        if (last) {
+                            dn[j] = ld2(dX + (t * d.N + I[t * k + j]) * C + c);
+                            x[j] = ld2(xact + (t * k + j) * C + c);
+                        } else {
+                            dn[j] = *reinterpret_cast<const float2*>(dxact + (t * k + j) * C + c);
+                        }
+                    }
+                } else if constexpr (KW > 0) {
+                    w[u] = f2z();
+                }
+                // dn, x and the unused components are zero where a term does not apply
+                float v[NB * 32];
+#pragma unroll
+                for (int q = 0; q < NB * 32; ++q) v[q] = 0.f;
+#pragma unroll
+                for (int j = 0; j < KM; ++j)
+#pragma unroll
+                    for (int a = 0; a < 4; ++a) v[j * 4 + a] = dot2(dn[j], uu[a]);
+                if (last) {
+#pragma unroll
+                    for (int j = 0; j < KM; ++j)
+#pragma unroll
+                        for (int i = 0; i < KM; ++i) v[KM * 4 + j * KM + i] = dot2(dn[j], x[i]);
+                }
+                if (gs) {
+                    int q = KM * 4 + KM * KM;
+#pragma unroll
+                    for (int a = 0; a < 4; ++a)
+#pragma unroll
+                        for (int bb = 0; bb <= a; ++bb) v[q++] = dot2(uu[a], uu[bb]);
+                }
+                float tot[NB];
+                wred32<NB>(v, lane, tot);
+                float* dst = wsh + ((t - t0) * (WT / 32) + warp) * (NB * 32);
+#pragma unroll
+                for (int bb = 0; bb < NB; ++bb) dst[bb * 32 + lane] = tot[bb];
+            }
+        }
+    }
+    __syncthreads();
+    const int ntok = (int)(t1 - t0);
+    for (int idx = threadIdx.x; idx < ntok * nv; idx += WT) {
+        const int tt = idx / nv, q = idx - tt * nv;
+        float sm = 0.f;
+#pragma unroll
+        for (int ww = 0; ww < WT / 32; ++ww) sm += wsh[(tt * (WT / 32) + ww) * (NB * 32) + q];
+        red[((t0 + tt) * nslice + slice) * NRED + q] = sm;
+    }
+}
+
+// ---------------------------------------------------------------------------------------------
+// wb_bapp: du_a = sum_j E[j][a] dXn_j + sum_b D[a][b] u_b;  dX_act_i = (H_res^T dXn)_i - cx x_i
+
+template <int KM, int KW>
+__global__ void __launch_bounds__(WT) k_wb_bapp(Dims d, int slot, int T, int TB,
+                                                const uint16_t* __restrict__ out, ConvPtrs cw,
+                                                const uint16_t* __restrict__ dX,
+                                                const int* __restrict__ I,
+                                                const uint16_t* __restrict__ xact,
+                                                const float* __restrict__ tokmat,
+                                                float* __restrict__ dxact,
+                                                float* __restrict__ du,
+                                                uint16_t* __restrict__ d_out) {
+    extern __shared__ float smf[];
+    const int k = d.k, K = d.K[slot], C = d.C;
+    const bool last = (slot == d.G - 1);
+    float* Esh = smf;                        // [TB][KM][4]
+    float* Dsh = Esh + TB * KM * 4;          // [TB][4][4]
+    float* Hsh = Dsh + TB * 16;              // [TB][KM][KM]
+    float* cxs = Hsh + TB * KM * KM;         // [TB]
+    int* Ish = (int*)(cxs + TB);             // [TB][KM]
+    const long long t0 = (long long)blockIdx.y * TB;
+    const long long t1 = min((long long)T, t0 + TB);
+    const int ntok = (int)(t1 - t0);
+    for (int idx = threadIdx.x; idx < ntok * 128; idx += WT) {
+        const int tt = idx >> 7, q = idx & 127;
+        const long long t = t0 + tt;
+        const float v = tokmat[t * TOKMAT + q];
+        if (q < 32) {
+            const int j = q >> 2, a = q & 3;
+            if (j < KM) Esh[(tt * KM + j) * 4 + a] = v;
+        } else if (q < 48) {
+            Dsh[tt * 16 + (q - 32)] = v;
+        } else if (q < 112) {
+            const int a = (q - 48) >> 3, b = (q - 48) & 7;
+            if (a < KM && b < KM) Hsh[(tt * KM + a) * KM + b] = v;
+        } else if (q == 112) {
+            cxs[tt] = v;
+        } else if (q >= 120 && q < 120 + KM) {
+            Ish[tt * KM + (q - 120)] = (q - 120 < k) ? I[t * k + (q - 120)] : 0;
+        }
+    }
+    const int c = blockIdx.x * WSL + 2 * threadIdx.x;
+    const bool act = c < C;
+    float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
+    if constexpr (KW > 0) {
+        taps_reg<KW>(d, cw, c, act, tw);
+        ring_init<KW>(out, C, c, act, t0, w);
+    }
+    __syncthreads();
+    const int RU = KW > 0 ? KW : 4;
+    for (long long tb = t0; tb < t1; tb += RU) {
+#pragma unroll
+        for (int u = 0; u < RU; ++u) {
+            const long long t = tb + u;
+            if (t < t1 && act) {
+                const int tt = (int)(t - t0);
+                const float2 o = ld2(out + t * C + c);
+                float2 uu[4] = {o, f2z(), f2z(), f2z()};
+                if constexpr (KW > 0) {
+                    w[u] = o;
+                    float2 g[3];
+                    conv_ring<KW>(tw, w, u, (int)(t % d.S), g);
+                    uu[1] = g[0];
+                    uu[2] = g[1];
+                    uu[3] = g[2];
+                }
+                float2 dn[KM], x[KM];
+#pragma unroll
+                for (int j = 0; j < KM; ++j) {
+                    if (j < k) {
+                        dn[j] = last ? ld2(dX + (t * d.N + Ish[tt * KM + j]) * C + c)
+                                     : *reinterpret_cast<const float2*>(dxact + (t * k + j) * C + c);
+                        x[j] = ld2(xact + (t * k + j) * C + c);
+                    } else {
+                        dn[j] = f2z();
+                        x[j] = f2z();
+                    }
+                }
+#pragma unroll
+                for (int a = 0; a < 4; ++a) {
+                    if (a >= K) continue;
+                    float2 gsum = f2z();
+#pragma unroll
+                    for (int j = 0; j < KM; ++j) gsum = fma2(Esh[(tt * KM + j) * 4 + a], dn[j], gsum);
+#pragma unroll
+                    for (int b = 0; b < 4; ++b)
+                        if (b < K) gsum = fma2(Dsh[tt * 16 + a * 4 + b], uu[b], gsum);
+                    if (K == 1)
+                        st2(d_out + t * C + c, gsum);
+                    else
+                        *reinterpret_cast<float2*>(du + (t * K + a) * C + c) = gsum;
+                }
+                const float cx = cxs[tt];
+#pragma unroll
+                for (int i = 0; i < KM; ++i) {
+                    if (i >= k) continue;
+                    float2 v;
+                    if (last) {
+                        v = f2z();
+#pragma unroll
+                        for (int j = 0; j < KM; ++j) v = fma2(Hsh[(tt * KM + j) * KM + i], dn[j], v);
+                    } else {
+                        v = dn[i];
+                    }
+                    v = fma2(-cx, x[i], v);
+                    *reinterpret_cast<float2*>(dxact + (t * k + i) * C + c) = v;
+                }
+            }
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------------------------
+// wb_dout: d_out[s] = du_0[s] + sum_j sum_{i, pos(s) + i < S} w_j[i] du_{1+j}[s + i].  Walks t
+// upwards keeping the last KW values of du_{1..3}; d_out[s] is emitted at t = s + KW - 1.
+
+template <int KW>
+__global__ void __launch_bounds__(WT) k_wb_dout(Dims d, int slot, int T, int TB,
+                                                ConvPtrs cw, const float* __restrict__ du,
+                                                uint16_t* __restrict__ d_out) {
+    const int K = d.K[slot], C = d.C;
+    const int c = blockIdx.x * WSL + 2 * threadIdx.x;
+    if (c >= C) return;
+    const long long t0 = (long long)blockIdx.y * TB;
+    const long long t1 = min((long long)T, t0 + TB);
+    float2 tw[3][KW];
+    taps_reg<KW>(d, cw, c, true, tw);
+    float2 r[3][KW];  // r[j][t mod KW] = du_{1+j}[t]
+#pragma unroll
+    for (int j = 0; j < 3; ++j)
+#pragma unroll
+        for (int s = 0; s < KW; ++s) r[j][s] = f2z();
+    // walk t over [t0, t1 + KW - 1); emit s = t - (KW - 1) when s >= t0
+    for (long long tb = t0; tb < t1 + KW - 1; tb += KW) {
+#pragma unroll
+        for (int u = 0; u < KW; ++u) {
+            const long long t = tb + u;
+            if (t < t1 + KW - 1) {
+#pragma unroll
+                for (int j = 0; j < 3; ++j)
+                    r[j][u] = (j < d.nconv && t < T) ? *reinterpret_cast<const float2*>(du + (t * K + 1 + j) * C + c)
+                                                     : f2z();
+                const long long s = t - (KW - 1);
+                if (s >= t0 && s < t1) {
+                    const int pos = (int)(s % d.S);
+                    float2 acc = *reinterpret_cast<const float2*>(du + (s * K) * C + c);
+#pragma unroll
+                    for (int i = 0; i < KW; ++i) {
+                        if (pos + i < d.S) {
+                            // du[s + i] sits at ring slot (s + i) mod KW = (u + 1 + i) mod KW
+#pragma unroll
+                            for (int j = 0; j < 3; ++j) {
+                                const float2 g = r[j][(u + 1 + i) % KW];
+                                acc.x = fmaf(tw[j][i].x, g.x, acc.x);
+                                acc.y = fmaf(tw[j][i].y, g.y, acc.y);
+                            }
+                        }
+                    }
+                    st2(d_out + s * C + c, acc);
+                }
+            }
+        }
+    }
+}
+
+// wb_dw: cpart[blockIdx.y][off_j + i][c] = sum_{t in run, pos(t) >= i} du_{1+j}[t] out[t - i]
+
+template <int KW>
+__global__ void __launch_bounds__(WT) k_wb_dw(Dims d, int slot, int T, int TB,
+                                              const uint16_t* __restrict__ out,
+                                              const float* __restrict__ du,
+                                              float* __restrict__ cpart) {
+    const int K = d.K[slot], C = d.C;
+    const int c = blockIdx.x * WSL + 2 * threadIdx.x;
+    if (c >= C) return;
+    const long long t0 = (long long)blockIdx.y * TB;
+    const long long t1 = min((long long)T, t0 + TB);
+    float2 w[KW], acc[3][KW];
+    ring_init<KW>(out, C, c, true, t0, w);
+#pragma unroll
+    for (int j = 0; j < 3; ++j)
+#pragma unroll
+        for (int i = 0; i < KW; ++i) acc[j][i] = f2z();
+    for (long long tb = t0; tb < t1; tb += KW) {
+#pragma unroll
+        for (int u = 0; u < KW; ++u) {
+            const long long t = tb + u;
+            if (t < t1) {
+                w[u] = ld2(out + t * C + c);
+                const int pos = (int)(t % d.S);
+#pragma unroll
+                for (int j = 0; j < 3; ++j) {
+                    if (j >= d.nconv) continue;
+                    const float2 g = *reinterpret_cast<const float2*>(du + (t * K + 1 + j) * C + c);
+#pragma unroll
+                    for (int i = 0; i < KW; ++i) {
+                        if (i <= pos) {
+                            const float2 o = w[(u - i + KW) % KW];
+                            acc[j][i].x = fmaf(g.x, o.x, acc[j][i].x);
+                            acc[j][i].y = fmaf(g.y, o.y, acc[j][i].y);
+                        }
+                    }
+                }
+            }
+        }
+    }
+    int off = 0;
+#pragma unroll
+    for (int j = 0; j < 3; ++j) {
+        if (j < d.nconv) {
+#pragma unroll
+            for (int i = 0; i < KW; ++i)
+                if (i < d.kap[j])
+                    *reinterpret_cast<float2*>(cpart + ((long long)blockIdx.y * d.kapsum + off + i) * C + c) = acc[j][i];
+            off += d.kap[j];
+        }
+    }
+}
+
+int kw_of(const Dims& d) {
+    const int km = d.kapmax;
+    return km <= 4 ? 4 : km <= 8 ? 8 : km <= 12 ? 12 : 16;
+}
+
+int run_len(int KW, int per) {  // tokens per CTA run: a multiple of KW near `per`
+    const int u = KW > 0 ? KW : 4;
+    int r = (per / u) * u;
+    return r < u ? u : r;
+}
+
+cudaError_t smem_attr(const void* fn, size_t bytes) {
+    if (bytes <= 48 * 1024) return cudaSuccess;
+    return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+}
+
+template <int KW>
+cudaError_t gram_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, int nslice,
+                    float* red, cudaStream_t st) {
+    const int TB = run_len(KW, 64);
+    const size_t sm = (size_t)TB * (WT / 32) * 16 * sizeof(float);
+    cudaError_t e = smem_attr((const void*)k_wb_gram<KW>, sm);
+    if (e != cudaSuccess) return e;
+    dim3 grid(nslice, (T + TB - 1) / TB);
+    k_wb_gram<KW><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, nslice, red); note_launch();
+    return cudaGetLastError();
+}
+
+template <int KM, int KW>
+cudaError_t fwd_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, const float* red,
+                   int nslice, const uint16_t* xact, const int* I, const float* p, const float* hpost,
+                   const float* hres, uint16_t* xact_next, uint16_t* X, int* err, cudaStream_t st) {
+    constexpr int BT = KW > 0 ? KW : 8;
+    const int TB = run_len(BT, 96);
+    const size_t sm = 64 + (size_t)TB * (KM * 4 + KM * KM + KM) * 4 + 128 +
+                      2 * (size_t)BT * (1 + d.k) * WSL * 2;
+    cudaError_t e = smem_attr((const void*)k_wb_fwd<KM, KW>, sm);
+    if (e != cudaSuccess) return e;
+    dim3 grid(nslice, (T + TB - 1) / TB);
+    k_wb_fwd<KM, KW><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, red, nslice, xact, I, p, hpost,
+                                           hres, xact_next, X, err); note_launch();
+    return cudaGetLastError();
+}
+
+template <int KM, int KW, int NB>
+cudaError_t bred_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, const uint16_t* dX,
+                    const int* I, const float* dxact, const uint16_t* xact, int nslice, float* red,
+                    int* err, cudaStream_t st) {
+    (void)err;
+    int TB = run_len(KW, 48);
+    while (TB > (KW > 0 ? KW : 4) && (size_t)TB * (WT / 32) * NB * 32 * 4 > 96 * 1024) TB -= (KW > 0 ? KW : 4);
+    const size_t sm = (size_t)TB * (WT / 32) * NB * 32 * sizeof(float);
+    cudaError_t e = smem_attr((const void*)k_wb_bred<KM, KW, NB>, sm);
+    if (e != cudaSuccess) return e;
+    dim3 grid(nslice, (T + TB - 1) / TB);
+    k_wb_bred<KM, KW, NB><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, dX, I, dxact, xact, nslice, red); note_launch();
+    return cudaGetLastError();
+}
+
+template <int KM, int KW>
+cudaError_t bapp_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, const uint16_t* dX,
+                    const int* I, const uint16_t* xact, const float* tokmat, float* dxact, float* du,
+                    uint16_t* d_out, int nslice, int* err, cudaStream_t st) {
+    (void)err;
+    const int TB = run_len(KW, 64);
+    const size_t sm = (size_t)TB * (KM * 4 + 16 + KM * KM + 1 + KM) * 4;
+    cudaError_t e = smem_attr((const void*)k_wb_bapp<KM, KW>, sm);
+    if (e != cudaSuccess) return e;
+    dim3 grid(nslice, (T + TB - 1) / TB);
+    k_wb_bapp<KM, KW><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, dX, I, xact, tokmat, dxact, du, d_out); note_launch();
+    return cudaGetLastError();
+}
+
+template <int KW>
+cudaError_t dout_kw(const Dims& d, int slot, int T, ConvPtrs cw, const float* du, uint16_t* d_out,
+                    float* cpart, const uint16_t* out, int nslice, int TBW, cudaStream_t st) {
+    const int TB = run_len(KW, 64);
+    dim3 grid(nslice, (T + TB - 1) / TB);
+    k_wb_dout<KW><<<grid, WT, 0, st>>>(d, slot, T, TB, cw, du, d_out); note_launch();
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    dim3 g2(nslice, (T + TBW - 1) / TBW);
+    k_wb_dw<KW><<<g2, WT, 0, st>>>(d, slot, T, TBW, out, du, cpart); note_launch();
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+int wb_nslice(int C) { return (C + WSL - 1) / WSL; }
+int wb_dw_run(const Dims& d) { return run_len(kw_of(d), 128); }
+
+#define XHC_KW_DISPATCH(KWV, CALL)                         \
+    switch (KWV) {                                         \
+        case 4: { constexpr int KWC = 4; return CALL; }    \
+        case 8: { constexpr int KWC = 8; return CALL; }    \
+        case 12: { constexpr int KWC = 12; return CALL; }  \
+        default: { constexpr int KWC = 16; return CALL; }  \
+    }
+
+cudaError_t launch_wb_gram(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
+                           int nslice, float* red, cudaStream_t st) {
+    XHC_KW_DISPATCH(kw_of(d), (gram_kw<KWC>(d, slot, T, out, cw, nslice, red, st)));
+}
+
+cudaError_t launch_wb_fwd(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
+                          const float* red, int nslice, const uint16_t* xact, const int* I,
+                          const float* p, const float* hpost, const float* hres,
+                          uint16_t* xact_next, uint16_t* X, int* err, cudaStream_t st) {
+    const bool conv = d.K[slot] > 1;
+    if (d.k <= 4) {
+        if (!conv) return fwd_kw<4, 0>(d, slot, T, out, cw, red, nslice, xact, I, p, hpost, hres, xact_next, X, err, st);
+        XHC_KW_DISPATCH(kw_of(d), (fwd_kw<4, KWC>(d, slot, T, out, cw, red, nslice, xact, I, p, hpost, hres, xact_next, X, err, st)));
+    }
+    if (!conv) return fwd_kw<8, 0>(d, slot, T, out, cw, red, nslice, xact, I, p, hpost, hres, xact_next, X, err, st);
+    XHC_KW_DISPATCH(kw_of(d), (fwd_kw<8, KWC>(d, slot, T, out, cw, red, nslice, xact, I, p, hpost, hres, xact_next, X, err, st)));
+}
+
+cudaError_t launch_wb_bred(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
+                           const uint16_t* dX, const int* I, const float* dxact,
+                           const uint16_t* xact, int nslice, float* red, int* err, cudaStream_t st) {
+    const bool conv = d.K[slot] > 1;
+    if (d.k <= 4) {
+        if (!conv) return bred_kw<4, 0, 2>(d, slot, T, out, cw, dX, I, dxact, xact, nslice, red, err, st);
+        XHC_KW_DISPATCH(kw_of(d), (bred_kw<4, KWC, 2>(d, slot, T, out, cw, dX, I, dxact, xact, nslice, red, err, st)));
+    }
+    if (!conv) return bred_kw<8, 0, 4>(d, slot, T, out, cw, dX, I, dxact, xact, nslice, red, err, st);
+    XHC_KW_DISPATCH(kw_of(d), (bred_kw<8, KWC, 4>(d, slot, T, out, cw, dX, I, dxact, xact, nslice, red, err, st)));
+}
+
+cudaError_t launch_wb_bapp(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
+                           const uint16_t* dX, const int* I, const uint16_t* xact,
+                           const float* tokmat, float* dxact, float* du, uint16_t* d_out,
+                           int* err, cudaStream_t st) {
+    const int nslice = wb_nslice(d.C);
+    const bool conv = d.K[slot] > 1;
+    if (d.k <= 4) {
+        if (!conv) return bapp_kw<4, 0>(d, slot, T, out, cw, dX, I, xact, tokmat, dxact, du, d_out, nslice, err, st);
+        XHC_KW_DISPATCH(kw_of(d), (bapp_kw<4, KWC>(d, slot, T, out, cw, dX, I, xact, tokmat, dxact, du, d_out, nslice, err, st)));
+    }
+    if (!conv) return bapp_kw<8, 0>(d, slot, T, out, cw, dX, I, xact, tokmat, dxact, du, d_out, nslice, err, st);
+    XHC_KW_DISPATCH(kw_of(d), (bapp_kw<8, KWC>(d, slot, T, out, cw, dX, I, xact, tokmat, dxact, du, d_out, nslice, err, st)));
+}
+
+cudaError_t launch_wb_dout(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
+                           const float* du, uint16_t* d_out, float* cpart, cudaStream_t st) {
+    const int nslice = wb_nslice(d.C);
+    const int TBW = wb_dw_run(d);
+    XHC_KW_DISPATCH(kw_of(d), (dout_kw<KWC>(d, slot, T, cw, du, d_out, cpart, out, nslice, TBW, st)));
+}
+
+}  // namespace xhc

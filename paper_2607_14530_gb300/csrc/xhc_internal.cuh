@@ -247,6 +247,23 @@ cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, 
                          uint16_t* w16, const uint16_t* X, const uint16_t* dinput, const float* hpre,
                          const int* I, const float* dxact, const float* scal, int scal_ld,
                          uint16_t* dX, int* err, cudaStream_t st);
+int wb_nslice(int C);
+int wb_dw_run(const Dims& d);
+cudaError_t launch_wb_gram(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
+                           int nslice, float* red, cudaStream_t st);
+cudaError_t launch_wb_fwd(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
+                          const float* red, int nslice, const uint16_t* xact, const int* I,
+                          const float* p, const float* hpost, const float* hres,
+                          uint16_t* xact_next, uint16_t* X, int* err, cudaStream_t st);
+cudaError_t launch_wb_bred(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
+                           const uint16_t* dX, const int* I, const float* dxact,
+                           const uint16_t* xact, int nslice, float* red, int* err, cudaStream_t st);
+cudaError_t launch_wb_bapp(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
+                           const uint16_t* dX, const int* I, const uint16_t* xact,
+                           const float* tokmat, float* dxact, float* du, uint16_t* d_out,
+                           int* err, cudaStream_t st);
+cudaError_t launch_wb_dout(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
+                           const float* du, uint16_t* d_out, float* cpart, cudaStream_t st);
 cudaError_t launch_wgrad_reduce(const float* wpart, int splits, int E, int n, const WSegsOut& G,
                                 cudaStream_t st);
 cudaError_t launch_colsum(const float* in, int rows, int ld, int n, float* out, int accumulate,
