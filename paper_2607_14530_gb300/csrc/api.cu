@@ -642,7 +642,8 @@ xhc_status xhc_pre_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
     if (d.hr)
         XHC_K("colsum", c.st, launch_colsum(P->W_r, d.N * d.C, d.N, d.N, c.W<float>(c.L.wsum), 0,
                                c.W<float>(c.L.colscr), c.st));
-    XHC_K("full_dots", c.st, launch_full_dots(d, T32, X, dinput, c.S<int>(c.L.I), c.W<float>(c.L.dhpre), c.st));
+    XHC_K("full_dots", c.st, launch_full_dots(d, T32, X, dinput, c.S<int>(c.L.I), c.S<float>(c.L.hpre), dX,
+                                              c.W<float>(c.L.dhpre), c.st));
     XHC_K("full_coef", c.st, launch_full_coef(d, T32, c.W<float>(c.L.dhpre), c.S<float>(c.L.hpre),
                               c.S<float>(c.L.zfull), c.S<float>(c.L.stats), c.W<float>(c.L.wsum),
                               c.S<int>(c.L.I), c.W<float>(c.L.dp), P->alpha_pre,

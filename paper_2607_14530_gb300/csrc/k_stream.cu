@@ -771,14 +771,18 @@ cudaError_t launch_dinput_act(const Dims& d, int slot, int T, const uint16_t* d_
 }
 
 // ---------------------------------------------------------------------------------------------
-// full_dots: dH_pre[t][q][i] = <x_i, d_input_q> for the non-active streams i
+// full_dots: for the non-active streams i, dH_pre[t][q][i] = <x_i, d_input_q> and the dense-read
+// gradient dX[t][i] += sum_q H_pre[t][q][i] d_input_q (Eq. dense_read reversed)
 
 __global__ void __launch_bounds__(256) k_full_dots(Dims d, int T, const uint16_t* __restrict__ X,
                                                    const uint16_t* __restrict__ dinput,
                                                    const int* __restrict__ I,
+                                                   const float* __restrict__ hpre,
+                                                   uint16_t* __restrict__ dX,
                                                    float* __restrict__ dhpre) {
     __shared__ float wsh[8][4];
     __shared__ int active[MAXN];
+    __shared__ float hs[4 * MAXN];
     const int t = blockIdx.x, C = d.C, G = d.G;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int nw = (blockDim.x + 31) / 32;
@@ -788,21 +792,29 @@ __global__ void __launch_bounds__(256) k_full_dots(Dims d, int T, const uint16_t
             if (I[(int64_t)t * d.k + q] == i) a = 1;
         active[i] = a;
     }
+    for (int q = threadIdx.x; q < G * d.N; q += blockDim.x) hs[q] = hpre[(int64_t)t * G * d.N + q];
     __syncthreads();
     for (int i = 0; i < d.N; ++i) {
         if (active[i]) continue;
         float acc[4] = {0.f, 0.f, 0.f, 0.f};
         for (int c8 = threadIdx.x; c8 < C / 8; c8 += blockDim.x) {
-            float x[8];
-            unpack8(__ldg(reinterpret_cast<const uint4*>(X + ((int64_t)t * d.N + i) * C + c8 * 8)), x);
+            float x[8], dx[8];
+            const int64_t off = ((int64_t)t * d.N + i) * C + c8 * 8;
+            unpack8(__ldg(reinterpret_cast<const uint4*>(X + off)), x);
+            unpack8(*reinterpret_cast<const uint4*>(dX + off), dx);
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 if (q >= G) continue;
                 float g[8];
                 unpack8(*reinterpret_cast<const uint4*>(dinput + ((int64_t)q * T + t) * C + c8 * 8), g);
+                const float h = hs[q * d.N + i];
 #pragma unroll
-                for (int e = 0; e < 8; ++e) acc[q] = fmaf(x[e], g[e], acc[q]);
+                for (int e = 0; e < 8; ++e) {
+                    acc[q] = fmaf(x[e], g[e], acc[q]);
+                    dx[e] = fmaf(h, g[e], dx[e]);
+                }
             }
+            *reinterpret_cast<uint4*>(dX + off) = pack8(dx);
         }
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
@@ -820,8 +832,9 @@ __global__ void __launch_bounds__(256) k_full_dots(Dims d, int T, const uint16_t
 }
 
 cudaError_t launch_full_dots(const Dims& d, int T, const uint16_t* X, const uint16_t* dinput,
-                             const int* I, float* dhpre, cudaStream_t st) {
-    k_full_dots<<<T, chunk_threads(d.C), 0, st>>>(d, T, X, dinput, I, dhpre); note_launch();
+                             const int* I, const float* hpre, uint16_t* dX, float* dhpre,
+                             cudaStream_t st) {
+    k_full_dots<<<T, chunk_threads(d.C), 0, st>>>(d, T, X, dinput, I, hpre, dX, dhpre); note_launch();
     return cudaGetLastError();
 }
 

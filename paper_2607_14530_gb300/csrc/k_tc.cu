@@ -655,75 +655,105 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
             }
         }
     } else {
+        // Each epilogue warp owns rows [32 q, 32 q + 32) x columns [32 cg, 32 cg + 32) of the tile.
+        // The accumulator is read row-per-lane from TMEM, bounced through a padded shared tile,
+        // and re-read with 4 lanes per row (8 channels each) so that the global reads and writes
+        // are contiguous along the channels.
         const int quarter = warp & 3;
-        const int r = quarter * 32 + lane;
         const int cg = (warp - 2) >> 2;            // column group of 32
+        const int ew = warp - 2;                   // epilogue warp index
+        float* tileb = reinterpret_cast<float*>(smem + 2 * STAGE + 128) + ew * (32 * 33 + 32 * 8);
+        float* meta = tileb + 32 * 33;             // per row: j, h0..h3, sa, sb
         for (long long n = 0; n < nloc; ++n) {
             const long long tile = blockIdx.x + n * a.P;
             const int i = (int)(tile % a.N);
             const long long rest = tile / a.N;
             const int ct = (int)(rest % a.CT), tt = (int)(rest / a.CT);
             const int s = (int)(n & 1);
+            {
+                // per-row metadata of this lane's row (row-per-lane, matches the TMEM layout)
+                const int t = tt * BM + quarter * 32 + lane;
+                int j = -1;
+                float h[4] = {0.f, 0.f, 0.f, 0.f};
+                float sa = 0.f, sb = 0.f;
+                if (t < a.T) {
+                    for (int q = 0; q < a.k; ++q)
+                        if (a.I[(long long)t * a.k + q] == i) j = q;
+                    for (int q = 0; q < a.G; ++q) h[q] = a.hpre[((long long)t * a.G + q) * a.N + i];
+                    sa = a.scal[(long long)t * a.scal_ld + 0];
+                    sb = a.scal[(long long)t * a.scal_ld + 1];
+                }
+                float* m = meta + lane * 8;
+                m[0] = __int_as_float(j); m[1] = h[0]; m[2] = h[1]; m[3] = h[2]; m[4] = h[3];
+                m[5] = sa; m[6] = sb;
+            }
             if (!mbar_wait(smem_u32(&bars[4 + s]), (uint32_t)((n >> 1) & 1))) {
                 atomicExch(a.err, 14);
                 break;
             }
             tc_fence_after();
-            const int t = tt * BM + r;
             const uint32_t tl = tmem + (uint32_t)(s * DX_BN) + ((uint32_t)(quarter * 32) << 16);
-            int j = -1;
-            float h[4] = {0.f, 0.f, 0.f, 0.f};
-            float sa = 0.f, sb = 0.f;
-            if (t < a.T) {
-                for (int q = 0; q < a.k; ++q)
-                    if (a.I[(long long)t * a.k + q] == i) j = q;
-                for (int q = 0; q < a.G; ++q) h[q] = a.hpre[((long long)t * a.G + q) * a.N + i];
-                sa = a.scal[(long long)t * a.scal_ld + 0];
-                sb = a.scal[(long long)t * a.scal_ld + 1];
-            }
-            const long long rowoff = ((long long)t * a.N + i) * a.C + ct * DX_BN;
-            for (int c0 = cg * (DX_BN / 4); c0 < (cg + 1) * (DX_BN / 4); c0 += 16) {
-                // global operands first (independent of the accumulator), then the TMEM read
-                float x[16], v[16];
-                const int c = ct * DX_BN + c0;
-                const bool tv = t < a.T;
-                if (tv) {
-                    unpack8(__ldg(reinterpret_cast<const uint4*>(a.X + rowoff + c0)), x);
-                    unpack8(__ldg(reinterpret_cast<const uint4*>(a.X + rowoff + c0 + 8)), x + 8);
-                    if (j >= 0) {
-                        const float4* b = reinterpret_cast<const float4*>(a.dxact + ((long long)t * a.k + j) * a.C + c);
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            const float4 f = b[q];
-                            v[4 * q] = f.x; v[4 * q + 1] = f.y; v[4 * q + 2] = f.z; v[4 * q + 3] = f.w;
-                        }
-                    } else {
-                        unpack8(*reinterpret_cast<const uint4*>(a.dX + rowoff + c0), v);
-                        unpack8(*reinterpret_cast<const uint4*>(a.dX + rowoff + c0 + 8), v + 8);
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            if (q >= a.G) continue;
-                            float g[16];
-                            const uint16_t* dp = a.dinput + ((long long)q * a.T + t) * a.C + c;
-                            unpack8(__ldg(reinterpret_cast<const uint4*>(dp)), g);
-                            unpack8(__ldg(reinterpret_cast<const uint4*>(dp + 8)), g + 8);
-#pragma unroll
-                            for (int e = 0; e < 16; ++e) v[e] = fmaf(h[q], g[e], v[e]);
-                        }
-                    }
-                }
+            {
                 float acc[16];
-                tmem_ld16(tl + (uint32_t)c0, acc);
-                if (!tv) continue;
-                float o[16];
+                tmem_ld16(tl + (uint32_t)(cg * 32), acc);
 #pragma unroll
-                for (int e = 0; e < 16; ++e) o[e] = v[e] + acc[e] + sa + sb * x[e];
-                *reinterpret_cast<uint4*>(a.dX + rowoff + c0) = pack8(o);
-                *reinterpret_cast<uint4*>(a.dX + rowoff + c0 + 8) = pack8(o + 8);
+                for (int e = 0; e < 16; ++e) tileb[lane * 33 + e] = acc[e];
+                tmem_ld16(tl + (uint32_t)(cg * 32 + 16), acc);
+#pragma unroll
+                for (int e = 0; e < 16; ++e) tileb[lane * 33 + 16 + e] = acc[e];
             }
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&bars[6 + s]));
+            if (lane == 0) mbar_arrive(smem_u32(&bars[6 + s]));  // TMEM buffer free
+            // 4 passes of 8 rows; lane -> row rr = 8 pass + lane / 4, channels 8 (lane % 4) ..
+            // Every pass's reads are issued before any write.
+            const int cq = (lane & 3) * 8;
+            const int c = ct * DX_BN + cg * 32 + cq;
+            uint4 xr[4], br[4], br2[4];
+#pragma unroll
+            for (int pass = 0; pass < 4; ++pass) {
+                const int rr = pass * 8 + (lane >> 2);
+                const int t = tt * BM + quarter * 32 + rr;
+                xr[pass] = make_uint4(0, 0, 0, 0);
+                br[pass] = make_uint4(0, 0, 0, 0);
+                br2[pass] = make_uint4(0, 0, 0, 0);
+                if (t >= a.T) continue;
+                const int j = __float_as_int(meta[rr * 8]);
+                const long long off = ((long long)t * a.N + i) * a.C + c;
+                xr[pass] = __ldg(reinterpret_cast<const uint4*>(a.X + off));
+                if (j >= 0) {
+                    const uint4* b = reinterpret_cast<const uint4*>(a.dxact + ((long long)t * a.k + j) * a.C + c);
+                    br[pass] = b[0];
+                    br2[pass] = b[1];
+                } else {
+                    br[pass] = *reinterpret_cast<const uint4*>(a.dX + off);
+                }
+            }
+#pragma unroll
+            for (int pass = 0; pass < 4; ++pass) {
+                const int rr = pass * 8 + (lane >> 2);
+                const int t = tt * BM + quarter * 32 + rr;
+                if (t >= a.T) continue;
+                const float* m = meta + rr * 8;
+                const int j = __float_as_int(m[0]);
+                const long long off = ((long long)t * a.N + i) * a.C + c;
+                float x[8], v[8];
+                unpack8(xr[pass], x);
+                if (j >= 0) {
+                    v[0] = __uint_as_float(br[pass].x); v[1] = __uint_as_float(br[pass].y);
+                    v[2] = __uint_as_float(br[pass].z); v[3] = __uint_as_float(br[pass].w);
+                    v[4] = __uint_as_float(br2[pass].x); v[5] = __uint_as_float(br2[pass].y);
+                    v[6] = __uint_as_float(br2[pass].z); v[7] = __uint_as_float(br2[pass].w);
+                } else {
+                    unpack8(br[pass], v);
+                }
+                const float sa = m[5], sb = m[6];
+                float o[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) o[e] = v[e] + tileb[rr * 33 + cq + e] + sa + sb * x[e];
+                *reinterpret_cast<uint4*>(a.dX + off) = pack8(o);
+            }
+            __syncwarp();
         }
     }
     tc_fence_before();
@@ -782,7 +812,8 @@ cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, 
     a.P = (int)std::min<long long>(num_sms(), a.ntiles);
     a.X = X; a.dX = dX; a.dinput = dinput; a.hpre = hpre; a.I = I; a.dxact = dxact;
     a.scal = scal; a.scal_ld = scal_ld; a.err = err;
-    const size_t sm = 2 * (size_t)a.nkb * (BM + DX_BN) * BK * 2 + 8 * 8 + 16 + 1024;
+    const size_t sm = 2 * (size_t)a.nkb * (BM + DX_BN) * BK * 2 + 128 +
+                      (size_t)DX_EW * (32 * 33 + 32 * 8) * 4 + 1024;
     e = cudaFuncSetAttribute((const void*)k_dx_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
     k_dx_tc<<<a.P, DX_THREADS, sm, st>>>(ma, mb, a); note_launch();

@@ -80,6 +80,22 @@ struct StageGeom {
     int tokb;       // bytes per token = nrow * rowb
 };
 
+// Per-thread prefetch of the next tokens' values with cp.async into a 4-slot ring in shared
+// memory (field-major [slot][field][thread], so a warp's accesses are consecutive words).
+constexpr int PD = 4;
+__device__ __forceinline__ void cpa4(void* dst, const void* src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(s_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cpa8(void* dst, const void* src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(s_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cpa_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cpa_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+__device__ __forceinline__ float2 u2f2(uint32_t u) {
+    return make_float2(__uint_as_float(u << 16), __uint_as_float(u & 0xffff0000u));
+}
+
 template <int KW>
 __device__ __forceinline__ void taps_reg(const Dims& d, const ConvPtrs& cw, int c, bool act,
                                          float2 (&tw)[3][KW]) {
@@ -212,7 +228,14 @@ __global__ void __launch_bounds__(WT) k_wb_gram(Dims d, int slot, int T, int TB,
 
 // ---------------------------------------------------------------------------------------------
 // wb_fwd: per-token coefficients E[j][a] (Gram-Schmidt folded in), H_res, I in shared memory;
-// the out row and the k active rows of every token are staged by bulk copies.
+// each thread prefetches the out value and the k active values of its channel pair 3 tokens
+// ahead with cp.async.
+
+template <int KM>
+struct FRing {
+    uint32_t o[PD][WT];
+    uint32_t x[PD][KM][WT];
+};
 
 template <int KM, int KW>
 __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
@@ -225,47 +248,32 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
                                                const float* __restrict__ hres,
                                                uint16_t* __restrict__ xact_next,
                                                uint16_t* __restrict__ X, int* __restrict__ err) {
-    constexpr int BT = KW > 0 ? KW : 8;      // tokens per staged batch
-    extern __shared__ __align__(128) unsigned char smu[];
+    (void)err;
+    extern __shared__ __align__(16) unsigned char smu[];
+    FRing<KM>& R = *reinterpret_cast<FRing<KM>*>(smu);
     const int k = d.k, K = d.K[slot], C = d.C;
     const bool last = (slot == d.G - 1);
     const bool gs = (K > 1) && d.gs;
-    const int c0 = blockIdx.x * WSL;
-    const int cs = min(WSL, C - c0);                 // channels of this slice
-    const uint32_t rowb = (uint32_t)cs * 2;
-    const int tokb = (1 + k) * WSL * 2;              // out row + k active rows
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smu);
-    float* Esh = reinterpret_cast<float*>(smu + 64);           // [TB][KM][4]
-    float* Hsh = Esh + TB * KM * 4;                           // [TB][KM][KM]
-    int* Ish = reinterpret_cast<int*>(Hsh + TB * KM * KM);     // [TB][KM]
-    unsigned char* stg = smu + 64 + (size_t)TB * (KM * 4 + KM * KM + KM) * 4;
-    stg = (unsigned char*)(((uintptr_t)stg + 127) & ~(uintptr_t)127);
+    float* Esh = reinterpret_cast<float*>(smu + sizeof(FRing<KM>));  // [TB][KM][4]
+    float* Hsh = Esh + TB * KM * 4;                                 // [TB][KM][KM]
+    int* Ish = reinterpret_cast<int*>(Hsh + TB * KM * KM);           // [TB][KM]
     const long long t0 = (long long)blockIdx.y * TB;
     const long long t1 = min((long long)T, t0 + TB);
     const int ntok = (int)(t1 - t0);
-    const int nb = (ntok + BT - 1) / BT;
-    if (threadIdx.x == 0) {
-        bar_init(&bars[0], 1);
-        bar_init(&bars[1], 1);
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    }
-    __syncthreads();
-    auto issue = [&](int b) {  // warp 0
-        const int s = b & 1;
-        const int tb0 = b * BT, nt = min(BT, ntok - tb0);
-        if (threadIdx.x == 0) bar_expect(&bars[s], (uint32_t)(nt * (1 + k)) * rowb);
-        __syncwarp();
-        for (int q = threadIdx.x; q < nt * (1 + k); q += 32) {
-            const int tt = q / (1 + k), r = q - tt * (1 + k);
-            const long long t = t0 + tb0 + tt;
-            const uint16_t* src = (r == 0) ? out + t * C + c0 : xact + (t * k + (r - 1)) * C + c0;
-            bulk_g2s(stg + (size_t)s * BT * tokb + (size_t)tt * tokb + (size_t)r * WSL * 2, src, rowb, &bars[s]);
+    const int c = blockIdx.x * WSL + 2 * threadIdx.x;
+    const bool act = c < C;
+    auto issue = [&](int sl, int tn) {
+        if (act && tn < ntok) {
+            const long long t = t0 + tn;
+            cpa4(&R.o[sl][threadIdx.x], out + t * C + c);
+#pragma unroll
+            for (int j = 0; j < KM; ++j)
+                if (j < k) cpa4(&R.x[sl][j][threadIdx.x], xact + (t * k + j) * C + c);
         }
+        cpa_commit();
     };
-    if (threadIdx.x < 32) {
-        issue(0);
-        if (nb > 1) issue(1);
-    }
+#pragma unroll
+    for (int q = 0; q < PD - 1; ++q) issue(q, q);
     for (int tt = threadIdx.x; tt < ntok; tt += WT) {
         const long long t = t0 + tt;
         double B[MAXCOMP][MAXCOMP];
@@ -299,29 +307,24 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
                 Hsh[(tt * KM + j) * KM + i] = (last && jv && i < k) ? hres[t * k * k + j * k + i] : 0.f;
         }
     }
-    const int cl = 2 * threadIdx.x;                 // channel pair within the slice
-    const int c = c0 + cl;
-    const bool act = cl < cs;
     float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
     if constexpr (KW > 0) {
         taps_reg<KW>(d, cw, c, act, tw);
         ring_init<KW>(out, C, c, act, t0, w);
     }
     __syncthreads();
-    for (int b = 0; b < nb; ++b) {
-        const int s = b & 1;
-        if (!bar_wait(&bars[s], (uint32_t)((b >> 1) & 1))) {
-            if (threadIdx.x == 0) atomicExch(err, 21);
-            break;
-        }
-        const unsigned char* sb = stg + (size_t)s * BT * tokb;
+    const int RU = KW > 0 ? KW : 4;
+    for (long long tb = t0; tb < t1; tb += RU) {
 #pragma unroll
-        for (int u = 0; u < BT; ++u) {
-            const int tt = b * BT + u;
-            if (tt < ntok && act) {
-                const long long t = t0 + tt;
-                const unsigned char* tk = sb + (size_t)u * tokb;
-                const float2 o = ld2(reinterpret_cast<const uint16_t*>(tk) + cl);
+        for (int u = 0; u < RU; ++u) {
+            const long long t = tb + u;
+            if (t < t1) {
+                const int tt = (int)(t - t0);
+                const int sl = u % PD;
+                issue((u + PD - 1) % PD, tt + PD - 1);
+                cpa_wait<PD - 1>();
+                if (!act) continue;
+                const float2 o = u2f2(R.o[sl][threadIdx.x]);
                 float2 uu[4] = {o, f2z(), f2z(), f2z()};
                 if constexpr (KW > 0) {
                     w[u] = o;
@@ -333,8 +336,8 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
                 }
                 float2 x[KM];
 #pragma unroll
-                for (int j = 0; j < KM; ++j)
-                    x[j] = (j < k) ? ld2(reinterpret_cast<const uint16_t*>(tk + (size_t)(1 + j) * WSL * 2) + cl) : f2z();
+                for (int j = 0; j < KM; ++j) x[j] = (j < k) ? u2f2(R.x[sl][j][threadIdx.x]) : f2z();
+                const float4* E4 = reinterpret_cast<const float4*>(Esh + tt * KM * 4);
 #pragma unroll
                 for (int j = 0; j < KM; ++j) {
                     if (j >= k) continue;
@@ -346,27 +349,52 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
                     } else {
                         v = x[j];
                     }
-#pragma unroll
-                    for (int a = 0; a < 4; ++a) v = fma2(Esh[(tt * KM + j) * 4 + a], uu[a], v);
+                    const float4 e = E4[j];
+                    v = fma2(e.x, uu[0], v);
+                    v = fma2(e.y, uu[1], v);
+                    v = fma2(e.z, uu[2], v);
+                    v = fma2(e.w, uu[3], v);
                     if (last)
                         st2(X + (t * d.N + Ish[tt * KM + j]) * C + c, v);
                     else
                         st2(xact_next + (t * k + j) * C + c, v);
                 }
-            } else if constexpr (KW > 0) {
-                if (tt < ntok) w[u] = f2z();
             }
         }
-        __syncthreads();
-        if (threadIdx.x < 32 && b + 2 < nb) issue(b + 2);
     }
+    cpa_wait<0>();
 }
 
-// ---------------------------------------------------------------------------------------------
-// wb_bred: backward reductions, fixed slots per token (zeros where a term does not apply):
-//   [j*4 + a]              P[j][a] = <dXn_j, u_a>
-//   [KM*4 + j*KM + i]      Q[j][i] = <dXn_j, x_i>          (last slot)
-//   [KM*4 + KM*KM + q]     Gram of u, lower triangle packed (Gram-Schmidt on)
+// prefetch ring of the backward kernels: per slot, out (bf16 pair), x_j (bf16 pairs), dn_j
+// (fp32 pair, or a bf16 pair in .x at the last slot)
+template <int KM>
+struct BRing {
+    uint32_t o[PD][WT];
+    uint32_t x[PD][KM][WT];
+    uint2 dn[PD][KM][WT];
+};
+
+template <int KM>
+__device__ __forceinline__ void bring_issue(BRing<KM>& R, int slot, long long t, bool ok, int k,
+                                            int N, int C, int c, bool last, bool with_x,
+                                            const uint16_t* out, const uint16_t* xact,
+                                            const uint16_t* dX, const int* Irow,
+                                            const float* dxact) {
+    const int tid = threadIdx.x;
+    if (ok) {
+        cpa4(&R.o[slot][tid], out + t * C + c);
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            if (j >= k) continue;
+            if (with_x) cpa4(&R.x[slot][j][tid], xact + (t * k + j) * C + c);
+            if (last)
+                cpa4(&R.dn[slot][j][tid], dX + (t * N + Irow[j]) * C + c);
+            else
+                cpa8(&R.dn[slot][j][tid], dxact + (t * k + j) * C + c);
+        }
+    }
+    cpa_commit();
+}
 
 template <int KM, int KW, int NB>
 __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
@@ -376,7 +404,10 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
                                                 const float* __restrict__ dxact,
                                                 const uint16_t* __restrict__ xact, int nslice,
                                                 float* __restrict__ red) {
-    extern __shared__ float wsh[];  // [TB][WT/32][NB*32]
+    extern __shared__ __align__(16) unsigned char smu[];
+    BRing<KM>& R = *reinterpret_cast<BRing<KM>*>(smu);
+    int* Ish = reinterpret_cast<int*>(smu + sizeof(BRing<KM>));          // [TB][KM]
+    float* wsh = reinterpret_cast<float*>(Ish + TB * KM);                 // [TB][WT/32][NB*32]
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int slice = blockIdx.x, C = d.C, k = d.k;
     const int K = d.K[slot];
@@ -387,6 +418,16 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
     const bool act = c < C;
     const long long t0 = (long long)blockIdx.y * TB;
     const long long t1 = min((long long)T, t0 + TB);
+    const int ntok = (int)(t1 - t0);
+    for (int q = threadIdx.x; q < ntok * KM; q += WT) {
+        const int tt = q / KM, j = q - tt * KM;
+        Ish[q] = (j < k) ? I[(t0 + tt) * k + j] : 0;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int q = 0; q < PD - 1; ++q)
+        bring_issue<KM>(R, q, t0 + q, act && q < ntok, k, d.N, C, c, last, last, out, xact, dX,
+                        Ish + q * KM, dxact);
     float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
     if constexpr (KW > 0) {
         taps_reg<KW>(d, cw, c, act, tw);
@@ -398,6 +439,14 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
         for (int u = 0; u < RU; ++u) {
             const long long t = tb + u;
             if (t < t1) {
+                const int tt = (int)(t - t0);
+                const int sl = u % PD;                       // == tt % PD (runs start on a multiple of 4)
+                {
+                    const int tn = tt + PD - 1;
+                    bring_issue<KM>(R, (u + PD - 1) % PD, t0 + tn, act && tn < ntok, k, d.N, C, c, last,
+                                    last, out, xact, dX, Ish + (tn < ntok ? tn : 0) * KM, dxact);
+                }
+                cpa_wait<PD - 1>();
                 float2 uu[4] = {f2z(), f2z(), f2z(), f2z()};
                 float2 dn[KM], x[KM];
 #pragma unroll
@@ -406,7 +455,7 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
                     x[j] = f2z();
                 }
                 if (act) {
-                    const float2 o = ld2(out + t * C + c);
+                    const float2 o = u2f2(R.o[sl][threadIdx.x]);
                     uu[0] = o;
                     if constexpr (KW > 0) {
                         w[u] = o;
@@ -419,11 +468,12 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
 #pragma unroll
                     for (int j = 0; j < KM; ++j) {
                         if (j >= k) continue;
+                        const uint2 r = R.dn[sl][j][threadIdx.x];
                         if (last) {
-                            dn[j] = ld2(dX + (t * d.N + I[t * k + j]) * C + c);
-                            x[j] = ld2(xact + (t * k + j) * C + c);
+                            dn[j] = u2f2(r.x);
+                            x[j] = u2f2(R.x[sl][j][threadIdx.x]);
                         } else {
-                            dn[j] = *reinterpret_cast<const float2*>(dxact + (t * k + j) * C + c);
+                            dn[j] = make_float2(__uint_as_float(r.x), __uint_as_float(r.y));
                         }
                     }
                 } else if constexpr (KW > 0) {
@@ -452,19 +502,19 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
                 }
                 float tot[NB];
                 wred32<NB>(v, lane, tot);
-                float* dst = wsh + ((t - t0) * (WT / 32) + warp) * (NB * 32);
+                float* dst = wsh + ((size_t)tt * (WT / 32) + warp) * (NB * 32);
 #pragma unroll
                 for (int bb = 0; bb < NB; ++bb) dst[bb * 32 + lane] = tot[bb];
             }
         }
     }
+    cpa_wait<0>();
     __syncthreads();
-    const int ntok = (int)(t1 - t0);
     for (int idx = threadIdx.x; idx < ntok * nv; idx += WT) {
         const int tt = idx / nv, q = idx - tt * nv;
         float sm = 0.f;
 #pragma unroll
-        for (int ww = 0; ww < WT / 32; ++ww) sm += wsh[(tt * (WT / 32) + ww) * (NB * 32) + q];
+        for (int ww = 0; ww < WT / 32; ++ww) sm += wsh[((size_t)tt * (WT / 32) + ww) * (NB * 32) + q];
         red[((t0 + tt) * nslice + slice) * NRED + q] = sm;
     }
 }
@@ -482,14 +532,15 @@ __global__ void __launch_bounds__(WT) k_wb_bapp(Dims d, int slot, int T, int TB,
                                                 float* __restrict__ dxact,
                                                 float* __restrict__ du,
                                                 uint16_t* __restrict__ d_out) {
-    extern __shared__ float smf[];
+    extern __shared__ __align__(16) unsigned char smu[];
+    BRing<KM>& R = *reinterpret_cast<BRing<KM>*>(smu);
     const int k = d.k, K = d.K[slot], C = d.C;
     const bool last = (slot == d.G - 1);
-    float* Esh = smf;                        // [TB][KM][4]
-    float* Dsh = Esh + TB * KM * 4;          // [TB][4][4]
-    float* Hsh = Dsh + TB * 16;              // [TB][KM][KM]
-    float* cxs = Hsh + TB * KM * KM;         // [TB]
-    int* Ish = (int*)(cxs + TB);             // [TB][KM]
+    float* Esh = reinterpret_cast<float*>(smu + sizeof(BRing<KM>));  // [TB][KM][4]
+    float* Dsh = Esh + TB * KM * 4;                                 // [TB][4][4]
+    float* Hsh = Dsh + TB * 16;                                     // [TB][KM][KM]
+    float* cxs = Hsh + TB * KM * KM;                                // [TB]
+    int* Ish = (int*)(cxs + TB);                                    // [TB][KM]
     const long long t0 = (long long)blockIdx.y * TB;
     const long long t1 = min((long long)T, t0 + TB);
     const int ntok = (int)(t1 - t0);
@@ -513,20 +564,32 @@ __global__ void __launch_bounds__(WT) k_wb_bapp(Dims d, int slot, int T, int TB,
     }
     const int c = blockIdx.x * WSL + 2 * threadIdx.x;
     const bool act = c < C;
+    __syncthreads();
+#pragma unroll
+    for (int q = 0; q < PD - 1; ++q)
+        bring_issue<KM>(R, q, t0 + q, act && q < ntok, k, d.N, C, c, last, true, out, xact, dX,
+                        Ish + q * KM, dxact);
     float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
     if constexpr (KW > 0) {
         taps_reg<KW>(d, cw, c, act, tw);
         ring_init<KW>(out, C, c, act, t0, w);
     }
-    __syncthreads();
     const int RU = KW > 0 ? KW : 4;
     for (long long tb = t0; tb < t1; tb += RU) {
 #pragma unroll
         for (int u = 0; u < RU; ++u) {
             const long long t = tb + u;
-            if (t < t1 && act) {
+            if (t < t1) {
                 const int tt = (int)(t - t0);
-                const float2 o = ld2(out + t * C + c);
+                const int sl = u % PD;
+                {
+                    const int tn = tt + PD - 1;
+                    bring_issue<KM>(R, (u + PD - 1) % PD, t0 + tn, act && tn < ntok, k, d.N, C, c, last,
+                                    true, out, xact, dX, Ish + (tn < ntok ? tn : 0) * KM, dxact);
+                }
+                cpa_wait<PD - 1>();
+                if (!act) continue;
+                const float2 o = u2f2(R.o[sl][threadIdx.x]);
                 float2 uu[4] = {o, f2z(), f2z(), f2z()};
                 if constexpr (KW > 0) {
                     w[u] = o;
@@ -540,9 +603,9 @@ __global__ void __launch_bounds__(WT) k_wb_bapp(Dims d, int slot, int T, int TB,
 #pragma unroll
                 for (int j = 0; j < KM; ++j) {
                     if (j < k) {
-                        dn[j] = last ? ld2(dX + (t * d.N + Ish[tt * KM + j]) * C + c)
-                                     : *reinterpret_cast<const float2*>(dxact + (t * k + j) * C + c);
-                        x[j] = ld2(xact + (t * k + j) * C + c);
+                        const uint2 r = R.dn[sl][j][threadIdx.x];
+                        dn[j] = last ? u2f2(r.x) : make_float2(__uint_as_float(r.x), __uint_as_float(r.y));
+                        x[j] = u2f2(R.x[sl][j][threadIdx.x]);
                     } else {
                         dn[j] = f2z();
                         x[j] = f2z();
@@ -580,6 +643,7 @@ __global__ void __launch_bounds__(WT) k_wb_bapp(Dims d, int slot, int T, int TB,
             }
         }
     }
+    cpa_wait<0>();
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -721,10 +785,8 @@ template <int KM, int KW>
 cudaError_t fwd_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, const float* red,
                    int nslice, const uint16_t* xact, const int* I, const float* p, const float* hpost,
                    const float* hres, uint16_t* xact_next, uint16_t* X, int* err, cudaStream_t st) {
-    constexpr int BT = KW > 0 ? KW : 8;
-    const int TB = run_len(BT, 96);
-    const size_t sm = 64 + (size_t)TB * (KM * 4 + KM * KM + KM) * 4 + 128 +
-                      2 * (size_t)BT * (1 + d.k) * WSL * 2;
+    const int TB = run_len(KW, 96);
+    const size_t sm = sizeof(FRing<KM>) + (size_t)TB * (KM * 4 + KM * KM + KM) * 4;
     cudaError_t e = smem_attr((const void*)k_wb_fwd<KM, KW>, sm);
     if (e != cudaSuccess) return e;
     dim3 grid(nslice, (T + TB - 1) / TB);
@@ -740,7 +802,7 @@ cudaError_t bred_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtr
     (void)err;
     int TB = run_len(KW, 48);
     while (TB > (KW > 0 ? KW : 4) && (size_t)TB * (WT / 32) * NB * 32 * 4 > 96 * 1024) TB -= (KW > 0 ? KW : 4);
-    const size_t sm = (size_t)TB * (WT / 32) * NB * 32 * sizeof(float);
+    const size_t sm = sizeof(BRing<KM>) + (size_t)TB * KM * 4 + (size_t)TB * (WT / 32) * NB * 32 * sizeof(float);
     cudaError_t e = smem_attr((const void*)k_wb_bred<KM, KW, NB>, sm);
     if (e != cudaSuccess) return e;
     dim3 grid(nslice, (T + TB - 1) / TB);
@@ -754,7 +816,7 @@ cudaError_t bapp_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtr
                     uint16_t* d_out, int nslice, int* err, cudaStream_t st) {
     (void)err;
     const int TB = run_len(KW, 64);
-    const size_t sm = (size_t)TB * (KM * 4 + 16 + KM * KM + 1 + KM) * 4;
+    const size_t sm = sizeof(BRing<KM>) + (size_t)TB * (KM * 4 + 16 + KM * KM + 1 + KM) * 4;
     cudaError_t e = smem_attr((const void*)k_wb_bapp<KM, KW>, sm);
     if (e != cudaSuccess) return e;
     dim3 grid(nslice, (T + TB - 1) / TB);

@@ -317,7 +317,8 @@ cudaError_t launch_dinput_act(const Dims& d, int slot, int T, const uint16_t* d_
                               float* dxact, float* dhpre, uint16_t* dinput_copy,
                               cudaStream_t st);
 cudaError_t launch_full_dots(const Dims& d, int T, const uint16_t* X, const uint16_t* dinput,
-                             const int* I, float* dhpre, cudaStream_t st);
+                             const int* I, const float* hpre, uint16_t* dX, float* dhpre,
+                             cudaStream_t st);
 cudaError_t launch_full_coef(const Dims& d, int T, const float* dhpre, const float* hpre,
                              const float* zfull, const float* stats, const float* wsum,
                              const int* I, const float* dp, const float* alpha_pre, float* dz,
