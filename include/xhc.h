@@ -190,15 +190,19 @@ xhc_status xhc_post_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
                         void* stream);
 
 /* Backward of post_fwd(slot).  Reads dX (slot G-1: the gradient w.r.t. the group output) or the
- * workspace-held active gradient, writes d_out [T, C] (= dL/d out, including the paths through
+ * workspace-held active gradient, leaves the post/res map-logit gradient in the workspace for
+ * pre_bwd(slot), writes d_out [T, C] (= dL/d out, including the paths through
  * later sublayer inputs), accumulates the post/res/conv parameter gradients.  slot G-1 also
  * restores the active rows of X to the group-entry state. */
 xhc_status xhc_post_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
                         uint16_t* X, uint16_t* dX, const uint16_t* out, uint16_t* d_out,
                         const xhc_grads* grads, void* saved, void* workspace, void* stream);
 
-/* Backward of pre_fwd(slot).  Adds the dense-read gradient of d_input to the active gradient;
- * slot 0 finishes the group: dX becomes the gradient w.r.t. the entry state (dense reads,
+/* Backward of pre_fwd(slot).  Adds the dense-read gradient of d_input and the gradient through
+ * the post/res map projections of this slot to the active gradient (the map-logit gradient is
+ * left in the workspace by post_bwd(slot), so the calls of one slot run back to back on the same
+ * workspace; P needs W_post[slot], and W_res at the last slot, on every slot); slot 0 finishes
+ * the group: dX becomes the gradient w.r.t. the entry state (dense reads,
  * norm statistics, router through the selected routed scores only) and the W_r / W_pre /
  * alpha_pre / b_pre gradients are accumulated. */
 xhc_status xhc_pre_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,

@@ -170,9 +170,12 @@ Layout make_layout(const Dims& d, int64_t T) {
     o = al(o + std::max((size_t)L.tc.NB * d.N * d.C, (size_t)L.tca.NB * d.k * d.C) * 2);
     L.dzpack = o; o = al(o + (size_t)std::max(L.twf.NB, L.twa.NB) * ((t + 7) / 8 * 8) * 2);
     {
+        // bf16 operands of the tensor-core input gradients: full maps [T][nfull] and [N C][nfull],
+        // active maps in three parts [T][3 nact] and [k C][3 nact] (rows padded to 8)
         const size_t ld = (size_t)(d.nfull + 7) / 8 * 8;
-        L.dz16 = o; o = al(o + t * ld * 2);
-        L.w16 = o; o = al(o + (size_t)d.N * d.C * ld * 2);
+        const size_t ld3 = (size_t)(3 * nact_max + 7) / 8 * 8;
+        L.dz16 = o; o = al(o + t * std::max(ld, ld3) * 2);
+        L.w16 = o; o = al(o + std::max((size_t)d.N * d.C * ld, (size_t)d.k * d.C * ld3) * 2);
     }
     L.part = o;
     o = al(o + std::max((size_t)L.splits_full * d.nfull, (size_t)L.splits_act * nact_max) * t * 4);
@@ -590,7 +593,9 @@ xhc_status xhc_post_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
                                           c.W<float>(c.L.tokmat), dxact, c.W<float>(c.L.du), d_out,
                                           c.W<int>(c.L.err), c.st));
     const WSegs wa = act_segs(d, P, slot);
-    XHC_K("gemm_dzw", c.st, launch_gemm_dzw(d, T32, c.W<float>(c.L.dz), n, n, wa, d.k * d.C, dxact, c.st));
+    // dZ_act stays in the workspace: pre_bwd(slot) applies it to dX_act on the tensor cores
+    if (!dxa_tc_ok(T32, d.k, d.C, n))
+        XHC_K("gemm_dzw", c.st, launch_gemm_dzw(d, T32, c.W<float>(c.L.dz), n, n, wa, d.k * d.C, dxact, c.st));
     if (T32 < 64 || d.k * d.C < 128) {
         const int ts = std::min(c.L.tsplits, pick_tsplits(d.k * d.C, T32));
         XHC_K("wgrad_active", c.st, launch_wgrad(c.xact(slot), (int64_t)d.k * d.C, d.k * d.C, T32,
@@ -628,16 +633,25 @@ xhc_status xhc_pre_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
     Ctx c;
     xhc_status s = common_check(h, slot, T, saved, workspace, c, stream);
     if (s != XHC_OK) return s;
-    if (!X || !d_input || !dX || !P || (slot == 0 && (!params_ok(c.d, P, slot, true) ||
-                                                      !grads_ok(c.d, g, slot, true))))
+    if (!X || !d_input || !dX || !params_ok(c.d, P, slot, slot == 0) ||
+        (slot == 0 && !grads_ok(c.d, g, slot, true)))
         return XHC_ERR_INVALID_ARG;
     if (!aligned16(X) || !aligned16(d_input) || !aligned16(dX)) return XHC_ERR_ALIGNMENT;
     const Dims& d = c.d;
     const int T32 = c.T;
     uint16_t* dinput = c.W<uint16_t>(c.L.dinput);
-    XHC_K("dinput_act", c.st, launch_dinput_act(d, slot, T32, d_input, c.xact(slot), c.S<float>(c.L.hpre),
-                               c.S<int>(c.L.I), c.W<float>(c.L.dxact), c.W<float>(c.L.dhpre),
-                               dinput, c.st));
+    const int n = d.nact[slot];
+    const bool tc = dxa_tc_ok(T32, d.k, d.C, n);
+    XHC_K("dinput_act", c.st, launch_dinput_act(d, slot, T32, tc ? 0 : 1, d_input, c.xact(slot),
+                               c.S<float>(c.L.hpre), c.S<int>(c.L.I), c.W<float>(c.L.dxact),
+                               c.W<float>(c.L.dhpre), dinput, c.st));
+    if (tc) {
+        // post_bwd(slot) left dZ_act of this slot in the workspace
+        XHC_K("dxa_tc", c.st, launch_dxa_tc(d, slot, T32, c.W<float>(c.L.dz), n, act_segs(d, P, slot),
+                                            c.W<uint16_t>(c.L.dz16), c.W<uint16_t>(c.L.w16), d_input,
+                                            c.S<float>(c.L.hpre), c.S<int>(c.L.I), c.W<float>(c.L.dxact),
+                                            c.W<int>(c.L.err), c.st));
+    }
     if (slot != 0) return XHC_OK;
     if (d.hr)
         XHC_K("colsum", c.st, launch_colsum(P->W_r, d.N * d.C, d.N, d.N, c.W<float>(c.L.wsum), 0,

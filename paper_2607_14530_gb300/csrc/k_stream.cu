@@ -703,7 +703,7 @@ cudaError_t launch_conv_wgrad_reduce(const Dims& d, int slot, const float* cpart
 // d_input is copied to the workspace for the full-state backward of slot 0.
 
 template <int KM>
-__global__ void __launch_bounds__(256) k_dinput_act(Dims d, int slot, int T,
+__global__ void __launch_bounds__(256) k_dinput_act(Dims d, int slot, int T, int add_dx,
                                                     const uint16_t* __restrict__ din,
                                                     const uint16_t* __restrict__ xact,
                                                     const float* __restrict__ hpre,
@@ -730,6 +730,9 @@ __global__ void __launch_bounds__(256) k_dinput_act(Dims d, int slot, int T,
             if (j >= k) continue;
             float x[8];
             unpack8(*reinterpret_cast<const uint4*>(xact + ((int64_t)t * k + j) * C + c8 * 8), x);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) dot[j] = fmaf(x[e], g[e], dot[j]);
+            if (!add_dx) continue;
             float* dp = dxact + ((int64_t)t * k + j) * C + c8 * 8;
             float4 a = *reinterpret_cast<float4*>(dp);
             float4 b = *reinterpret_cast<float4*>(dp + 4);
@@ -738,8 +741,6 @@ __global__ void __launch_bounds__(256) k_dinput_act(Dims d, int slot, int T,
             b.x = fmaf(h, g[4], b.x); b.y = fmaf(h, g[5], b.y); b.z = fmaf(h, g[6], b.z); b.w = fmaf(h, g[7], b.w);
             *reinterpret_cast<float4*>(dp) = a;
             *reinterpret_cast<float4*>(dp + 4) = b;
-#pragma unroll
-            for (int e = 0; e < 8; ++e) dot[j] = fmaf(x[e], g[e], dot[j]);
         }
     }
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -757,14 +758,14 @@ __global__ void __launch_bounds__(256) k_dinput_act(Dims d, int slot, int T,
     }
 }
 
-cudaError_t launch_dinput_act(const Dims& d, int slot, int T, const uint16_t* d_input,
+cudaError_t launch_dinput_act(const Dims& d, int slot, int T, int add_dx, const uint16_t* d_input,
                               const uint16_t* xact, const float* hpre, const int* I, float* dxact,
                               float* dhpre, uint16_t* dinput_copy, cudaStream_t st) {
     if (d.k <= 4) {
-        k_dinput_act<4><<<T, chunk_threads(d.C), 0, st>>>(d, slot, T, d_input, xact, hpre, I, dxact,
+        k_dinput_act<4><<<T, chunk_threads(d.C), 0, st>>>(d, slot, T, add_dx, d_input, xact, hpre, I, dxact,
                                                            dhpre, dinput_copy); note_launch();
     } else {
-        k_dinput_act<8><<<T, chunk_threads(d.C), 0, st>>>(d, slot, T, d_input, xact, hpre, I, dxact,
+        k_dinput_act<8><<<T, chunk_threads(d.C), 0, st>>>(d, slot, T, add_dx, d_input, xact, hpre, I, dxact,
                                                            dhpre, dinput_copy); note_launch();
     }
     return cudaGetLastError();

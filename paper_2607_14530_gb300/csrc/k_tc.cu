@@ -560,6 +560,9 @@ constexpr int DX_THREADS = (2 + DX_EW) * 32;    // + TMA warp + MMA warp
 
 struct DxArgs {
     int T, C, N, k, G;
+    int slot;             // active epilogue: slot of the pre-map
+    int NH;               // active epilogue: streams of the H_pre rows
+    float* dxa;           // active epilogue: dX_act [T][k][C] fp32, updated in place
     int nkb, ksteps;      // k-blocks of 64, MMA k-steps of 16
     int TT, CT;           // token tiles, channel tiles per stream
     long long ntiles;
@@ -575,6 +578,10 @@ struct DxArgs {
     int* err;
 };
 
+// ACT = false: full-state dX epilogue (streams i of N, tiles of one stream).
+// ACT = true : active-state epilogue, "streams" are the k active slots j:
+//              dX_act[t][j][c] += acc + H_pre[t][slot][I_j] d_input[t][c].
+template <bool ACT>
 __global__ void __launch_bounds__(DX_THREADS, 1)
 k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, DxArgs a) {
     extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -677,11 +684,16 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
                 float h[4] = {0.f, 0.f, 0.f, 0.f};
                 float sa = 0.f, sb = 0.f;
                 if (t < a.T) {
-                    for (int q = 0; q < a.k; ++q)
-                        if (a.I[(long long)t * a.k + q] == i) j = q;
-                    for (int q = 0; q < a.G; ++q) h[q] = a.hpre[((long long)t * a.G + q) * a.N + i];
-                    sa = a.scal[(long long)t * a.scal_ld + 0];
-                    sb = a.scal[(long long)t * a.scal_ld + 1];
+                    if (ACT) {
+                        j = i;
+                        h[0] = a.hpre[((long long)t * a.G + a.slot) * a.NH + a.I[(long long)t * a.k + i]];
+                    } else {
+                        for (int q = 0; q < a.k; ++q)
+                            if (a.I[(long long)t * a.k + q] == i) j = q;
+                        for (int q = 0; q < a.G; ++q) h[q] = a.hpre[((long long)t * a.G + q) * a.N + i];
+                        sa = a.scal[(long long)t * a.scal_ld + 0];
+                        sb = a.scal[(long long)t * a.scal_ld + 1];
+                    }
                 }
                 float* m = meta + lane * 8;
                 m[0] = __int_as_float(j); m[1] = h[0]; m[2] = h[1]; m[3] = h[2]; m[4] = h[3];
@@ -709,6 +721,48 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
             // Every pass's reads are issued before any write.
             const int cq = (lane & 3) * 8;
             const int c = ct * DX_BN + cg * 32 + cq;
+            if (ACT) {
+                // dX_act[t][i][c..c+8) += acc + h din[t][c..c+8)   (i = active slot here)
+                float4 b0[4], b1[4];
+                uint4 gr[4];
+#pragma unroll
+                for (int pass = 0; pass < 4; ++pass) {
+                    const int rr = pass * 8 + (lane >> 2);
+                    const int t = tt * BM + quarter * 32 + rr;
+                    b0[pass] = make_float4(0.f, 0.f, 0.f, 0.f);
+                    b1[pass] = b0[pass];
+                    gr[pass] = make_uint4(0, 0, 0, 0);
+                    if (t >= a.T) continue;
+                    const float4* b = reinterpret_cast<const float4*>(a.dxa + ((long long)t * a.k + i) * a.C + c);
+                    b0[pass] = b[0];
+                    b1[pass] = b[1];
+                    gr[pass] = __ldg(reinterpret_cast<const uint4*>(a.dinput + (long long)t * a.C + c));
+                }
+#pragma unroll
+                for (int pass = 0; pass < 4; ++pass) {
+                    const int rr = pass * 8 + (lane >> 2);
+                    const int t = tt * BM + quarter * 32 + rr;
+                    if (t >= a.T) continue;
+                    const float hq = meta[rr * 8 + 1];
+                    float g[8];
+                    unpack8(gr[pass], g);
+                    const float* ac = tileb + rr * 33 + cq;
+                    float4 o0, o1;
+                    o0.x = b0[pass].x + ac[0] + hq * g[0];
+                    o0.y = b0[pass].y + ac[1] + hq * g[1];
+                    o0.z = b0[pass].z + ac[2] + hq * g[2];
+                    o0.w = b0[pass].w + ac[3] + hq * g[3];
+                    o1.x = b1[pass].x + ac[4] + hq * g[4];
+                    o1.y = b1[pass].y + ac[5] + hq * g[5];
+                    o1.z = b1[pass].z + ac[6] + hq * g[6];
+                    o1.w = b1[pass].w + ac[7] + hq * g[7];
+                    float4* dst = reinterpret_cast<float4*>(a.dxa + ((long long)t * a.k + i) * a.C + c);
+                    dst[0] = o0;
+                    dst[1] = o1;
+                }
+                __syncwarp();
+                continue;
+            }
             uint4 xr[4], br[4], br2[4];
 #pragma unroll
             for (int pass = 0; pass < 4; ++pass) {
@@ -778,10 +832,72 @@ __global__ void k_pack_rows(WSegs W, int n, int rows, int ld, uint16_t* __restri
     dst[idx] = __bfloat16_as_ushort(__float2bfloat16_rn(v));
 }
 
+// rows of three bf16 parts along K: A rows [hi | lo | hi] of dz, B rows [hi | hi | lo] of W, so
+// that sum_k A B = dz_hi W_hi + dz_lo W_hi + dz_hi W_lo (~2^-16 relative)
+__global__ void k_pack3(WSegs W, int n, int rows, int ld, int lo_part, uint16_t* __restrict__ dst) {
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)rows * ld) return;
+    const int r = (int)(idx / ld), col = (int)(idx - (long long)r * ld);
+    float v = 0.f;
+    if (col < 3 * n) {
+        const int part = col / n, o = col - part * n;
+        const int sg = seg_of(W, o);
+        const float w = W.ptr[sg][(long long)r * W.width[sg] + (o - W.off[sg])];
+        const float hi = __bfloat162float(__float2bfloat16_rn(w));
+        v = (part == lo_part) ? (w - hi) : hi;
+    }
+    dst[idx] = __bfloat16_as_ushort(__float2bfloat16_rn(v));
+}
+
 }  // namespace
 
+// two operand stages of up to two k-blocks each fit the 227 KB of shared memory
+bool dxa_tc_ok(int T, int k, int C, int nact) {
+    (void)k;
+    return T >= BM && C % DX_BN == 0 && 3 * nact <= 2 * BK;
+}
+
+cudaError_t launch_dxa_tc(const Dims& d, int slot, int T, const float* dzs, int nact, const WSegs& W,
+                          uint16_t* dz3, uint16_t* w3, const uint16_t* d_input, const float* hpre,
+                          const int* I, float* dxact, int* err, cudaStream_t st) {
+    const int KC = d.k * d.C;
+    const int K3 = 3 * nact;
+    const int ld = (K3 + 7) / 8 * 8;
+    WSegs dzsg;
+    memset(&dzsg, 0, sizeof(dzsg));
+    dzsg.ptr[0] = dzs; dzsg.width[0] = nact; dzsg.off[0] = 0; dzsg.off[1] = nact; dzsg.n = 1;
+    long long tot = (long long)T * ld;
+    k_pack3<<<(unsigned)((tot + 255) / 256), 256, 0, st>>>(dzsg, nact, T, ld, 1, dz3); note_launch();
+    tot = (long long)KC * ld;
+    k_pack3<<<(unsigned)((tot + 255) / 256), 256, 0, st>>>(W, nact, KC, ld, 2, w3); note_launch();
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    CUtensorMap ma, mb;
+    if (!make_map_box(&ma, dz3, (uint64_t)K3, (uint64_t)T, BK, BM, (uint64_t)ld * 2)) return cudaErrorInvalidValue;
+    if (!make_map_box(&mb, w3, (uint64_t)K3, (uint64_t)KC, BK, DX_BN, (uint64_t)ld * 2)) return cudaErrorInvalidValue;
+    DxArgs a;
+    memset(&a, 0, sizeof(a));
+    a.T = T; a.C = d.C; a.N = d.N; a.k = d.k; a.G = d.G; a.slot = slot;
+    a.nkb = (K3 + BK - 1) / BK;
+    a.ksteps = (K3 + 15) / 16;
+    a.TT = (T + BM - 1) / BM;
+    a.CT = d.C / DX_BN;
+    a.ntiles = (long long)a.TT * a.CT * d.k;
+    a.P = (int)std::min<long long>(num_sms(), a.ntiles);
+    a.N = d.k;  // tile "streams" are the active slots
+    a.NH = d.N;
+    a.dinput = d_input; a.hpre = hpre; a.I = I; a.dxa = dxact; a.err = err;
+    const size_t sm = 2 * (size_t)a.nkb * (BM + DX_BN) * BK * 2 + 128 +
+                      (size_t)DX_EW * (32 * 33 + 32 * 8) * 4 + 1024;
+    e = cudaFuncSetAttribute((const void*)k_dx_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+    k_dx_tc<true><<<a.P, DX_THREADS, sm, st>>>(ma, mb, a); note_launch();
+    return cudaGetLastError();
+}
+
 bool dx_tc_ok(int T, int N, int C, int nfull) {
-    return T >= BM && C % DX_BN == 0 && nfull <= 3 * BK;
+    (void)N;
+    return T >= BM && C % DX_BN == 0 && nfull <= 2 * BK;
 }
 
 cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, uint16_t* dz16,
@@ -803,6 +919,7 @@ cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, 
     if (!make_map_box(&ma, dz16, (uint64_t)n, (uint64_t)T, BK, BM, (uint64_t)ld * 2)) return cudaErrorInvalidValue;
     if (!make_map_box(&mb, w16, (uint64_t)n, (uint64_t)NC, BK, DX_BN, (uint64_t)ld * 2)) return cudaErrorInvalidValue;
     DxArgs a;
+    memset(&a, 0, sizeof(a));
     a.T = T; a.C = d.C; a.N = d.N; a.k = d.k; a.G = d.G;
     a.nkb = (n + BK - 1) / BK;
     a.ksteps = (n + 15) / 16;
@@ -814,9 +931,9 @@ cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, 
     a.scal = scal; a.scal_ld = scal_ld; a.err = err;
     const size_t sm = 2 * (size_t)a.nkb * (BM + DX_BN) * BK * 2 + 128 +
                       (size_t)DX_EW * (32 * 33 + 32 * 8) * 4 + 1024;
-    e = cudaFuncSetAttribute((const void*)k_dx_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    e = cudaFuncSetAttribute((const void*)k_dx_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
-    k_dx_tc<<<a.P, DX_THREADS, sm, st>>>(ma, mb, a); note_launch();
+    k_dx_tc<false><<<a.P, DX_THREADS, sm, st>>>(ma, mb, a); note_launch();
     return cudaGetLastError();
 }
 

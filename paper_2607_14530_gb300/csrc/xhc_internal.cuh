@@ -243,6 +243,11 @@ cudaError_t launch_wgrad_tc(const uint16_t* A, int T, int E, const float* dz, in
                             uint16_t* dzpack, const ProjTcPlan& p, float* part, int* err,
                             cudaStream_t st);
 bool dx_tc_ok(int T, int N, int C, int nfull);
+bool dxa_tc_ok(int T, int k, int C, int nact);
+// dX_act += dZ_act W_act^T (three-term bf16 split on the tensor cores) + H_pre[slot][I_j] d_input
+cudaError_t launch_dxa_tc(const Dims& d, int slot, int T, const float* dzs, int nact, const WSegs& W,
+                          uint16_t* dz3, uint16_t* w3, const uint16_t* d_input, const float* hpre,
+                          const int* I, float* dxact, int* err, cudaStream_t st);
 cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, uint16_t* dz16,
                          uint16_t* w16, const uint16_t* X, const uint16_t* dinput, const float* hpre,
                          const int* I, const float* dxact, const float* scal, int scal_ld,
@@ -312,7 +317,7 @@ cudaError_t launch_conv_wgrad_reduce(const Dims& d, int slot, const float* cpart
                                      ConvGradPtrs gconv, cudaStream_t st);
 cudaError_t launch_wgrad(const uint16_t* A, int64_t lda, int E, int T, const float* dz, int ldz,
                          int n, int tsplits, float* wpart, const WSegsOut& G, cudaStream_t st);
-cudaError_t launch_dinput_act(const Dims& d, int slot, int T, const uint16_t* d_input,
+cudaError_t launch_dinput_act(const Dims& d, int slot, int T, int add_dx, const uint16_t* d_input,
                               const uint16_t* xact, const float* hpre, const int* I,
                               float* dxact, float* dhpre, uint16_t* dinput_copy,
                               cudaStream_t st);
