@@ -128,10 +128,9 @@ Layout make_layout(const Dims& d, int64_t T) {
     Layout L;
     memset(&L, 0, sizeof(L));
     const size_t t = (size_t)T;
-    int nact_max = 0, Kmax = 1;
+    int nact_max = 0;
     for (int q = 0; q < d.G; ++q) {
         nact_max = std::max(nact_max, d.nact[q]);
-        Kmax = std::max(Kmax, d.K[q]);
     }
     size_t o = 0;
     L.xact = o; o = al(o + (size_t)d.G * t * d.k * d.C * 2);
@@ -146,6 +145,8 @@ Layout make_layout(const Dims& d, int64_t T) {
         L.hpost[q] = o; o = al(o + t * d.k * d.K[q] * 4);
     }
     L.hres = o; o = al(o + t * d.k * d.k * 4);
+    for (int q = 0; q < d.G; ++q)
+        if (d.K[q] > 1 && d.gs) { L.gram[q] = o; o = al(o + t * NGRAM * 8); }
     L.saved_total = o;
 
     const int rowblocks = (int)((T + 63) / 64);
@@ -190,7 +191,6 @@ Layout make_layout(const Dims& d, int64_t T) {
     L.dhpre = o; o = al(o + t * d.G * d.N * 4);
     L.tokmat = o; o = al(o + t * TOKMAT * 4);
     L.dz = o; o = al(o + t * std::max(d.nfull, nact_max) * 4);
-    L.du = o; o = al(o + (Kmax > 1 ? t * Kmax * d.C * 4 : 0));
     L.tokgrad = o; o = al(o + t * NTG * 4);
     L.wpart = o;
     {
@@ -556,7 +556,7 @@ xhc_status xhc_post_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
     XHC_K("wb_fwd", c.st, launch_wb_fwd(d, slot, c.T, out, cw, c.W<float>(c.L.red), c.L.nslice, c.xact(slot),
                                c.S<int>(c.L.I), c.S<float>(c.L.p), c.S<float>(c.L.hpost[slot]),
                                c.S<float>(c.L.hres), last ? nullptr : c.xact(slot + 1), X,
-                               c.W<int>(c.L.err), c.st));
+                               (d.K[slot] > 1 && d.gs) ? c.S<double>(c.L.gram[slot]) : nullptr, c.st));
     return XHC_OK;
 }
 
@@ -583,15 +583,19 @@ xhc_status xhc_post_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
         XHC_K("restore", c.st, launch_restore(d, T32, c.xact(0), c.S<int>(c.L.I), X, c.st));
     }
     XHC_K("wb_bred", c.st, launch_wb_bred(d, slot, T32, out, cw, dX, c.S<int>(c.L.I), dxact, c.xact(slot),
-                                          c.L.nslice, red, c.W<int>(c.L.err), c.st));
+                                          c.L.nslice, red, c.st));
     XHC_K("bwd_coef", c.st, launch_bwd_coef(d, slot, T32, red, c.L.nslice, c.S<float>(c.L.zact[slot]),
                              c.S<float>(c.L.rs[slot]), c.S<float>(c.L.p),
-                             c.S<float>(c.L.hpost[slot]), P->alpha_post, P->b_post[slot],
+                             c.S<float>(c.L.hpost[slot]),
+                             (d.K[slot] > 1 && d.gs) ? c.S<double>(c.L.gram[slot]) : nullptr,
+                             P->alpha_post, P->b_post[slot],
                              P->alpha_res, P->b_res, c.W<float>(c.L.tokmat), c.W<float>(c.L.dz),
                              c.W<float>(c.L.dp), c.W<float>(c.L.tokgrad), c.st));
-    XHC_K("wb_bapp", c.st, launch_wb_bapp(d, slot, T32, out, cw, dX, c.S<int>(c.L.I), c.xact(slot),
-                                          c.W<float>(c.L.tokmat), dxact, c.W<float>(c.L.du), d_out,
-                                          c.W<int>(c.L.err), c.st));
+    // d_out, conv weight-gradient partials and (last slot) the mixed active gradient; the
+    // active gradient of earlier slots is read in place and completed by pre_bwd(slot)
+    XHC_K("wb_bapp", c.st, launch_wb_bapp(d, slot, T32, out, cw, dX, c.S<int>(c.L.I), dxact,
+                                          c.W<float>(c.L.tokmat), dxact, d_out,
+                                          c.W<float>(c.L.cpart), c.st));
     const WSegs wa = act_segs(d, P, slot);
     // dZ_act stays in the workspace: pre_bwd(slot) applies it to dX_act on the tensor cores
     if (!dxa_tc_ok(T32, d.k, d.C, n))
@@ -618,8 +622,6 @@ xhc_status xhc_post_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
         XHC_K("colsum", c.st, launch_colsum(tg + d.k * K + 1 + d.k * d.k, T32, NTG, 1, g->alpha_res, 1, scr, c.st));
     }
     if (K > 1) {
-        XHC_K("wb_dout", c.st, launch_wb_dout(d, slot, T32, out, cw, c.W<float>(c.L.du), d_out,
-                                              c.W<float>(c.L.cpart), c.st));
         ConvGradPtrs gc;
         for (int j = 0; j < 3; ++j) gc.w[j] = (j < d.nconv) ? g->conv_w[slot][j] : nullptr;
         XHC_K("conv_wgrad_reduce", c.st, launch_conv_wgrad_reduce(d, slot, c.W<float>(c.L.cpart), c.L.ntiles, gc, c.st));
@@ -644,12 +646,13 @@ xhc_status xhc_pre_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
     const bool tc = dxa_tc_ok(T32, d.k, d.C, n);
     XHC_K("dinput_act", c.st, launch_dinput_act(d, slot, T32, tc ? 0 : 1, d_input, c.xact(slot),
                                c.S<float>(c.L.hpre), c.S<int>(c.L.I), c.W<float>(c.L.dxact),
-                               c.W<float>(c.L.dhpre), dinput, c.st));
+                               c.W<float>(c.L.dhpre), dinput, c.W<float>(c.L.tokmat), c.st));
     if (tc) {
         // post_bwd(slot) left dZ_act of this slot in the workspace
         XHC_K("dxa_tc", c.st, launch_dxa_tc(d, slot, T32, c.W<float>(c.L.dz), n, act_segs(d, P, slot),
                                             c.W<uint16_t>(c.L.dz16), c.W<uint16_t>(c.L.w16), d_input,
-                                            c.S<float>(c.L.hpre), c.S<int>(c.L.I), c.W<float>(c.L.dxact),
+                                            c.S<float>(c.L.hpre), c.S<int>(c.L.I), c.xact(slot),
+                                            c.W<float>(c.L.tokmat), c.W<float>(c.L.dxact),
                                             c.W<int>(c.L.err), c.st));
     }
     if (slot != 0) return XHC_OK;

@@ -297,6 +297,7 @@ template <int KM>
 __global__ void k_bwd_coef(Dims d, int slot, int T, const float* __restrict__ red, int nslice,
                            const float* __restrict__ zact, const float* __restrict__ rs,
                            const float* __restrict__ p, const float* __restrict__ hpost,
+                           const double* __restrict__ gram,
                            const float* __restrict__ alpha_post, const float* __restrict__ b_post,
                            const float* __restrict__ alpha_res, const float* __restrict__ b_res,
                            float* __restrict__ tokmat, float* __restrict__ dzs,
@@ -306,9 +307,9 @@ __global__ void k_bwd_coef(Dims d, int slot, int T, const float* __restrict__ re
     const int k = d.k, K = d.K[slot], n = d.nact[slot];
     const bool last = (slot == d.G - 1);
     const bool gs = (K > 1) && d.gs;
-    // reduction slots per token (see wb_bred): P at j*4 + a, Q at KM*4 + j*KM + i, Gram at
-    // KM*4 + KM*KM (lower triangle packed)
-    const int offQ = KM * 4, offG = KM * 4 + KM * KM;
+    // reduction slots per token (see wb_bred): P at j*4 + a, Q at KM*4 + j*KM + i; the Gram
+    // matrix of the components comes from the forward (lower triangle packed, fp64)
+    const int offQ = KM * 4;
     float Pm[KM][MAXCOMP], Q[KM][KM];
     double Gm[MAXCOMP][MAXCOMP];
 #pragma unroll
@@ -334,11 +335,11 @@ __global__ void k_bwd_coef(Dims d, int slot, int T, const float* __restrict__ re
                 for (int i = 0; i < KM; ++i)
                     if (j < k && i < k) Q[j][i] += rp[offQ + j * KM + i];
         }
-        if (gs) {
-            int q = 0;
-            for (int a = 0; a < K; ++a)
-                for (int b = 0; b <= a; ++b) Gm[a][b] += (double)rp[offG + q++];
-        }
+    }
+    if (gs) {
+        int q = 0;
+        for (int a = 0; a < K; ++a)
+            for (int b = 0; b <= a; ++b) Gm[a][b] = gram[(int64_t)t * NGRAM + q++];
     }
     for (int a = 0; a < K; ++a)
         for (int b = a + 1; b < K; ++b) Gm[a][b] = Gm[b][a];
@@ -432,16 +433,16 @@ __global__ void k_bwd_coef(Dims d, int slot, int T, const float* __restrict__ re
 
 cudaError_t launch_bwd_coef(const Dims& d, int slot, int T, const float* red, int nslice,
                             const float* zact, const float* rs, const float* p,
-                            const float* hpost, const float* alpha_post, const float* b_post,
-                            const float* alpha_res, const float* b_res, float* tokmat,
-                            float* dz, float* dp, float* tokgrad, cudaStream_t st) {
+                            const float* hpost, const double* gram, const float* alpha_post,
+                            const float* b_post, const float* alpha_res, const float* b_res,
+                            float* tokmat, float* dz, float* dp, float* tokgrad, cudaStream_t st) {
     (void)b_post;
     if (d.k <= 4) {
-        k_bwd_coef<4><<<(T + 63) / 64, 64, 0, st>>>(d, slot, T, red, nslice, zact, rs, p, hpost,
+        k_bwd_coef<4><<<(T + 63) / 64, 64, 0, st>>>(d, slot, T, red, nslice, zact, rs, p, hpost, gram,
                                                      alpha_post, b_post, alpha_res, b_res, tokmat,
                                                      dz, dp, tokgrad); note_launch();
     } else {
-        k_bwd_coef<8><<<(T + 63) / 64, 64, 0, st>>>(d, slot, T, red, nslice, zact, rs, p, hpost,
+        k_bwd_coef<8><<<(T + 63) / 64, 64, 0, st>>>(d, slot, T, red, nslice, zact, rs, p, hpost, gram,
                                                      alpha_post, b_post, alpha_res, b_res, tokmat,
                                                      dz, dp, tokgrad); note_launch();
     }

@@ -580,7 +580,8 @@ struct DxArgs {
 
 // ACT = false: full-state dX epilogue (streams i of N, tiles of one stream).
 // ACT = true : active-state epilogue, "streams" are the k active slots j:
-//              dX_act[t][j][c] += acc + H_pre[t][slot][I_j] d_input[t][c].
+//              dX_act[t][j][c] += acc + H_pre[t][slot][I_j] d_input[t][c] - cx_t x_act[t][j][c]
+//              (X = x_act of the slot, scal = the per-token matrices with cx at 112).
 template <bool ACT>
 __global__ void __launch_bounds__(DX_THREADS, 1)
 k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, DxArgs a) {
@@ -687,6 +688,7 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
                     if (ACT) {
                         j = i;
                         h[0] = a.hpre[((long long)t * a.G + a.slot) * a.NH + a.I[(long long)t * a.k + i]];
+                        h[1] = a.scal[(long long)t * a.scal_ld + 112];  // cx
                     } else {
                         for (int q = 0; q < a.k; ++q)
                             if (a.I[(long long)t * a.k + q] == i) j = q;
@@ -724,7 +726,7 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
             if (ACT) {
                 // dX_act[t][i][c..c+8) += acc + h din[t][c..c+8)   (i = active slot here)
                 float4 b0[4], b1[4];
-                uint4 gr[4];
+                uint4 gr[4], xr[4];
 #pragma unroll
                 for (int pass = 0; pass < 4; ++pass) {
                     const int rr = pass * 8 + (lane >> 2);
@@ -732,30 +734,34 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
                     b0[pass] = make_float4(0.f, 0.f, 0.f, 0.f);
                     b1[pass] = b0[pass];
                     gr[pass] = make_uint4(0, 0, 0, 0);
+                    xr[pass] = gr[pass];
                     if (t >= a.T) continue;
-                    const float4* b = reinterpret_cast<const float4*>(a.dxa + ((long long)t * a.k + i) * a.C + c);
+                    const long long row = ((long long)t * a.k + i) * a.C + c;
+                    const float4* b = reinterpret_cast<const float4*>(a.dxa + row);
                     b0[pass] = b[0];
                     b1[pass] = b[1];
                     gr[pass] = __ldg(reinterpret_cast<const uint4*>(a.dinput + (long long)t * a.C + c));
+                    xr[pass] = __ldg(reinterpret_cast<const uint4*>(a.X + row));
                 }
 #pragma unroll
                 for (int pass = 0; pass < 4; ++pass) {
                     const int rr = pass * 8 + (lane >> 2);
                     const int t = tt * BM + quarter * 32 + rr;
                     if (t >= a.T) continue;
-                    const float hq = meta[rr * 8 + 1];
-                    float g[8];
+                    const float hq = meta[rr * 8 + 1], cx = meta[rr * 8 + 2];
+                    float g[8], x[8];
                     unpack8(gr[pass], g);
+                    unpack8(xr[pass], x);
                     const float* ac = tileb + rr * 33 + cq;
                     float4 o0, o1;
-                    o0.x = b0[pass].x + ac[0] + hq * g[0];
-                    o0.y = b0[pass].y + ac[1] + hq * g[1];
-                    o0.z = b0[pass].z + ac[2] + hq * g[2];
-                    o0.w = b0[pass].w + ac[3] + hq * g[3];
-                    o1.x = b1[pass].x + ac[4] + hq * g[4];
-                    o1.y = b1[pass].y + ac[5] + hq * g[5];
-                    o1.z = b1[pass].z + ac[6] + hq * g[6];
-                    o1.w = b1[pass].w + ac[7] + hq * g[7];
+                    o0.x = b0[pass].x + ac[0] + (hq * g[0] - cx * x[0]);
+                    o0.y = b0[pass].y + ac[1] + (hq * g[1] - cx * x[1]);
+                    o0.z = b0[pass].z + ac[2] + (hq * g[2] - cx * x[2]);
+                    o0.w = b0[pass].w + ac[3] + (hq * g[3] - cx * x[3]);
+                    o1.x = b1[pass].x + ac[4] + (hq * g[4] - cx * x[4]);
+                    o1.y = b1[pass].y + ac[5] + (hq * g[5] - cx * x[5]);
+                    o1.z = b1[pass].z + ac[6] + (hq * g[6] - cx * x[6]);
+                    o1.w = b1[pass].w + ac[7] + (hq * g[7] - cx * x[7]);
                     float4* dst = reinterpret_cast<float4*>(a.dxa + ((long long)t * a.k + i) * a.C + c);
                     dst[0] = o0;
                     dst[1] = o1;
@@ -859,7 +865,8 @@ bool dxa_tc_ok(int T, int k, int C, int nact) {
 
 cudaError_t launch_dxa_tc(const Dims& d, int slot, int T, const float* dzs, int nact, const WSegs& W,
                           uint16_t* dz3, uint16_t* w3, const uint16_t* d_input, const float* hpre,
-                          const int* I, float* dxact, int* err, cudaStream_t st) {
+                          const int* I, const uint16_t* xact, const float* tokmat, float* dxact,
+                          int* err, cudaStream_t st) {
     const int KC = d.k * d.C;
     const int K3 = 3 * nact;
     const int ld = (K3 + 7) / 8 * 8;
@@ -887,6 +894,7 @@ cudaError_t launch_dxa_tc(const Dims& d, int slot, int T, const float* dzs, int 
     a.N = d.k;  // tile "streams" are the active slots
     a.NH = d.N;
     a.dinput = d_input; a.hpre = hpre; a.I = I; a.dxa = dxact; a.err = err;
+    a.X = xact; a.scal = tokmat; a.scal_ld = TOKMAT;
     const size_t sm = 2 * (size_t)a.nkb * (BM + DX_BN) * BK * 2 + 128 +
                       (size_t)DX_EW * (32 * 33 + 32 * 8) * 4 + 1024;
     e = cudaFuncSetAttribute((const void*)k_dx_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);

@@ -3,16 +3,19 @@
 // Every kernel here walks a run of consecutive tokens for one pair of channels per thread.  The
 // conv taps of the pair (zero past kappa_j) and a ring of the last KW values of `out` stay in
 // registers; the token loop is unrolled by KW so the ring positions are compile-time constants,
-// and each out value is loaded once per run instead of once per tap.  Per-token reductions over
-// the channels (Gram matrix, write-back gradients) use a reduce-scatter butterfly inside the warp
-// (about V shuffles for V values instead of 5 V), then shared memory across warps.
+// and each out value is loaded once per run instead of once per tap.  KS = 1 specialises the
+// tap counts to the (4, 8, 12) kernels of the MLP sublayers, so no FMA is spent on zero taps.
+// Per-token reductions over the channels (Gram matrix, write-back gradients) use a
+// reduce-scatter butterfly inside the warp (about V shuffles for V values instead of 5 V), then
+// shared memory across warps.
 //   wb_gram   Gram matrix of u = [out, g_1..g_r] (Eq. aug, Eq. gs), partial per channel slice
 //   wb_fwd    X_act_new = (H_res) X_act + p (H_post out_aug) (Eq. sparse_write_delta,
-//             Eq. sparse_write), scatter into X on the last slot
-//   wb_bred   backward reductions <dXn_j, u_a>, <dXn_j, x_i>, <u_a, u_b>
-//   wb_bapp   component gradients du_a and the active-state gradient
-//   wb_dout   d_out = du_0 + conv^T(du_1..r) (anti-causal, computed with a lag of KW - 1 tokens)
-//   wb_dw     conv weight-gradient partials sum_t du_{1+j}[t] out[t - i]
+//             Eq. sparse_write), scatter into X on the last slot; keeps the token's Gram matrix
+//             for the backward
+//   wb_bred   backward reductions <dXn_j, u_a> and, on the last slot, <dXn_j, x_i>
+//   wb_bapp   component gradients du_a consumed on the fly: d_out = du_0 + conv^T(du_1..r)
+//             (emitted KW - 1 tokens late), conv weight-gradient partials, and on the last slot
+//             the mixed active-state gradient H_res^T dXn
 #include "xhc_internal.cuh"
 
 namespace xhc {
@@ -96,7 +99,13 @@ __device__ __forceinline__ float2 u2f2(uint32_t u) {
     return make_float2(__uint_as_float(u << 16), __uint_as_float(u & 0xffff0000u));
 }
 
-template <int KW>
+// taps of component j held in registers: KS = 1 is the (4, 8, 12) kernel set, else KW each
+template <int KW, int KS>
+__host__ __device__ constexpr int ntap(int j) {
+    return KS == 1 ? (j == 0 ? 4 : (j == 1 ? 8 : 12)) : KW;
+}
+
+template <int KW, int KS>
 __device__ __forceinline__ void taps_reg(const Dims& d, const ConvPtrs& cw, int c, bool act,
                                          float2 (&tw)[3][KW]) {
 #pragma unroll
@@ -104,7 +113,7 @@ __device__ __forceinline__ void taps_reg(const Dims& d, const ConvPtrs& cw, int 
 #pragma unroll
         for (int i = 0; i < KW; ++i) {
             float2 v = f2z();
-            if (act && j < d.nconv && i < d.kap[j])
+            if (i < ntap<KW, KS>(j) && act && j < d.nconv && i < d.kap[j])
                 v = make_float2(cw.w[j][(size_t)i * d.C + c], cw.w[j][(size_t)i * d.C + c + 1]);
             tw[j][i] = v;
         }
@@ -123,7 +132,7 @@ __device__ __forceinline__ void ring_init(const uint16_t* out, int C, int c, boo
 }
 
 // g_j = sum_{i <= pos} tw[j][i] out[t - i], with out[t - i] at ring slot (U - i) mod KW
-template <int KW>
+template <int KW, int KS>
 __device__ __forceinline__ void conv_ring(const float2 (&tw)[3][KW], const float2 (&w)[KW], int U,
                                           int pos, float2 (&g)[3]) {
 #pragma unroll
@@ -134,6 +143,7 @@ __device__ __forceinline__ void conv_ring(const float2 (&tw)[3][KW], const float
             const float2 o = w[(U - i + KW) % KW];
 #pragma unroll
             for (int j = 0; j < 3; ++j) {
+                if (i >= ntap<KW, KS>(j)) continue;
                 g[j].x = fmaf(tw[j][i].x, o.x, g[j].x);
                 g[j].y = fmaf(tw[j][i].y, o.y, g[j].y);
             }
@@ -176,7 +186,7 @@ __device__ __forceinline__ void wred32(float (&v)[NB * 32], int lane, float (&to
 // ---------------------------------------------------------------------------------------------
 // wb_gram
 
-template <int KW>
+template <int KW, int KS>
 __global__ void __launch_bounds__(WT) k_wb_gram(Dims d, int slot, int T, int TB,
                                                 const uint16_t* __restrict__ out, ConvPtrs cw,
                                                 int nslice, float* __restrict__ red) {
@@ -190,7 +200,7 @@ __global__ void __launch_bounds__(WT) k_wb_gram(Dims d, int slot, int T, int TB,
     const int K = d.K[slot];
     const int nq = K * (K + 1) / 2;
     float2 tw[3][KW], w[KW];
-    taps_reg<KW>(d, cw, c, act, tw);
+    taps_reg<KW, KS>(d, cw, c, act, tw);
     ring_init<KW>(out, C, c, act, t0, w);
     for (long long tb = t0; tb < t1; tb += KW) {
 #pragma unroll
@@ -200,7 +210,7 @@ __global__ void __launch_bounds__(WT) k_wb_gram(Dims d, int slot, int T, int TB,
                 const float2 o = act ? ld2(out + t * C + c) : f2z();
                 w[u] = o;
                 float2 g[3];
-                conv_ring<KW>(tw, w, u, (int)(t % d.S), g);
+                conv_ring<KW, KS>(tw, w, u, (int)(t % d.S), g);
                 const float2 uu[4] = {o, g[0], g[1], g[2]};
                 float v[16];
                 int q = 0;
@@ -229,7 +239,8 @@ __global__ void __launch_bounds__(WT) k_wb_gram(Dims d, int slot, int T, int TB,
 // ---------------------------------------------------------------------------------------------
 // wb_fwd: per-token coefficients E[j][a] (Gram-Schmidt folded in), H_res, I in shared memory;
 // each thread prefetches the out value and the k active values of its channel pair 3 tokens
-// ahead with cp.async.
+// ahead with cp.async.  The CTAs of channel slice 0 also store the token's Gram matrix (fp64,
+// lower triangle) for the backward of Eq. gs.
 
 template <int KM>
 struct FRing {
@@ -237,7 +248,7 @@ struct FRing {
     uint32_t x[PD][KM][WT];
 };
 
-template <int KM, int KW>
+template <int KM, int KW, int KS>
 __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
                                                const uint16_t* __restrict__ out, ConvPtrs cw,
                                                const float* __restrict__ red, int nslice,
@@ -247,8 +258,8 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
                                                const float* __restrict__ hpost,
                                                const float* __restrict__ hres,
                                                uint16_t* __restrict__ xact_next,
-                                               uint16_t* __restrict__ X, int* __restrict__ err) {
-    (void)err;
+                                               uint16_t* __restrict__ X,
+                                               double* __restrict__ gram) {
     extern __shared__ __align__(16) unsigned char smu[];
     FRing<KM>& R = *reinterpret_cast<FRing<KM>*>(smu);
     const int k = d.k, K = d.K[slot], C = d.C;
@@ -289,6 +300,11 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
                 for (int a = 0; a < K; ++a)
                     for (int b = 0; b <= a; ++b) Gm[a][b] += (double)rp[q++];
             }
+            if (blockIdx.x == 0) {
+                int q = 0;
+                for (int a = 0; a < K; ++a)
+                    for (int b = 0; b <= a; ++b) gram[t * NGRAM + q++] = Gm[a][b];
+            }
             for (int a = 0; a < K; ++a)
                 for (int b = a + 1; b < K; ++b) Gm[a][b] = Gm[b][a];
             gs_coef(Gm, K, (double)d.eps_gs, B, cc, vv);
@@ -309,7 +325,7 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
     }
     float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
     if constexpr (KW > 0) {
-        taps_reg<KW>(d, cw, c, act, tw);
+        taps_reg<KW, KS>(d, cw, c, act, tw);
         ring_init<KW>(out, C, c, act, t0, w);
     }
     __syncthreads();
@@ -329,7 +345,7 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
                 if constexpr (KW > 0) {
                     w[u] = o;
                     float2 g[3];
-                    conv_ring<KW>(tw, w, u, (int)(t % d.S), g);
+                    conv_ring<KW, KS>(tw, w, u, (int)(t % d.S), g);
                     uu[1] = g[0];
                     uu[2] = g[1];
                     uu[3] = g[2];
@@ -396,7 +412,10 @@ __device__ __forceinline__ void bring_issue(BRing<KM>& R, int slot, long long t,
     cpa_commit();
 }
 
-template <int KM, int KW, int NB>
+// Per token, NV partial sums over this CTA's channel slice: P[j][a] = <dXn_j, u_a> at j*4 + a
+// and, on the last slot, Q[j][i] = <dXn_j, x_i> at KM*4 + j*KM + i.  NV = 16 is reduced to
+// lane pairs, larger NV in blocks of 32.
+template <int KM, int KW, int NV, int KS>
 __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
                                                 const uint16_t* __restrict__ out, ConvPtrs cw,
                                                 const uint16_t* __restrict__ dX,
@@ -404,16 +423,16 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
                                                 const float* __restrict__ dxact,
                                                 const uint16_t* __restrict__ xact, int nslice,
                                                 float* __restrict__ red) {
+    static_assert(NV == 16 || NV % 32 == 0, "reduction width");
+    constexpr int NVP = NV < 32 ? 16 : NV;      // values per token and warp in shared memory
     extern __shared__ __align__(16) unsigned char smu[];
     BRing<KM>& R = *reinterpret_cast<BRing<KM>*>(smu);
     int* Ish = reinterpret_cast<int*>(smu + sizeof(BRing<KM>));          // [TB][KM]
-    float* wsh = reinterpret_cast<float*>(Ish + TB * KM);                 // [TB][WT/32][NB*32]
+    float* wsh = reinterpret_cast<float*>(Ish + TB * KM);                 // [TB][WT/32][NVP]
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int slice = blockIdx.x, C = d.C, k = d.k;
-    const int K = d.K[slot];
     const bool last = (slot == d.G - 1);
-    const bool gs = (K > 1) && d.gs;
-    const int nv = KM * 4 + KM * KM + 10;
+    const int nv = last ? KM * 4 + KM * KM : KM * 4;
     const int c = slice * WSL + 2 * threadIdx.x;
     const bool act = c < C;
     const long long t0 = (long long)blockIdx.y * TB;
@@ -430,7 +449,7 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
                         Ish + q * KM, dxact);
     float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
     if constexpr (KW > 0) {
-        taps_reg<KW>(d, cw, c, act, tw);
+        taps_reg<KW, KS>(d, cw, c, act, tw);
         ring_init<KW>(out, C, c, act, t0, w);
     }
     const int RU = KW > 0 ? KW : 4;
@@ -460,7 +479,7 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
                     if constexpr (KW > 0) {
                         w[u] = o;
                         float2 g[3];
-                        conv_ring<KW>(tw, w, u, (int)(t % d.S), g);
+                        conv_ring<KW, KS>(tw, w, u, (int)(t % d.S), g);
                         uu[1] = g[0];
                         uu[2] = g[1];
                         uu[3] = g[2];
@@ -480,31 +499,32 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
                     w[u] = f2z();
                 }
                 // dn, x and the unused components are zero where a term does not apply
-                float v[NB * 32];
+                float v[NVP];
 #pragma unroll
-                for (int q = 0; q < NB * 32; ++q) v[q] = 0.f;
+                for (int q = 0; q < NVP; ++q) v[q] = 0.f;
 #pragma unroll
                 for (int j = 0; j < KM; ++j)
 #pragma unroll
-                    for (int a = 0; a < 4; ++a) v[j * 4 + a] = dot2(dn[j], uu[a]);
-                if (last) {
-#pragma unroll
-                    for (int j = 0; j < KM; ++j)
-#pragma unroll
-                        for (int i = 0; i < KM; ++i) v[KM * 4 + j * KM + i] = dot2(dn[j], x[i]);
-                }
-                if (gs) {
-                    int q = KM * 4 + KM * KM;
-#pragma unroll
                     for (int a = 0; a < 4; ++a)
+                        if (j * 4 + a < NVP) v[j * 4 + a] = dot2(dn[j], uu[a]);
+                if constexpr (NVP >= KM * 4 + KM * KM) {
+                    if (last) {
 #pragma unroll
-                        for (int bb = 0; bb <= a; ++bb) v[q++] = dot2(uu[a], uu[bb]);
+                        for (int j = 0; j < KM; ++j)
+#pragma unroll
+                            for (int i = 0; i < KM; ++i) v[KM * 4 + j * KM + i] = dot2(dn[j], x[i]);
+                    }
                 }
-                float tot[NB];
-                wred32<NB>(v, lane, tot);
-                float* dst = wsh + ((size_t)tt * (WT / 32) + warp) * (NB * 32);
+                float* dst = wsh + ((size_t)tt * (WT / 32) + warp) * NVP;
+                if constexpr (NV == 16) {
+                    const float tot = WRed<16, 16>::run(v, lane);
+                    if ((lane & 1) == 0) dst[lane >> 1] = tot;
+                } else {
+                    float tot[NV / 32];
+                    wred32<NV / 32>(v, lane, tot);
 #pragma unroll
-                for (int bb = 0; bb < NB; ++bb) dst[bb * 32 + lane] = tot[bb];
+                    for (int bb = 0; bb < NV / 32; ++bb) dst[bb * 32 + lane] = tot[bb];
+                }
             }
         }
     }
@@ -514,241 +534,216 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
         const int tt = idx / nv, q = idx - tt * nv;
         float sm = 0.f;
 #pragma unroll
-        for (int ww = 0; ww < WT / 32; ++ww) sm += wsh[((size_t)tt * (WT / 32) + ww) * (NB * 32) + q];
+        for (int ww = 0; ww < WT / 32; ++ww) sm += wsh[((size_t)tt * (WT / 32) + ww) * NVP + q];
         red[((t0 + tt) * nslice + slice) * NRED + q] = sm;
     }
 }
 
 // ---------------------------------------------------------------------------------------------
-// wb_bapp: du_a = sum_j E[j][a] dXn_j + sum_b D[a][b] u_b;  dX_act_i = (H_res^T dXn)_i - cx x_i
+// wb_bapp: du_a = sum_j E[j][a] dXn_j + sum_b D[a][b] u_b (Eq. sparse_write reversed, with the
+// Gram-Schmidt Jacobian in D), never stored:
+//   d_out[s] = du_0[s] + sum_j sum_{i < kappa_j, pos(s) + i < S} w_j[i] du_{1+j}[s + i]
+// (the transpose of the causal conv of Eq. aug) is accumulated in a ring of KW pending outputs
+// and emitted once token s + KW - 1 has been seen; each run therefore recomputes du for the first
+// KW - 1 tokens of the next run.  The conv weight gradient sum_t du_{1+j}[t] out[t - i] is
+// accumulated per run.  Last slot: dX_act_i = sum_j H_res[j][i] dXn_j.  The -cx x_i term of the
+// active-state gradient is added by the backward of the slot's pre-map.
 
-template <int KM, int KW>
-__global__ void __launch_bounds__(WT) k_wb_bapp(Dims d, int slot, int T, int TB,
-                                                const uint16_t* __restrict__ out, ConvPtrs cw,
-                                                const uint16_t* __restrict__ dX,
-                                                const int* __restrict__ I,
-                                                const uint16_t* __restrict__ xact,
-                                                const float* __restrict__ tokmat,
-                                                float* __restrict__ dxact,
-                                                float* __restrict__ du,
-                                                uint16_t* __restrict__ d_out) {
+template <int KM>
+struct ARing {
+    uint32_t o[PD][WT];
+    uint2 dn[PD][KM][WT];
+};
+
+template <int KM, int KW, int KS>
+__global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int TB,
+                                                   const uint16_t* __restrict__ out, ConvPtrs cw,
+                                                   const uint16_t* __restrict__ dX,
+                                                   const int* __restrict__ I,
+                                                   const float* dn_in,  // may alias dxact_out
+                                                   const float* __restrict__ tokmat,
+                                                   float* dxact_out,
+                                                   uint16_t* __restrict__ d_out,
+                                                   float* __restrict__ cpart) {
+    constexpr int HL = KW > 0 ? KW - 1 : 0;   // tokens of the next run whose du this run needs
+    constexpr int RU = KW > 0 ? KW : 4;
     extern __shared__ __align__(16) unsigned char smu[];
-    BRing<KM>& R = *reinterpret_cast<BRing<KM>*>(smu);
+    ARing<KM>& R = *reinterpret_cast<ARing<KM>*>(smu);
     const int k = d.k, K = d.K[slot], C = d.C;
     const bool last = (slot == d.G - 1);
-    float* Esh = reinterpret_cast<float*>(smu + sizeof(BRing<KM>));  // [TB][KM][4]
-    float* Dsh = Esh + TB * KM * 4;                                 // [TB][4][4]
-    float* Hsh = Dsh + TB * 16;                                     // [TB][KM][KM]
-    float* cxs = Hsh + TB * KM * KM;                                // [TB]
-    int* Ish = (int*)(cxs + TB);                                    // [TB][KM]
+    const int TH = TB + HL;
+    float* Esh = reinterpret_cast<float*>(smu + sizeof(ARing<KM>));  // [TH][KM][4]
+    float* Dsh = Esh + TH * KM * 4;                                 // [TH][4][4]
+    float* Hsh = Dsh + TH * 16;                                     // [TH][KM][KM]
+    int* Ish = reinterpret_cast<int*>(Hsh + TH * KM * KM);           // [TH][KM]
     const long long t0 = (long long)blockIdx.y * TB;
     const long long t1 = min((long long)T, t0 + TB);
-    const int ntok = (int)(t1 - t0);
+    const long long te = min((long long)T, t1 + HL);                // tokens with data
+    const long long tend = t1 + HL;                                 // loop end (emission lag)
+    const int ntok = (int)(te - t0);
     for (int idx = threadIdx.x; idx < ntok * 128; idx += WT) {
         const int tt = idx >> 7, q = idx & 127;
         const long long t = t0 + tt;
-        const float v = tokmat[t * TOKMAT + q];
         if (q < 32) {
-            const int j = q >> 2, a = q & 3;
-            if (j < KM) Esh[(tt * KM + j) * 4 + a] = v;
+            const int j = q >> 2;
+            if (j < KM) Esh[tt * KM * 4 + q] = tokmat[t * TOKMAT + q];
         } else if (q < 48) {
-            Dsh[tt * 16 + (q - 32)] = v;
+            Dsh[tt * 16 + (q - 32)] = tokmat[t * TOKMAT + q];
         } else if (q < 112) {
             const int a = (q - 48) >> 3, b = (q - 48) & 7;
-            if (a < KM && b < KM) Hsh[(tt * KM + a) * KM + b] = v;
-        } else if (q == 112) {
-            cxs[tt] = v;
+            if (a < KM && b < KM) Hsh[(tt * KM + a) * KM + b] = last ? tokmat[t * TOKMAT + q] : 0.f;
         } else if (q >= 120 && q < 120 + KM) {
-            Ish[tt * KM + (q - 120)] = (q - 120 < k) ? I[t * k + (q - 120)] : 0;
+            Ish[tt * KM + (q - 120)] = (last && q - 120 < k) ? I[t * k + (q - 120)] : 0;
         }
     }
     const int c = blockIdx.x * WSL + 2 * threadIdx.x;
     const bool act = c < C;
     __syncthreads();
+    auto issue = [&](int sl, int tn) {
+        if (act && tn < ntok) {
+            const long long t = t0 + tn;
+            cpa4(&R.o[sl][threadIdx.x], out + t * C + c);
 #pragma unroll
-    for (int q = 0; q < PD - 1; ++q)
-        bring_issue<KM>(R, q, t0 + q, act && q < ntok, k, d.N, C, c, last, true, out, xact, dX,
-                        Ish + q * KM, dxact);
-    float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
+            for (int j = 0; j < KM; ++j) {
+                if (j >= k) continue;
+                if (last)
+                    cpa4(&R.dn[sl][j][threadIdx.x], dX + (t * d.N + Ish[tn * KM + j]) * C + c);
+                else
+                    cpa8(&R.dn[sl][j][threadIdx.x], dn_in + (t * k + j) * C + c);
+            }
+        }
+        cpa_commit();
+    };
+#pragma unroll
+    for (int q = 0; q < PD - 1; ++q) issue(q, q);
+    float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1], pend[KW > 0 ? KW : 1];
+    float2 acc[3][KW > 0 ? KW : 1];
     if constexpr (KW > 0) {
-        taps_reg<KW>(d, cw, c, act, tw);
+        taps_reg<KW, KS>(d, cw, c, act, tw);
         ring_init<KW>(out, C, c, act, t0, w);
+#pragma unroll
+        for (int s = 0; s < KW; ++s) pend[s] = f2z();
+#pragma unroll
+        for (int j = 0; j < 3; ++j)
+#pragma unroll
+            for (int i = 0; i < KW; ++i) acc[j][i] = f2z();
     }
-    const int RU = KW > 0 ? KW : 4;
-    for (long long tb = t0; tb < t1; tb += RU) {
+    for (long long tb = t0; tb < tend; tb += RU) {
 #pragma unroll
         for (int u = 0; u < RU; ++u) {
             const long long t = tb + u;
-            if (t < t1) {
+            if (t < tend) {
                 const int tt = (int)(t - t0);
                 const int sl = u % PD;
-                {
-                    const int tn = tt + PD - 1;
-                    bring_issue<KM>(R, (u + PD - 1) % PD, t0 + tn, act && tn < ntok, k, d.N, C, c, last,
-                                    true, out, xact, dX, Ish + (tn < ntok ? tn : 0) * KM, dxact);
-                }
+                issue((u + PD - 1) % PD, tt + PD - 1);
                 cpa_wait<PD - 1>();
                 if (!act) continue;
-                const float2 o = u2f2(R.o[sl][threadIdx.x]);
-                float2 uu[4] = {o, f2z(), f2z(), f2z()};
-                if constexpr (KW > 0) {
-                    w[u] = o;
-                    float2 g[3];
-                    conv_ring<KW>(tw, w, u, (int)(t % d.S), g);
-                    uu[1] = g[0];
-                    uu[2] = g[1];
-                    uu[3] = g[2];
-                }
-                float2 dn[KM], x[KM];
+                const bool has = t < te;
+                const int pos = (int)(t % d.S);
+                float2 uu[4] = {f2z(), f2z(), f2z(), f2z()};
+                float2 du[4] = {f2z(), f2z(), f2z(), f2z()};
+                if (has) {
+                    uu[0] = u2f2(R.o[sl][threadIdx.x]);
+                    float2 dn[KM];
 #pragma unroll
-                for (int j = 0; j < KM; ++j) {
-                    if (j < k) {
-                        const uint2 r = R.dn[sl][j][threadIdx.x];
-                        dn[j] = last ? u2f2(r.x) : make_float2(__uint_as_float(r.x), __uint_as_float(r.y));
-                        x[j] = u2f2(R.x[sl][j][threadIdx.x]);
-                    } else {
+                    for (int j = 0; j < KM; ++j) {
                         dn[j] = f2z();
-                        x[j] = f2z();
+                        if (j < k) {
+                            const uint2 r = R.dn[sl][j][threadIdx.x];
+                            dn[j] = last ? u2f2(r.x) : make_float2(__uint_as_float(r.x), __uint_as_float(r.y));
+                        }
                     }
-                }
-#pragma unroll
-                for (int a = 0; a < 4; ++a) {
-                    if (a >= K) continue;
-                    float2 gsum = f2z();
-#pragma unroll
-                    for (int j = 0; j < KM; ++j) gsum = fma2(Esh[(tt * KM + j) * 4 + a], dn[j], gsum);
-#pragma unroll
-                    for (int b = 0; b < 4; ++b)
-                        if (b < K) gsum = fma2(Dsh[tt * 16 + a * 4 + b], uu[b], gsum);
-                    if (K == 1)
-                        st2(d_out + t * C + c, gsum);
-                    else
-                        *reinterpret_cast<float2*>(du + (t * K + a) * C + c) = gsum;
-                }
-                const float cx = cxs[tt];
-#pragma unroll
-                for (int i = 0; i < KM; ++i) {
-                    if (i >= k) continue;
-                    float2 v;
-                    if (last) {
-                        v = f2z();
-#pragma unroll
-                        for (int j = 0; j < KM; ++j) v = fma2(Hsh[(tt * KM + j) * KM + i], dn[j], v);
-                    } else {
-                        v = dn[i];
+                    if constexpr (KW > 0) {
+                        w[u] = uu[0];
+                        float2 g[3];
+                        conv_ring<KW, KS>(tw, w, u, pos, g);
+                        uu[1] = g[0];
+                        uu[2] = g[1];
+                        uu[3] = g[2];
                     }
-                    v = fma2(-cx, x[i], v);
-                    *reinterpret_cast<float2*>(dxact + (t * k + i) * C + c) = v;
+                    const float4* E4 = reinterpret_cast<const float4*>(Esh + tt * KM * 4);
+                    const float4* D4 = reinterpret_cast<const float4*>(Dsh + tt * 16);
+#pragma unroll
+                    for (int j = 0; j < KM; ++j) {
+                        if (j >= k) continue;
+                        const float4 e = E4[j];
+                        du[0] = fma2(e.x, dn[j], du[0]);
+                        du[1] = fma2(e.y, dn[j], du[1]);
+                        du[2] = fma2(e.z, dn[j], du[2]);
+                        du[3] = fma2(e.w, dn[j], du[3]);
+                    }
+                    if constexpr (KW > 0) {
+#pragma unroll
+                        for (int a = 0; a < 4; ++a) {
+                            const float4 m = D4[a];
+                            du[a] = fma2(m.x, uu[0], du[a]);
+                            du[a] = fma2(m.y, uu[1], du[a]);
+                            du[a] = fma2(m.z, uu[2], du[a]);
+                            du[a] = fma2(m.w, uu[3], du[a]);
+                        }
+                    }
+                    if (last && t < t1) {
+#pragma unroll
+                        for (int i = 0; i < KM; ++i) {
+                            if (i >= k) continue;
+                            float2 v = f2z();
+#pragma unroll
+                            for (int j = 0; j < KM; ++j) v = fma2(Hsh[(tt * KM + j) * KM + i], dn[j], v);
+                            *reinterpret_cast<float2*>(dxact_out + (t * k + i) * C + c) = v;
+                        }
+                    }
+                } else if constexpr (KW > 0) {
+                    w[u] = f2z();
+                }
+                if constexpr (KW == 0) {
+                    if (has) st2(d_out + t * C + c, du[0]);
+                } else {
+                    // conv weight gradient of this run's tokens
+                    if (t < t1) {
+#pragma unroll
+                        for (int j = 0; j < 3; ++j)
+#pragma unroll
+                            for (int i = 0; i < KW; ++i) {
+                                if (i >= ntap<KW, KS>(j) || i > pos) continue;
+                                const float2 o = w[(u - i + KW) % KW];
+                                acc[j][i].x = fmaf(du[1 + j].x, o.x, acc[j][i].x);
+                                acc[j][i].y = fmaf(du[1 + j].y, o.y, acc[j][i].y);
+                            }
+                    }
+                    // d_out[t - i] += w_j[i] du_{1+j}[t] for the pending outputs of this run
+                    pend[u] = du[0];
+#pragma unroll
+                    for (int i = 0; i < KW; ++i) {
+                        if (i > pos || i > tt) continue;
+#pragma unroll
+                        for (int j = 0; j < 3; ++j) {
+                            if (i >= ntap<KW, KS>(j)) continue;
+                            float2& q = pend[(u - i + KW) % KW];
+                            q.x = fmaf(tw[j][i].x, du[1 + j].x, q.x);
+                            q.y = fmaf(tw[j][i].y, du[1 + j].y, q.y);
+                        }
+                    }
+                    // token t - (KW - 1) has all its terms
+                    const long long s = t - (KW - 1);
+                    if (s >= t0 && s < t1) st2(d_out + s * C + c, pend[(u + 1) % KW]);
                 }
             }
         }
     }
     cpa_wait<0>();
-}
-
-// ---------------------------------------------------------------------------------------------
-// wb_dout: d_out[s] = du_0[s] + sum_j sum_{i, pos(s) + i < S} w_j[i] du_{1+j}[s + i].  Walks t
-// upwards keeping the last KW values of du_{1..3}; d_out[s] is emitted at t = s + KW - 1.
-
-template <int KW>
-__global__ void __launch_bounds__(WT) k_wb_dout(Dims d, int slot, int T, int TB,
-                                                ConvPtrs cw, const float* __restrict__ du,
-                                                uint16_t* __restrict__ d_out) {
-    const int K = d.K[slot], C = d.C;
-    const int c = blockIdx.x * WSL + 2 * threadIdx.x;
-    if (c >= C) return;
-    const long long t0 = (long long)blockIdx.y * TB;
-    const long long t1 = min((long long)T, t0 + TB);
-    float2 tw[3][KW];
-    taps_reg<KW>(d, cw, c, true, tw);
-    float2 r[3][KW];  // r[j][t mod KW] = du_{1+j}[t]
+    if constexpr (KW > 0) {
+        if (!act) return;
+        int off = 0;
 #pragma unroll
-    for (int j = 0; j < 3; ++j)
+        for (int j = 0; j < 3; ++j) {
+            if (j < d.nconv) {
 #pragma unroll
-        for (int s = 0; s < KW; ++s) r[j][s] = f2z();
-    // walk t over [t0, t1 + KW - 1); emit s = t - (KW - 1) when s >= t0
-    for (long long tb = t0; tb < t1 + KW - 1; tb += KW) {
-#pragma unroll
-        for (int u = 0; u < KW; ++u) {
-            const long long t = tb + u;
-            if (t < t1 + KW - 1) {
-#pragma unroll
-                for (int j = 0; j < 3; ++j)
-                    r[j][u] = (j < d.nconv && t < T) ? *reinterpret_cast<const float2*>(du + (t * K + 1 + j) * C + c)
-                                                     : f2z();
-                const long long s = t - (KW - 1);
-                if (s >= t0 && s < t1) {
-                    const int pos = (int)(s % d.S);
-                    float2 acc = *reinterpret_cast<const float2*>(du + (s * K) * C + c);
-#pragma unroll
-                    for (int i = 0; i < KW; ++i) {
-                        if (pos + i < d.S) {
-                            // du[s + i] sits at ring slot (s + i) mod KW = (u + 1 + i) mod KW
-#pragma unroll
-                            for (int j = 0; j < 3; ++j) {
-                                const float2 g = r[j][(u + 1 + i) % KW];
-                                acc.x = fmaf(tw[j][i].x, g.x, acc.x);
-                                acc.y = fmaf(tw[j][i].y, g.y, acc.y);
-                            }
-                        }
-                    }
-                    st2(d_out + s * C + c, acc);
-                }
+                for (int i = 0; i < KW; ++i)
+                    if (i < d.kap[j])
+                        *reinterpret_cast<float2*>(cpart + ((long long)blockIdx.y * d.kapsum + off + i) * C + c) =
+                            acc[j][i];
+                off += d.kap[j];
             }
-        }
-    }
-}
-
-// wb_dw: cpart[blockIdx.y][off_j + i][c] = sum_{t in run, pos(t) >= i} du_{1+j}[t] out[t - i]
-
-template <int KW>
-__global__ void __launch_bounds__(WT) k_wb_dw(Dims d, int slot, int T, int TB,
-                                              const uint16_t* __restrict__ out,
-                                              const float* __restrict__ du,
-                                              float* __restrict__ cpart) {
-    const int K = d.K[slot], C = d.C;
-    const int c = blockIdx.x * WSL + 2 * threadIdx.x;
-    if (c >= C) return;
-    const long long t0 = (long long)blockIdx.y * TB;
-    const long long t1 = min((long long)T, t0 + TB);
-    float2 w[KW], acc[3][KW];
-    ring_init<KW>(out, C, c, true, t0, w);
-#pragma unroll
-    for (int j = 0; j < 3; ++j)
-#pragma unroll
-        for (int i = 0; i < KW; ++i) acc[j][i] = f2z();
-    for (long long tb = t0; tb < t1; tb += KW) {
-#pragma unroll
-        for (int u = 0; u < KW; ++u) {
-            const long long t = tb + u;
-            if (t < t1) {
-                w[u] = ld2(out + t * C + c);
-                const int pos = (int)(t % d.S);
-#pragma unroll
-                for (int j = 0; j < 3; ++j) {
-                    if (j >= d.nconv) continue;
-                    const float2 g = *reinterpret_cast<const float2*>(du + (t * K + 1 + j) * C + c);
-#pragma unroll
-                    for (int i = 0; i < KW; ++i) {
-                        if (i <= pos) {
-                            const float2 o = w[(u - i + KW) % KW];
-                            acc[j][i].x = fmaf(g.x, o.x, acc[j][i].x);
-                            acc[j][i].y = fmaf(g.y, o.y, acc[j][i].y);
-                        }
-                    }
-                }
-            }
-        }
-    }
-    int off = 0;
-#pragma unroll
-    for (int j = 0; j < 3; ++j) {
-        if (j < d.nconv) {
-#pragma unroll
-            for (int i = 0; i < KW; ++i)
-                if (i < d.kap[j])
-                    *reinterpret_cast<float2*>(cpart + ((long long)blockIdx.y * d.kapsum + off + i) * C + c) = acc[j][i];
-            off += d.kap[j];
         }
     }
 }
@@ -756,6 +751,11 @@ __global__ void __launch_bounds__(WT) k_wb_dw(Dims d, int slot, int T, int TB,
 int kw_of(const Dims& d) {
     const int km = d.kapmax;
     return km <= 4 ? 4 : km <= 8 ? 8 : km <= 12 ? 12 : 16;
+}
+
+// the (4, 8, 12) kernels of the MLP sublayers
+bool paper_kaps(const Dims& d) {
+    return d.nconv == 3 && d.kap[0] == 4 && d.kap[1] == 8 && d.kap[2] == 12;
 }
 
 int run_len(int KW, int per) {  // tokens per CTA run: a multiple of KW near `per`
@@ -769,71 +769,59 @@ cudaError_t smem_attr(const void* fn, size_t bytes) {
     return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
 }
 
-template <int KW>
+template <int KW, int KS>
 cudaError_t gram_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, int nslice,
                     float* red, cudaStream_t st) {
     const int TB = run_len(KW, 64);
     const size_t sm = (size_t)TB * (WT / 32) * 16 * sizeof(float);
-    cudaError_t e = smem_attr((const void*)k_wb_gram<KW>, sm);
+    cudaError_t e = smem_attr((const void*)k_wb_gram<KW, KS>, sm);
     if (e != cudaSuccess) return e;
     dim3 grid(nslice, (T + TB - 1) / TB);
-    k_wb_gram<KW><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, nslice, red); note_launch();
+    k_wb_gram<KW, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, nslice, red); note_launch();
     return cudaGetLastError();
 }
 
-template <int KM, int KW>
+template <int KM, int KW, int KS>
 cudaError_t fwd_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, const float* red,
                    int nslice, const uint16_t* xact, const int* I, const float* p, const float* hpost,
-                   const float* hres, uint16_t* xact_next, uint16_t* X, int* err, cudaStream_t st) {
+                   const float* hres, uint16_t* xact_next, uint16_t* X, double* gram, cudaStream_t st) {
     const int TB = run_len(KW, 96);
     const size_t sm = sizeof(FRing<KM>) + (size_t)TB * (KM * 4 + KM * KM + KM) * 4;
-    cudaError_t e = smem_attr((const void*)k_wb_fwd<KM, KW>, sm);
+    cudaError_t e = smem_attr((const void*)k_wb_fwd<KM, KW, KS>, sm);
     if (e != cudaSuccess) return e;
     dim3 grid(nslice, (T + TB - 1) / TB);
-    k_wb_fwd<KM, KW><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, red, nslice, xact, I, p, hpost,
-                                           hres, xact_next, X, err); note_launch();
+    k_wb_fwd<KM, KW, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, red, nslice, xact, I, p, hpost,
+                                               hres, xact_next, X, gram); note_launch();
     return cudaGetLastError();
 }
 
-template <int KM, int KW, int NB>
+template <int KM, int KW, int NV, int KS>
 cudaError_t bred_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, const uint16_t* dX,
                     const int* I, const float* dxact, const uint16_t* xact, int nslice, float* red,
-                    int* err, cudaStream_t st) {
-    (void)err;
+                    cudaStream_t st) {
+    constexpr int NVP = NV < 32 ? 16 : NV;
     int TB = run_len(KW, 48);
-    while (TB > (KW > 0 ? KW : 4) && (size_t)TB * (WT / 32) * NB * 32 * 4 > 96 * 1024) TB -= (KW > 0 ? KW : 4);
-    const size_t sm = sizeof(BRing<KM>) + (size_t)TB * KM * 4 + (size_t)TB * (WT / 32) * NB * 32 * sizeof(float);
-    cudaError_t e = smem_attr((const void*)k_wb_bred<KM, KW, NB>, sm);
+    while (TB > (KW > 0 ? KW : 4) && (size_t)TB * (WT / 32) * NVP * 4 > 96 * 1024) TB -= (KW > 0 ? KW : 4);
+    const size_t sm = sizeof(BRing<KM>) + (size_t)TB * KM * 4 + (size_t)TB * (WT / 32) * NVP * sizeof(float);
+    cudaError_t e = smem_attr((const void*)k_wb_bred<KM, KW, NV, KS>, sm);
     if (e != cudaSuccess) return e;
     dim3 grid(nslice, (T + TB - 1) / TB);
-    k_wb_bred<KM, KW, NB><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, dX, I, dxact, xact, nslice, red); note_launch();
+    k_wb_bred<KM, KW, NV, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, dX, I, dxact, xact, nslice, red); note_launch();
     return cudaGetLastError();
 }
 
-template <int KM, int KW>
+template <int KM, int KW, int KS>
 cudaError_t bapp_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, const uint16_t* dX,
-                    const int* I, const uint16_t* xact, const float* tokmat, float* dxact, float* du,
-                    uint16_t* d_out, int nslice, int* err, cudaStream_t st) {
-    (void)err;
-    const int TB = run_len(KW, 64);
-    const size_t sm = sizeof(BRing<KM>) + (size_t)TB * (KM * 4 + 16 + KM * KM + 1 + KM) * 4;
-    cudaError_t e = smem_attr((const void*)k_wb_bapp<KM, KW>, sm);
+                    const int* I, const float* dn_in, const float* tokmat, float* dxact_out,
+                    uint16_t* d_out, float* cpart, int nslice, cudaStream_t st) {
+    const int TB = KW > 0 ? run_len(KW, 128) : 64;
+    const int TH = TB + (KW > 0 ? KW - 1 : 0);
+    const size_t sm = sizeof(ARing<KM>) + (size_t)TH * (KM * 4 + 16 + KM * KM + KM) * 4;
+    cudaError_t e = smem_attr((const void*)k_wb_bapp<KM, KW, KS>, sm);
     if (e != cudaSuccess) return e;
     dim3 grid(nslice, (T + TB - 1) / TB);
-    k_wb_bapp<KM, KW><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, dX, I, xact, tokmat, dxact, du, d_out); note_launch();
-    return cudaGetLastError();
-}
-
-template <int KW>
-cudaError_t dout_kw(const Dims& d, int slot, int T, ConvPtrs cw, const float* du, uint16_t* d_out,
-                    float* cpart, const uint16_t* out, int nslice, int TBW, cudaStream_t st) {
-    const int TB = run_len(KW, 64);
-    dim3 grid(nslice, (T + TB - 1) / TB);
-    k_wb_dout<KW><<<grid, WT, 0, st>>>(d, slot, T, TB, cw, du, d_out); note_launch();
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    dim3 g2(nslice, (T + TBW - 1) / TBW);
-    k_wb_dw<KW><<<g2, WT, 0, st>>>(d, slot, T, TBW, out, du, cpart); note_launch();
+    k_wb_bapp<KM, KW, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, dX, I, dn_in, tokmat, dxact_out,
+                                                d_out, cpart); note_launch();
     return cudaGetLastError();
 }
 
@@ -842,63 +830,66 @@ cudaError_t dout_kw(const Dims& d, int slot, int T, ConvPtrs cw, const float* du
 int wb_nslice(int C) { return (C + WSL - 1) / WSL; }
 int wb_dw_run(const Dims& d) { return run_len(kw_of(d), 128); }
 
-#define XHC_KW_DISPATCH(KWV, CALL)                         \
-    switch (KWV) {                                         \
-        case 4: { constexpr int KWC = 4; return CALL; }    \
-        case 8: { constexpr int KWC = 8; return CALL; }    \
-        case 12: { constexpr int KWC = 12; return CALL; }  \
-        default: { constexpr int KWC = 16; return CALL; }  \
+// KWC: conv taps held per component (0: no conv); KSC: 1 for the (4, 8, 12) kernel set
+#define XHC_KW_DISPATCH(D, CALL)                                              \
+    switch (kw_of(D)) {                                                       \
+        case 4: { constexpr int KWC = 4, KSC = 0; return CALL; }              \
+        case 8: { constexpr int KWC = 8, KSC = 0; return CALL; }              \
+        case 12:                                                              \
+            if (paper_kaps(D)) { constexpr int KWC = 12, KSC = 1; return CALL; } \
+            else { constexpr int KWC = 12, KSC = 0; return CALL; }            \
+        default: { constexpr int KWC = 16, KSC = 0; return CALL; }            \
     }
 
 cudaError_t launch_wb_gram(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
                            int nslice, float* red, cudaStream_t st) {
-    XHC_KW_DISPATCH(kw_of(d), (gram_kw<KWC>(d, slot, T, out, cw, nslice, red, st)));
+    XHC_KW_DISPATCH(d, (gram_kw<KWC, KSC>(d, slot, T, out, cw, nslice, red, st)));
 }
 
 cudaError_t launch_wb_fwd(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
                           const float* red, int nslice, const uint16_t* xact, const int* I,
                           const float* p, const float* hpost, const float* hres,
-                          uint16_t* xact_next, uint16_t* X, int* err, cudaStream_t st) {
+                          uint16_t* xact_next, uint16_t* X, double* gram, cudaStream_t st) {
     const bool conv = d.K[slot] > 1;
     if (d.k <= 4) {
-        if (!conv) return fwd_kw<4, 0>(d, slot, T, out, cw, red, nslice, xact, I, p, hpost, hres, xact_next, X, err, st);
-        XHC_KW_DISPATCH(kw_of(d), (fwd_kw<4, KWC>(d, slot, T, out, cw, red, nslice, xact, I, p, hpost, hres, xact_next, X, err, st)));
+        if (!conv) return fwd_kw<4, 0, 0>(d, slot, T, out, cw, red, nslice, xact, I, p, hpost, hres, xact_next, X, gram, st);
+        XHC_KW_DISPATCH(d, (fwd_kw<4, KWC, KSC>(d, slot, T, out, cw, red, nslice, xact, I, p, hpost, hres, xact_next, X, gram, st)));
     }
-    if (!conv) return fwd_kw<8, 0>(d, slot, T, out, cw, red, nslice, xact, I, p, hpost, hres, xact_next, X, err, st);
-    XHC_KW_DISPATCH(kw_of(d), (fwd_kw<8, KWC>(d, slot, T, out, cw, red, nslice, xact, I, p, hpost, hres, xact_next, X, err, st)));
+    if (!conv) return fwd_kw<8, 0, 0>(d, slot, T, out, cw, red, nslice, xact, I, p, hpost, hres, xact_next, X, gram, st);
+    XHC_KW_DISPATCH(d, (fwd_kw<8, KWC, KSC>(d, slot, T, out, cw, red, nslice, xact, I, p, hpost, hres, xact_next, X, gram, st)));
 }
 
 cudaError_t launch_wb_bred(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
                            const uint16_t* dX, const int* I, const float* dxact,
-                           const uint16_t* xact, int nslice, float* red, int* err, cudaStream_t st) {
+                           const uint16_t* xact, int nslice, float* red, cudaStream_t st) {
     const bool conv = d.K[slot] > 1;
+    const bool last = (slot == d.G - 1);
+#define XHC_BRED(KM_, NV_)                                                                          \
+    do {                                                                                            \
+        if (!conv) return bred_kw<KM_, 0, NV_, 0>(d, slot, T, out, cw, dX, I, dxact, xact, nslice, red, st); \
+        XHC_KW_DISPATCH(d, (bred_kw<KM_, KWC, NV_, KSC>(d, slot, T, out, cw, dX, I, dxact, xact, nslice, red, st))); \
+    } while (0)
     if (d.k <= 4) {
-        if (!conv) return bred_kw<4, 0, 2>(d, slot, T, out, cw, dX, I, dxact, xact, nslice, red, err, st);
-        XHC_KW_DISPATCH(kw_of(d), (bred_kw<4, KWC, 2>(d, slot, T, out, cw, dX, I, dxact, xact, nslice, red, err, st)));
+        if (last) XHC_BRED(4, 32);
+        XHC_BRED(4, 16);
     }
-    if (!conv) return bred_kw<8, 0, 4>(d, slot, T, out, cw, dX, I, dxact, xact, nslice, red, err, st);
-    XHC_KW_DISPATCH(kw_of(d), (bred_kw<8, KWC, 4>(d, slot, T, out, cw, dX, I, dxact, xact, nslice, red, err, st)));
+    if (last) XHC_BRED(8, 96);
+    XHC_BRED(8, 32);
+#undef XHC_BRED
 }
 
 cudaError_t launch_wb_bapp(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
-                           const uint16_t* dX, const int* I, const uint16_t* xact,
-                           const float* tokmat, float* dxact, float* du, uint16_t* d_out,
-                           int* err, cudaStream_t st) {
+                           const uint16_t* dX, const int* I, const float* dn_in,
+                           const float* tokmat, float* dxact_out, uint16_t* d_out, float* cpart,
+                           cudaStream_t st) {
     const int nslice = wb_nslice(d.C);
     const bool conv = d.K[slot] > 1;
     if (d.k <= 4) {
-        if (!conv) return bapp_kw<4, 0>(d, slot, T, out, cw, dX, I, xact, tokmat, dxact, du, d_out, nslice, err, st);
-        XHC_KW_DISPATCH(kw_of(d), (bapp_kw<4, KWC>(d, slot, T, out, cw, dX, I, xact, tokmat, dxact, du, d_out, nslice, err, st)));
+        if (!conv) return bapp_kw<4, 0, 0>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st);
+        XHC_KW_DISPATCH(d, (bapp_kw<4, KWC, KSC>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st)));
     }
-    if (!conv) return bapp_kw<8, 0>(d, slot, T, out, cw, dX, I, xact, tokmat, dxact, du, d_out, nslice, err, st);
-    XHC_KW_DISPATCH(kw_of(d), (bapp_kw<8, KWC>(d, slot, T, out, cw, dX, I, xact, tokmat, dxact, du, d_out, nslice, err, st)));
-}
-
-cudaError_t launch_wb_dout(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
-                           const float* du, uint16_t* d_out, float* cpart, cudaStream_t st) {
-    const int nslice = wb_nslice(d.C);
-    const int TBW = wb_dw_run(d);
-    XHC_KW_DISPATCH(kw_of(d), (dout_kw<KWC>(d, slot, T, cw, du, d_out, cpart, out, nslice, TBW, st)));
+    if (!conv) return bapp_kw<8, 0, 0>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st);
+    XHC_KW_DISPATCH(d, (bapp_kw<8, KWC, KSC>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st)));
 }
 
 }  // namespace xhc

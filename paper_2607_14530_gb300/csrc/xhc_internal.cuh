@@ -74,6 +74,8 @@ struct Layout {
     size_t rs[4];           // f32 [T]: active rstd
     size_t hpost[4];        // f32 [T][k*K_t]
     size_t hres;            // f32 [T][k*k]
+    size_t gram[4];         // f64 [T][NGRAM]: Gram matrix of the write-back components (lower
+                            // triangle), slots with a temporal conv and Gram-Schmidt
     size_t saved_total;
     // workspace
     size_t err;             // int: device error word (first 256 bytes of the workspace)
@@ -90,7 +92,6 @@ struct Layout {
     size_t dhpre;           // f32 [T][G][N]
     size_t tokmat;          // f32 [T][TOKMAT]: per-token matrices (E, D, H_res, scalars)
     size_t dz;              // f32 [T][max(nfull, nact)]: projection-output gradients
-    size_t du;              // f32 [T][K][C]: gradients of the write-back components
     size_t tokgrad;         // f32 [T][NTG]: per-token alpha / b gradient contributions
     size_t wpart;           // f32 [tsplits][rows * n]: weight-gradient partials
     size_t cpart;           // f32 [ntiles][kapsum][C]: conv weight-gradient partials
@@ -106,6 +107,7 @@ struct Layout {
     size_t w16;             // bf16 [N*C][ld]: full-state projection weight rows
 };
 
+constexpr int NGRAM = 10;    // lower triangle of the 4 x 4 component Gram matrix
 constexpr int NRED = 112;    // per-token reduction slots (>= k*K + k*k + K*K)
 constexpr int TOKMAT = 176;  // E[k][4] + D[4][4] + Hres[k][k] + dX_act mix + scalars (k<=8)
 constexpr int NTG = 208;     // per-token alpha/b gradient contributions
@@ -245,9 +247,11 @@ cudaError_t launch_wgrad_tc(const uint16_t* A, int T, int E, const float* dz, in
 bool dx_tc_ok(int T, int N, int C, int nfull);
 bool dxa_tc_ok(int T, int k, int C, int nact);
 // dX_act += dZ_act W_act^T (three-term bf16 split on the tensor cores) + H_pre[slot][I_j] d_input
+//           - cx x_act (the write-back's own term, cx per token in tokmat)
 cudaError_t launch_dxa_tc(const Dims& d, int slot, int T, const float* dzs, int nact, const WSegs& W,
                           uint16_t* dz3, uint16_t* w3, const uint16_t* d_input, const float* hpre,
-                          const int* I, float* dxact, int* err, cudaStream_t st);
+                          const int* I, const uint16_t* xact, const float* tokmat, float* dxact,
+                          int* err, cudaStream_t st);
 cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, uint16_t* dz16,
                          uint16_t* w16, const uint16_t* X, const uint16_t* dinput, const float* hpre,
                          const int* I, const float* dxact, const float* scal, int scal_ld,
@@ -259,16 +263,14 @@ cudaError_t launch_wb_gram(const Dims& d, int slot, int T, const uint16_t* out, 
 cudaError_t launch_wb_fwd(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
                           const float* red, int nslice, const uint16_t* xact, const int* I,
                           const float* p, const float* hpost, const float* hres,
-                          uint16_t* xact_next, uint16_t* X, int* err, cudaStream_t st);
+                          uint16_t* xact_next, uint16_t* X, double* gram, cudaStream_t st);
 cudaError_t launch_wb_bred(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
                            const uint16_t* dX, const int* I, const float* dxact,
-                           const uint16_t* xact, int nslice, float* red, int* err, cudaStream_t st);
+                           const uint16_t* xact, int nslice, float* red, cudaStream_t st);
 cudaError_t launch_wb_bapp(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
-                           const uint16_t* dX, const int* I, const uint16_t* xact,
-                           const float* tokmat, float* dxact, float* du, uint16_t* d_out,
-                           int* err, cudaStream_t st);
-cudaError_t launch_wb_dout(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
-                           const float* du, uint16_t* d_out, float* cpart, cudaStream_t st);
+                           const uint16_t* dX, const int* I, const float* dn_in,
+                           const float* tokmat, float* dxact_out, uint16_t* d_out, float* cpart,
+                           cudaStream_t st);
 cudaError_t launch_wgrad_reduce(const float* wpart, int splits, int E, int n, const WSegsOut& G,
                                 cudaStream_t st);
 cudaError_t launch_colsum(const float* in, int rows, int ld, int n, float* out, int accumulate,
@@ -286,33 +288,15 @@ cudaError_t launch_read(const Dims& d, int T, const uint16_t* X, const float* hp
                         uint16_t* input0, float* base, uint16_t* xact0, cudaStream_t st);
 cudaError_t launch_input(const Dims& d, int slot, int T, const float* base, const uint16_t* xact,
                          const float* hpre, const int* I, uint16_t* input, cudaStream_t st);
-cudaError_t launch_aug_gram(const Dims& d, int slot, int T, const uint16_t* out,
-                            ConvPtrs convw, int nslice, float* red, cudaStream_t st);
-cudaError_t launch_post_apply(const Dims& d, int slot, int T, const uint16_t* out,
-                              ConvPtrs convw, const float* red, int nslice,
-                              const uint16_t* xact, const int* I, const float* p,
-                              const float* hpost, const float* hres, uint16_t* xact_next,
-                              uint16_t* X, cudaStream_t st);
 cudaError_t launch_restore(const Dims& d, int T, const uint16_t* xact0, const int* I,
                            uint16_t* X, cudaStream_t st);
-cudaError_t launch_bwd_reduce(const Dims& d, int slot, int T, const uint16_t* out,
-                              ConvPtrs convw, const uint16_t* dX, const int* I,
-                              const float* dxact, const uint16_t* xact, int nslice, float* red,
-                              cudaStream_t st);
 cudaError_t launch_bwd_coef(const Dims& d, int slot, int T, const float* red, int nslice,
                             const float* zact, const float* rs, const float* p,
-                            const float* hpost, const float* alpha_post, const float* b_post,
-                            const float* alpha_res, const float* b_res, float* tokmat,
-                            float* dz, float* dp, float* tokgrad, cudaStream_t st);
-cudaError_t launch_bwd_apply(const Dims& d, int slot, int T, const uint16_t* out,
-                             ConvPtrs convw, const uint16_t* dX, const int* I,
-                             const uint16_t* xact, const float* tokmat, float* dxact, float* du,
-                             uint16_t* d_out, cudaStream_t st);
+                            const float* hpost, const double* gram, const float* alpha_post,
+                            const float* b_post, const float* alpha_res, const float* b_res,
+                            float* tokmat, float* dz, float* dp, float* tokgrad, cudaStream_t st);
 cudaError_t launch_gemm_dzw(const Dims& d, int T, const float* dz, int ldz, int n,
                             const WSegs& W, int E, float* dxact, cudaStream_t st);
-cudaError_t launch_bwd_conv(const Dims& d, int slot, int T, const uint16_t* out,
-                            ConvPtrs convw, const float* du, uint16_t* d_out,
-                            float* cpart, int ntiles, cudaStream_t st);
 cudaError_t launch_conv_wgrad_reduce(const Dims& d, int slot, const float* cpart, int ntiles,
                                      ConvGradPtrs gconv, cudaStream_t st);
 cudaError_t launch_wgrad(const uint16_t* A, int64_t lda, int E, int T, const float* dz, int ldz,
@@ -320,7 +304,7 @@ cudaError_t launch_wgrad(const uint16_t* A, int64_t lda, int E, int T, const flo
 cudaError_t launch_dinput_act(const Dims& d, int slot, int T, int add_dx, const uint16_t* d_input,
                               const uint16_t* xact, const float* hpre, const int* I,
                               float* dxact, float* dhpre, uint16_t* dinput_copy,
-                              cudaStream_t st);
+                              const float* tokmat, cudaStream_t st);
 cudaError_t launch_full_dots(const Dims& d, int T, const uint16_t* X, const uint16_t* dinput,
                              const int* I, const float* hpre, uint16_t* dX, float* dhpre,
                              cudaStream_t st);
