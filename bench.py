@@ -72,7 +72,12 @@ def kernel_model(cfg, T):
 
     X = T * N * C * b16
     xa = T * k * C * b16
+    xa32 = T * k * C * f32
     row = T * C * b16
+    kw = max(cfg.conv_k) if cfg.conv_k else 0
+    kw = 0 if kw == 0 else (4 if kw <= 4 else 8 if kw <= 8 else 12 if kw <= 12 else 16)
+    runs = -(-T // max(kw, (128 // kw) * kw if kw else 128)) if kw else 0
+    cpart = runs * sum(cfg.conv_k) * C * f32
     # forward
     if hr:
         add("colsum", N * C * N * f32)
@@ -89,34 +94,36 @@ def kernel_model(cfg, T):
         add("proj_tc_active", xa + T * nact[t] * f32, 2.0 * T * k * C * 2 * nact[t], "hbm")
         add("coef_act", T * nact[t] * f32 * 2)
         if Ks[t] > 1 and gs:
-            add("aug_gram", row)
-        add("post_apply", xa + row + xa)
+            add("wb_gram", row)
+        add("wb_fwd", row + xa + xa)
     # backward
     for t in reversed(range(G)):
         last = t == G - 1
-        dxn = xa if last else T * k * C * f32
+        dxn = xa if last else xa32
         if last:
             add("restore", 2 * xa)
-        add("bwd_reduce", dxn + (xa if last else 0) + row)
+        add("wb_bred", row + dxn + (xa if last else 0))
         add("bwd_coef", T * nact[t] * f32 * 2)
-        add("bwd_apply", dxn + xa + row + T * k * C * f32 + (T * Ks[t] * C * f32 if Ks[t] > 1 else row))
-        add("gemm_dzw", T * nact[t] * f32 + 2 * T * k * C * f32, 2.0 * T * k * C * nact[t], "alu")
+        # out, dXn read; d_out written; last slot writes the mixed active gradient; conv partials
+        add("wb_bapp", row + dxn + row + (xa32 if last else 0) + (cpart if Ks[t] > 1 else 0))
         add("wgrad_tc_active", xa + T * nact[t] * f32 + 2 * T * nact[t] * b16 + k * C * nact[t] * f32,
             2.0 * T * k * C * 2 * nact[t], "hbm")
         add("wgrad_reduce", 2 * k * C * nact[t] * f32)
         for _ in range(4 if last else 2):
             add("colsum", T * 16 * f32)
         if Ks[t] > 1:
-            add("bwd_conv", T * Ks[t] * C * f32 + 2 * row)
-            add("conv_wgrad_reduce", sum(cfg.conv_k) * C * f32 * 2)
-        add("dinput_act", row + xa + 2 * T * k * C * f32 + row)
+            add("conv_wgrad_reduce", cpart)
+        # pre-map backward of the slot: dH_pre dots and the d_input copy, then the active-state
+        # gradient update dX_act += dZ W^T + H_pre d_input - cx x_act on the tensor cores
+        add("dinput_act", row + xa + row)
+        add("dxa_tc", 2 * xa32 + xa + row + 3 * T * nact[t] * b16, 2.0 * T * k * C * 3 * nact[t], "hbm")
     if hr:
         add("colsum", N * C * N * f32)
-    add("full_dots", T * (N - k) * C * b16 + G * row)
+    # dH_pre of the inactive streams and their dense-read gradient (dX rows read and written)
+    add("full_dots", 3 * T * (N - k) * C * b16 + G * row)
     add("full_coef", T * (nfull + G * N) * f32)
-    # tensor-core dX: X read, inactive dX rows read, active-row gradient read, d_input (once per
-    # token block), dX written
-    add("dx_tc", X + T * (N - k) * C * b16 + T * k * C * f32 + G * row + X, 2.0 * T * N * C * nfull, "hbm")
+    # tensor-core dX: X read, inactive dX rows read, active-row gradient read, dX written
+    add("dx_tc", X + T * (N - k) * C * b16 + xa32 + X, 2.0 * T * N * C * nfull, "hbm")
     add("wgrad_tc_full", X + T * nfull * f32 + 2 * T * nfull * b16 + N * C * nfull * f32,
         2.0 * T * N * C * 2 * nfull, "hbm")
     add("wgrad_reduce", 2 * N * C * nfull * f32)
@@ -417,7 +424,9 @@ def run_xhc(args, wl_name):
 
     if args.kernels_out and rank == 0:
         with open(args.kernels_out, "w") as f:
-            json.dump({"workload": wl_name, "kernels": kernels, "model": model}, f, indent=1)
+            seq = [[n, t_ms] for n, t_ms in recs[:len(recs) // max(1, args.steps)]]
+            json.dump({"workload": wl_name, "kernels": kernels, "model": model, "sequence": seq}, f,
+                      indent=1)
 
     # end to end through the public API with host buffers: H2D of the step's inputs from pinned
     # memory, the step, D2H of its results

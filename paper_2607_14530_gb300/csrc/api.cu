@@ -553,10 +553,13 @@ xhc_status xhc_post_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
     if (d.K[slot] > 1 && d.gs)
         XHC_K("wb_gram", c.st, launch_wb_gram(d, slot, c.T, out, cw, c.L.nslice, c.W<float>(c.L.red), c.st));
     const bool last = (slot == d.G - 1);
-    XHC_K("wb_fwd", c.st, launch_wb_fwd(d, slot, c.T, out, cw, c.W<float>(c.L.red), c.L.nslice, c.xact(slot),
-                               c.S<int>(c.L.I), c.S<float>(c.L.p), c.S<float>(c.L.hpost[slot]),
-                               c.S<float>(c.L.hres), last ? nullptr : c.xact(slot + 1), X,
-                               (d.K[slot] > 1 && d.gs) ? c.S<double>(c.L.gram[slot]) : nullptr, c.st));
+    XHC_K("wb_coef", c.st, launch_wb_coef(d, slot, c.T, c.W<float>(c.L.red), c.L.nslice, c.S<float>(c.L.p),
+                                          c.S<float>(c.L.hpost[slot]),
+                                          (d.K[slot] > 1 && d.gs) ? c.S<double>(c.L.gram[slot]) : nullptr,
+                                          c.W<float>(c.L.tokmat), c.st));
+    XHC_K("wb_fwd", c.st, launch_wb_fwd(d, slot, c.T, out, cw, c.W<float>(c.L.tokmat), c.L.nslice,
+                                        c.xact(slot), c.S<int>(c.L.I), c.S<float>(c.L.hres),
+                                        last ? nullptr : c.xact(slot + 1), X, c.st));
     return XHC_OK;
 }
 

@@ -365,9 +365,10 @@ __global__ void k_bwd_coef(Dims d, int slot, int T, const float* __restrict__ re
         if (j >= k) continue;
         const float pj = p[(int64_t)t * k + j];
         float dpj = 0.f;
-        for (int a = 0; a < K; ++a) {
+        for (int a = 0; a < 4; ++a) {
             float e = 0.f;
-            for (int q = 0; q < K; ++q) e += hpost[((int64_t)t * k + j) * K + q] * (float)B[q][a];
+            if (a < K)
+                for (int q = 0; q < K; ++q) e += hpost[((int64_t)t * k + j) * K + q] * (float)B[q][a];
             tm[j * 4 + a] = pj * e;
         }
         for (int q = 0; q < K; ++q) {

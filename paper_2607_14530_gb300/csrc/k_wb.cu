@@ -1,17 +1,18 @@
 // Write-back kernels of the connection op with the causal conv held in registers.
 //
 // Every kernel here walks a run of consecutive tokens for one pair of channels per thread.  The
-// conv taps of the pair (zero past kappa_j) and a ring of the last KW values of `out` stay in
-// registers; the token loop is unrolled by KW so the ring positions are compile-time constants,
-// and each out value is loaded once per run instead of once per tap.  KS = 1 specialises the
-// tap counts to the (4, 8, 12) kernels of the MLP sublayers, so no FMA is spent on zero taps.
-// Per-token reductions over the channels (Gram matrix, write-back gradients) use a
-// reduce-scatter butterfly inside the warp (about V shuffles for V values instead of 5 V), then
-// shared memory across warps.
+// conv taps of the pair and a ring of the last KW values of `out` stay in registers; the token
+// loop is unrolled by KW so the ring positions are compile-time constants, and each out value
+// is loaded once per run instead of once per tap.  The ring is zeroed at every sequence start,
+// so the conv (which never reaches into the previous sequence) needs no per-tap test.  KS = 1
+// specialises the tap counts to the (4, 8, 12) kernels of the MLP sublayers, so no FMA is spent
+// on zero taps.  Per-token reductions over the channels use a reduce-scatter butterfly inside
+// the warp (about V shuffles for V values instead of 5 V), then shared memory across warps.
 //   wb_gram   Gram matrix of u = [out, g_1..g_r] (Eq. aug, Eq. gs), partial per channel slice
-//   wb_fwd    X_act_new = (H_res) X_act + p (H_post out_aug) (Eq. sparse_write_delta,
-//             Eq. sparse_write), scatter into X on the last slot; keeps the token's Gram matrix
-//             for the backward
+//   wb_coef   per token: Gram-Schmidt coefficients (Eq. gs) folded with p and H_post into
+//             E[j][a]; keeps the token's Gram matrix for the backward
+//   wb_fwd    X_act_new = (H_res) X_act + sum_a E[j][a] u_a (Eq. sparse_write_delta,
+//             Eq. sparse_write), scatter into X on the last slot
 //   wb_bred   backward reductions <dXn_j, u_a> and, on the last slot, <dXn_j, x_i>
 //   wb_bapp   component gradients du_a consumed on the fly: d_out = du_0 + conv^T(du_1..r)
 //             (emitted KW - 1 tokens late), conv weight-gradient partials, and on the last slot
@@ -37,53 +38,11 @@ __device__ __forceinline__ float2 fma2(float s, float2 a, float2 acc) {
     return make_float2(fmaf(s, a.x, acc.x), fmaf(s, a.y, acc.y));
 }
 __device__ __forceinline__ float2 f2z() { return make_float2(0.f, 0.f); }
-
 __device__ __forceinline__ uint32_t s_u32(const void* p) {
     return (uint32_t)__cvta_generic_to_shared(p);
 }
-__device__ __forceinline__ void bar_init(uint64_t* b, uint32_t n) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(s_u32(b)), "r"(n) : "memory");
-}
-__device__ __forceinline__ void bar_expect(uint64_t* b, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(s_u32(b)), "r"(bytes) : "memory");
-}
-// bounded wait (~4 s of global time); false when it gives up
-__device__ __forceinline__ bool bar_wait(uint64_t* b, uint32_t parity) {
-    uint64_t t0 = 0;
-    for (uint32_t it = 0;; ++it) {
-        uint32_t ok;
-        asm volatile(
-            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-            " selp.u32 %0, 1, 0, p;\n}\n"
-            : "=r"(ok) : "r"(s_u32(b)), "r"(parity) : "memory");
-        if (ok) return true;
-        if ((it & 255u) == 255u) {
-            uint64_t now;
-            asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(now));
-            if (t0 == 0) t0 = now;
-            else if (now - t0 > 4000000000ull) return false;
-        }
-    }
-}
-// 1-D bulk copy global -> shared completing on an mbarrier (16-byte aligned, size % 16 == 0)
-__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-            s_u32(dst)), "l"(src), "r"(bytes), "r"(s_u32(bar))
-        : "memory");
-}
 
-// Row staging of a run of tokens: per token, `nrow` rows of this CTA's channel slice are copied
-// into a shared-memory stage (two stages, batches of B tokens).  row_src(t, r) gives the global
-// address of row r of token t and its element size.
-struct StageGeom {
-    int B;          // tokens per batch
-    int nrow;       // rows per token
-    int rowb;       // bytes reserved per row in shared memory
-    int tokb;       // bytes per token = nrow * rowb
-};
-
-// Per-thread prefetch of the next tokens' values with cp.async into a 4-slot ring in shared
+// Per-thread prefetch of the next tokens' values with cp.async into a PD-slot ring in shared
 // memory (field-major [slot][field][thread], so a warp's accesses are consecutive words).
 constexpr int PD = 4;
 __device__ __forceinline__ void cpa4(void* dst, const void* src) {
@@ -98,6 +57,9 @@ __device__ __forceinline__ void cpa_wait() { asm volatile("cp.async.wait_group %
 __device__ __forceinline__ float2 u2f2(uint32_t u) {
     return make_float2(__uint_as_float(u << 16), __uint_as_float(u & 0xffff0000u));
 }
+
+// position within the sequence of the next token
+__device__ __forceinline__ int next_pos(int pos, int S) { return (pos + 1 == S) ? 0 : pos + 1; }
 
 // taps of component j held in registers: KS = 1 is the (4, 8, 12) kernel set, else KW each
 template <int KW, int KS>
@@ -119,34 +81,41 @@ __device__ __forceinline__ void taps_reg(const Dims& d, const ConvPtrs& cw, int 
         }
 }
 
-// ring w[s] = out[t] for t = s (mod KW); prepare the run starting at t0 (t0 % KW == 0)
+// ring w[s] = out[t] for t = s (mod KW); prepares the run starting at t0 (t0 % KW == 0), whose
+// position in its sequence is pos0: values before the sequence start are zero
 template <int KW>
 __device__ __forceinline__ void ring_init(const uint16_t* out, int C, int c, bool act, long long t0,
-                                          float2 (&w)[KW]) {
+                                          int pos0, float2 (&w)[KW]) {
     w[0] = f2z();
 #pragma unroll
-    for (int i = 1; i < KW; ++i) {
-        const long long t = t0 - i;
-        w[KW - i] = (act && t >= 0) ? ld2(out + t * C + c) : f2z();
+    for (int i = 1; i < KW; ++i) w[KW - i] = (act && i <= pos0) ? ld2(out + (t0 - i) * C + c) : f2z();
+}
+
+// store out[t] at slot U; at a sequence start the older slots are cleared
+template <int KW>
+__device__ __forceinline__ void ring_push(float2 (&w)[KW], int U, float2 o, bool seq_start) {
+    w[U] = o;
+    if (seq_start) {
+#pragma unroll
+        for (int s = 0; s < KW; ++s)
+            if (s != U) w[s] = f2z();
     }
 }
 
-// g_j = sum_{i <= pos} tw[j][i] out[t - i], with out[t - i] at ring slot (U - i) mod KW
+// g_j = sum_i tw[j][i] out[t - i], with out[t - i] at ring slot (U - i) mod KW
 template <int KW, int KS>
 __device__ __forceinline__ void conv_ring(const float2 (&tw)[3][KW], const float2 (&w)[KW], int U,
-                                          int pos, float2 (&g)[3]) {
+                                          float2 (&g)[3]) {
 #pragma unroll
     for (int j = 0; j < 3; ++j) g[j] = f2z();
 #pragma unroll
     for (int i = 0; i < KW; ++i) {
-        if (i <= pos) {
-            const float2 o = w[(U - i + KW) % KW];
+        const float2 o = w[(U - i + KW) % KW];
 #pragma unroll
-            for (int j = 0; j < 3; ++j) {
-                if (i >= ntap<KW, KS>(j)) continue;
-                g[j].x = fmaf(tw[j][i].x, o.x, g[j].x);
-                g[j].y = fmaf(tw[j][i].y, o.y, g[j].y);
-            }
+        for (int j = 0; j < 3; ++j) {
+            if (i >= ntap<KW, KS>(j)) continue;
+            g[j].x = fmaf(tw[j][i].x, o.x, g[j].x);
+            g[j].y = fmaf(tw[j][i].y, o.y, g[j].y);
         }
     }
 }
@@ -199,18 +168,21 @@ __global__ void __launch_bounds__(WT) k_wb_gram(Dims d, int slot, int T, int TB,
     const long long t1 = min((long long)T, t0 + TB);
     const int K = d.K[slot];
     const int nq = K * (K + 1) / 2;
+    int pos = (int)(t0 % d.S);
     float2 tw[3][KW], w[KW];
     taps_reg<KW, KS>(d, cw, c, act, tw);
-    ring_init<KW>(out, C, c, act, t0, w);
+    ring_init<KW>(out, C, c, act, t0, pos, w);
+    const uint16_t* po = out + t0 * C + c;
     for (long long tb = t0; tb < t1; tb += KW) {
 #pragma unroll
         for (int u = 0; u < KW; ++u) {
             const long long t = tb + u;
             if (t < t1) {
-                const float2 o = act ? ld2(out + t * C + c) : f2z();
-                w[u] = o;
+                const float2 o = act ? ld2(po) : f2z();
+                po += C;
+                ring_push<KW>(w, u, o, pos == 0);
                 float2 g[3];
-                conv_ring<KW, KS>(tw, w, u, (int)(t % d.S), g);
+                conv_ring<KW, KS>(tw, w, u, g);
                 const float2 uu[4] = {o, g[0], g[1], g[2]};
                 float v[16];
                 int q = 0;
@@ -222,6 +194,7 @@ __global__ void __launch_bounds__(WT) k_wb_gram(Dims d, int slot, int T, int TB,
                 for (int r = 10; r < 16; ++r) v[r] = 0.f;
                 const float tot = WRed<16, 16>::run(v, lane);
                 if ((lane & 1) == 0) wsh[((t - t0) * (WT / 32) + warp) * 16 + (lane >> 1)] = tot;
+                pos = next_pos(pos, d.S);
             }
         }
     }
@@ -237,10 +210,55 @@ __global__ void __launch_bounds__(WT) k_wb_gram(Dims d, int slot, int T, int TB,
 }
 
 // ---------------------------------------------------------------------------------------------
-// wb_fwd: per-token coefficients E[j][a] (Gram-Schmidt folded in), H_res, I in shared memory;
-// each thread prefetches the out value and the k active values of its channel pair 3 tokens
-// ahead with cp.async.  The CTAs of channel slice 0 also store the token's Gram matrix (fp64,
-// lower triangle) for the backward of Eq. gs.
+// wb_coef: one thread per token.  With Gram-Schmidt, the slice partials of the Gram matrix are
+// summed in fp64, kept in `gram` for the backward and turned into the coefficients B of Eq. gs
+// (orthogonalised component q = sum_a B[q][a] u_a), so that the write-back of active slot j is
+// sum_a E[j][a] u_a with E[j][a] = p_j sum_q H_post[j][q] B[q][a]; without it B is the
+// identity.  E goes to the per-token matrix buffer (rows j < k, four entries each).
+
+__global__ void __launch_bounds__(64) k_wb_coef(Dims d, int slot, int T, const float* __restrict__ red,
+                                                int nslice, const float* __restrict__ p,
+                                                const float* __restrict__ hpost,
+                                                double* __restrict__ gram, float* __restrict__ emat) {
+    const int t = blockIdx.x * blockDim.x + threadIdx.x;
+    if (t >= T) return;
+    const int k = d.k, K = d.K[slot];
+    const bool gs = (K > 1) && d.gs;
+    double B[MAXCOMP][MAXCOMP];
+    for (int a = 0; a < MAXCOMP; ++a)
+        for (int b = 0; b < MAXCOMP; ++b) B[a][b] = (a == b) ? 1.0 : 0.0;
+    if (gs) {
+        double Gm[MAXCOMP][MAXCOMP], cc[MAXCOMP][MAXCOMP], vv[MAXCOMP];
+        for (int a = 0; a < MAXCOMP; ++a)
+            for (int b = 0; b < MAXCOMP; ++b) Gm[a][b] = 0.0;
+        for (int sl = 0; sl < nslice; ++sl) {
+            const float* rp = red + ((int64_t)t * nslice + sl) * NRED;
+            int q = 0;
+            for (int a = 0; a < K; ++a)
+                for (int b = 0; b <= a; ++b) Gm[a][b] += (double)rp[q++];
+        }
+        int q = 0;
+        for (int a = 0; a < K; ++a)
+            for (int b = 0; b <= a; ++b) gram[(int64_t)t * NGRAM + q++] = Gm[a][b];
+        for (int a = 0; a < K; ++a)
+            for (int b = a + 1; b < K; ++b) Gm[a][b] = Gm[b][a];
+        gs_coef(Gm, K, (double)d.eps_gs, B, cc, vv);
+    }
+    float* em = emat + (int64_t)t * TOKMAT;
+    for (int j = 0; j < k; ++j) {
+        const float pj = p[(int64_t)t * k + j];
+        for (int a = 0; a < 4; ++a) {
+            float e = 0.f;
+            if (a < K)
+                for (int q = 0; q < K; ++q) e += hpost[((int64_t)t * k + j) * K + q] * (float)B[q][a];
+            em[j * 4 + a] = pj * e;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------------------------
+// wb_fwd: per-token coefficients E[j][a], H_res and I in shared memory; each thread prefetches
+// the out value and the k active values of its channel pair PD - 1 tokens ahead with cp.async.
 
 template <int KM>
 struct FRing {
@@ -251,20 +269,16 @@ struct FRing {
 template <int KM, int KW, int KS>
 __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
                                                const uint16_t* __restrict__ out, ConvPtrs cw,
-                                               const float* __restrict__ red, int nslice,
+                                               const float* __restrict__ emat,
                                                const uint16_t* __restrict__ xact,
                                                const int* __restrict__ I,
-                                               const float* __restrict__ p,
-                                               const float* __restrict__ hpost,
                                                const float* __restrict__ hres,
                                                uint16_t* __restrict__ xact_next,
-                                               uint16_t* __restrict__ X,
-                                               double* __restrict__ gram) {
+                                               uint16_t* __restrict__ X) {
     extern __shared__ __align__(16) unsigned char smu[];
     FRing<KM>& R = *reinterpret_cast<FRing<KM>*>(smu);
-    const int k = d.k, K = d.K[slot], C = d.C;
+    const int k = d.k, C = d.C;
     const bool last = (slot == d.G - 1);
-    const bool gs = (K > 1) && d.gs;
     float* Esh = reinterpret_cast<float*>(smu + sizeof(FRing<KM>));  // [TB][KM][4]
     float* Hsh = Esh + TB * KM * 4;                                 // [TB][KM][KM]
     int* Ish = reinterpret_cast<int*>(Hsh + TB * KM * KM);           // [TB][KM]
@@ -273,60 +287,37 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
     const int ntok = (int)(t1 - t0);
     const int c = blockIdx.x * WSL + 2 * threadIdx.x;
     const bool act = c < C;
+    const uint16_t* po = out + t0 * C + c;
+    const uint16_t* px = xact + t0 * k * C + c;
     auto issue = [&](int sl, int tn) {
         if (act && tn < ntok) {
-            const long long t = t0 + tn;
-            cpa4(&R.o[sl][threadIdx.x], out + t * C + c);
+            cpa4(&R.o[sl][threadIdx.x], po + (long long)tn * C);
 #pragma unroll
             for (int j = 0; j < KM; ++j)
-                if (j < k) cpa4(&R.x[sl][j][threadIdx.x], xact + (t * k + j) * C + c);
+                if (j < k) cpa4(&R.x[sl][j][threadIdx.x], px + ((long long)tn * k + j) * C);
         }
         cpa_commit();
     };
 #pragma unroll
     for (int q = 0; q < PD - 1; ++q) issue(q, q);
-    for (int tt = threadIdx.x; tt < ntok; tt += WT) {
-        const long long t = t0 + tt;
-        double B[MAXCOMP][MAXCOMP];
-        for (int a = 0; a < MAXCOMP; ++a)
-            for (int b = 0; b < MAXCOMP; ++b) B[a][b] = (a == b) ? 1.0 : 0.0;
-        if (gs) {
-            double Gm[MAXCOMP][MAXCOMP], cc[MAXCOMP][MAXCOMP], vv[MAXCOMP];
-            for (int a = 0; a < MAXCOMP; ++a)
-                for (int b = 0; b < MAXCOMP; ++b) Gm[a][b] = 0.0;
-            for (int sl = 0; sl < nslice; ++sl) {
-                const float* rp = red + (t * nslice + sl) * NRED;
-                int q = 0;
-                for (int a = 0; a < K; ++a)
-                    for (int b = 0; b <= a; ++b) Gm[a][b] += (double)rp[q++];
-            }
-            if (blockIdx.x == 0) {
-                int q = 0;
-                for (int a = 0; a < K; ++a)
-                    for (int b = 0; b <= a; ++b) gram[t * NGRAM + q++] = Gm[a][b];
-            }
-            for (int a = 0; a < K; ++a)
-                for (int b = a + 1; b < K; ++b) Gm[a][b] = Gm[b][a];
-            gs_coef(Gm, K, (double)d.eps_gs, B, cc, vv);
-        }
-        for (int j = 0; j < KM; ++j) {
-            const bool jv = j < k;
-            const float pj = jv ? p[t * k + j] : 0.f;
-            for (int a = 0; a < 4; ++a) {
-                float e = 0.f;
-                if (jv && a < K)
-                    for (int q = 0; q < K; ++q) e += hpost[(t * k + j) * K + q] * (float)B[q][a];
-                Esh[(tt * KM + j) * 4 + a] = pj * e;
-            }
-            Ish[tt * KM + j] = jv ? I[t * k + j] : 0;
-            for (int i = 0; i < KM; ++i)
-                Hsh[(tt * KM + j) * KM + i] = (last && jv && i < k) ? hres[t * k * k + j * k + i] : 0.f;
-        }
+    for (int idx = threadIdx.x; idx < ntok * KM * 4; idx += WT) {
+        const int tt = idx / (KM * 4), q = idx - tt * (KM * 4);
+        Esh[idx] = (q < k * 4) ? emat[(t0 + tt) * TOKMAT + q] : 0.f;
     }
+    for (int idx = threadIdx.x; idx < ntok * KM * KM; idx += WT) {
+        const int tt = idx / (KM * KM), q = idx - tt * (KM * KM);
+        const int j = q / KM, i = q - j * KM;
+        Hsh[idx] = (last && j < k && i < k) ? hres[(t0 + tt) * k * k + j * k + i] : 0.f;
+    }
+    for (int idx = threadIdx.x; idx < ntok * KM; idx += WT) {
+        const int tt = idx / KM, j = idx - tt * KM;
+        Ish[idx] = (j < k) ? I[(t0 + tt) * k + j] : 0;
+    }
+    int pos = (int)(t0 % d.S);
     float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
     if constexpr (KW > 0) {
         taps_reg<KW, KS>(d, cw, c, act, tw);
-        ring_init<KW>(out, C, c, act, t0, w);
+        ring_init<KW>(out, C, c, act, t0, pos, w);
     }
     __syncthreads();
     const int RU = KW > 0 ? KW : 4;
@@ -339,49 +330,60 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
                 const int sl = u % PD;
                 issue((u + PD - 1) % PD, tt + PD - 1);
                 cpa_wait<PD - 1>();
-                if (!act) continue;
-                const float2 o = u2f2(R.o[sl][threadIdx.x]);
-                float2 uu[4] = {o, f2z(), f2z(), f2z()};
-                if constexpr (KW > 0) {
-                    w[u] = o;
-                    float2 g[3];
-                    conv_ring<KW, KS>(tw, w, u, (int)(t % d.S), g);
-                    uu[1] = g[0];
-                    uu[2] = g[1];
-                    uu[3] = g[2];
-                }
-                float2 x[KM];
-#pragma unroll
-                for (int j = 0; j < KM; ++j) x[j] = (j < k) ? u2f2(R.x[sl][j][threadIdx.x]) : f2z();
-                const float4* E4 = reinterpret_cast<const float4*>(Esh + tt * KM * 4);
-#pragma unroll
-                for (int j = 0; j < KM; ++j) {
-                    if (j >= k) continue;
-                    float2 v;
-                    if (last) {
-                        v = f2z();
-#pragma unroll
-                        for (int i = 0; i < KM; ++i) v = fma2(Hsh[(tt * KM + j) * KM + i], x[i], v);
-                    } else {
-                        v = x[j];
+                if (act) {
+                    const float2 o = u2f2(R.o[sl][threadIdx.x]);
+                    float2 uu[4] = {o, f2z(), f2z(), f2z()};
+                    if constexpr (KW > 0) {
+                        ring_push<KW>(w, u, o, pos == 0);
+                        float2 g[3];
+                        conv_ring<KW, KS>(tw, w, u, g);
+                        uu[1] = g[0];
+                        uu[2] = g[1];
+                        uu[3] = g[2];
                     }
-                    const float4 e = E4[j];
-                    v = fma2(e.x, uu[0], v);
-                    v = fma2(e.y, uu[1], v);
-                    v = fma2(e.z, uu[2], v);
-                    v = fma2(e.w, uu[3], v);
-                    if (last)
-                        st2(X + (t * d.N + Ish[tt * KM + j]) * C + c, v);
-                    else
-                        st2(xact_next + (t * k + j) * C + c, v);
+                    float2 x[KM];
+#pragma unroll
+                    for (int j = 0; j < KM; ++j) x[j] = (j < k) ? u2f2(R.x[sl][j][threadIdx.x]) : f2z();
+                    const float4* E4 = reinterpret_cast<const float4*>(Esh + tt * KM * 4);
+                    const float4* H4 = reinterpret_cast<const float4*>(Hsh + tt * KM * KM);
+#pragma unroll
+                    for (int j = 0; j < KM; ++j) {
+                        if (j >= k) continue;
+                        float2 v;
+                        if (last) {
+                            v = f2z();
+#pragma unroll
+                            for (int q = 0; q < KM / 4; ++q) {
+                                const float4 h = H4[j * (KM / 4) + q];
+                                v = fma2(h.x, x[4 * q + 0], v);
+                                v = fma2(h.y, x[4 * q + 1], v);
+                                v = fma2(h.z, x[4 * q + 2], v);
+                                v = fma2(h.w, x[4 * q + 3], v);
+                            }
+                        } else {
+                            v = x[j];
+                        }
+                        const float4 e = E4[j];
+                        v = fma2(e.x, uu[0], v);
+                        if constexpr (KW > 0) {
+                            v = fma2(e.y, uu[1], v);
+                            v = fma2(e.z, uu[2], v);
+                            v = fma2(e.w, uu[3], v);
+                        }
+                        if (last)
+                            st2(X + (t * d.N + Ish[tt * KM + j]) * C + c, v);
+                        else
+                            st2(xact_next + (t * k + j) * C + c, v);
+                    }
                 }
+                pos = next_pos(pos, d.S);
             }
         }
     }
     cpa_wait<0>();
 }
 
-// prefetch ring of the backward kernels: per slot, out (bf16 pair), x_j (bf16 pairs), dn_j
+// prefetch ring of the backward reductions: per slot, out (bf16 pair), x_j (bf16 pairs), dn_j
 // (fp32 pair, or a bf16 pair in .x at the last slot)
 template <int KM>
 struct BRing {
@@ -389,28 +391,6 @@ struct BRing {
     uint32_t x[PD][KM][WT];
     uint2 dn[PD][KM][WT];
 };
-
-template <int KM>
-__device__ __forceinline__ void bring_issue(BRing<KM>& R, int slot, long long t, bool ok, int k,
-                                            int N, int C, int c, bool last, bool with_x,
-                                            const uint16_t* out, const uint16_t* xact,
-                                            const uint16_t* dX, const int* Irow,
-                                            const float* dxact) {
-    const int tid = threadIdx.x;
-    if (ok) {
-        cpa4(&R.o[slot][tid], out + t * C + c);
-#pragma unroll
-        for (int j = 0; j < KM; ++j) {
-            if (j >= k) continue;
-            if (with_x) cpa4(&R.x[slot][j][tid], xact + (t * k + j) * C + c);
-            if (last)
-                cpa4(&R.dn[slot][j][tid], dX + (t * N + Irow[j]) * C + c);
-            else
-                cpa8(&R.dn[slot][j][tid], dxact + (t * k + j) * C + c);
-        }
-    }
-    cpa_commit();
-}
 
 // Per token, NV partial sums over this CTA's channel slice: P[j][a] = <dXn_j, u_a> at j*4 + a
 // and, on the last slot, Q[j][i] = <dXn_j, x_i> at KM*4 + j*KM + i.  NV = 16 is reduced to
@@ -443,14 +423,33 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
         Ish[q] = (j < k) ? I[(t0 + tt) * k + j] : 0;
     }
     __syncthreads();
+    const uint16_t* po = out + t0 * C + c;
+    const uint16_t* px = xact + t0 * k * C + c;
+    const uint16_t* pX = dX + t0 * d.N * C + c;
+    const float* pd = dxact + t0 * k * C + c;
+    auto issue = [&](int sl, int tn) {
+        if (act && tn < ntok) {
+            cpa4(&R.o[sl][threadIdx.x], po + (long long)tn * C);
 #pragma unroll
-    for (int q = 0; q < PD - 1; ++q)
-        bring_issue<KM>(R, q, t0 + q, act && q < ntok, k, d.N, C, c, last, last, out, xact, dX,
-                        Ish + q * KM, dxact);
+            for (int j = 0; j < KM; ++j) {
+                if (j >= k) continue;
+                if (last) {
+                    cpa4(&R.x[sl][j][threadIdx.x], px + ((long long)tn * k + j) * C);
+                    cpa4(&R.dn[sl][j][threadIdx.x], pX + ((long long)tn * d.N + Ish[tn * KM + j]) * C);
+                } else {
+                    cpa8(&R.dn[sl][j][threadIdx.x], pd + ((long long)tn * k + j) * C);
+                }
+            }
+        }
+        cpa_commit();
+    };
+#pragma unroll
+    for (int q = 0; q < PD - 1; ++q) issue(q, q);
+    int pos = (int)(t0 % d.S);
     float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
     if constexpr (KW > 0) {
         taps_reg<KW, KS>(d, cw, c, act, tw);
-        ring_init<KW>(out, C, c, act, t0, w);
+        ring_init<KW>(out, C, c, act, t0, pos, w);
     }
     const int RU = KW > 0 ? KW : 4;
     for (long long tb = t0; tb < t1; tb += RU) {
@@ -460,11 +459,7 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
             if (t < t1) {
                 const int tt = (int)(t - t0);
                 const int sl = u % PD;                       // == tt % PD (runs start on a multiple of 4)
-                {
-                    const int tn = tt + PD - 1;
-                    bring_issue<KM>(R, (u + PD - 1) % PD, t0 + tn, act && tn < ntok, k, d.N, C, c, last,
-                                    last, out, xact, dX, Ish + (tn < ntok ? tn : 0) * KM, dxact);
-                }
+                issue((u + PD - 1) % PD, tt + PD - 1);
                 cpa_wait<PD - 1>();
                 float2 uu[4] = {f2z(), f2z(), f2z(), f2z()};
                 float2 dn[KM], x[KM];
@@ -477,9 +472,9 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
                     const float2 o = u2f2(R.o[sl][threadIdx.x]);
                     uu[0] = o;
                     if constexpr (KW > 0) {
-                        w[u] = o;
+                        ring_push<KW>(w, u, o, pos == 0);
                         float2 g[3];
-                        conv_ring<KW, KS>(tw, w, u, (int)(t % d.S), g);
+                        conv_ring<KW, KS>(tw, w, u, g);
                         uu[1] = g[0];
                         uu[2] = g[1];
                         uu[3] = g[2];
@@ -495,8 +490,6 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
                             dn[j] = make_float2(__uint_as_float(r.x), __uint_as_float(r.y));
                         }
                     }
-                } else if constexpr (KW > 0) {
-                    w[u] = f2z();
                 }
                 // dn, x and the unused components are zero where a term does not apply
                 float v[NVP];
@@ -506,7 +499,7 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
                 for (int j = 0; j < KM; ++j)
 #pragma unroll
                     for (int a = 0; a < 4; ++a)
-                        if (j * 4 + a < NVP) v[j * 4 + a] = dot2(dn[j], uu[a]);
+                        if (j * 4 + a < NVP && (KW > 0 || a == 0)) v[j * 4 + a] = dot2(dn[j], uu[a]);
                 if constexpr (NVP >= KM * 4 + KM * KM) {
                     if (last) {
 #pragma unroll
@@ -525,6 +518,7 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
 #pragma unroll
                     for (int bb = 0; bb < NV / 32; ++bb) dst[bb * 32 + lane] = tot[bb];
                 }
+                pos = next_pos(pos, d.S);
             }
         }
     }
@@ -543,11 +537,13 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
 // wb_bapp: du_a = sum_j E[j][a] dXn_j + sum_b D[a][b] u_b (Eq. sparse_write reversed, with the
 // Gram-Schmidt Jacobian in D), never stored:
 //   d_out[s] = du_0[s] + sum_j sum_{i < kappa_j, pos(s) + i < S} w_j[i] du_{1+j}[s + i]
-// (the transpose of the causal conv of Eq. aug) is accumulated in a ring of KW pending outputs
-// and emitted once token s + KW - 1 has been seen; each run therefore recomputes du for the first
-// KW - 1 tokens of the next run.  The conv weight gradient sum_t du_{1+j}[t] out[t - i] is
-// accumulated per run.  Last slot: dX_act_i = sum_j H_res[j][i] dXn_j.  The -cx x_i term of the
-// active-state gradient is added by the backward of the slot's pre-map.
+// (the transpose of the causal conv of Eq. aug) is accumulated in a ring of KW pending outputs.
+// An output is complete once token s + KW - 1 of its sequence has been seen, or when its
+// sequence (or the data) ends: it is stored then, and later terms that land in its ring slot
+// are never stored.  Each run therefore recomputes du for the first KW - 1 tokens of the next
+// run.  The conv weight gradient sum_t du_{1+j}[t] out[t - i] is accumulated per run.  Last
+// slot: dX_act_i = sum_j H_res[j][i] dXn_j.  The -cx x_i term of the active-state gradient is
+// added by the backward of the slot's pre-map.
 
 template <int KM>
 struct ARing {
@@ -569,7 +565,7 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
     constexpr int RU = KW > 0 ? KW : 4;
     extern __shared__ __align__(16) unsigned char smu[];
     ARing<KM>& R = *reinterpret_cast<ARing<KM>*>(smu);
-    const int k = d.k, K = d.K[slot], C = d.C;
+    const int k = d.k, C = d.C;
     const bool last = (slot == d.G - 1);
     const int TH = TB + HL;
     float* Esh = reinterpret_cast<float*>(smu + sizeof(ARing<KM>));  // [TH][KM][4]
@@ -581,46 +577,54 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
     const long long te = min((long long)T, t1 + HL);                // tokens with data
     const long long tend = t1 + HL;                                 // loop end (emission lag)
     const int ntok = (int)(te - t0);
-    for (int idx = threadIdx.x; idx < ntok * 128; idx += WT) {
-        const int tt = idx >> 7, q = idx & 127;
-        const long long t = t0 + tt;
-        if (q < 32) {
-            const int j = q >> 2;
-            if (j < KM) Esh[tt * KM * 4 + q] = tokmat[t * TOKMAT + q];
-        } else if (q < 48) {
-            Dsh[tt * 16 + (q - 32)] = tokmat[t * TOKMAT + q];
-        } else if (q < 112) {
-            const int a = (q - 48) >> 3, b = (q - 48) & 7;
-            if (a < KM && b < KM) Hsh[(tt * KM + a) * KM + b] = last ? tokmat[t * TOKMAT + q] : 0.f;
-        } else if (q >= 120 && q < 120 + KM) {
-            Ish[tt * KM + (q - 120)] = (last && q - 120 < k) ? I[t * k + (q - 120)] : 0;
+    for (int idx = threadIdx.x; idx < ntok * KM * 4; idx += WT) {
+        const int tt = idx / (KM * 4), q = idx - tt * (KM * 4);
+        Esh[idx] = tokmat[(t0 + tt) * TOKMAT + q];
+    }
+    if constexpr (KW > 0) {
+        for (int idx = threadIdx.x; idx < ntok * 16; idx += WT) {
+            const int tt = idx >> 4, q = idx & 15;
+            Dsh[idx] = tokmat[(t0 + tt) * TOKMAT + 32 + q];
+        }
+    }
+    if (last) {
+        for (int idx = threadIdx.x; idx < ntok * KM * KM; idx += WT) {
+            const int tt = idx / (KM * KM), q = idx - tt * (KM * KM);
+            Hsh[idx] = tokmat[(t0 + tt) * TOKMAT + 48 + (q / KM) * 8 + (q % KM)];
+        }
+        for (int idx = threadIdx.x; idx < ntok * KM; idx += WT) {
+            const int tt = idx / KM, j = idx - tt * KM;
+            Ish[idx] = (j < k) ? I[(t0 + tt) * k + j] : 0;
         }
     }
     const int c = blockIdx.x * WSL + 2 * threadIdx.x;
     const bool act = c < C;
     __syncthreads();
+    const uint16_t* po = out + t0 * C + c;
+    const uint16_t* pX = dX + t0 * d.N * C + c;
+    const float* pd = dn_in + t0 * k * C + c;
     auto issue = [&](int sl, int tn) {
         if (act && tn < ntok) {
-            const long long t = t0 + tn;
-            cpa4(&R.o[sl][threadIdx.x], out + t * C + c);
+            cpa4(&R.o[sl][threadIdx.x], po + (long long)tn * C);
 #pragma unroll
             for (int j = 0; j < KM; ++j) {
                 if (j >= k) continue;
                 if (last)
-                    cpa4(&R.dn[sl][j][threadIdx.x], dX + (t * d.N + Ish[tn * KM + j]) * C + c);
+                    cpa4(&R.dn[sl][j][threadIdx.x], pX + ((long long)tn * d.N + Ish[tn * KM + j]) * C);
                 else
-                    cpa8(&R.dn[sl][j][threadIdx.x], dn_in + (t * k + j) * C + c);
+                    cpa8(&R.dn[sl][j][threadIdx.x], pd + ((long long)tn * k + j) * C);
             }
         }
         cpa_commit();
     };
 #pragma unroll
     for (int q = 0; q < PD - 1; ++q) issue(q, q);
+    int pos = (int)(t0 % d.S);
     float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1], pend[KW > 0 ? KW : 1];
     float2 acc[3][KW > 0 ? KW : 1];
     if constexpr (KW > 0) {
         taps_reg<KW, KS>(d, cw, c, act, tw);
-        ring_init<KW>(out, C, c, act, t0, w);
+        ring_init<KW>(out, C, c, act, t0, pos, w);
 #pragma unroll
         for (int s = 0; s < KW; ++s) pend[s] = f2z();
 #pragma unroll
@@ -637,96 +641,117 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
                 const int sl = u % PD;
                 issue((u + PD - 1) % PD, tt + PD - 1);
                 cpa_wait<PD - 1>();
-                if (!act) continue;
-                const bool has = t < te;
-                const int pos = (int)(t % d.S);
-                float2 uu[4] = {f2z(), f2z(), f2z(), f2z()};
-                float2 du[4] = {f2z(), f2z(), f2z(), f2z()};
-                if (has) {
-                    uu[0] = u2f2(R.o[sl][threadIdx.x]);
-                    float2 dn[KM];
+                if (act) {
+                    const bool has = t < te;
+                    float2 du[4] = {f2z(), f2z(), f2z(), f2z()};
+                    if (has) {
+                        const float2 o = u2f2(R.o[sl][threadIdx.x]);
+                        float2 dn[KM];
 #pragma unroll
-                    for (int j = 0; j < KM; ++j) {
-                        dn[j] = f2z();
-                        if (j < k) {
-                            const uint2 r = R.dn[sl][j][threadIdx.x];
-                            dn[j] = last ? u2f2(r.x) : make_float2(__uint_as_float(r.x), __uint_as_float(r.y));
-                        }
-                    }
-                    if constexpr (KW > 0) {
-                        w[u] = uu[0];
-                        float2 g[3];
-                        conv_ring<KW, KS>(tw, w, u, pos, g);
-                        uu[1] = g[0];
-                        uu[2] = g[1];
-                        uu[3] = g[2];
-                    }
-                    const float4* E4 = reinterpret_cast<const float4*>(Esh + tt * KM * 4);
-                    const float4* D4 = reinterpret_cast<const float4*>(Dsh + tt * 16);
-#pragma unroll
-                    for (int j = 0; j < KM; ++j) {
-                        if (j >= k) continue;
-                        const float4 e = E4[j];
-                        du[0] = fma2(e.x, dn[j], du[0]);
-                        du[1] = fma2(e.y, dn[j], du[1]);
-                        du[2] = fma2(e.z, dn[j], du[2]);
-                        du[3] = fma2(e.w, dn[j], du[3]);
-                    }
-                    if constexpr (KW > 0) {
-#pragma unroll
-                        for (int a = 0; a < 4; ++a) {
-                            const float4 m = D4[a];
-                            du[a] = fma2(m.x, uu[0], du[a]);
-                            du[a] = fma2(m.y, uu[1], du[a]);
-                            du[a] = fma2(m.z, uu[2], du[a]);
-                            du[a] = fma2(m.w, uu[3], du[a]);
-                        }
-                    }
-                    if (last && t < t1) {
-#pragma unroll
-                        for (int i = 0; i < KM; ++i) {
-                            if (i >= k) continue;
-                            float2 v = f2z();
-#pragma unroll
-                            for (int j = 0; j < KM; ++j) v = fma2(Hsh[(tt * KM + j) * KM + i], dn[j], v);
-                            *reinterpret_cast<float2*>(dxact_out + (t * k + i) * C + c) = v;
-                        }
-                    }
-                } else if constexpr (KW > 0) {
-                    w[u] = f2z();
-                }
-                if constexpr (KW == 0) {
-                    if (has) st2(d_out + t * C + c, du[0]);
-                } else {
-                    // conv weight gradient of this run's tokens
-                    if (t < t1) {
-#pragma unroll
-                        for (int j = 0; j < 3; ++j)
-#pragma unroll
-                            for (int i = 0; i < KW; ++i) {
-                                if (i >= ntap<KW, KS>(j) || i > pos) continue;
-                                const float2 o = w[(u - i + KW) % KW];
-                                acc[j][i].x = fmaf(du[1 + j].x, o.x, acc[j][i].x);
-                                acc[j][i].y = fmaf(du[1 + j].y, o.y, acc[j][i].y);
+                        for (int j = 0; j < KM; ++j) {
+                            dn[j] = f2z();
+                            if (j < k) {
+                                const uint2 r = R.dn[sl][j][threadIdx.x];
+                                dn[j] = last ? u2f2(r.x) : make_float2(__uint_as_float(r.x), __uint_as_float(r.y));
                             }
+                        }
+                        const float4* E4 = reinterpret_cast<const float4*>(Esh + tt * KM * 4);
+#pragma unroll
+                        for (int j = 0; j < KM; ++j) {
+                            if (j >= k) continue;
+                            const float4 e = E4[j];
+                            du[0] = fma2(e.x, dn[j], du[0]);
+                            if constexpr (KW > 0) {
+                                du[1] = fma2(e.y, dn[j], du[1]);
+                                du[2] = fma2(e.z, dn[j], du[2]);
+                                du[3] = fma2(e.w, dn[j], du[3]);
+                            }
+                        }
+                        if constexpr (KW > 0) {
+                            ring_push<KW>(w, u, o, pos == 0);
+                            float2 g[3];
+                            conv_ring<KW, KS>(tw, w, u, g);
+                            const float2 uu[4] = {o, g[0], g[1], g[2]};
+                            const float4* D4 = reinterpret_cast<const float4*>(Dsh + tt * 16);
+#pragma unroll
+                            for (int a = 0; a < 4; ++a) {
+                                const float4 m = D4[a];
+                                du[a] = fma2(m.x, uu[0], du[a]);
+                                du[a] = fma2(m.y, uu[1], du[a]);
+                                du[a] = fma2(m.z, uu[2], du[a]);
+                                du[a] = fma2(m.w, uu[3], du[a]);
+                            }
+                        }
+                        if (last && t < t1) {
+                            const float4* H4 = reinterpret_cast<const float4*>(Hsh + tt * KM * KM);
+                            float2 v[KM];
+#pragma unroll
+                            for (int i = 0; i < KM; ++i) v[i] = f2z();
+#pragma unroll
+                            for (int j = 0; j < KM; ++j) {
+                                if (j >= k) continue;
+#pragma unroll
+                                for (int q = 0; q < KM / 4; ++q) {
+                                    const float4 h = H4[j * (KM / 4) + q];
+                                    v[4 * q + 0] = fma2(h.x, dn[j], v[4 * q + 0]);
+                                    v[4 * q + 1] = fma2(h.y, dn[j], v[4 * q + 1]);
+                                    v[4 * q + 2] = fma2(h.z, dn[j], v[4 * q + 2]);
+                                    v[4 * q + 3] = fma2(h.w, dn[j], v[4 * q + 3]);
+                                }
+                            }
+#pragma unroll
+                            for (int i = 0; i < KM; ++i)
+                                if (i < k) *reinterpret_cast<float2*>(dxact_out + (t * k + i) * C + c) = v[i];
+                        }
+                    } else if constexpr (KW > 0) {
+                        w[u] = f2z();
                     }
-                    // d_out[t - i] += w_j[i] du_{1+j}[t] for the pending outputs of this run
-                    pend[u] = du[0];
+                    if constexpr (KW == 0) {
+                        if (has) st2(d_out + t * C + c, du[0]);
+                    } else {
+                        // conv weight gradient of this run's tokens (the ring is zero before the
+                        // sequence start)
+                        if (t < t1) {
 #pragma unroll
-                    for (int i = 0; i < KW; ++i) {
-                        if (i > pos || i > tt) continue;
+                            for (int j = 0; j < 3; ++j)
 #pragma unroll
-                        for (int j = 0; j < 3; ++j) {
-                            if (i >= ntap<KW, KS>(j)) continue;
-                            float2& q = pend[(u - i + KW) % KW];
-                            q.x = fmaf(tw[j][i].x, du[1 + j].x, q.x);
-                            q.y = fmaf(tw[j][i].y, du[1 + j].y, q.y);
+                                for (int i = 0; i < KW; ++i) {
+                                    if (i >= ntap<KW, KS>(j)) continue;
+                                    const float2 o = w[(u - i + KW) % KW];
+                                    acc[j][i].x = fmaf(du[1 + j].x, o.x, acc[j][i].x);
+                                    acc[j][i].y = fmaf(du[1 + j].y, o.y, acc[j][i].y);
+                                }
+                        }
+                        // a sequence starts at t, or the data ends: the pending outputs of the
+                        // finished sequence (the last min(S, pos) or S tokens) are complete
+                        if (pos == 0 || t == T) {
+                            const int lim = (pos == 0) ? d.S : pos;
+#pragma unroll
+                            for (int i = 1; i < KW; ++i) {
+                                const long long s = t - i;
+                                if (i <= lim && s >= t0 && s < t1) st2(d_out + s * C + c, pend[(u - i + KW) % KW]);
+                            }
+                        }
+                        // d_out[t - i] += w_j[i] du_{1+j}[t]
+                        pend[u] = du[0];
+#pragma unroll
+                        for (int i = 0; i < KW; ++i) {
+#pragma unroll
+                            for (int j = 0; j < 3; ++j) {
+                                if (i >= ntap<KW, KS>(j)) continue;
+                                float2& q = pend[(u - i + KW) % KW];
+                                q.x = fmaf(tw[j][i].x, du[1 + j].x, q.x);
+                                q.y = fmaf(tw[j][i].y, du[1 + j].y, q.y);
+                            }
+                        }
+                        // token t - (KW - 1) of the same sequence has all its terms
+                        if (has && pos >= KW - 1) {
+                            const long long s = t - (KW - 1);
+                            if (s >= t0 && s < t1) st2(d_out + s * C + c, pend[(u + 1) % KW]);
                         }
                     }
-                    // token t - (KW - 1) has all its terms
-                    const long long s = t - (KW - 1);
-                    if (s >= t0 && s < t1) st2(d_out + s * C + c, pend[(u + 1) % KW]);
                 }
+                pos = next_pos(pos, d.S);
             }
         }
     }
@@ -782,16 +807,16 @@ cudaError_t gram_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtr
 }
 
 template <int KM, int KW, int KS>
-cudaError_t fwd_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, const float* red,
-                   int nslice, const uint16_t* xact, const int* I, const float* p, const float* hpost,
-                   const float* hres, uint16_t* xact_next, uint16_t* X, double* gram, cudaStream_t st) {
+cudaError_t fwd_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, const float* emat,
+                   int nslice, const uint16_t* xact, const int* I, const float* hres,
+                   uint16_t* xact_next, uint16_t* X, cudaStream_t st) {
     const int TB = run_len(KW, 96);
     const size_t sm = sizeof(FRing<KM>) + (size_t)TB * (KM * 4 + KM * KM + KM) * 4;
     cudaError_t e = smem_attr((const void*)k_wb_fwd<KM, KW, KS>, sm);
     if (e != cudaSuccess) return e;
     dim3 grid(nslice, (T + TB - 1) / TB);
-    k_wb_fwd<KM, KW, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, red, nslice, xact, I, p, hpost,
-                                               hres, xact_next, X, gram); note_launch();
+    k_wb_fwd<KM, KW, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, emat, xact, I, hres, xact_next,
+                                               X); note_launch();
     return cudaGetLastError();
 }
 
@@ -846,17 +871,22 @@ cudaError_t launch_wb_gram(const Dims& d, int slot, int T, const uint16_t* out, 
     XHC_KW_DISPATCH(d, (gram_kw<KWC, KSC>(d, slot, T, out, cw, nslice, red, st)));
 }
 
+cudaError_t launch_wb_coef(const Dims& d, int slot, int T, const float* red, int nslice, const float* p,
+                           const float* hpost, double* gram, float* emat, cudaStream_t st) {
+    k_wb_coef<<<(T + 63) / 64, 64, 0, st>>>(d, slot, T, red, nslice, p, hpost, gram, emat); note_launch();
+    return cudaGetLastError();
+}
+
 cudaError_t launch_wb_fwd(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
-                          const float* red, int nslice, const uint16_t* xact, const int* I,
-                          const float* p, const float* hpost, const float* hres,
-                          uint16_t* xact_next, uint16_t* X, double* gram, cudaStream_t st) {
+                          const float* emat, int nslice, const uint16_t* xact, const int* I,
+                          const float* hres, uint16_t* xact_next, uint16_t* X, cudaStream_t st) {
     const bool conv = d.K[slot] > 1;
     if (d.k <= 4) {
-        if (!conv) return fwd_kw<4, 0, 0>(d, slot, T, out, cw, red, nslice, xact, I, p, hpost, hres, xact_next, X, gram, st);
-        XHC_KW_DISPATCH(d, (fwd_kw<4, KWC, KSC>(d, slot, T, out, cw, red, nslice, xact, I, p, hpost, hres, xact_next, X, gram, st)));
+        if (!conv) return fwd_kw<4, 0, 0>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st);
+        XHC_KW_DISPATCH(d, (fwd_kw<4, KWC, KSC>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st)));
     }
-    if (!conv) return fwd_kw<8, 0, 0>(d, slot, T, out, cw, red, nslice, xact, I, p, hpost, hres, xact_next, X, gram, st);
-    XHC_KW_DISPATCH(d, (fwd_kw<8, KWC, KSC>(d, slot, T, out, cw, red, nslice, xact, I, p, hpost, hres, xact_next, X, gram, st)));
+    if (!conv) return fwd_kw<8, 0, 0>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st);
+    XHC_KW_DISPATCH(d, (fwd_kw<8, KWC, KSC>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st)));
 }
 
 cudaError_t launch_wb_bred(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,

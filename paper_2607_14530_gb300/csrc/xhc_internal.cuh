@@ -260,10 +260,11 @@ int wb_nslice(int C);
 int wb_dw_run(const Dims& d);
 cudaError_t launch_wb_gram(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
                            int nslice, float* red, cudaStream_t st);
+cudaError_t launch_wb_coef(const Dims& d, int slot, int T, const float* red, int nslice, const float* p,
+                           const float* hpost, double* gram, float* emat, cudaStream_t st);
 cudaError_t launch_wb_fwd(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
-                          const float* red, int nslice, const uint16_t* xact, const int* I,
-                          const float* p, const float* hpost, const float* hres,
-                          uint16_t* xact_next, uint16_t* X, double* gram, cudaStream_t st);
+                          const float* emat, int nslice, const uint16_t* xact, const int* I,
+                          const float* hres, uint16_t* xact_next, uint16_t* X, cudaStream_t st);
 cudaError_t launch_wb_bred(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
                            const uint16_t* dX, const int* I, const float* dxact,
                            const uint16_t* xact, int nslice, float* red, cudaStream_t st);
