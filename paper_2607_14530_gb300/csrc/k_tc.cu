@@ -558,6 +558,14 @@ constexpr int DX_BN = 128;
 constexpr int DX_EW = 16;                       // epilogue warps: 4 per TMEM lane quarter
 constexpr int DX_THREADS = (2 + DX_EW) * 32;    // + TMA warp + MMA warp
 
+// 16-byte global read (plain LDG: measured faster here than the non-coherent or no-allocate forms)
+__device__ __forceinline__ uint4 ld_stream(const void* p) {
+    uint4 r;
+    asm volatile("ld.global.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "l"(p));
+    return r;
+}
+
 struct DxArgs {
     int T, C, N, k, G;
     int slot;             // active epilogue: slot of the pre-map
@@ -701,6 +709,42 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
                 m[0] = __int_as_float(j); m[1] = h[0]; m[2] = h[1]; m[3] = h[2]; m[4] = h[3];
                 m[5] = sa; m[6] = sb;
             }
+            __syncwarp();
+            // 4 passes of 8 rows; lane -> row rr = 8 pass + lane / 4, channels 8 (lane % 4) ..
+            // The global reads of passes 0-1 are issued before the accumulator is waited for, so
+            // they overlap the MMA and the TMEM read-out; those of passes 2-3 follow the read-out.
+            const int cq = (lane & 3) * 8;
+            const int c = ct * DX_BN + cg * 32 + cq;
+            uint4 xr[4], br[4], br2[4], gr[4];
+            auto load_pass = [&](int pass) {
+                const int rr = pass * 8 + (lane >> 2);
+                const int t = tt * BM + quarter * 32 + rr;
+                xr[pass] = make_uint4(0, 0, 0, 0);
+                br[pass] = xr[pass];
+                br2[pass] = xr[pass];
+                gr[pass] = xr[pass];
+                if (t >= a.T) return;
+                if (ACT) {
+                    const long long row = ((long long)t * a.k + i) * a.C + c;
+                    br[pass] = ld_stream(a.dxa + row);
+                    br2[pass] = ld_stream(a.dxa + row + 4);
+                    gr[pass] = ld_stream(a.dinput + (long long)t * a.C + c);
+                    xr[pass] = ld_stream(a.X + row);
+                } else {
+                    const int j = __float_as_int(meta[rr * 8]);
+                    const long long off = ((long long)t * a.N + i) * a.C + c;
+                    xr[pass] = ld_stream(a.X + off);
+                    if (j >= 0) {
+                        const float* b = a.dxact + ((long long)t * a.k + j) * a.C + c;
+                        br[pass] = ld_stream(b);
+                        br2[pass] = ld_stream(b + 4);
+                    } else {
+                        br[pass] = ld_stream(a.dX + off);
+                    }
+                }
+            };
+            load_pass(0);
+            load_pass(1);
             if (!mbar_wait(smem_u32(&bars[4 + s]), (uint32_t)((n >> 1) & 1))) {
                 atomicExch(a.err, 14);
                 break;
@@ -719,99 +763,55 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&bars[6 + s]));  // TMEM buffer free
-            // 4 passes of 8 rows; lane -> row rr = 8 pass + lane / 4, channels 8 (lane % 4) ..
-            // Every pass's reads are issued before any write.
-            const int cq = (lane & 3) * 8;
-            const int c = ct * DX_BN + cg * 32 + cq;
-            if (ACT) {
-                // dX_act[t][i][c..c+8) += acc + h din[t][c..c+8)   (i = active slot here)
-                float4 b0[4], b1[4];
-                uint4 gr[4], xr[4];
-#pragma unroll
-                for (int pass = 0; pass < 4; ++pass) {
-                    const int rr = pass * 8 + (lane >> 2);
-                    const int t = tt * BM + quarter * 32 + rr;
-                    b0[pass] = make_float4(0.f, 0.f, 0.f, 0.f);
-                    b1[pass] = b0[pass];
-                    gr[pass] = make_uint4(0, 0, 0, 0);
-                    xr[pass] = gr[pass];
-                    if (t >= a.T) continue;
-                    const long long row = ((long long)t * a.k + i) * a.C + c;
-                    const float4* b = reinterpret_cast<const float4*>(a.dxa + row);
-                    b0[pass] = b[0];
-                    b1[pass] = b[1];
-                    gr[pass] = __ldg(reinterpret_cast<const uint4*>(a.dinput + (long long)t * a.C + c));
-                    xr[pass] = __ldg(reinterpret_cast<const uint4*>(a.X + row));
-                }
-#pragma unroll
-                for (int pass = 0; pass < 4; ++pass) {
-                    const int rr = pass * 8 + (lane >> 2);
-                    const int t = tt * BM + quarter * 32 + rr;
-                    if (t >= a.T) continue;
-                    const float hq = meta[rr * 8 + 1], cx = meta[rr * 8 + 2];
-                    float g[8], x[8];
-                    unpack8(gr[pass], g);
-                    unpack8(xr[pass], x);
-                    const float* ac = tileb + rr * 33 + cq;
-                    float4 o0, o1;
-                    o0.x = b0[pass].x + ac[0] + (hq * g[0] - cx * x[0]);
-                    o0.y = b0[pass].y + ac[1] + (hq * g[1] - cx * x[1]);
-                    o0.z = b0[pass].z + ac[2] + (hq * g[2] - cx * x[2]);
-                    o0.w = b0[pass].w + ac[3] + (hq * g[3] - cx * x[3]);
-                    o1.x = b1[pass].x + ac[4] + (hq * g[4] - cx * x[4]);
-                    o1.y = b1[pass].y + ac[5] + (hq * g[5] - cx * x[5]);
-                    o1.z = b1[pass].z + ac[6] + (hq * g[6] - cx * x[6]);
-                    o1.w = b1[pass].w + ac[7] + (hq * g[7] - cx * x[7]);
-                    float4* dst = reinterpret_cast<float4*>(a.dxa + ((long long)t * a.k + i) * a.C + c);
-                    dst[0] = o0;
-                    dst[1] = o1;
-                }
-                __syncwarp();
-                continue;
-            }
-            uint4 xr[4], br[4], br2[4];
-#pragma unroll
-            for (int pass = 0; pass < 4; ++pass) {
-                const int rr = pass * 8 + (lane >> 2);
-                const int t = tt * BM + quarter * 32 + rr;
-                xr[pass] = make_uint4(0, 0, 0, 0);
-                br[pass] = make_uint4(0, 0, 0, 0);
-                br2[pass] = make_uint4(0, 0, 0, 0);
-                if (t >= a.T) continue;
-                const int j = __float_as_int(meta[rr * 8]);
-                const long long off = ((long long)t * a.N + i) * a.C + c;
-                xr[pass] = __ldg(reinterpret_cast<const uint4*>(a.X + off));
-                if (j >= 0) {
-                    const uint4* b = reinterpret_cast<const uint4*>(a.dxact + ((long long)t * a.k + j) * a.C + c);
-                    br[pass] = b[0];
-                    br2[pass] = b[1];
-                } else {
-                    br[pass] = *reinterpret_cast<const uint4*>(a.dX + off);
-                }
-            }
+            load_pass(2);
+            load_pass(3);
 #pragma unroll
             for (int pass = 0; pass < 4; ++pass) {
                 const int rr = pass * 8 + (lane >> 2);
                 const int t = tt * BM + quarter * 32 + rr;
                 if (t >= a.T) continue;
                 const float* m = meta + rr * 8;
-                const int j = __float_as_int(m[0]);
-                const long long off = ((long long)t * a.N + i) * a.C + c;
+                const float* ac = tileb + rr * 33 + cq;
                 float x[8], v[8];
                 unpack8(xr[pass], x);
-                if (j >= 0) {
+                if (ACT) {
+                    // dX_act[t][i][c..c+8) += acc + h din[t][c..c+8) - cx x   (i = active slot here)
+                    const float hq = m[1], cx = m[2];
+                    float g[8];
+                    unpack8(gr[pass], g);
                     v[0] = __uint_as_float(br[pass].x); v[1] = __uint_as_float(br[pass].y);
                     v[2] = __uint_as_float(br[pass].z); v[3] = __uint_as_float(br[pass].w);
                     v[4] = __uint_as_float(br2[pass].x); v[5] = __uint_as_float(br2[pass].y);
                     v[6] = __uint_as_float(br2[pass].z); v[7] = __uint_as_float(br2[pass].w);
+                    float4 o0, o1;
+                    o0.x = v[0] + ac[0] + (hq * g[0] - cx * x[0]);
+                    o0.y = v[1] + ac[1] + (hq * g[1] - cx * x[1]);
+                    o0.z = v[2] + ac[2] + (hq * g[2] - cx * x[2]);
+                    o0.w = v[3] + ac[3] + (hq * g[3] - cx * x[3]);
+                    o1.x = v[4] + ac[4] + (hq * g[4] - cx * x[4]);
+                    o1.y = v[5] + ac[5] + (hq * g[5] - cx * x[5]);
+                    o1.z = v[6] + ac[6] + (hq * g[6] - cx * x[6]);
+                    o1.w = v[7] + ac[7] + (hq * g[7] - cx * x[7]);
+                    float4* dst = reinterpret_cast<float4*>(a.dxa + ((long long)t * a.k + i) * a.C + c);
+                    dst[0] = o0;
+                    dst[1] = o1;
                 } else {
-                    unpack8(br[pass], v);
-                }
-                const float sa = m[5], sb = m[6];
-                float o[8];
+                    const int j = __float_as_int(m[0]);
+                    const long long off = ((long long)t * a.N + i) * a.C + c;
+                    if (j >= 0) {
+                        v[0] = __uint_as_float(br[pass].x); v[1] = __uint_as_float(br[pass].y);
+                        v[2] = __uint_as_float(br[pass].z); v[3] = __uint_as_float(br[pass].w);
+                        v[4] = __uint_as_float(br2[pass].x); v[5] = __uint_as_float(br2[pass].y);
+                        v[6] = __uint_as_float(br2[pass].z); v[7] = __uint_as_float(br2[pass].w);
+                    } else {
+                        unpack8(br[pass], v);
+                    }
+                    const float sa = m[5], sb = m[6];
+                    float o[8];
 #pragma unroll
-                for (int e = 0; e < 8; ++e) o[e] = v[e] + tileb[rr * 33 + cq + e] + sa + sb * x[e];
-                *reinterpret_cast<uint4*>(a.dX + off) = pack8(o);
+                    for (int e = 0; e < 8; ++e) o[e] = v[e] + ac[e] + sa + sb * x[e];
+                    *reinterpret_cast<uint4*>(a.dX + off) = pack8(o);
+                }
             }
             __syncwarp();
         }
