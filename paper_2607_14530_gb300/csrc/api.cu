@@ -162,8 +162,7 @@ Layout make_layout(const Dims& d, int64_t T) {
     const int ts_act = pick_tsplits(d.k * d.C, (int)T);
     L.tsplits = std::max(ts_full, ts_act);
     {
-        const int run = d.nconv > 0 ? wb_dw_run(d) : 128;
-        L.ntiles = (int)((T + run - 1) / run);
+        L.ntiles = d.nconv > 0 ? wb_conv_runs(d, T) : 1;
     }
     o = 0;
     L.err = o; o = al(o + 256);

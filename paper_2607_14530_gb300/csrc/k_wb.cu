@@ -3,8 +3,8 @@
 // Every kernel here walks a run of consecutive tokens for one pair of channels per thread.  The
 // conv taps of the pair and a ring of the last KW values of `out` stay in registers; the token
 // loop is unrolled by KW so the ring positions are compile-time constants, and each out value
-// is loaded once per run instead of once per tap.  The ring is zeroed at every sequence start,
-// so the conv (which never reaches into the previous sequence) needs no per-tap test.  KS = 1
+// is loaded once per run instead of once per tap.  Runs never cross a sequence boundary (Sec.
+// 3.3.4: the conv restarts with every sequence), so the conv needs no per-tap test.  KS = 1
 // specialises the tap counts to the (4, 8, 12) kernels of the MLP sublayers, so no FMA is spent
 // on zero taps.  Per-token reductions over the channels use a reduce-scatter butterfly inside
 // the warp (about V shuffles for V values instead of 5 V), then shared memory across warps.
@@ -58,8 +58,28 @@ __device__ __forceinline__ float2 u2f2(uint32_t u) {
     return make_float2(__uint_as_float(u << 16), __uint_as_float(u & 0xffff0000u));
 }
 
-// position within the sequence of the next token
-__device__ __forceinline__ int next_pos(int pos, int S) { return (pos + 1 == S) ? 0 : pos + 1; }
+// Runs of tokens: with a conv (KW > 0) every run lies inside one sequence (runs of TB tokens
+// from each sequence start, the last one shorter), so a conv window never crosses a run's
+// sequence boundary except at the run start; without a conv, runs of TB tokens.
+template <int KW>
+__device__ __forceinline__ void run_bounds(const Dims& d, int T, int TB, long long& t0, long long& t1,
+                                           long long& send, int& pos0) {
+    if constexpr (KW == 0) {
+        t0 = (long long)blockIdx.y * TB;
+        t1 = min((long long)T, t0 + TB);
+        send = t1;
+        pos0 = 0;
+    } else {
+        const int rps = (d.S + TB - 1) / TB;
+        const long long seq = blockIdx.y / rps;
+        const int r = (int)(blockIdx.y - seq * rps);
+        const long long s0 = seq * d.S;
+        send = min((long long)T, s0 + d.S);
+        pos0 = r * TB;
+        t0 = s0 + pos0;
+        t1 = min(send, t0 + TB);
+    }
+}
 
 // taps of component j held in registers: KS = 1 is the (4, 8, 12) kernel set, else KW each
 template <int KW, int KS>
@@ -81,25 +101,14 @@ __device__ __forceinline__ void taps_reg(const Dims& d, const ConvPtrs& cw, int 
         }
 }
 
-// ring w[s] = out[t] for t = s (mod KW); prepares the run starting at t0 (t0 % KW == 0), whose
-// position in its sequence is pos0: values before the sequence start are zero
+// ring w[s] = out[t] for t - t0 = s (mod KW); prepares the run starting at t0, whose position in
+// its sequence is pos0: values before the sequence start are zero
 template <int KW>
 __device__ __forceinline__ void ring_init(const uint16_t* out, int C, int c, bool act, long long t0,
                                           int pos0, float2 (&w)[KW]) {
     w[0] = f2z();
 #pragma unroll
     for (int i = 1; i < KW; ++i) w[KW - i] = (act && i <= pos0) ? ld2(out + (t0 - i) * C + c) : f2z();
-}
-
-// store out[t] at slot U; at a sequence start the older slots are cleared
-template <int KW>
-__device__ __forceinline__ void ring_push(float2 (&w)[KW], int U, float2 o, bool seq_start) {
-    w[U] = o;
-    if (seq_start) {
-#pragma unroll
-        for (int s = 0; s < KW; ++s)
-            if (s != U) w[s] = f2z();
-    }
 }
 
 // g_j = sum_i tw[j][i] out[t - i], with out[t - i] at ring slot (U - i) mod KW
@@ -164,23 +173,24 @@ __global__ void __launch_bounds__(WT) k_wb_gram(Dims d, int slot, int T, int TB,
     const int slice = blockIdx.x, C = d.C;
     const int c = slice * WSL + 2 * threadIdx.x;
     const bool act = c < C;
-    const long long t0 = (long long)blockIdx.y * TB;
-    const long long t1 = min((long long)T, t0 + TB);
+    long long t0, t1, send;
+    int pos0;
+    run_bounds<KW>(d, T, TB, t0, t1, send, pos0);
+    const int n1 = (int)(t1 - t0);
     const int K = d.K[slot];
     const int nq = K * (K + 1) / 2;
-    int pos = (int)(t0 % d.S);
     float2 tw[3][KW], w[KW];
     taps_reg<KW, KS>(d, cw, c, act, tw);
-    ring_init<KW>(out, C, c, act, t0, pos, w);
+    ring_init<KW>(out, C, c, act, t0, pos0, w);
     const uint16_t* po = out + t0 * C + c;
-    for (long long tb = t0; tb < t1; tb += KW) {
+    for (int tb = 0; tb < n1; tb += KW) {
 #pragma unroll
         for (int u = 0; u < KW; ++u) {
-            const long long t = tb + u;
-            if (t < t1) {
+            const int tt = tb + u;
+            if (tt < n1) {
                 const float2 o = act ? ld2(po) : f2z();
                 po += C;
-                ring_push<KW>(w, u, o, pos == 0);
+                w[u] = o;
                 float2 g[3];
                 conv_ring<KW, KS>(tw, w, u, g);
                 const float2 uu[4] = {o, g[0], g[1], g[2]};
@@ -193,8 +203,7 @@ __global__ void __launch_bounds__(WT) k_wb_gram(Dims d, int slot, int T, int TB,
 #pragma unroll
                 for (int r = 10; r < 16; ++r) v[r] = 0.f;
                 const float tot = WRed<16, 16>::run(v, lane);
-                if ((lane & 1) == 0) wsh[((t - t0) * (WT / 32) + warp) * 16 + (lane >> 1)] = tot;
-                pos = next_pos(pos, d.S);
+                if ((lane & 1) == 0) wsh[(tt * (WT / 32) + warp) * 16 + (lane >> 1)] = tot;
             }
         }
     }
@@ -282,8 +291,9 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
     float* Esh = reinterpret_cast<float*>(smu + sizeof(FRing<KM>));  // [TB][KM][4]
     float* Hsh = Esh + TB * KM * 4;                                 // [TB][KM][KM]
     int* Ish = reinterpret_cast<int*>(Hsh + TB * KM * KM);           // [TB][KM]
-    const long long t0 = (long long)blockIdx.y * TB;
-    const long long t1 = min((long long)T, t0 + TB);
+    long long t0, t1, send;
+    int pos0;
+    run_bounds<KW>(d, T, TB, t0, t1, send, pos0);
     const int ntok = (int)(t1 - t0);
     const int c = blockIdx.x * WSL + 2 * threadIdx.x;
     const bool act = c < C;
@@ -313,20 +323,20 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
         const int tt = idx / KM, j = idx - tt * KM;
         Ish[idx] = (j < k) ? I[(t0 + tt) * k + j] : 0;
     }
-    int pos = (int)(t0 % d.S);
     float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
     if constexpr (KW > 0) {
         taps_reg<KW, KS>(d, cw, c, act, tw);
-        ring_init<KW>(out, C, c, act, t0, pos, w);
+        ring_init<KW>(out, C, c, act, t0, pos0, w);
     }
+    uint16_t* pX = X + t0 * d.N * C + c;
+    uint16_t* pn = last ? nullptr : xact_next + t0 * k * C + c;
     __syncthreads();
     const int RU = KW > 0 ? KW : 4;
-    for (long long tb = t0; tb < t1; tb += RU) {
+    for (int tb = 0; tb < ntok; tb += RU) {
 #pragma unroll
         for (int u = 0; u < RU; ++u) {
-            const long long t = tb + u;
-            if (t < t1) {
-                const int tt = (int)(t - t0);
+            const int tt = tb + u;
+            if (tt < ntok) {
                 const int sl = u % PD;
                 issue((u + PD - 1) % PD, tt + PD - 1);
                 cpa_wait<PD - 1>();
@@ -334,7 +344,7 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
                     const float2 o = u2f2(R.o[sl][threadIdx.x]);
                     float2 uu[4] = {o, f2z(), f2z(), f2z()};
                     if constexpr (KW > 0) {
-                        ring_push<KW>(w, u, o, pos == 0);
+                        w[u] = o;
                         float2 g[3];
                         conv_ring<KW, KS>(tw, w, u, g);
                         uu[1] = g[0];
@@ -371,12 +381,11 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
                             v = fma2(e.w, uu[3], v);
                         }
                         if (last)
-                            st2(X + (t * d.N + Ish[tt * KM + j]) * C + c, v);
+                            st2(pX + ((long long)tt * d.N + Ish[tt * KM + j]) * C, v);
                         else
-                            st2(xact_next + (t * k + j) * C + c, v);
+                            st2(pn + ((long long)tt * k + j) * C, v);
                     }
                 }
-                pos = next_pos(pos, d.S);
             }
         }
     }
@@ -415,8 +424,9 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
     const int nv = last ? KM * 4 + KM * KM : KM * 4;
     const int c = slice * WSL + 2 * threadIdx.x;
     const bool act = c < C;
-    const long long t0 = (long long)blockIdx.y * TB;
-    const long long t1 = min((long long)T, t0 + TB);
+    long long t0, t1, send;
+    int pos0;
+    run_bounds<KW>(d, T, TB, t0, t1, send, pos0);
     const int ntok = (int)(t1 - t0);
     for (int q = threadIdx.x; q < ntok * KM; q += WT) {
         const int tt = q / KM, j = q - tt * KM;
@@ -445,19 +455,17 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
     };
 #pragma unroll
     for (int q = 0; q < PD - 1; ++q) issue(q, q);
-    int pos = (int)(t0 % d.S);
     float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
     if constexpr (KW > 0) {
         taps_reg<KW, KS>(d, cw, c, act, tw);
-        ring_init<KW>(out, C, c, act, t0, pos, w);
+        ring_init<KW>(out, C, c, act, t0, pos0, w);
     }
     const int RU = KW > 0 ? KW : 4;
-    for (long long tb = t0; tb < t1; tb += RU) {
+    for (int tb = 0; tb < ntok; tb += RU) {
 #pragma unroll
         for (int u = 0; u < RU; ++u) {
-            const long long t = tb + u;
-            if (t < t1) {
-                const int tt = (int)(t - t0);
+            const int tt = tb + u;
+            if (tt < ntok) {
                 const int sl = u % PD;                       // == tt % PD (runs start on a multiple of 4)
                 issue((u + PD - 1) % PD, tt + PD - 1);
                 cpa_wait<PD - 1>();
@@ -472,7 +480,7 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
                     const float2 o = u2f2(R.o[sl][threadIdx.x]);
                     uu[0] = o;
                     if constexpr (KW > 0) {
-                        ring_push<KW>(w, u, o, pos == 0);
+                        w[u] = o;
                         float2 g[3];
                         conv_ring<KW, KS>(tw, w, u, g);
                         uu[1] = g[0];
@@ -518,7 +526,6 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
 #pragma unroll
                     for (int bb = 0; bb < NV / 32; ++bb) dst[bb * 32 + lane] = tot[bb];
                 }
-                pos = next_pos(pos, d.S);
             }
         }
     }
@@ -536,14 +543,13 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
 // ---------------------------------------------------------------------------------------------
 // wb_bapp: du_a = sum_j E[j][a] dXn_j + sum_b D[a][b] u_b (Eq. sparse_write reversed, with the
 // Gram-Schmidt Jacobian in D), never stored:
-//   d_out[s] = du_0[s] + sum_j sum_{i < kappa_j, pos(s) + i < S} w_j[i] du_{1+j}[s + i]
-// (the transpose of the causal conv of Eq. aug) is accumulated in a ring of KW pending outputs.
-// An output is complete once token s + KW - 1 of its sequence has been seen, or when its
-// sequence (or the data) ends: it is stored then, and later terms that land in its ring slot
-// are never stored.  Each run therefore recomputes du for the first KW - 1 tokens of the next
-// run.  The conv weight gradient sum_t du_{1+j}[t] out[t - i] is accumulated per run.  Last
-// slot: dX_act_i = sum_j H_res[j][i] dXn_j.  The -cx x_i term of the active-state gradient is
-// added by the backward of the slot's pre-map.
+//   d_out[s] = du_0[s] + sum_j sum_{i < kappa_j, s + i in the sequence} w_j[i] du_{1+j}[s + i]
+// (the transpose of the causal conv of Eq. aug) is accumulated in a ring of KW pending outputs;
+// output s is complete, and stored, once token s + KW - 1 has been seen (du is taken as zero
+// past the sequence end).  Each run therefore recomputes du for up to KW - 1 tokens after it.
+// The conv weight gradient sum_t du_{1+j}[t] out[t - i] is accumulated per run.  Last slot:
+// dX_act_i = sum_j H_res[j][i] dXn_j.  The -cx x_i term of the active-state gradient is added by
+// the backward of the slot's pre-map.
 
 template <int KM>
 struct ARing {
@@ -561,7 +567,7 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
                                                    float* dxact_out,
                                                    uint16_t* __restrict__ d_out,
                                                    float* __restrict__ cpart) {
-    constexpr int HL = KW > 0 ? KW - 1 : 0;   // tokens of the next run whose du this run needs
+    constexpr int HL = KW > 0 ? KW - 1 : 0;   // tokens after the run whose du the run needs
     constexpr int RU = KW > 0 ? KW : 4;
     extern __shared__ __align__(16) unsigned char smu[];
     ARing<KM>& R = *reinterpret_cast<ARing<KM>*>(smu);
@@ -572,11 +578,12 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
     float* Dsh = Esh + TH * KM * 4;                                 // [TH][4][4]
     float* Hsh = Dsh + TH * 16;                                     // [TH][KM][KM]
     int* Ish = reinterpret_cast<int*>(Hsh + TH * KM * KM);           // [TH][KM]
-    const long long t0 = (long long)blockIdx.y * TB;
-    const long long t1 = min((long long)T, t0 + TB);
-    const long long te = min((long long)T, t1 + HL);                // tokens with data
-    const long long tend = t1 + HL;                                 // loop end (emission lag)
-    const int ntok = (int)(te - t0);
+    long long t0, t1, send;
+    int pos0;
+    run_bounds<KW>(d, T, TB, t0, t1, send, pos0);
+    const int n1 = (int)(t1 - t0);                                  // tokens of the run
+    const int ntok = (int)(min(t1 + HL, send) - t0);                // + the halo inside the sequence
+    const int nloop = n1 + HL;                                      // + the emission lag
     for (int idx = threadIdx.x; idx < ntok * KM * 4; idx += WT) {
         const int tt = idx / (KM * 4), q = idx - tt * (KM * 4);
         Esh[idx] = tokmat[(t0 + tt) * TOKMAT + q];
@@ -603,6 +610,8 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
     const uint16_t* po = out + t0 * C + c;
     const uint16_t* pX = dX + t0 * d.N * C + c;
     const float* pd = dn_in + t0 * k * C + c;
+    float* pxo = dxact_out + t0 * k * C + c;
+    uint16_t* pdo = d_out + t0 * C + c;
     auto issue = [&](int sl, int tn) {
         if (act && tn < ntok) {
             cpa4(&R.o[sl][threadIdx.x], po + (long long)tn * C);
@@ -619,12 +628,11 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
     };
 #pragma unroll
     for (int q = 0; q < PD - 1; ++q) issue(q, q);
-    int pos = (int)(t0 % d.S);
     float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1], pend[KW > 0 ? KW : 1];
     float2 acc[3][KW > 0 ? KW : 1];
     if constexpr (KW > 0) {
         taps_reg<KW, KS>(d, cw, c, act, tw);
-        ring_init<KW>(out, C, c, act, t0, pos, w);
+        ring_init<KW>(out, C, c, act, t0, pos0, w);
 #pragma unroll
         for (int s = 0; s < KW; ++s) pend[s] = f2z();
 #pragma unroll
@@ -632,19 +640,17 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
 #pragma unroll
             for (int i = 0; i < KW; ++i) acc[j][i] = f2z();
     }
-    for (long long tb = t0; tb < tend; tb += RU) {
+    for (int tb = 0; tb < nloop; tb += RU) {
 #pragma unroll
         for (int u = 0; u < RU; ++u) {
-            const long long t = tb + u;
-            if (t < tend) {
-                const int tt = (int)(t - t0);
+            const int tt = tb + u;
+            if (tt < nloop) {
                 const int sl = u % PD;
                 issue((u + PD - 1) % PD, tt + PD - 1);
                 cpa_wait<PD - 1>();
                 if (act) {
-                    const bool has = t < te;
                     float2 du[4] = {f2z(), f2z(), f2z(), f2z()};
-                    if (has) {
+                    if (tt < ntok) {
                         const float2 o = u2f2(R.o[sl][threadIdx.x]);
                         float2 dn[KM];
 #pragma unroll
@@ -668,7 +674,7 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
                             }
                         }
                         if constexpr (KW > 0) {
-                            ring_push<KW>(w, u, o, pos == 0);
+                            w[u] = o;
                             float2 g[3];
                             conv_ring<KW, KS>(tw, w, u, g);
                             const float2 uu[4] = {o, g[0], g[1], g[2]};
@@ -682,7 +688,7 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
                                 du[a] = fma2(m.w, uu[3], du[a]);
                             }
                         }
-                        if (last && t < t1) {
+                        if (last && tt < n1) {
                             const float4* H4 = reinterpret_cast<const float4*>(Hsh + tt * KM * KM);
                             float2 v[KM];
 #pragma unroll
@@ -701,17 +707,16 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
                             }
 #pragma unroll
                             for (int i = 0; i < KM; ++i)
-                                if (i < k) *reinterpret_cast<float2*>(dxact_out + (t * k + i) * C + c) = v[i];
+                                if (i < k) *reinterpret_cast<float2*>(pxo + ((long long)tt * k + i) * C) = v[i];
                         }
                     } else if constexpr (KW > 0) {
-                        w[u] = f2z();
+                        w[u] = f2z();   // past the sequence end
                     }
                     if constexpr (KW == 0) {
-                        if (has) st2(d_out + t * C + c, du[0]);
+                        if (tt < n1) st2(pdo + (long long)tt * C, du[0]);
                     } else {
-                        // conv weight gradient of this run's tokens (the ring is zero before the
-                        // sequence start)
-                        if (t < t1) {
+                        // conv weight gradient of the run's tokens
+                        if (tt < n1) {
 #pragma unroll
                             for (int j = 0; j < 3; ++j)
 #pragma unroll
@@ -721,16 +726,6 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
                                     acc[j][i].x = fmaf(du[1 + j].x, o.x, acc[j][i].x);
                                     acc[j][i].y = fmaf(du[1 + j].y, o.y, acc[j][i].y);
                                 }
-                        }
-                        // a sequence starts at t, or the data ends: the pending outputs of the
-                        // finished sequence (the last min(S, pos) or S tokens) are complete
-                        if (pos == 0 || t == T) {
-                            const int lim = (pos == 0) ? d.S : pos;
-#pragma unroll
-                            for (int i = 1; i < KW; ++i) {
-                                const long long s = t - i;
-                                if (i <= lim && s >= t0 && s < t1) st2(d_out + s * C + c, pend[(u - i + KW) % KW]);
-                            }
                         }
                         // d_out[t - i] += w_j[i] du_{1+j}[t]
                         pend[u] = du[0];
@@ -744,14 +739,10 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
                                 q.y = fmaf(tw[j][i].y, du[1 + j].y, q.y);
                             }
                         }
-                        // token t - (KW - 1) of the same sequence has all its terms
-                        if (has && pos >= KW - 1) {
-                            const long long s = t - (KW - 1);
-                            if (s >= t0 && s < t1) st2(d_out + s * C + c, pend[(u + 1) % KW]);
-                        }
+                        // token tt - (KW - 1) has all its terms (du is zero past the sequence end)
+                        if (tt >= KW - 1) st2(pdo + (long long)(tt - (KW - 1)) * C, pend[(u + 1) % KW]);
                     }
                 }
-                pos = next_pos(pos, d.S);
             }
         }
     }
@@ -789,6 +780,17 @@ int run_len(int KW, int per) {  // tokens per CTA run: a multiple of KW near `pe
     return r < u ? u : r;
 }
 
+// number of runs of TB tokens (with a conv: runs inside each sequence of S tokens)
+long long n_runs(const Dims& d, int T, int TB, bool conv) {
+    if (!conv || d.S <= 0) return ((long long)T + TB - 1) / TB;
+    const long long rps = (d.S + TB - 1) / TB;
+    const long long rem = T % d.S;
+    return (T / d.S) * rps + (rem + TB - 1) / TB;
+}
+
+// tokens per run of the backward apply (longer runs amortise the KW - 1 recomputed tokens)
+int bapp_run(int KW) { return KW > 0 ? run_len(KW, 240) : 64; }
+
 cudaError_t smem_attr(const void* fn, size_t bytes) {
     if (bytes <= 48 * 1024) return cudaSuccess;
     return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
@@ -801,7 +803,7 @@ cudaError_t gram_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtr
     const size_t sm = (size_t)TB * (WT / 32) * 16 * sizeof(float);
     cudaError_t e = smem_attr((const void*)k_wb_gram<KW, KS>, sm);
     if (e != cudaSuccess) return e;
-    dim3 grid(nslice, (T + TB - 1) / TB);
+    dim3 grid(nslice, (unsigned)n_runs(d, T, TB, true));
     k_wb_gram<KW, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, nslice, red); note_launch();
     return cudaGetLastError();
 }
@@ -814,7 +816,7 @@ cudaError_t fwd_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs
     const size_t sm = sizeof(FRing<KM>) + (size_t)TB * (KM * 4 + KM * KM + KM) * 4;
     cudaError_t e = smem_attr((const void*)k_wb_fwd<KM, KW, KS>, sm);
     if (e != cudaSuccess) return e;
-    dim3 grid(nslice, (T + TB - 1) / TB);
+    dim3 grid(nslice, (unsigned)n_runs(d, T, TB, KW > 0));
     k_wb_fwd<KM, KW, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, emat, xact, I, hres, xact_next,
                                                X); note_launch();
     return cudaGetLastError();
@@ -830,7 +832,7 @@ cudaError_t bred_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtr
     const size_t sm = sizeof(BRing<KM>) + (size_t)TB * KM * 4 + (size_t)TB * (WT / 32) * NVP * sizeof(float);
     cudaError_t e = smem_attr((const void*)k_wb_bred<KM, KW, NV, KS>, sm);
     if (e != cudaSuccess) return e;
-    dim3 grid(nslice, (T + TB - 1) / TB);
+    dim3 grid(nslice, (unsigned)n_runs(d, T, TB, KW > 0));
     k_wb_bred<KM, KW, NV, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, dX, I, dxact, xact, nslice, red); note_launch();
     return cudaGetLastError();
 }
@@ -839,12 +841,12 @@ template <int KM, int KW, int KS>
 cudaError_t bapp_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, const uint16_t* dX,
                     const int* I, const float* dn_in, const float* tokmat, float* dxact_out,
                     uint16_t* d_out, float* cpart, int nslice, cudaStream_t st) {
-    const int TB = KW > 0 ? run_len(KW, 128) : 64;
+    const int TB = bapp_run(KW);
     const int TH = TB + (KW > 0 ? KW - 1 : 0);
     const size_t sm = sizeof(ARing<KM>) + (size_t)TH * (KM * 4 + 16 + KM * KM + KM) * 4;
     cudaError_t e = smem_attr((const void*)k_wb_bapp<KM, KW, KS>, sm);
     if (e != cudaSuccess) return e;
-    dim3 grid(nslice, (T + TB - 1) / TB);
+    dim3 grid(nslice, (unsigned)n_runs(d, T, TB, KW > 0));
     k_wb_bapp<KM, KW, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, dX, I, dn_in, tokmat, dxact_out,
                                                 d_out, cpart); note_launch();
     return cudaGetLastError();
@@ -853,7 +855,10 @@ cudaError_t bapp_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtr
 }  // namespace
 
 int wb_nslice(int C) { return (C + WSL - 1) / WSL; }
-int wb_dw_run(const Dims& d) { return run_len(kw_of(d), 128); }
+int wb_conv_runs(const Dims& d, int64_t T) {
+    const int KW = kw_of(d);
+    return (int)n_runs(d, (int)T, bapp_run(KW), true);
+}
 
 // KWC: conv taps held per component (0: no conv); KSC: 1 for the (4, 8, 12) kernel set
 #define XHC_KW_DISPATCH(D, CALL)                                              \
