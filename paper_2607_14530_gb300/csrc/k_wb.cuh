@@ -17,6 +17,7 @@
 //   wb_bapp   component gradients du_a consumed on the fly: d_out = du_0 + conv^T(du_1..r)
 //             (emitted KW - 1 tokens late), conv weight-gradient partials, and on the last slot
 //             the mixed active-state gradient H_res^T dXn
+#pragma once
 #include "xhc_internal.cuh"
 
 namespace xhc {
@@ -81,10 +82,13 @@ __device__ __forceinline__ void run_bounds(const Dims& d, int T, int TB, long lo
     }
 }
 
-// taps of component j held in registers: KS = 1 is the (4, 8, 12) kernel set, else KW each
+// Kernel variants: KS = 0 generic; KS = 1 the (4, 8, 12) kernel set of the MLP sublayers (taps
+// of component j held in registers: 4, 8, 12, else KW each); KS = 2 as KS = 1 (or no conv) with,
+// in addition, k equal to the compile-time KM and every thread of a channel slice in range, so
+// that the loops over active slots and the range tests fold away.
 template <int KW, int KS>
 __host__ __device__ constexpr int ntap(int j) {
-    return KS == 1 ? (j == 0 ? 4 : (j == 1 ? 8 : 12)) : KW;
+    return KS >= 1 ? (j == 0 ? 4 : (j == 1 ? 8 : 12)) : KW;
 }
 
 template <int KW, int KS>
@@ -172,7 +176,7 @@ __global__ void __launch_bounds__(WT) k_wb_gram(Dims d, int slot, int T, int TB,
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int slice = blockIdx.x, C = d.C;
     const int c = slice * WSL + 2 * threadIdx.x;
-    const bool act = c < C;
+    const bool act = (KS == 2) || c < C;
     long long t0, t1, send;
     int pos0;
     run_bounds<KW>(d, T, TB, t0, t1, send, pos0);
@@ -219,53 +223,6 @@ __global__ void __launch_bounds__(WT) k_wb_gram(Dims d, int slot, int T, int TB,
 }
 
 // ---------------------------------------------------------------------------------------------
-// wb_coef: one thread per token.  With Gram-Schmidt, the slice partials of the Gram matrix are
-// summed in fp64, kept in `gram` for the backward and turned into the coefficients B of Eq. gs
-// (orthogonalised component q = sum_a B[q][a] u_a), so that the write-back of active slot j is
-// sum_a E[j][a] u_a with E[j][a] = p_j sum_q H_post[j][q] B[q][a]; without it B is the
-// identity.  E goes to the per-token matrix buffer (rows j < k, four entries each).
-
-__global__ void __launch_bounds__(64) k_wb_coef(Dims d, int slot, int T, const float* __restrict__ red,
-                                                int nslice, const float* __restrict__ p,
-                                                const float* __restrict__ hpost,
-                                                double* __restrict__ gram, float* __restrict__ emat) {
-    const int t = blockIdx.x * blockDim.x + threadIdx.x;
-    if (t >= T) return;
-    const int k = d.k, K = d.K[slot];
-    const bool gs = (K > 1) && d.gs;
-    double B[MAXCOMP][MAXCOMP];
-    for (int a = 0; a < MAXCOMP; ++a)
-        for (int b = 0; b < MAXCOMP; ++b) B[a][b] = (a == b) ? 1.0 : 0.0;
-    if (gs) {
-        double Gm[MAXCOMP][MAXCOMP], cc[MAXCOMP][MAXCOMP], vv[MAXCOMP];
-        for (int a = 0; a < MAXCOMP; ++a)
-            for (int b = 0; b < MAXCOMP; ++b) Gm[a][b] = 0.0;
-        for (int sl = 0; sl < nslice; ++sl) {
-            const float* rp = red + ((int64_t)t * nslice + sl) * NRED;
-            int q = 0;
-            for (int a = 0; a < K; ++a)
-                for (int b = 0; b <= a; ++b) Gm[a][b] += (double)rp[q++];
-        }
-        int q = 0;
-        for (int a = 0; a < K; ++a)
-            for (int b = 0; b <= a; ++b) gram[(int64_t)t * NGRAM + q++] = Gm[a][b];
-        for (int a = 0; a < K; ++a)
-            for (int b = a + 1; b < K; ++b) Gm[a][b] = Gm[b][a];
-        gs_coef(Gm, K, (double)d.eps_gs, B, cc, vv);
-    }
-    float* em = emat + (int64_t)t * TOKMAT;
-    for (int j = 0; j < k; ++j) {
-        const float pj = p[(int64_t)t * k + j];
-        for (int a = 0; a < 4; ++a) {
-            float e = 0.f;
-            if (a < K)
-                for (int q = 0; q < K; ++q) e += hpost[((int64_t)t * k + j) * K + q] * (float)B[q][a];
-            em[j * 4 + a] = pj * e;
-        }
-    }
-}
-
-// ---------------------------------------------------------------------------------------------
 // wb_fwd: per-token coefficients E[j][a], H_res and I in shared memory; each thread prefetches
 // the out value and the k active values of its channel pair PD - 1 tokens ahead with cp.async.
 
@@ -286,7 +243,7 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
                                                uint16_t* __restrict__ X) {
     extern __shared__ __align__(16) unsigned char smu[];
     FRing<KM>& R = *reinterpret_cast<FRing<KM>*>(smu);
-    const int k = d.k, C = d.C;
+    const int k = (KS == 2) ? KM : d.k, C = d.C;
     const bool last = (slot == d.G - 1);
     float* Esh = reinterpret_cast<float*>(smu + sizeof(FRing<KM>));  // [TB][KM][4]
     float* Hsh = Esh + TB * KM * 4;                                 // [TB][KM][KM]
@@ -296,7 +253,7 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
     run_bounds<KW>(d, T, TB, t0, t1, send, pos0);
     const int ntok = (int)(t1 - t0);
     const int c = blockIdx.x * WSL + 2 * threadIdx.x;
-    const bool act = c < C;
+    const bool act = (KS == 2) || c < C;
     const uint16_t* po = out + t0 * C + c;
     const uint16_t* px = xact + t0 * k * C + c;
     auto issue = [&](int sl, int tn) {
@@ -419,11 +376,11 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
     int* Ish = reinterpret_cast<int*>(smu + sizeof(BRing<KM>));          // [TB][KM]
     float* wsh = reinterpret_cast<float*>(Ish + TB * KM);                 // [TB][WT/32][NVP]
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int slice = blockIdx.x, C = d.C, k = d.k;
+    const int slice = blockIdx.x, C = d.C, k = (KS == 2) ? KM : d.k;
     const bool last = (slot == d.G - 1);
     const int nv = last ? KM * 4 + KM * KM : KM * 4;
     const int c = slice * WSL + 2 * threadIdx.x;
-    const bool act = c < C;
+    const bool act = (KS == 2) || c < C;
     long long t0, t1, send;
     int pos0;
     run_bounds<KW>(d, T, TB, t0, t1, send, pos0);
@@ -571,7 +528,7 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
     constexpr int RU = KW > 0 ? KW : 4;
     extern __shared__ __align__(16) unsigned char smu[];
     ARing<KM>& R = *reinterpret_cast<ARing<KM>*>(smu);
-    const int k = d.k, C = d.C;
+    const int k = (KS == 2) ? KM : d.k, C = d.C;
     const bool last = (slot == d.G - 1);
     const int TH = TB + HL;
     float* Esh = reinterpret_cast<float*>(smu + sizeof(ARing<KM>));  // [TH][KM][4]
@@ -605,7 +562,7 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
         }
     }
     const int c = blockIdx.x * WSL + 2 * threadIdx.x;
-    const bool act = c < C;
+    const bool act = (KS == 2) || c < C;
     __syncthreads();
     const uint16_t* po = out + t0 * C + c;
     const uint16_t* pX = dX + t0 * d.N * C + c;
@@ -764,24 +721,24 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
     }
 }
 
-int kw_of(const Dims& d) {
+inline int kw_of(const Dims& d) {
     const int km = d.kapmax;
     return km <= 4 ? 4 : km <= 8 ? 8 : km <= 12 ? 12 : 16;
 }
 
 // the (4, 8, 12) kernels of the MLP sublayers
-bool paper_kaps(const Dims& d) {
+inline bool paper_kaps(const Dims& d) {
     return d.nconv == 3 && d.kap[0] == 4 && d.kap[1] == 8 && d.kap[2] == 12;
 }
 
-int run_len(int KW, int per) {  // tokens per CTA run: a multiple of KW near `per`
+inline int run_len(int KW, int per) {  // tokens per CTA run: a multiple of KW near `per`
     const int u = KW > 0 ? KW : 4;
     int r = (per / u) * u;
     return r < u ? u : r;
 }
 
 // number of runs of TB tokens (with a conv: runs inside each sequence of S tokens)
-long long n_runs(const Dims& d, int T, int TB, bool conv) {
+inline long long n_runs(const Dims& d, int T, int TB, bool conv) {
     if (!conv || d.S <= 0) return ((long long)T + TB - 1) / TB;
     const long long rps = (d.S + TB - 1) / TB;
     const long long rem = T % d.S;
@@ -789,142 +746,28 @@ long long n_runs(const Dims& d, int T, int TB, bool conv) {
 }
 
 // tokens per run of the backward apply (longer runs amortise the KW - 1 recomputed tokens)
-int bapp_run(int KW) { return KW > 0 ? run_len(KW, 240) : 64; }
+inline int bapp_run(int KW) { return KW > 0 ? run_len(KW, 240) : 64; }
 
-cudaError_t smem_attr(const void* fn, size_t bytes) {
+inline cudaError_t smem_attr(const void* fn, size_t bytes) {
     if (bytes <= 48 * 1024) return cudaSuccess;
     return cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
 }
 
-template <int KW, int KS>
-cudaError_t gram_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, int nslice,
-                    float* red, cudaStream_t st) {
-    const int TB = run_len(KW, 64);
-    const size_t sm = (size_t)TB * (WT / 32) * 16 * sizeof(float);
-    cudaError_t e = smem_attr((const void*)k_wb_gram<KW, KS>, sm);
-    if (e != cudaSuccess) return e;
-    dim3 grid(nslice, (unsigned)n_runs(d, T, TB, true));
-    k_wb_gram<KW, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, nslice, red); note_launch();
-    return cudaGetLastError();
-}
-
-template <int KM, int KW, int KS>
-cudaError_t fwd_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, const float* emat,
-                   int nslice, const uint16_t* xact, const int* I, const float* hres,
-                   uint16_t* xact_next, uint16_t* X, cudaStream_t st) {
-    const int TB = run_len(KW, 96);
-    const size_t sm = sizeof(FRing<KM>) + (size_t)TB * (KM * 4 + KM * KM + KM) * 4;
-    cudaError_t e = smem_attr((const void*)k_wb_fwd<KM, KW, KS>, sm);
-    if (e != cudaSuccess) return e;
-    dim3 grid(nslice, (unsigned)n_runs(d, T, TB, KW > 0));
-    k_wb_fwd<KM, KW, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, emat, xact, I, hres, xact_next,
-                                               X); note_launch();
-    return cudaGetLastError();
-}
-
-template <int KM, int KW, int NV, int KS>
-cudaError_t bred_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, const uint16_t* dX,
-                    const int* I, const float* dxact, const uint16_t* xact, int nslice, float* red,
-                    cudaStream_t st) {
-    constexpr int NVP = NV < 32 ? 16 : NV;
-    int TB = run_len(KW, 48);
-    while (TB > (KW > 0 ? KW : 4) && (size_t)TB * (WT / 32) * NVP * 4 > 96 * 1024) TB -= (KW > 0 ? KW : 4);
-    const size_t sm = sizeof(BRing<KM>) + (size_t)TB * KM * 4 + (size_t)TB * (WT / 32) * NVP * sizeof(float);
-    cudaError_t e = smem_attr((const void*)k_wb_bred<KM, KW, NV, KS>, sm);
-    if (e != cudaSuccess) return e;
-    dim3 grid(nslice, (unsigned)n_runs(d, T, TB, KW > 0));
-    k_wb_bred<KM, KW, NV, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, dX, I, dxact, xact, nslice, red); note_launch();
-    return cudaGetLastError();
-}
-
-template <int KM, int KW, int KS>
-cudaError_t bapp_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, const uint16_t* dX,
-                    const int* I, const float* dn_in, const float* tokmat, float* dxact_out,
-                    uint16_t* d_out, float* cpart, int nslice, cudaStream_t st) {
-    const int TB = bapp_run(KW);
-    const int TH = TB + (KW > 0 ? KW - 1 : 0);
-    const size_t sm = sizeof(ARing<KM>) + (size_t)TH * (KM * 4 + 16 + KM * KM + KM) * 4;
-    cudaError_t e = smem_attr((const void*)k_wb_bapp<KM, KW, KS>, sm);
-    if (e != cudaSuccess) return e;
-    dim3 grid(nslice, (unsigned)n_runs(d, T, TB, KW > 0));
-    k_wb_bapp<KM, KW, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, dX, I, dn_in, tokmat, dxact_out,
-                                                d_out, cpart); note_launch();
-    return cudaGetLastError();
-}
-
-}  // namespace
-
-int wb_nslice(int C) { return (C + WSL - 1) / WSL; }
-int wb_conv_runs(const Dims& d, int64_t T) {
-    const int KW = kw_of(d);
-    return (int)n_runs(d, (int)T, bapp_run(KW), true);
-}
-
-// KWC: conv taps held per component (0: no conv); KSC: 1 for the (4, 8, 12) kernel set
-#define XHC_KW_DISPATCH(D, CALL)                                              \
+// KWC: conv taps held per component (0: no conv); KSC: the kernel variant (see ntap)
+#define XHC_KW_DISPATCH(D, FAST, CALL)                                        \
     switch (kw_of(D)) {                                                       \
         case 4: { constexpr int KWC = 4, KSC = 0; return CALL; }              \
         case 8: { constexpr int KWC = 8, KSC = 0; return CALL; }              \
         case 12:                                                              \
+            if (paper_kaps(D) && (FAST)) { constexpr int KWC = 12, KSC = 2; return CALL; } \
             if (paper_kaps(D)) { constexpr int KWC = 12, KSC = 1; return CALL; } \
-            else { constexpr int KWC = 12, KSC = 0; return CALL; }            \
+            { constexpr int KWC = 12, KSC = 0; return CALL; }                 \
         default: { constexpr int KWC = 16, KSC = 0; return CALL; }            \
     }
 
-cudaError_t launch_wb_gram(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
-                           int nslice, float* red, cudaStream_t st) {
-    XHC_KW_DISPATCH(d, (gram_kw<KWC, KSC>(d, slot, T, out, cw, nslice, red, st)));
-}
+// the KS = 2 variants: four active slots and whole channel slices
+inline bool wb_fast(const Dims& d) { return d.k == 4 && d.C % WSL == 0; }
 
-cudaError_t launch_wb_coef(const Dims& d, int slot, int T, const float* red, int nslice, const float* p,
-                           const float* hpost, double* gram, float* emat, cudaStream_t st) {
-    k_wb_coef<<<(T + 63) / 64, 64, 0, st>>>(d, slot, T, red, nslice, p, hpost, gram, emat); note_launch();
-    return cudaGetLastError();
-}
 
-cudaError_t launch_wb_fwd(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
-                          const float* emat, int nslice, const uint16_t* xact, const int* I,
-                          const float* hres, uint16_t* xact_next, uint16_t* X, cudaStream_t st) {
-    const bool conv = d.K[slot] > 1;
-    if (d.k <= 4) {
-        if (!conv) return fwd_kw<4, 0, 0>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st);
-        XHC_KW_DISPATCH(d, (fwd_kw<4, KWC, KSC>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st)));
-    }
-    if (!conv) return fwd_kw<8, 0, 0>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st);
-    XHC_KW_DISPATCH(d, (fwd_kw<8, KWC, KSC>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st)));
-}
-
-cudaError_t launch_wb_bred(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
-                           const uint16_t* dX, const int* I, const float* dxact,
-                           const uint16_t* xact, int nslice, float* red, cudaStream_t st) {
-    const bool conv = d.K[slot] > 1;
-    const bool last = (slot == d.G - 1);
-#define XHC_BRED(KM_, NV_)                                                                          \
-    do {                                                                                            \
-        if (!conv) return bred_kw<KM_, 0, NV_, 0>(d, slot, T, out, cw, dX, I, dxact, xact, nslice, red, st); \
-        XHC_KW_DISPATCH(d, (bred_kw<KM_, KWC, NV_, KSC>(d, slot, T, out, cw, dX, I, dxact, xact, nslice, red, st))); \
-    } while (0)
-    if (d.k <= 4) {
-        if (last) XHC_BRED(4, 32);
-        XHC_BRED(4, 16);
-    }
-    if (last) XHC_BRED(8, 96);
-    XHC_BRED(8, 32);
-#undef XHC_BRED
-}
-
-cudaError_t launch_wb_bapp(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
-                           const uint16_t* dX, const int* I, const float* dn_in,
-                           const float* tokmat, float* dxact_out, uint16_t* d_out, float* cpart,
-                           cudaStream_t st) {
-    const int nslice = wb_nslice(d.C);
-    const bool conv = d.K[slot] > 1;
-    if (d.k <= 4) {
-        if (!conv) return bapp_kw<4, 0, 0>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st);
-        XHC_KW_DISPATCH(d, (bapp_kw<4, KWC, KSC>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st)));
-    }
-    if (!conv) return bapp_kw<8, 0, 0>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st);
-    XHC_KW_DISPATCH(d, (bapp_kw<8, KWC, KSC>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st)));
-}
-
+}  // namespace
 }  // namespace xhc

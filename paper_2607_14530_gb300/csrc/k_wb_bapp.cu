@@ -1,0 +1,39 @@
+// Launcher of the backward write-back apply (wb_bapp).
+#include "k_wb.cuh"
+
+namespace xhc {
+namespace {
+
+template <int KM, int KW, int KS>
+cudaError_t bapp_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, const uint16_t* dX,
+                    const int* I, const float* dn_in, const float* tokmat, float* dxact_out,
+                    uint16_t* d_out, float* cpart, int nslice, cudaStream_t st) {
+    const int TB = bapp_run(KW);
+    const int TH = TB + (KW > 0 ? KW - 1 : 0);
+    const size_t sm = sizeof(ARing<KM>) + (size_t)TH * (KM * 4 + 16 + KM * KM + KM) * 4;
+    cudaError_t e = smem_attr((const void*)k_wb_bapp<KM, KW, KS>, sm);
+    if (e != cudaSuccess) return e;
+    dim3 grid(nslice, (unsigned)n_runs(d, T, TB, KW > 0));
+    k_wb_bapp<KM, KW, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, dX, I, dn_in, tokmat, dxact_out,
+                                                d_out, cpart); note_launch();
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_wb_bapp(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
+                           const uint16_t* dX, const int* I, const float* dn_in,
+                           const float* tokmat, float* dxact_out, uint16_t* d_out, float* cpart,
+                           cudaStream_t st) {
+    const int nslice = wb_nslice(d.C);
+    const bool conv = d.K[slot] > 1;
+    if (d.k <= 4) {
+        if (!conv && wb_fast(d)) return bapp_kw<4, 0, 2>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st);
+        if (!conv) return bapp_kw<4, 0, 0>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st);
+        XHC_KW_DISPATCH(d, wb_fast(d), (bapp_kw<4, KWC, KSC>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st)));
+    }
+    if (!conv) return bapp_kw<8, 0, 0>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st);
+    XHC_KW_DISPATCH(d, false, (bapp_kw<8, KWC, KSC>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st)));
+}
+
+}  // namespace xhc

@@ -1,0 +1,112 @@
+// Launchers of the forward write-back kernels (wb_gram, wb_coef, wb_fwd).
+#include "k_wb.cuh"
+
+namespace xhc {
+namespace {
+
+// ---------------------------------------------------------------------------------------------
+// wb_coef: one thread per token.  With Gram-Schmidt, the slice partials of the Gram matrix are
+// summed in fp64, kept in `gram` for the backward and turned into the coefficients B of Eq. gs
+// (orthogonalised component q = sum_a B[q][a] u_a), so that the write-back of active slot j is
+// sum_a E[j][a] u_a with E[j][a] = p_j sum_q H_post[j][q] B[q][a]; without it B is the
+// identity.  E goes to the per-token matrix buffer (rows j < k, four entries each).
+
+__global__ void __launch_bounds__(64) k_wb_coef(Dims d, int slot, int T, const float* __restrict__ red,
+                                                int nslice, const float* __restrict__ p,
+                                                const float* __restrict__ hpost,
+                                                double* __restrict__ gram, float* __restrict__ emat) {
+    const int t = blockIdx.x * blockDim.x + threadIdx.x;
+    if (t >= T) return;
+    const int k = d.k, K = d.K[slot];
+    const bool gs = (K > 1) && d.gs;
+    double B[MAXCOMP][MAXCOMP];
+    for (int a = 0; a < MAXCOMP; ++a)
+        for (int b = 0; b < MAXCOMP; ++b) B[a][b] = (a == b) ? 1.0 : 0.0;
+    if (gs) {
+        double Gm[MAXCOMP][MAXCOMP], cc[MAXCOMP][MAXCOMP], vv[MAXCOMP];
+        for (int a = 0; a < MAXCOMP; ++a)
+            for (int b = 0; b < MAXCOMP; ++b) Gm[a][b] = 0.0;
+        for (int sl = 0; sl < nslice; ++sl) {
+            const float* rp = red + ((int64_t)t * nslice + sl) * NRED;
+            int q = 0;
+            for (int a = 0; a < K; ++a)
+                for (int b = 0; b <= a; ++b) Gm[a][b] += (double)rp[q++];
+        }
+        int q = 0;
+        for (int a = 0; a < K; ++a)
+            for (int b = 0; b <= a; ++b) gram[(int64_t)t * NGRAM + q++] = Gm[a][b];
+        for (int a = 0; a < K; ++a)
+            for (int b = a + 1; b < K; ++b) Gm[a][b] = Gm[b][a];
+        gs_coef(Gm, K, (double)d.eps_gs, B, cc, vv);
+    }
+    float* em = emat + (int64_t)t * TOKMAT;
+    for (int j = 0; j < k; ++j) {
+        const float pj = p[(int64_t)t * k + j];
+        for (int a = 0; a < 4; ++a) {
+            float e = 0.f;
+            if (a < K)
+                for (int q = 0; q < K; ++q) e += hpost[((int64_t)t * k + j) * K + q] * (float)B[q][a];
+            em[j * 4 + a] = pj * e;
+        }
+    }
+}
+
+template <int KW, int KS>
+cudaError_t gram_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, int nslice,
+                    float* red, cudaStream_t st) {
+    const int TB = run_len(KW, 64);
+    const size_t sm = (size_t)TB * (WT / 32) * 16 * sizeof(float);
+    cudaError_t e = smem_attr((const void*)k_wb_gram<KW, KS>, sm);
+    if (e != cudaSuccess) return e;
+    dim3 grid(nslice, (unsigned)n_runs(d, T, TB, true));
+    k_wb_gram<KW, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, nslice, red); note_launch();
+    return cudaGetLastError();
+}
+
+template <int KM, int KW, int KS>
+cudaError_t fwd_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, const float* emat,
+                   int nslice, const uint16_t* xact, const int* I, const float* hres,
+                   uint16_t* xact_next, uint16_t* X, cudaStream_t st) {
+    const int TB = run_len(KW, 96);
+    const size_t sm = sizeof(FRing<KM>) + (size_t)TB * (KM * 4 + KM * KM + KM) * 4;
+    cudaError_t e = smem_attr((const void*)k_wb_fwd<KM, KW, KS>, sm);
+    if (e != cudaSuccess) return e;
+    dim3 grid(nslice, (unsigned)n_runs(d, T, TB, KW > 0));
+    k_wb_fwd<KM, KW, KS><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, emat, xact, I, hres, xact_next,
+                                               X); note_launch();
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+int wb_nslice(int C) { return (C + WSL - 1) / WSL; }
+int wb_conv_runs(const Dims& d, int64_t T) {
+    const int KW = kw_of(d);
+    return (int)n_runs(d, (int)T, bapp_run(KW), true);
+}
+
+cudaError_t launch_wb_gram(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
+                           int nslice, float* red, cudaStream_t st) {
+    XHC_KW_DISPATCH(d, d.C % WSL == 0, (gram_kw<KWC, KSC>(d, slot, T, out, cw, nslice, red, st)));
+}
+
+cudaError_t launch_wb_coef(const Dims& d, int slot, int T, const float* red, int nslice, const float* p,
+                           const float* hpost, double* gram, float* emat, cudaStream_t st) {
+    k_wb_coef<<<(T + 63) / 64, 64, 0, st>>>(d, slot, T, red, nslice, p, hpost, gram, emat); note_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_wb_fwd(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
+                          const float* emat, int nslice, const uint16_t* xact, const int* I,
+                          const float* hres, uint16_t* xact_next, uint16_t* X, cudaStream_t st) {
+    const bool conv = d.K[slot] > 1;
+    if (d.k <= 4) {
+        if (!conv && wb_fast(d)) return fwd_kw<4, 0, 2>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st);
+        if (!conv) return fwd_kw<4, 0, 0>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st);
+        XHC_KW_DISPATCH(d, wb_fast(d), (fwd_kw<4, KWC, KSC>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st)));
+    }
+    if (!conv) return fwd_kw<8, 0, 0>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st);
+    XHC_KW_DISPATCH(d, false, (fwd_kw<8, KWC, KSC>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st)));
+}
+
+}  // namespace xhc
