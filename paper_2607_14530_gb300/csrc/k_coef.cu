@@ -71,14 +71,27 @@ __device__ __forceinline__ void sinkhorn_fwd(const float (&M)[KM][KM], int k, in
     }
 }
 
-// Reverse mode of sinkhorn_fwd: given dH returns dM (and H).  The iterates are recomputed from
-// the logits for every half-step (no storage), as the paper's backward kernel does.
+// Reverse mode of sinkhorn_fwd: given dH returns dM (and H).  The forward iterates are rebuilt
+// from checkpoints: the matrix entering every L-th half-step is kept in shared memory (ck, laid
+// out [segment][entry][thread] with stride nth), and the half-steps of a segment are replayed
+// from its checkpoint, so the reverse sweep costs O(iters * L) half-steps instead of O(iters^2).
+// The replayed values are bit-identical to the forward ones.
 template <int KM>
-__device__ void sinkhorn_bwd(const float (&M)[KM][KM], int k, int iters,
+__device__ void sinkhorn_bwd(const float (&M)[KM][KM], int k, int iters, int L, float* ck, int nth,
                              const float (&dH)[KM][KM], float (&H)[KM][KM], float (&dM)[KM][KM]) {
+    const int nh = 2 * iters;
     float A[KM][KM], dA[KM][KM];
     sk_init<KM>(M, k, A);
-    for (int h = 0; h < 2 * iters; ++h) sk_half<KM>(A, k, h);
+    for (int h = 0; h < nh; ++h) {
+        if (h % L == 0) {
+            float* c = ck + (size_t)(h / L) * KM * KM * nth;
+#pragma unroll
+            for (int a = 0; a < KM; ++a)
+#pragma unroll
+                for (int b = 0; b < KM; ++b) c[(a * KM + b) * nth] = A[a][b];
+        }
+        sk_half<KM>(A, k, h);
+    }
     // clamp
 #pragma unroll
     for (int a = 0; a < KM; ++a) {
@@ -102,11 +115,16 @@ __device__ void sinkhorn_bwd(const float (&M)[KM][KM], int k, int iters,
             }
         }
     }
-    // half-steps in reverse; B = output of step h = A (current), input recomputed
-    for (int h = 2 * iters - 1; h >= 0; --h) {
+    // half-steps in reverse; the input of step h is replayed from its segment's checkpoint
+    for (int h = nh - 1; h >= 0; --h) {
+        const int h0 = (h / L) * L;
         float In[KM][KM];
-        sk_init<KM>(M, k, In);
-        for (int q = 0; q < h; ++q) sk_half<KM>(In, k, q);
+        const float* c = ck + (size_t)(h / L) * KM * KM * nth;
+#pragma unroll
+        for (int a = 0; a < KM; ++a)
+#pragma unroll
+            for (int b = 0; b < KM; ++b) In[a][b] = c[(a * KM + b) * nth];
+        for (int q = h0; q < h; ++q) sk_half<KM>(In, k, q);
         // output of step h
         float Out[KM][KM];
 #pragma unroll
@@ -297,7 +315,7 @@ template <int KM>
 __global__ void k_bwd_coef(Dims d, int slot, int T, const float* __restrict__ red, int nslice,
                            const float* __restrict__ zact, const float* __restrict__ rs,
                            const float* __restrict__ p, const float* __restrict__ hpost,
-                           const double* __restrict__ gram,
+                           const double* __restrict__ gram, int skL,
                            const float* __restrict__ alpha_post, const float* __restrict__ b_post,
                            const float* __restrict__ alpha_res, const float* __restrict__ b_res,
                            float* __restrict__ tokmat, float* __restrict__ dzs,
@@ -408,7 +426,8 @@ __global__ void k_bwd_coef(Dims d, int slot, int T, const float* __restrict__ re
                 M[a][b] = v ? ar * (za[k * K + a * k + b] * r) + b_res[a * k + b] : 0.f;
                 dH[a][b] = v ? Q[a][b] : 0.f;
             }
-        sinkhorn_bwd<KM>(M, k, d.iters, dH, H, dM);
+        extern __shared__ float sk_ck[];
+        sinkhorn_bwd<KM>(M, k, d.iters, skL, sk_ck + threadIdx.x, blockDim.x, dH, H, dM);
         float dar = 0.f;
 #pragma unroll
         for (int a = 0; a < KM; ++a)
@@ -438,14 +457,28 @@ cudaError_t launch_bwd_coef(const Dims& d, int slot, int T, const float* red, in
                             const float* b_post, const float* alpha_res, const float* b_res,
                             float* tokmat, float* dz, float* dp, float* tokgrad, cudaStream_t st) {
     (void)b_post;
+    // Sinkhorn checkpoints (last slot): segments of L half-steps, at most ~96 KB per block
+    const int KMv = d.k <= 4 ? 4 : 8, nth = 64;
+    const int nh = 2 * d.iters;
+    const int segmax = std::max(1, (96 * 1024) / (KMv * KMv * 4 * nth));
+    const int L = std::max(8, (nh + segmax - 1) / segmax);
+    const int nseg = std::max(1, (nh + L - 1) / L);
+    const size_t sm = (slot == d.G - 1) ? (size_t)nseg * KMv * KMv * 4 * nth : 0;
+    cudaError_t e;
     if (d.k <= 4) {
-        k_bwd_coef<4><<<(T + 63) / 64, 64, 0, st>>>(d, slot, T, red, nslice, zact, rs, p, hpost, gram,
-                                                     alpha_post, b_post, alpha_res, b_res, tokmat,
-                                                     dz, dp, tokgrad); note_launch();
+        if ((e = cudaFuncSetAttribute((const void*)k_bwd_coef<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)std::max<size_t>(sm, 1))) != cudaSuccess)
+            return e;
+        k_bwd_coef<4><<<(T + nth - 1) / nth, nth, sm, st>>>(d, slot, T, red, nslice, zact, rs, p, hpost, gram,
+                                                            L, alpha_post, b_post, alpha_res, b_res, tokmat,
+                                                            dz, dp, tokgrad); note_launch();
     } else {
-        k_bwd_coef<8><<<(T + 63) / 64, 64, 0, st>>>(d, slot, T, red, nslice, zact, rs, p, hpost, gram,
-                                                     alpha_post, b_post, alpha_res, b_res, tokmat,
-                                                     dz, dp, tokgrad); note_launch();
+        if ((e = cudaFuncSetAttribute((const void*)k_bwd_coef<8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)std::max<size_t>(sm, 1))) != cudaSuccess)
+            return e;
+        k_bwd_coef<8><<<(T + nth - 1) / nth, nth, sm, st>>>(d, slot, T, red, nslice, zact, rs, p, hpost, gram,
+                                                            L, alpha_post, b_post, alpha_res, b_res, tokmat,
+                                                            dz, dp, tokgrad); note_launch();
     }
     return cudaGetLastError();
 }
