@@ -607,7 +607,7 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
             mbar_init(smem_u32(&bars[s]), 1);
             mbar_init(smem_u32(&bars[2 + s]), 1);
             mbar_init(smem_u32(&bars[4 + s]), 1);
-            mbar_init(smem_u32(&bars[6 + s]), DX_EW);
+            mbar_init(smem_u32(&bars[6 + s]), DX_EW / 2);  // one group of epilogue warps per buffer
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -671,16 +671,19 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
             }
         }
     } else {
-        // Each epilogue warp owns rows [32 q, 32 q + 32) x columns [32 cg, 32 cg + 32) of the tile.
-        // The accumulator is read row-per-lane from TMEM, bounced through a padded shared tile,
-        // and re-read with 4 lanes per row (8 channels each) so that the global reads and writes
-        // are contiguous along the channels.
-        const int quarter = warp & 3;
-        const int cg = (warp - 2) >> 2;            // column group of 32
+        // Two groups of 8 epilogue warps take alternate tiles (group g: tiles n = g mod 2, TMEM
+        // buffer g), so one group's global reads overlap the other's arithmetic and stores.  In a
+        // group, warp w owns rows [32 (w % 4), +32) and columns [64 (w / 4), +64) of the tile,
+        // taken as two halves of 32 columns.  The accumulator is read row-per-lane from TMEM,
+        // bounced through a padded shared tile and re-read with 4 lanes per row (8 channels each)
+        // so that the global reads and writes are contiguous along the channels.
         const int ew = warp - 2;                   // epilogue warp index
+        const int grp = ew >> 3;                   // tile parity of this warp's group
+        const int quarter = warp & 3;              // TMEM lane quarter (warp id % 4)
+        const int chalf = (ew & 7) >> 2;           // 64-column half of the tile
         float* tileb = reinterpret_cast<float*>(smem + 2 * STAGE + 128) + ew * (32 * 33 + 32 * 8);
         float* meta = tileb + 32 * 33;             // per row: j, h0..h3, sa, sb
-        for (long long n = 0; n < nloc; ++n) {
+        for (long long n = grp; n < nloc; n += 2) {
             const long long tile = blockIdx.x + n * a.P;
             const int i = (int)(tile % a.N);
             const long long rest = tile / a.N;
@@ -710,110 +713,121 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
                 m[5] = sa; m[6] = sb;
             }
             __syncwarp();
-            // 4 passes of 8 rows; lane -> row rr = 8 pass + lane / 4, channels 8 (lane % 4) ..
-            // The global reads of passes 0-1 are issued before the accumulator is waited for, so
-            // they overlap the MMA and the TMEM read-out; those of passes 2-3 follow the read-out.
-            const int cq = (lane & 3) * 8;
-            const int c = ct * DX_BN + cg * 32 + cq;
-            uint4 xr[4], br[4], br2[4], gr[4];
-            auto load_pass = [&](int pass) {
-                const int rr = pass * 8 + (lane >> 2);
-                const int t = tt * BM + quarter * 32 + rr;
-                xr[pass] = make_uint4(0, 0, 0, 0);
-                br[pass] = xr[pass];
-                br2[pass] = xr[pass];
-                gr[pass] = xr[pass];
-                if (t >= a.T) return;
-                if (ACT) {
-                    const long long row = ((long long)t * a.k + i) * a.C + c;
-                    br[pass] = ld_stream(a.dxa + row);
-                    br2[pass] = ld_stream(a.dxa + row + 4);
-                    gr[pass] = ld_stream(a.dinput + (long long)t * a.C + c);
-                    xr[pass] = ld_stream(a.X + row);
-                } else {
-                    const int j = __float_as_int(meta[rr * 8]);
-                    const long long off = ((long long)t * a.N + i) * a.C + c;
-                    xr[pass] = ld_stream(a.X + off);
-                    if (j >= 0) {
-                        const float* b = a.dxact + ((long long)t * a.k + j) * a.C + c;
-                        br[pass] = ld_stream(b);
-                        br2[pass] = ld_stream(b + 4);
-                    } else {
-                        br[pass] = ld_stream(a.dX + off);
-                    }
-                }
-            };
-            load_pass(0);
-            load_pass(1);
-            if (!mbar_wait(smem_u32(&bars[4 + s]), (uint32_t)((n >> 1) & 1))) {
-                atomicExch(a.err, 14);
-                break;
-            }
-            tc_fence_after();
             const uint32_t tl = tmem + (uint32_t)(s * DX_BN) + ((uint32_t)(quarter * 32) << 16);
-            {
-                float acc[16];
-                tmem_ld16(tl + (uint32_t)(cg * 32), acc);
+            bool ok = true;
+#pragma unroll 1
+            for (int hh = 0; hh < 2; ++hh) {
+                const int cg = chalf * 2 + hh;     // column group of 32
+                // 4 passes of 8 rows; lane -> row rr = 8 pass + lane / 4, channels 8 (lane % 4)..
+                // The reads of passes 0-1 are issued before the accumulator is read out.
+                const int cq = (lane & 3) * 8;
+                const int c = ct * DX_BN + cg * 32 + cq;
+                uint4 xr[4], br[4], br2[4], gr[4];
+                auto load_pass = [&](int pass) {
+                    const int rr = pass * 8 + (lane >> 2);
+                    const int t = tt * BM + quarter * 32 + rr;
+                    xr[pass] = make_uint4(0, 0, 0, 0);
+                    br[pass] = xr[pass];
+                    br2[pass] = xr[pass];
+                    gr[pass] = xr[pass];
+                    if (t >= a.T) return;
+                    if (ACT) {
+                        const long long row = ((long long)t * a.k + i) * a.C + c;
+                        br[pass] = ld_stream(a.dxa + row);
+                        br2[pass] = ld_stream(a.dxa + row + 4);
+                        gr[pass] = ld_stream(a.dinput + (long long)t * a.C + c);
+                        xr[pass] = ld_stream(a.X + row);
+                    } else {
+                        const int j = __float_as_int(meta[rr * 8]);
+                        const long long off = ((long long)t * a.N + i) * a.C + c;
+                        xr[pass] = ld_stream(a.X + off);
+                        if (j >= 0) {
+                            const float* bp = a.dxact + ((long long)t * a.k + j) * a.C + c;
+                            br[pass] = ld_stream(bp);
+                            br2[pass] = ld_stream(bp + 4);
+                        } else {
+                            br[pass] = ld_stream(a.dX + off);
+                        }
+                    }
+                };
+                load_pass(0);
+                load_pass(1);
+                if (hh == 0) {
+                    if (!mbar_wait(smem_u32(&bars[4 + s]), (uint32_t)((n >> 1) & 1))) {
+                        atomicExch(a.err, 14);
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                }
+                {
+                    float acc[16];
+                    tmem_ld16(tl + (uint32_t)(cg * 32), acc);
 #pragma unroll
-                for (int e = 0; e < 16; ++e) tileb[lane * 33 + e] = acc[e];
-                tmem_ld16(tl + (uint32_t)(cg * 32 + 16), acc);
+                    for (int e = 0; e < 16; ++e) tileb[lane * 33 + e] = acc[e];
+                    tmem_ld16(tl + (uint32_t)(cg * 32 + 16), acc);
 #pragma unroll
-                for (int e = 0; e < 16; ++e) tileb[lane * 33 + 16 + e] = acc[e];
-            }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&bars[6 + s]));  // TMEM buffer free
-            load_pass(2);
-            load_pass(3);
+                    for (int e = 0; e < 16; ++e) tileb[lane * 33 + 16 + e] = acc[e];
+                }
+                if (hh == 1) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(smem_u32(&bars[6 + s]));  // TMEM buffer free
+                }
+                __syncwarp();
+                load_pass(2);
+                load_pass(3);
 #pragma unroll
-            for (int pass = 0; pass < 4; ++pass) {
-                const int rr = pass * 8 + (lane >> 2);
-                const int t = tt * BM + quarter * 32 + rr;
-                if (t >= a.T) continue;
-                const float* m = meta + rr * 8;
-                const float* ac = tileb + rr * 33 + cq;
-                float x[8], v[8];
-                unpack8(xr[pass], x);
-                if (ACT) {
-                    // dX_act[t][i][c..c+8) += acc + h din[t][c..c+8) - cx x   (i = active slot here)
-                    const float hq = m[1], cx = m[2];
-                    float g[8];
-                    unpack8(gr[pass], g);
-                    v[0] = __uint_as_float(br[pass].x); v[1] = __uint_as_float(br[pass].y);
-                    v[2] = __uint_as_float(br[pass].z); v[3] = __uint_as_float(br[pass].w);
-                    v[4] = __uint_as_float(br2[pass].x); v[5] = __uint_as_float(br2[pass].y);
-                    v[6] = __uint_as_float(br2[pass].z); v[7] = __uint_as_float(br2[pass].w);
-                    float4 o0, o1;
-                    o0.x = v[0] + ac[0] + (hq * g[0] - cx * x[0]);
-                    o0.y = v[1] + ac[1] + (hq * g[1] - cx * x[1]);
-                    o0.z = v[2] + ac[2] + (hq * g[2] - cx * x[2]);
-                    o0.w = v[3] + ac[3] + (hq * g[3] - cx * x[3]);
-                    o1.x = v[4] + ac[4] + (hq * g[4] - cx * x[4]);
-                    o1.y = v[5] + ac[5] + (hq * g[5] - cx * x[5]);
-                    o1.z = v[6] + ac[6] + (hq * g[6] - cx * x[6]);
-                    o1.w = v[7] + ac[7] + (hq * g[7] - cx * x[7]);
-                    float4* dst = reinterpret_cast<float4*>(a.dxa + ((long long)t * a.k + i) * a.C + c);
-                    dst[0] = o0;
-                    dst[1] = o1;
-                } else {
-                    const int j = __float_as_int(m[0]);
-                    const long long off = ((long long)t * a.N + i) * a.C + c;
-                    if (j >= 0) {
+                for (int pass = 0; pass < 4; ++pass) {
+                    const int rr = pass * 8 + (lane >> 2);
+                    const int t = tt * BM + quarter * 32 + rr;
+                    if (t >= a.T) continue;
+                    const float* m = meta + rr * 8;
+                    const float* ac = tileb + rr * 33 + cq;
+                    float x[8], v[8];
+                    unpack8(xr[pass], x);
+                    if (ACT) {
+                        // dX_act[t][i][c..c+8) += acc + h din - cx x   (i = active slot here)
+                        const float hq = m[1], cx = m[2];
+                        float g[8];
+                        unpack8(gr[pass], g);
                         v[0] = __uint_as_float(br[pass].x); v[1] = __uint_as_float(br[pass].y);
                         v[2] = __uint_as_float(br[pass].z); v[3] = __uint_as_float(br[pass].w);
                         v[4] = __uint_as_float(br2[pass].x); v[5] = __uint_as_float(br2[pass].y);
                         v[6] = __uint_as_float(br2[pass].z); v[7] = __uint_as_float(br2[pass].w);
+                        float4 o0, o1;
+                        o0.x = v[0] + ac[0] + (hq * g[0] - cx * x[0]);
+                        o0.y = v[1] + ac[1] + (hq * g[1] - cx * x[1]);
+                        o0.z = v[2] + ac[2] + (hq * g[2] - cx * x[2]);
+                        o0.w = v[3] + ac[3] + (hq * g[3] - cx * x[3]);
+                        o1.x = v[4] + ac[4] + (hq * g[4] - cx * x[4]);
+                        o1.y = v[5] + ac[5] + (hq * g[5] - cx * x[5]);
+                        o1.z = v[6] + ac[6] + (hq * g[6] - cx * x[6]);
+                        o1.w = v[7] + ac[7] + (hq * g[7] - cx * x[7]);
+                        float4* dst = reinterpret_cast<float4*>(a.dxa + ((long long)t * a.k + i) * a.C + c);
+                        dst[0] = o0;
+                        dst[1] = o1;
                     } else {
-                        unpack8(br[pass], v);
-                    }
-                    const float sa = m[5], sb = m[6];
-                    float o[8];
+                        const int j = __float_as_int(m[0]);
+                        const long long off = ((long long)t * a.N + i) * a.C + c;
+                        if (j >= 0) {
+                            v[0] = __uint_as_float(br[pass].x); v[1] = __uint_as_float(br[pass].y);
+                            v[2] = __uint_as_float(br[pass].z); v[3] = __uint_as_float(br[pass].w);
+                            v[4] = __uint_as_float(br2[pass].x); v[5] = __uint_as_float(br2[pass].y);
+                            v[6] = __uint_as_float(br2[pass].z); v[7] = __uint_as_float(br2[pass].w);
+                        } else {
+                            unpack8(br[pass], v);
+                        }
+                        const float sa = m[5], sb = m[6];
+                        float o[8];
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) o[e] = v[e] + ac[e] + sa + sb * x[e];
-                    *reinterpret_cast<uint4*>(a.dX + off) = pack8(o);
+                        for (int e = 0; e < 8; ++e) o[e] = v[e] + ac[e] + sa + sb * x[e];
+                        *reinterpret_cast<uint4*>(a.dX + off) = pack8(o);
+                    }
                 }
+                __syncwarp();
             }
-            __syncwarp();
+            if (!ok) break;
         }
     }
     tc_fence_before();
