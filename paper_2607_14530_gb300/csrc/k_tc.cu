@@ -153,7 +153,7 @@ __device__ __forceinline__ long long range_start(long long W, int P, int c) {
 // A_MN = true : rows of A are state elements e, K = tokens; the A tile is X[t0.., e0..] as stored
 //               (two 64-wide e blocks, MN-major); no statistics (weight gradients).
 template <bool A_MN>
-__global__ void __launch_bounds__(NTHREADS, 1)
+__global__ void __launch_bounds__(NTHREADS, 2)
 k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
           ProjTcArgs a) {
     extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -421,25 +421,27 @@ int proj_tc_nb(int nfull) {
     return nb;
 }
 
+// Two CTAs per SM (each with its own TMA ring and 256 TMEM columns) keep twice the loads in
+// flight; with more than 256 accumulator columns a CTA takes the whole TMEM and runs alone.
 ProjTcPlan plan_proj_tc(int T, int K, int nfull, int nsm) {
     ProjTcPlan p;
     p.KB = (K + BK - 1) / BK;
     p.MT = (T + BM - 1) / BM;
     p.W = (long long)p.KB * p.MT;
-    const int sms = nsm > 0 ? nsm : 148;
+    p.NB = proj_tc_nb(nfull);
+    p.nchunk = p.NB > 256 ? 2 : 1;
+    const int sms = (p.NB <= 256 ? 2 : 1) * (nsm > 0 ? nsm : 148);
     long long P = std::min<long long>(sms, std::max<long long>(1, p.W / 4));
     p.P = (int)P;
     const long long per = p.W / p.P;  // >= 4
     p.nseg = (int)((p.KB + per - 1) / per) + 1;
     if (p.nseg > p.P) p.nseg = p.P;
-    p.NB = proj_tc_nb(nfull);
-    p.nchunk = p.NB > 256 ? 2 : 1;
     return p;
 }
-
 int proj_tc_stages(int NB) {
     const size_t stage = (size_t)BM * BK * 2 + (size_t)NB * BK * 2;
-    int s = (int)((220 * 1024 - 2048) / stage);
+    const size_t budget = (NB <= 256 ? 110 : 220) * 1024;  // two CTAs per SM, or one
+    int s = (int)((budget - 2048) / stage);
     return s > MAXSTAGES ? MAXSTAGES : s;
 }
 
