@@ -841,6 +841,231 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
     }
 }
 
+// ---------------------------------------------------------------------------------------------
+// Full-state dX with TMA-staged epilogue tiles.  Per tile (128 tokens x 128 channels of stream i):
+// the producer loads the MMA operands (one stage) and, into the epilogue stage of the tile's
+// warp group, the X and dX tiles of the stream (two 64-channel boxes each, 128-byte swizzle);
+// the epilogue warps read their row from TMEM (row per lane) and from the staged tiles, write
+// the bf16 result over the X tile, and one thread of the group stores the tile with TMA.  Rows
+// of active streams take their base from dX_act (fp32) with plain loads; the dX tile supplies
+// the base of the other rows.
+
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, uint32_t src, int x, int y) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                     (uint64_t)map), "r"(src), "r"(x), "r"(y)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read0() {
+    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+// named barrier over `nthreads` threads that also returns, to every one of them, the OR of `p`
+__device__ __forceinline__ bool named_bar_or(int id, int nthreads, bool p) {
+    uint32_t r;
+    asm volatile(
+        "{\n .reg .pred a, b;\n setp.ne.u32 a, %3, 0;\n"
+        " barrier.red.or.pred b, %1, %2, a;\n selp.u32 %0, 1, 0, b;\n}\n"
+        : "=r"(r) : "r"(id), "r"(nthreads), "r"((uint32_t)p) : "memory");
+    return r != 0;
+}
+
+constexpr int DXF_TILE = 2 * BM * 64 * 2;   // X (or dX) tile: two 64-channel boxes, 32 KB
+
+__global__ void __launch_bounds__(DX_THREADS, 1)
+k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+         const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmD, DxArgs a) {
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    const uint32_t A_BYTES = (uint32_t)a.nkb * BM * BK * 2;
+    const uint32_t B_BYTES = (uint32_t)a.nkb * DX_BN * BK * 2;
+    const uint32_t OPS = A_BYTES + B_BYTES;
+    unsigned char* epi = smem + OPS;                 // [2 groups][X tile | dX tile]
+    uint64_t* bars = reinterpret_cast<uint64_t*>(epi + 2 * 2 * DXF_TILE);
+    // [0] ops full, [1] ops empty, [2,4) tmem full, [4,6) tmem empty, [6,8) epi full, [8,10) epi empty
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 10);
+    volatile int* s_abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        *s_abort = 0;
+        mbar_init(smem_u32(&bars[0]), 1);
+        mbar_init(smem_u32(&bars[1]), 1);
+        for (int g = 0; g < 2; ++g) {
+            mbar_init(smem_u32(&bars[2 + g]), 1);
+            mbar_init(smem_u32(&bars[4 + g]), DX_EW / 2);
+            mbar_init(smem_u32(&bars[6 + g]), 1);
+            mbar_init(smem_u32(&bars[8 + g]), 1);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(tmem_slot)), "r"(256u) : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const long long nloc = (a.ntiles > blockIdx.x) ? (a.ntiles - 1 - blockIdx.x) / a.P + 1 : 0;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            for (long long n = 0; n < nloc; ++n) {
+                if (*s_abort) break;
+                const long long tile = blockIdx.x + n * a.P;
+                const int i = (int)(tile % a.N);
+                const long long rest = tile / a.N;
+                const int ct = (int)(rest % a.CT), tt = (int)(rest / a.CT);
+                if (n >= 1 && !mbar_wait(smem_u32(&bars[1]), (uint32_t)((n - 1) & 1))) {
+                    atomicExch(a.err, 21);
+                    *s_abort = 1;
+                    break;
+                }
+                const uint32_t full = smem_u32(&bars[0]);
+                mbar_expect_tx(full, OPS);
+                for (int kb = 0; kb < a.nkb; ++kb) {
+                    tma_load_2d(smem_u32(smem + kb * BM * BK * 2), &tmA, kb * BK, tt * BM, full);
+                    tma_load_2d(smem_u32(smem + A_BYTES + kb * DX_BN * BK * 2), &tmB, kb * BK,
+                                i * a.C + ct * DX_BN, full);
+                }
+                const int g = (int)(n & 1);
+                if (n >= 2 && !mbar_wait(smem_u32(&bars[8 + g]), (uint32_t)(((n >> 1) - 1) & 1))) {
+                    atomicExch(a.err, 22);
+                    *s_abort = 1;
+                    break;
+                }
+                const uint32_t ef = smem_u32(&bars[6 + g]);
+                mbar_expect_tx(ef, 2 * DXF_TILE);
+                unsigned char* xt = epi + (size_t)g * 2 * DXF_TILE;
+                for (int h = 0; h < 2; ++h) {
+                    const int x = i * a.C + ct * DX_BN + h * 64;
+                    tma_load_2d(smem_u32(xt + h * (DXF_TILE / 2)), &tmX, x, tt * BM, ef);
+                    tma_load_2d(smem_u32(xt + DXF_TILE + h * (DXF_TILE / 2)), &tmD, x, tt * BM, ef);
+                }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16(BM, DX_BN);
+            for (long long n = 0; n < nloc; ++n) {
+                const int s = (int)(n & 1);
+                if (!mbar_wait(smem_u32(&bars[0]), (uint32_t)(n & 1))) {
+                    atomicExch(a.err, 23);
+                    *s_abort = 1;
+                    break;
+                }
+                if (n >= 2 && !mbar_wait(smem_u32(&bars[4 + s]), (uint32_t)(((n >> 1) - 1) & 1))) {
+                    atomicExch(a.err, 24);
+                    *s_abort = 1;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t abase = smem_u32(smem);
+                const uint32_t bbase = abase + A_BYTES;
+                for (int ks = 0; ks < a.ksteps; ++ks) {
+                    const int kb = ks >> 2, kk = ks & 3;
+                    mma_bf16(tmem + (uint32_t)(s * DX_BN), sw128_desc(abase + kb * BM * BK * 2 + kk * 32),
+                             sw128_desc(bbase + kb * DX_BN * BK * 2 + kk * 32), idesc, ks > 0 ? 1u : 0u);
+                }
+                mma_commit(smem_u32(&bars[1]));       // operands consumed
+                mma_commit(smem_u32(&bars[2 + s]));   // accumulator ready
+            }
+        }
+    } else {
+        // group g = tiles n = g mod 2 (TMEM buffer g, epilogue stage g); in the group, warp w owns
+        // the TMEM lane quarter warp % 4 (rows) and the 64-channel box (w % 8) / 4
+        const int ew = warp - 2;
+        const int grp = ew >> 3;
+        const int quarter = warp & 3;
+        const int box = (ew & 7) >> 2;
+        const int r = quarter * 32 + lane;          // tile row
+        const bool leader = (ew & 7) == 0 && lane == 0;
+        unsigned char* xt = epi + (size_t)grp * 2 * DXF_TILE;
+        unsigned char* xrow = xt + box * (DXF_TILE / 2) + r * 128;                // this row, X box
+        const unsigned char* drow = xt + DXF_TILE + box * (DXF_TILE / 2) + r * 128; // dX box
+        const int sw = r & 7;                                                     // 128B swizzle
+        bool stored = false;
+        for (long long n = grp; n < nloc; n += 2) {
+            const long long tile = blockIdx.x + n * a.P;
+            const int i = (int)(tile % a.N);
+            const long long rest = tile / a.N;
+            const int ct = (int)(rest % a.CT), tt = (int)(rest / a.CT);
+            const int t = tt * BM + r;
+            int j = -1;
+            float sa = 0.f, sb = 0.f;
+            if (t < a.T) {
+                for (int q = 0; q < a.k; ++q)
+                    if (a.I[(long long)t * a.k + q] == i) j = q;
+                sa = a.scal[(long long)t * a.scal_ld + 0];
+                sb = a.scal[(long long)t * a.scal_ld + 1];
+            }
+            bool ok = mbar_wait(smem_u32(&bars[6 + grp]), (uint32_t)((n >> 1) & 1));
+            ok = ok && mbar_wait(smem_u32(&bars[2 + grp]), (uint32_t)((n >> 1) & 1));
+            if (!ok) {
+                atomicExch(a.err, 25);
+                *s_abort = 1;
+            } else {
+                tc_fence_after();
+                const uint32_t tl = tmem + (uint32_t)(grp * DX_BN + box * 64) + ((uint32_t)(quarter * 32) << 16);
+                const float* brow = a.dxact + ((long long)t * a.k + (j < 0 ? 0 : j)) * a.C + ct * DX_BN + box * 64;
+#pragma unroll 1
+                for (int q2 = 0; q2 < 2; ++q2) {
+                    float acc[32];
+                    tmem_ld16(tl + (uint32_t)(q2 * 32), acc);
+                    tmem_ld16(tl + (uint32_t)(q2 * 32 + 16), acc + 16);
+#pragma unroll
+                    for (int cc = 0; cc < 4; ++cc) {
+                        const int q = q2 * 4 + cc;                 // logical 16-byte chunk
+                        const int ph = (q ^ sw) * 16;
+                        float x[8], v[8];
+                        unpack8(*reinterpret_cast<const uint4*>(xrow + ph), x);
+                        if (j >= 0) {
+                            const uint4 b0 = ld_stream(brow + q * 8);
+                            const uint4 b1 = ld_stream(brow + q * 8 + 4);
+                            v[0] = __uint_as_float(b0.x); v[1] = __uint_as_float(b0.y);
+                            v[2] = __uint_as_float(b0.z); v[3] = __uint_as_float(b0.w);
+                            v[4] = __uint_as_float(b1.x); v[5] = __uint_as_float(b1.y);
+                            v[6] = __uint_as_float(b1.z); v[7] = __uint_as_float(b1.w);
+                        } else {
+                            unpack8(*reinterpret_cast<const uint4*>(drow + ph), v);
+                        }
+                        float o[8];
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) o[e] = v[e] + acc[cc * 8 + e] + sa + sb * x[e];
+                        *reinterpret_cast<uint4*>(xrow + ph) = pack8(o);
+                    }
+                }
+                tc_fence_before();
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&bars[4 + grp]));  // TMEM buffer free
+            fence_async_smem();                                     // results visible to TMA
+            if (named_bar_or(1 + grp, (DX_EW / 2) * 32, *s_abort != 0)) break;  // same decision in the group
+            if (leader) {
+                for (int h = 0; h < 2; ++h)
+                    tma_store_2d(&tmD, smem_u32(xt + h * (DXF_TILE / 2)), i * a.C + ct * DX_BN + h * 64, tt * BM);
+                bulk_commit();
+                bulk_wait_read0();                                  // the stage may be reloaded
+                mbar_arrive(smem_u32(&bars[8 + grp]));
+                stored = true;
+            }
+        }
+        if (leader && stored) bulk_wait0();
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(256u)
+                     : "memory");
+    }
+}
+
 // bf16 copies with a padded row stride: dst[r][o] = src[r][o] (o < n), 0 for n <= o < ld
 __global__ void k_pack_rows(WSegs W, int n, int rows, int ld, uint16_t* __restrict__ dst) {
     const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
@@ -953,11 +1178,13 @@ cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, 
     a.P = (int)std::min<long long>(num_sms(), a.ntiles);
     a.X = X; a.dX = dX; a.dinput = dinput; a.hpre = hpre; a.I = I; a.dxact = dxact;
     a.scal = scal; a.scal_ld = scal_ld; a.err = err;
-    const size_t sm = 2 * (size_t)a.nkb * (BM + DX_BN) * BK * 2 + 128 +
-                      (size_t)DX_EW * (32 * 33 + 32 * 8) * 4 + 1024;
-    e = cudaFuncSetAttribute((const void*)k_dx_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    CUtensorMap mx, md;
+    if (!make_map_box(&mx, X, (uint64_t)NC, (uint64_t)T, 64, BM)) return cudaErrorInvalidValue;
+    if (!make_map_box(&md, dX, (uint64_t)NC, (uint64_t)T, 64, BM)) return cudaErrorInvalidValue;
+    const size_t sm = (size_t)a.nkb * (BM + DX_BN) * BK * 2 + 4 * (size_t)DXF_TILE + 128 + 1024;
+    e = cudaFuncSetAttribute((const void*)k_dxf_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
-    k_dx_tc<false><<<a.P, DX_THREADS, sm, st>>>(ma, mb, a); note_launch();
+    k_dxf_tc<<<a.P, DX_THREADS, sm, st>>>(ma, mb, mx, md, a); note_launch();
     return cudaGetLastError();
 }
 
