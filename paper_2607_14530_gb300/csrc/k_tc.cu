@@ -574,6 +574,7 @@ struct DxArgs {
     int NH;               // active epilogue: streams of the H_pre rows
     float* dxa;           // active epilogue: dX_act [T][k][C] fp32, updated in place
     int nkb, ksteps;      // k-blocks of 64, MMA k-steps of 16
+    int ns;               // operand stages in shared memory (1 or 2)
     int TT, CT;           // token tiles, channel tiles per stream
     long long ntiles;
     int P;
@@ -600,8 +601,10 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
     const uint32_t A_BYTES = (uint32_t)a.nkb * BM * BK * 2;
     const uint32_t B_BYTES = (uint32_t)a.nkb * DX_BN * BK * 2;
     const uint32_t STAGE = A_BYTES + B_BYTES;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 2 * STAGE);
-    // [0,2) full, [2,4) empty, [4,6) tmem full, [6,8) tmem empty
+    const int NS = a.ns;                             // operand stages (1 or 2)
+    const int nsh = NS - 1;                          // log2(NS)
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + NS * STAGE);
+    // [0,2) operands full, [2,4) operands empty, [4,6) tmem full, [6,8) tmem empty
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 8);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
@@ -632,8 +635,8 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
                 const int i = (int)(tile % a.N);
                 const long long rest = tile / a.N;
                 const int ct = (int)(rest % a.CT), tt = (int)(rest / a.CT);
-                const int s = (int)(n & 1);
-                if (n >= 2 && !mbar_wait(smem_u32(&bars[2 + s]), (uint32_t)(((n >> 1) - 1) & 1))) {
+                const int s = (int)(n & nsh);
+                if (n >= NS && !mbar_wait(smem_u32(&bars[2 + s]), (uint32_t)(((n >> nsh) - 1) & 1))) {
                     atomicExch(a.err, 11);
                     break;
                 }
@@ -651,8 +654,9 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
         if (lane == 0) {
             const uint32_t idesc = idesc_bf16(BM, DX_BN);
             for (long long n = 0; n < nloc; ++n) {
-                const int s = (int)(n & 1);
-                if (!mbar_wait(smem_u32(&bars[s]), (uint32_t)((n >> 1) & 1))) {
+                const int s = (int)(n & 1);        // TMEM buffer
+                const int os = (int)(n & nsh);     // operand stage
+                if (!mbar_wait(smem_u32(&bars[os]), (uint32_t)((n >> nsh) & 1))) {
                     atomicExch(a.err, 12);
                     break;
                 }
@@ -661,14 +665,14 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
                     break;
                 }
                 tc_fence_after();
-                const uint32_t abase = smem_u32(smem + (size_t)s * STAGE);
+                const uint32_t abase = smem_u32(smem + (size_t)os * STAGE);
                 const uint32_t bbase = abase + A_BYTES;
                 for (int ks = 0; ks < a.ksteps; ++ks) {
                     const int kb = ks >> 2, kk = ks & 3;
                     mma_bf16(tmem + (uint32_t)(s * DX_BN), sw128_desc(abase + kb * BM * BK * 2 + kk * 32),
                              sw128_desc(bbase + kb * DX_BN * BK * 2 + kk * 32), idesc, ks > 0 ? 1u : 0u);
                 }
-                mma_commit(smem_u32(&bars[2 + s]));  // operands consumed
+                mma_commit(smem_u32(&bars[2 + os]));  // operands consumed
                 mma_commit(smem_u32(&bars[4 + s]));  // accumulator ready
             }
         }
@@ -683,7 +687,7 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
         const int grp = ew >> 3;                   // tile parity of this warp's group
         const int quarter = warp & 3;              // TMEM lane quarter (warp id % 4)
         const int chalf = (ew & 7) >> 2;           // 64-column half of the tile
-        float* tileb = reinterpret_cast<float*>(smem + 2 * STAGE + 128) + ew * (32 * 33 + 32 * 8);
+        float* tileb = reinterpret_cast<float*>(smem + NS * STAGE + 128) + ew * (32 * 33 + 32 * 8);
         float* meta = tileb + 32 * 33;             // per row: j, h0..h3, sa, sb
         for (long long n = grp; n < nloc; n += 2) {
             const long long tile = blockIdx.x + n * a.P;
@@ -1136,7 +1140,10 @@ cudaError_t launch_dxa_tc(const Dims& d, int slot, int T, const float* dzs, int 
     a.NH = d.N;
     a.dinput = d_input; a.hpre = hpre; a.I = I; a.dxa = dxact; a.err = err;
     a.X = xact; a.scal = tokmat; a.scal_ld = TOKMAT;
-    const size_t sm = 2 * (size_t)a.nkb * (BM + DX_BN) * BK * 2 + 128 +
+    // one operand stage (the MMA of a tile is short next to its epilogue): the shared memory
+    // left over is L1 for the epilogue's in-flight reads
+    a.ns = 1;
+    const size_t sm = (size_t)a.ns * a.nkb * (BM + DX_BN) * BK * 2 + 128 +
                       (size_t)DX_EW * (32 * 33 + 32 * 8) * 4 + 1024;
     e = cudaFuncSetAttribute((const void*)k_dx_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
