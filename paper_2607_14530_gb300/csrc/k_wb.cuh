@@ -39,6 +39,16 @@ __device__ __forceinline__ float2 fma2(float s, float2 a, float2 acc) {
     return make_float2(fmaf(s, a.x, acc.x), fmaf(s, a.y, acc.y));
 }
 __device__ __forceinline__ float2 f2z() { return make_float2(0.f, 0.f); }
+// a * b + c on both channels of a pair in one packed instruction (each lane rounded as fmaf)
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+    float2 d;
+    asm("{\n .reg .b64 ra, rb, rc, rd;\n"
+        " mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n mov.b64 rc, {%6, %7};\n"
+        " fma.rn.f32x2 rd, ra, rb, rc;\n mov.b64 {%0, %1}, rd;\n}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+    return d;
+}
 __device__ __forceinline__ uint32_t s_u32(const void* p) {
     return (uint32_t)__cvta_generic_to_shared(p);
 }
@@ -127,8 +137,7 @@ __device__ __forceinline__ void conv_ring(const float2 (&tw)[3][KW], const float
 #pragma unroll
         for (int j = 0; j < 3; ++j) {
             if (i >= ntap<KW, KS>(j)) continue;
-            g[j].x = fmaf(tw[j][i].x, o.x, g[j].x);
-            g[j].y = fmaf(tw[j][i].y, o.y, g[j].y);
+            g[j] = ffma2(tw[j][i], o, g[j]);
         }
     }
 }
@@ -680,8 +689,7 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
                                 for (int i = 0; i < KW; ++i) {
                                     if (i >= ntap<KW, KS>(j)) continue;
                                     const float2 o = w[(u - i + KW) % KW];
-                                    acc[j][i].x = fmaf(du[1 + j].x, o.x, acc[j][i].x);
-                                    acc[j][i].y = fmaf(du[1 + j].y, o.y, acc[j][i].y);
+                                    acc[j][i] = ffma2(du[1 + j], o, acc[j][i]);
                                 }
                         }
                         // d_out[t - i] += w_j[i] du_{1+j}[t]
@@ -692,8 +700,7 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
                             for (int j = 0; j < 3; ++j) {
                                 if (i >= ntap<KW, KS>(j)) continue;
                                 float2& q = pend[(u - i + KW) % KW];
-                                q.x = fmaf(tw[j][i].x, du[1 + j].x, q.x);
-                                q.y = fmaf(tw[j][i].y, du[1 + j].y, q.y);
+                                q = ffma2(tw[j][i], du[1 + j], q);
                             }
                         }
                         // token tt - (KW - 1) has all its terms (du is zero past the sequence end)
