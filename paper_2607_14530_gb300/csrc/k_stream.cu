@@ -249,7 +249,9 @@ cudaError_t launch_dinput_act(const Dims& d, int slot, int T, int add_dx, const 
 
 // ---------------------------------------------------------------------------------------------
 // full_dots: for the non-active streams i, dH_pre[t][q][i] = <x_i, d_input_q> and the dense-read
-// gradient dX[t][i] += sum_q H_pre[t][q][i] d_input_q (Eq. dense_read reversed)
+// gradient dX[t][i] += sum_q H_pre[t][q][i] d_input_q (Eq. dense_read reversed).  One CTA per
+// token: the token's G d_input rows are staged in shared memory, then each warp takes whole
+// non-active streams (warp-level reductions only, no block barrier per stream).
 
 __global__ void __launch_bounds__(256) k_full_dots(Dims d, int T, const uint16_t* __restrict__ X,
                                                    const uint16_t* __restrict__ dinput,
@@ -257,61 +259,73 @@ __global__ void __launch_bounds__(256) k_full_dots(Dims d, int T, const uint16_t
                                                    const float* __restrict__ hpre,
                                                    uint16_t* __restrict__ dX,
                                                    float* __restrict__ dhpre) {
-    __shared__ float wsh[8][4];
-    __shared__ int active[MAXN];
+    extern __shared__ __align__(16) uint16_t din[];   // [G][C]
+    __shared__ int list[MAXN];
+    __shared__ int nlist;
     __shared__ float hs[4 * MAXN];
     const int t = blockIdx.x, C = d.C, G = d.G;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int nw = (blockDim.x + 31) / 32;
-    for (int i = threadIdx.x; i < d.N; i += blockDim.x) {
-        int a = 0;
-        for (int q = 0; q < d.k; ++q)
-            if (I[(int64_t)t * d.k + q] == i) a = 1;
-        active[i] = a;
+    const int nw = blockDim.x >> 5;
+    if (threadIdx.x == 0) {
+        int n = 0;
+        for (int i = 0; i < d.N; ++i) {
+            bool a = false;
+            for (int q = 0; q < d.k; ++q)
+                if (I[(int64_t)t * d.k + q] == i) a = true;
+            if (!a) list[n++] = i;
+        }
+        nlist = n;
     }
     for (int q = threadIdx.x; q < G * d.N; q += blockDim.x) hs[q] = hpre[(int64_t)t * G * d.N + q];
+    for (int idx = threadIdx.x; idx < G * C / 8; idx += blockDim.x) {
+        const int q = idx / (C / 8), c8 = idx - q * (C / 8);
+        reinterpret_cast<uint4*>(din)[idx] =
+            *reinterpret_cast<const uint4*>(dinput + ((int64_t)q * T + t) * C + c8 * 8);
+    }
     __syncthreads();
-    for (int i = 0; i < d.N; ++i) {
-        if (active[i]) continue;
+    for (int li = warp; li < nlist; li += nw) {
+        const int i = list[li];
         float acc[4] = {0.f, 0.f, 0.f, 0.f};
-        for (int c8 = threadIdx.x; c8 < C / 8; c8 += blockDim.x) {
+        float h[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) h[q] = (q < G) ? hs[q * d.N + i] : 0.f;
+        const int64_t row = ((int64_t)t * d.N + i) * C;
+#pragma unroll 4
+        for (int c8 = lane; c8 < C / 8; c8 += 32) {
             float x[8], dx[8];
-            const int64_t off = ((int64_t)t * d.N + i) * C + c8 * 8;
-            unpack8(__ldg(reinterpret_cast<const uint4*>(X + off)), x);
-            unpack8(*reinterpret_cast<const uint4*>(dX + off), dx);
+            unpack8(__ldg(reinterpret_cast<const uint4*>(X + row + c8 * 8)), x);
+            unpack8(*reinterpret_cast<const uint4*>(dX + row + c8 * 8), dx);
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 if (q >= G) continue;
                 float g[8];
-                unpack8(*reinterpret_cast<const uint4*>(dinput + ((int64_t)q * T + t) * C + c8 * 8), g);
-                const float h = hs[q * d.N + i];
+                unpack8(reinterpret_cast<const uint4*>(din + q * C)[c8], g);
 #pragma unroll
                 for (int e = 0; e < 8; ++e) {
                     acc[q] = fmaf(x[e], g[e], acc[q]);
-                    dx[e] = fmaf(h, g[e], dx[e]);
+                    dx[e] = fmaf(h[q], g[e], dx[e]);
                 }
             }
-            *reinterpret_cast<uint4*>(dX + off) = pack8(dx);
+            *reinterpret_cast<uint4*>(dX + row + c8 * 8) = pack8(dx);
         }
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
             const float v = warp_sum(acc[q]);
-            if (lane == 0) wsh[warp][q] = v;
+            if (lane == 0 && q < G) dhpre[((int64_t)t * G + q) * d.N + i] = v;
         }
-        __syncthreads();
-        if (threadIdx.x < G) {
-            float s = 0.f;
-            for (int w = 0; w < nw; ++w) s += wsh[w][threadIdx.x];
-            dhpre[((int64_t)t * G + threadIdx.x) * d.N + i] = s;
-        }
-        __syncthreads();
     }
 }
 
 cudaError_t launch_full_dots(const Dims& d, int T, const uint16_t* X, const uint16_t* dinput,
                              const int* I, const float* hpre, uint16_t* dX, float* dhpre,
                              cudaStream_t st) {
-    k_full_dots<<<T, chunk_threads(d.C), 0, st>>>(d, T, X, dinput, I, hpre, dX, dhpre); note_launch();
+    const size_t sm = (size_t)d.G * d.C * 2;
+    if (sm > 48 * 1024) {
+        cudaError_t e = cudaFuncSetAttribute((const void*)k_full_dots, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)sm);
+        if (e != cudaSuccess) return e;
+    }
+    k_full_dots<<<T, 256, sm, st>>>(d, T, X, dinput, I, hpre, dX, dhpre); note_launch();
     return cudaGetLastError();
 }
 
