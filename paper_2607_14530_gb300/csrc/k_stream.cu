@@ -44,26 +44,34 @@ __global__ void __launch_bounds__(256) k_read(Dims d, int T, const uint16_t* __r
         for (int q = 0; q < 4; ++q)
 #pragma unroll
             for (int e = 0; e < 8; ++e) acc[q][e] = 0.f;
-#pragma unroll 4
-        for (int i = 0; i < N; ++i) {
-            const uint4 u = __ldg(reinterpret_cast<const uint4*>(xt + (int64_t)i * C + c8 * 8));
-            float x[8];
-            unpack8(u, x);
-            const int j = slotmap[i];
-            const float h0 = sh[i];
+        // streams in blocks of 8: the block's 8 reads are issued before any is used
+        for (int i0 = 0; i0 < N; i0 += 8) {
+            uint4 ub[8];
 #pragma unroll
-            for (int e = 0; e < 8; ++e) acc[0][e] = fmaf(h0, x[e], acc[0][e]);
-            if (j < 0) {
+            for (int ii = 0; ii < 8; ++ii)
+                if (i0 + ii < N) ub[ii] = __ldg(reinterpret_cast<const uint4*>(xt + (int64_t)(i0 + ii) * C + c8 * 8));
 #pragma unroll
-                for (int q = 1; q < 4; ++q) {
-                    if (q < G) {
-                        const float h = sh[q * N + i];
+            for (int ii = 0; ii < 8; ++ii) {
+                const int i = i0 + ii;
+                if (i >= N) continue;
+                float x[8];
+                unpack8(ub[ii], x);
+                const int j = slotmap[i];
+                const float h0 = sh[i];
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) acc[q][e] = fmaf(h, x[e], acc[q][e]);
+                for (int e = 0; e < 8; ++e) acc[0][e] = fmaf(h0, x[e], acc[0][e]);
+                if (j < 0) {
+#pragma unroll
+                    for (int q = 1; q < 4; ++q) {
+                        if (q < G) {
+                            const float h = sh[q * N + i];
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) acc[q][e] = fmaf(h, x[e], acc[q][e]);
+                        }
                     }
+                } else {
+                    *reinterpret_cast<uint4*>(xact0 + ((int64_t)t * d.k + j) * C + c8 * 8) = ub[ii];
                 }
-            } else {
-                *reinterpret_cast<uint4*>(xact0 + ((int64_t)t * d.k + j) * C + c8 * 8) = u;
             }
         }
         *reinterpret_cast<uint4*>(input0 + (int64_t)t * C + c8 * 8) = pack8(acc[0]);
