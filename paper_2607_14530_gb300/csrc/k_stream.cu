@@ -298,23 +298,37 @@ __global__ void __launch_bounds__(256) k_full_dots(Dims d, int T, const uint16_t
 #pragma unroll
         for (int q = 0; q < 4; ++q) h[q] = (q < G) ? hs[q * d.N + i] : 0.f;
         const int64_t row = ((int64_t)t * d.N + i) * C;
-#pragma unroll 4
-        for (int c8 = lane; c8 < C / 8; c8 += 32) {
-            float x[8], dx[8];
-            unpack8(__ldg(reinterpret_cast<const uint4*>(X + row + c8 * 8)), x);
-            unpack8(*reinterpret_cast<const uint4*>(dX + row + c8 * 8), dx);
+        // 4 chunks per lane per step: their 8 reads are issued before any is used
+        for (int c0 = lane; c0 < C / 8; c0 += 128) {
+            uint4 xr[4], dr[4];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                if (q >= G) continue;
-                float g[8];
-                unpack8(reinterpret_cast<const uint4*>(din + q * C)[c8], g);
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    acc[q] = fmaf(x[e], g[e], acc[q]);
-                    dx[e] = fmaf(h[q], g[e], dx[e]);
+            for (int u = 0; u < 4; ++u) {
+                const int c8 = c0 + 32 * u;
+                if (c8 < C / 8) {
+                    xr[u] = __ldg(reinterpret_cast<const uint4*>(X + row + c8 * 8));
+                    dr[u] = *reinterpret_cast<const uint4*>(dX + row + c8 * 8);
                 }
             }
-            *reinterpret_cast<uint4*>(dX + row + c8 * 8) = pack8(dx);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int c8 = c0 + 32 * u;
+                if (c8 >= C / 8) continue;
+                float x[8], dx[8];
+                unpack8(xr[u], x);
+                unpack8(dr[u], dx);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    if (q >= G) continue;
+                    float g[8];
+                    unpack8(reinterpret_cast<const uint4*>(din + q * C)[c8], g);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        acc[q] = fmaf(x[e], g[e], acc[q]);
+                        dx[e] = fmaf(h[q], g[e], dx[e]);
+                    }
+                }
+                *reinterpret_cast<uint4*>(dX + row + c8 * 8) = pack8(dx);
+            }
         }
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
