@@ -24,6 +24,9 @@ constexpr int BK = 64;         // k-elements per stage (128 bytes of bf16 = one 
 constexpr int MAXSTAGES = 8;
 constexpr int NTHREADS = 192;  // warp 0 TMA, warp 1 MMA + TMEM, warps 2..5 statistics + epilogue
 constexpr uint64_t WAIT_NS = 4000000000ull;  // give up a wait after ~4 s
+// a waiting thread may be suspended up to this long per try (it resumes as soon as the phase
+// completes); fewer polls leave the shared-memory pipe to the TMA writes and the epilogues
+constexpr uint32_t WAIT_HINT_NS = 20000;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return (uint32_t)__cvta_generic_to_shared(p);
@@ -44,9 +47,9 @@ __device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity) {
     for (uint32_t it = 0;; ++it) {
         uint32_t ok;
         asm volatile(
-            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n"
             " selp.u32 %0, 1, 0, p;\n}\n"
-            : "=r"(ok) : "r"(a), "r"(parity) : "memory");
+            : "=r"(ok) : "r"(a), "r"(parity), "r"(WAIT_HINT_NS) : "memory");
         if (ok) return true;
         if ((it & 255u) == 255u) {
             uint64_t now;
