@@ -1011,6 +1011,18 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
                 sa = a.scal[(long long)t * a.scal_ld + 0];
                 sb = a.scal[(long long)t * a.scal_ld + 1];
             }
+            // fp32 base of an active row: 16 channels (two chunks) per step, each step's reads
+            // issued one step ahead, the first before the waits
+            const bool arow = (j >= 0) && (t < a.T);
+            const float* brow = a.dxact + ((long long)t * a.k + (j < 0 ? 0 : j)) * a.C + ct * DX_BN + box * 64;
+            uint4 pfa[4], pfb[4];
+            auto prefetch = [&](int step, uint4 (&dst)[4]) {
+                if (arow) {
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) dst[e] = ld_stream(brow + step * 16 + e * 4);
+                }
+            };
+            prefetch(0, pfa);
             bool ok = mbar_wait(smem_u32(&bars[6 + grp]), (uint32_t)((n >> 1) & 1));
             ok = ok && mbar_wait(smem_u32(&bars[2 + grp]), (uint32_t)((n >> 1) & 1));
             if (!ok) {
@@ -1019,21 +1031,17 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
             } else {
                 tc_fence_after();
                 const uint32_t tl = tmem + (uint32_t)(grp * DX_BN + box * 64) + ((uint32_t)(quarter * 32) << 16);
-                const float* brow = a.dxact + ((long long)t * a.k + (j < 0 ? 0 : j)) * a.C + ct * DX_BN + box * 64;
-#pragma unroll 1
-                for (int q2 = 0; q2 < 2; ++q2) {
-                    float acc[32];
-                    tmem_ld16(tl + (uint32_t)(q2 * 32), acc);
-                    tmem_ld16(tl + (uint32_t)(q2 * 32 + 16), acc + 16);
+                auto step_body = [&](int step, const uint4 (&pf)[4]) {
+                    float acc[16];
+                    tmem_ld16(tl + (uint32_t)(step * 16), acc);
 #pragma unroll
-                    for (int cc = 0; cc < 4; ++cc) {
-                        const int q = q2 * 4 + cc;                 // logical 16-byte chunk
+                    for (int cc = 0; cc < 2; ++cc) {
+                        const int q = step * 2 + cc;               // logical 16-byte chunk
                         const int ph = (q ^ sw) * 16;
                         float x[8], v[8];
                         unpack8(*reinterpret_cast<const uint4*>(xrow + ph), x);
-                        if (j >= 0) {
-                            const uint4 b0 = ld_stream(brow + q * 8);
-                            const uint4 b1 = ld_stream(brow + q * 8 + 4);
+                        if (arow) {
+                            const uint4 b0 = pf[cc * 2], b1 = pf[cc * 2 + 1];
                             v[0] = __uint_as_float(b0.x); v[1] = __uint_as_float(b0.y);
                             v[2] = __uint_as_float(b0.z); v[3] = __uint_as_float(b0.w);
                             v[4] = __uint_as_float(b1.x); v[5] = __uint_as_float(b1.y);
@@ -1046,7 +1054,14 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
                         for (int e = 0; e < 8; ++e) o[e] = v[e] + acc[cc * 8 + e] + sa + sb * x[e];
                         *reinterpret_cast<uint4*>(xrow + ph) = pack8(o);
                     }
-                }
+                };
+                prefetch(1, pfb);
+                step_body(0, pfa);
+                prefetch(2, pfa);
+                step_body(1, pfb);
+                prefetch(3, pfb);
+                step_body(2, pfa);
+                step_body(3, pfb);
                 tc_fence_before();
             }
             __syncwarp();
