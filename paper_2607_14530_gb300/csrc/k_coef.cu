@@ -28,7 +28,8 @@ __device__ __forceinline__ void sk_init(const float (&M)[KM][KM], int k, float (
     }
 }
 
-// one half-step: h even = row normalisation, h odd = column normalisation
+// one half-step: h even = row normalisation, h odd = column normalisation (one reciprocal per
+// row or column, then products)
 template <int KM>
 __device__ __forceinline__ void sk_half(float (&A)[KM][KM], int k, int h) {
     if ((h & 1) == 0) {
@@ -38,8 +39,9 @@ __device__ __forceinline__ void sk_half(float (&A)[KM][KM], int k, int h) {
             float s = 0.f;
 #pragma unroll
             for (int b = 0; b < KM; ++b) s += A[a][b];
+            const float r = 1.0f / s;
 #pragma unroll
-            for (int b = 0; b < KM; ++b) A[a][b] = A[a][b] / s;
+            for (int b = 0; b < KM; ++b) A[a][b] = A[a][b] * r;
         }
     } else {
 #pragma unroll
@@ -48,8 +50,9 @@ __device__ __forceinline__ void sk_half(float (&A)[KM][KM], int k, int h) {
             float s = 0.f;
 #pragma unroll
             for (int a = 0; a < KM; ++a) s += A[a][b];
+            const float r = 1.0f / s;
 #pragma unroll
-            for (int a = 0; a < KM; ++a) A[a][b] = A[a][b] / s;
+            for (int a = 0; a < KM; ++a) A[a][b] = A[a][b] * r;
         }
     }
 }
@@ -143,7 +146,7 @@ __device__ void sinkhorn_bwd(const float (&M)[KM][KM], int k, int iters, int L, 
                     dot += dA[a][b] * Out[a][b];
                 }
 #pragma unroll
-                for (int b = 0; b < KM; ++b) dA[a][b] = (dA[a][b] - dot) / s;
+                for (int b = 0; b < KM; ++b) dA[a][b] = (dA[a][b] - dot) * (1.0f / s);
             }
         } else {
 #pragma unroll
@@ -156,7 +159,7 @@ __device__ void sinkhorn_bwd(const float (&M)[KM][KM], int k, int iters, int L, 
                     dot += dA[a][b] * Out[a][b];
                 }
 #pragma unroll
-                for (int a = 0; a < KM; ++a) dA[a][b] = (dA[a][b] - dot) / s;
+                for (int a = 0; a < KM; ++a) dA[a][b] = (dA[a][b] - dot) * (1.0f / s);
             }
         }
     }
