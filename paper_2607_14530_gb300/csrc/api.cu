@@ -151,10 +151,10 @@ Layout make_layout(const Dims& d, int64_t T) {
 
     const int rowblocks = (int)((T + 63) / 64);
     const int sms = device_sms();
-    L.tc = plan_proj_tc((int)T, d.N * d.C, d.nfull, sms);
-    L.tca = plan_proj_tc((int)T, d.k * d.C, nact_max, sms);
-    L.twf = plan_proj_tc(d.N * d.C, (int)T, d.nfull, sms);
-    L.twa = plan_proj_tc(d.k * d.C, (int)T, nact_max, sms);
+    L.tc = plan_proj_tc((int)T, d.N * d.C, d.nfull, sms, true);
+    L.tca = plan_proj_tc((int)T, d.k * d.C, nact_max, sms, true);
+    L.twf = plan_proj_tc(d.N * d.C, (int)T, d.nfull, sms, false);
+    L.twa = plan_proj_tc(d.k * d.C, (int)T, nact_max, sms, false);
     L.splits_full = std::max(L.tc.nseg, pick_splits(rowblocks, d.N * d.C));
     L.splits_act = std::max(L.tca.nseg, pick_splits(rowblocks, d.k * d.C));
     L.nslice = wb_nslice(d.C);
@@ -481,7 +481,7 @@ xhc_status active_maps(const Ctx& c, int slot, const xhc_params* P) {
                                                      d.nact[slot], c.L.splits_act, c.W<float>(c.L.part),
                                                      c.W<float>(c.L.pstats), c.st));
     } else {
-        ProjTcPlan pl = plan_proj_tc(c.T, d.k * d.C, d.nact[slot], device_sms());
+        ProjTcPlan pl = plan_proj_tc(c.T, d.k * d.C, d.nact[slot], device_sms(), true);
         splits = pl.nseg;
         XHC_K("pack_w", c.st, launch_pack_w(wa, d.nact[slot], pl.NB, d.k * d.C,
                                             c.W<uint16_t>(c.L.wpack), c.st));
@@ -514,12 +514,15 @@ xhc_status xhc_pre_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
             XHC_K("colsum", c.st, launch_colsum(P->W_r, d.N * d.C, d.N, d.N, c.W<float>(c.L.wsum), 0,
                                    c.W<float>(c.L.colscr), c.st));
         const WSegs wf = full_segs(d, P);
+        // partial slots written (and summed by coef_full): the split count of the path taken
+        int fsplits = c.L.splits_full;
         if (c.T < 128 || d.N * d.C < 64) {
             // smaller than one tensor-core tile: fp32 CUDA-core projection
             XHC_K("rowproj_full", c.st, launch_rowproj(X, (int64_t)d.N * d.C, d.N * d.C, c.T, wf,
                                                        d.nfull, c.L.splits_full, c.W<float>(c.L.part),
                                                        c.W<float>(c.L.pstats), c.st));
         } else {
+        fsplits = c.L.tc.nseg;
         XHC_K("pack_w", c.st, launch_pack_w(wf, d.nfull, c.L.tc.NB, d.N * d.C,
                                             c.W<uint16_t>(c.L.wpack), c.st));
         XHC_K("proj_tc", c.st, launch_proj_tc(X, c.T, d.N * d.C, c.W<uint16_t>(c.L.wpack), d.nfull,
@@ -527,7 +530,7 @@ xhc_status xhc_pre_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
                                               c.W<int>(c.L.err), c.st));
         }
         XHC_K("coef_full", c.st, launch_coef_full(d, c.T, c.W<float>(c.L.part), c.W<float>(c.L.pstats),
-                                  c.L.splits_full, c.W<float>(c.L.wsum), P->alpha_pre, P->b_pre,
+                                  fsplits, c.W<float>(c.L.wsum), P->alpha_pre, P->b_pre,
                                   c.S<float>(c.L.zfull), c.S<float>(c.L.stats),
                                   c.S<float>(c.L.hpre), c.S<int>(c.L.I), c.S<float>(c.L.p), c.st));
         XHC_K("read", c.st, launch_read(d, c.T, X, c.S<float>(c.L.hpre), c.S<int>(c.L.I), input,
@@ -608,7 +611,7 @@ xhc_status xhc_post_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
                                                  c.W<float>(c.L.dz), n, n, ts, c.W<float>(c.L.wpart),
                                                  act_segs_g(d, g, slot), c.st));
     } else {
-        ProjTcPlan pl = plan_proj_tc(d.k * d.C, T32, n, device_sms());
+        ProjTcPlan pl = plan_proj_tc(d.k * d.C, T32, n, device_sms(), false);
         XHC_K("wgrad_tc_active", c.st, launch_wgrad_tc(c.xact(slot), T32, d.k * d.C, c.W<float>(c.L.dz), n, n,
                                                        c.W<uint16_t>(c.L.dzpack), pl, c.W<float>(c.L.wpart),
                                                        c.W<int>(c.L.err), c.st));

@@ -143,6 +143,7 @@ struct ProjTcArgs {
     int nchunk;         // MMA instructions per k-step (N split in chunks of NB / nchunk <= 256)
     int nseg;           // partial slots per tile
     int stages;         // smem ring depth
+    int kps;            // k-blocks of 64 per stage (projections; 1 for the weight gradients)
     float* part;        // [nseg][T][nfull]
     float* pstats;      // [nseg][T][2]
     int* err;           // set to a nonzero code when a wait gives up
@@ -162,8 +163,9 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     const int STAGES = a.stages;
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    const uint32_t A_BYTES = BM * BK * 2;
-    const uint32_t B_BYTES = (uint32_t)a.NB * BK * 2;
+    const int KPS = A_MN ? 1 : a.kps;               // k-blocks of 64 per stage
+    const uint32_t A_BYTES = (uint32_t)KPS * BM * BK * 2;
+    const uint32_t B_BYTES = (uint32_t)KPS * a.NB * BK * 2;
     const uint32_t STAGE = A_BYTES + B_BYTES;  // both multiples of 1024
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE);
     // bars[0..S) full, [S..2S) empty, [2S] acc full, [2S+1] acc empty
@@ -219,12 +221,14 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                     tma_load_2d(smem_u32(st), &tmA, m * BM, kb * BK, full);
                     tma_load_2d(smem_u32(st + A_BYTES / 2), &tmA, m * BM + 64, kb * BK, full);
                 } else {
-                    tma_load_2d(smem_u32(st), &tmA, kb * BK, m * BM, full);
+                    for (int p2 = 0; p2 < KPS; ++p2)
+                        tma_load_2d(smem_u32(st + p2 * BM * BK * 2), &tmA, (kb * KPS + p2) * BK, m * BM, full);
                 }
                 const int nb_box = a.NB / a.nchunk;
-                for (int q = 0; q < a.nchunk; ++q)
-                    tma_load_2d(smem_u32(st + A_BYTES + (size_t)q * nb_box * 128), &tmB, kb * BK,
-                                q * nb_box, full);
+                for (int p2 = 0; p2 < KPS; ++p2)
+                    for (int q = 0; q < a.nchunk; ++q)
+                        tma_load_2d(smem_u32(st + A_BYTES + (size_t)p2 * a.NB * 128 + (size_t)q * nb_box * 128),
+                                    &tmB, (kb * KPS + p2) * BK, q * nb_box, full);
             }
         }
     } else if (warp == 1) {
@@ -256,16 +260,19 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                     tc_fence_after();
                     const uint32_t abase = smem_u32(smem + (size_t)s * STAGE);
                     const uint32_t bbase = abase + A_BYTES;
+                    for (int p2 = 0; p2 < KPS; ++p2) {
 #pragma unroll
-                    for (int kk = 0; kk < BK / 16; ++kk) {
-                        // K-major: +32 B per 16 k-elements inside the swizzled row; MN-major:
-                        // +16 K-rows of 128 B
-                        const uint64_t ad = A_MN ? sw128_desc_mn(abase + kk * 2048, A_BYTES / 2)
-                                                 : sw128_desc(abase + kk * 32);
-                        for (int q = 0; q < a.nchunk; ++q) {
-                            const uint64_t bd = sw128_desc(bbase + q * nb_chunk * 128 + kk * 32);
-                            mma_bf16(tmem + (uint32_t)(q * nb_chunk), ad, bd, idesc,
-                                     (first && kk == 0) ? 0u : 1u);
+                        for (int kk = 0; kk < BK / 16; ++kk) {
+                            // K-major: +32 B per 16 k-elements inside the swizzled row; MN-major:
+                            // +16 K-rows of 128 B
+                            const uint64_t ad = A_MN ? sw128_desc_mn(abase + kk * 2048, A_BYTES / 2)
+                                                     : sw128_desc(abase + p2 * BM * BK * 2 + kk * 32);
+                            for (int q = 0; q < a.nchunk; ++q) {
+                                const uint64_t bd =
+                                    sw128_desc(bbase + p2 * a.NB * 128 + q * nb_chunk * 128 + kk * 32);
+                                mma_bf16(tmem + (uint32_t)(q * nb_chunk), ad, bd, idesc,
+                                         (first && p2 == 0 && kk == 0) ? 0u : 1u);
+                            }
                         }
                     }
                     first = false;
@@ -299,15 +306,18 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                 if (!A_MN) {
                     // row r of the A tile: 128 bytes, 16-byte chunks permuted by the swizzle (the
                     // sum over the row does not depend on the order)
-                    const uint4* row = reinterpret_cast<const uint4*>(smem + (size_t)s * STAGE + r * 128);
+                    for (int p2 = 0; p2 < KPS; ++p2) {
+                        const uint4* row = reinterpret_cast<const uint4*>(smem + (size_t)s * STAGE +
+                                                                          p2 * BM * BK * 2 + r * 128);
 #pragma unroll
-                    for (int q = 0; q < 8; ++q) {
-                        float f[8];
-                        unpack8(row[q], f);
+                        for (int q = 0; q < 8; ++q) {
+                            float f[8];
+                            unpack8(row[q], f);
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) {
-                            s1 += f[e];
-                            s2 = fmaf(f[e], f[e], s2);
+                            for (int e = 0; e < 8; ++e) {
+                                s1 += f[e];
+                                s2 = fmaf(f[e], f[e], s2);
+                            }
                         }
                     }
                 }
@@ -424,16 +434,30 @@ int proj_tc_nb(int nfull) {
     return nb;
 }
 
-// Two CTAs per SM (each with its own TMA ring and 256 TMEM columns) keep twice the loads in
-// flight; with more than 256 accumulator columns a CTA takes the whole TMEM and runs alone.
-ProjTcPlan plan_proj_tc(int T, int K, int nfull, int nsm) {
+// ring depth that fits the shared memory of one of `ctas` CTAs per SM
+int proj_tc_stages_for(int NB, int kps, int ctas) {
+    const size_t stage = (size_t)kps * ((size_t)BM * BK * 2 + (size_t)NB * BK * 2);
+    const size_t budget = (size_t)(ctas == 2 ? 110 : 220) * 1024;
+    int s = (int)((budget - 2048) / stage);
+    return s > MAXSTAGES ? MAXSTAGES : s;
+}
+
+// Projections (A = X rows, K-major) with a narrow B load two k-blocks per stage, so every row of
+// an A tile is read as 256 contiguous bytes (measured faster for the active projections; the wide
+// full-state projection keeps one k-block per stage and two CTAs per SM); the weight gradients
+// (A MN-major) already read 256 bytes per row with one k-block.  Two CTAs per SM (each with its
+// own TMA ring and 256 TMEM columns) keep twice the loads in flight when two rings fit;
+// otherwise (or with more than 256 accumulator columns) one CTA per SM.
+ProjTcPlan plan_proj_tc(int T, int K, int nfull, int nsm, bool proj) {
     ProjTcPlan p;
-    p.KB = (K + BK - 1) / BK;
+    p.NB = proj_tc_nb(nfull);
+    p.kps = (proj && proj_tc_stages_for(p.NB, 2, 2) >= 2) ? 2 : 1;
+    p.KB = (K + BK * p.kps - 1) / (BK * p.kps);
     p.MT = (T + BM - 1) / BM;
     p.W = (long long)p.KB * p.MT;
-    p.NB = proj_tc_nb(nfull);
     p.nchunk = p.NB > 256 ? 2 : 1;
-    const int sms = (p.NB <= 256 ? 2 : 1) * (nsm > 0 ? nsm : 148);
+    p.ctas = (p.NB <= 256 && proj_tc_stages_for(p.NB, p.kps, 2) >= 2) ? 2 : 1;
+    const int sms = p.ctas * (nsm > 0 ? nsm : 148);
     long long P = std::min<long long>(sms, std::max<long long>(1, p.W / 4));
     p.P = (int)P;
     const long long per = p.W / p.P;  // >= 4
@@ -441,16 +465,10 @@ ProjTcPlan plan_proj_tc(int T, int K, int nfull, int nsm) {
     if (p.nseg > p.P) p.nseg = p.P;
     return p;
 }
-int proj_tc_stages(int NB) {
-    const size_t stage = (size_t)BM * BK * 2 + (size_t)NB * BK * 2;
-    const size_t budget = (NB <= 256 ? 110 : 220) * 1024;  // two CTAs per SM, or one
-    int s = (int)((budget - 2048) / stage);
-    return s > MAXSTAGES ? MAXSTAGES : s;
-}
 
-size_t proj_tc_smem(int NB) {
-    const int S = proj_tc_stages(NB);
-    return (size_t)S * (BM * BK * 2 + (size_t)NB * BK * 2) + (2 * S + 2) * 8 + 16 + 1024;
+size_t proj_tc_smem(const ProjTcPlan& p) {
+    const int S = proj_tc_stages_for(p.NB, p.kps, p.ctas);
+    return (size_t)S * p.kps * (BM * BK * 2 + (size_t)p.NB * BK * 2) + (2 * S + 2) * 8 + 16 + 1024;
 }
 
 cudaError_t launch_pack_w(const WSegs& W, int nfull, int NB, int K, uint16_t* Wpack, cudaStream_t st) {
@@ -469,7 +487,7 @@ cudaError_t launch_proj_tc(const uint16_t* X, int T, int K, const uint16_t* Wpac
     if (e != cudaSuccess) return e;
     e = cudaMemsetAsync(pstats, 0, (size_t)p.nseg * T * 2 * sizeof(float), st);
     if (e != cudaSuccess) return e;
-    const size_t sm = proj_tc_smem(p.NB);
+    const size_t sm = proj_tc_smem(p);
     e = cudaFuncSetAttribute((const void*)k_proj_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
     ProjTcArgs a;
@@ -482,7 +500,8 @@ cudaError_t launch_proj_tc(const uint16_t* X, int T, int K, const uint16_t* Wpac
     a.NB = p.NB;
     a.nchunk = p.nchunk;
     a.nseg = p.nseg;
-    a.stages = proj_tc_stages(p.NB);
+    a.stages = proj_tc_stages_for(p.NB, p.kps, p.ctas);
+    a.kps = p.kps;
     if (a.stages < 2) return cudaErrorInvalidValue;
     a.part = part;
     a.pstats = pstats;
@@ -523,7 +542,7 @@ cudaError_t launch_wgrad_tc(const uint16_t* A, int T, int E, const float* dz, in
         return cudaErrorInvalidValue;
     e = cudaMemsetAsync(part, 0, (size_t)p.nseg * E * n * sizeof(float), st);
     if (e != cudaSuccess) return e;
-    const size_t sm = proj_tc_smem(p.NB);
+    const size_t sm = proj_tc_smem(p);
     e = cudaFuncSetAttribute((const void*)k_proj_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
     ProjTcArgs a;
@@ -536,7 +555,8 @@ cudaError_t launch_wgrad_tc(const uint16_t* A, int T, int E, const float* dz, in
     a.NB = p.NB;
     a.nchunk = p.nchunk;
     a.nseg = p.nseg;
-    a.stages = proj_tc_stages(p.NB);
+    a.stages = proj_tc_stages_for(p.NB, p.kps, p.ctas);
+    a.kps = p.kps;
     if (a.stages < 2) return cudaErrorInvalidValue;
     a.part = part;
     a.pstats = nullptr;

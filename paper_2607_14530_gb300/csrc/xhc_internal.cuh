@@ -57,8 +57,10 @@ struct ProjTcPlan {
     int nseg;        // partial slots per tile
     int NB;          // B rows (hi + lo + pad)
     int nchunk;      // MMA instructions per k-step
+    int kps;         // k-blocks of 64 per stage
+    int ctas;        // CTAs per SM
 };
-ProjTcPlan plan_proj_tc(int T, int K, int nfull, int nsm);
+ProjTcPlan plan_proj_tc(int T, int K, int nfull, int nsm, bool proj);  // proj: A = X rows (else weight gradient)
 int device_sms();
 
 // Byte offsets of the per-group buffers for a given T (all 256-byte aligned).

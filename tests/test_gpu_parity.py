@@ -52,8 +52,12 @@ def run_case(cfg, T, seed=0, alpha=0.01):
     outs = [Guarded(o.cuda()) for o in inp["outs"]]
     inputs = [Guarded(torch.zeros(T, cfg.C, dtype=torch.bfloat16)) for _ in range(cfg.G)]
     saved, ws = g.alloc(T)
-    saved_g = Guarded(torch.zeros(saved.numel(), dtype=torch.uint8))
-    ws_g = Guarded(torch.zeros(ws.numel(), dtype=torch.uint8))
+    # saved and workspace start poisoned (0xFF bytes: NaN as fp32 / bf16, -1 as int32), except the
+    # workspace's device error word: nothing may be read before this call sequence wrote it
+    saved_g = Guarded(torch.full((saved.numel(),), 0xFF, dtype=torch.uint8))
+    ws0 = torch.full((ws.numel(),), 0xFF, dtype=torch.uint8)
+    ws0[:256] = 0
+    ws_g = Guarded(ws0)
     g.forward(Pd, Xg.t, [o.t for o in outs], saved_g.t, ws_g.t, inputs=[i.t for i in inputs])
     torch.cuda.synchronize()
     return g, inp, P, Pd, grads_in, ref, Xg, outs, inputs, saved_g, ws_g
