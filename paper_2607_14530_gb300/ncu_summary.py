@@ -1,33 +1,60 @@
-"""Summarise an ncu launch list (``--metrics gpu__time_duration.sum --csv``) per kernel.
+"""Summaries of ncu CSV logs.
 
-Usage: python -m paper_2607_14530_gb300.ncu_summary launches.csv [--last N]
-Prints, per kernel, the number of launches, total device time and share of the total.  ``--last N``
-keeps only the last N launches (one timed step after the warm-up steps).  The per-launch times
-of such a list are cold-cache and serialised: compare shares, not absolute times.
+Launch list (``--metrics gpu__time_duration.sum --csv``)::
+
+    python -m paper_2607_14530_gb300.ncu_summary launches.csv [--last N]
+
+prints, per kernel, the number of launches, total device time and share of the total.  ``--last
+N`` keeps only the last N launches (one timed step after the warm-up steps).  The per-launch
+times of such a list are cold-cache and serialised: compare shares, not absolute times.
+
+DRAM traffic (``--metrics dram__bytes_read.sum,dram__bytes_write.sum --csv``)::
+
+    python -m paper_2607_14530_gb300.ncu_summary traffic.csv --traffic OUT.json --workload W
+        --scale S --map NAME=KERNEL [--map ...]
+
+writes, for every trace name NAME mapped to a kernel, the mean DRAM bytes (read + write) per
+launch of that kernel times S (the ratio of the benchmark's token count to the captured one:
+every kernel's traffic is linear in the tokens), tagged with the hash of the kernel sources, so
+that ``bench.py`` reports it only while the sources are unchanged.
 """
 from __future__ import annotations
 
 import csv
+import hashlib
+import glob
 import io
+import json
+import os
 import re
 import sys
 
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
-def load(path):
+
+def _rows(path):
     with open(path) as f:
         text = f.read()
     start = text.find('"ID"')
-    rows = list(csv.DictReader(io.StringIO(text[start:])))
+    return list(csv.DictReader(io.StringIO(text[start:])))
+
+
+def kernel_base(name: str) -> str:
+    """`void xhc::<unnamed>::k_dx_tc<1>(CUtensorMap_st, ...)` -> `k_dx_tc<1>`."""
+    name = name.replace("(anonymous namespace)", "").replace("<unnamed>", "")
+    name = re.sub(r"\(.*$", "", name).replace("void ", "").strip()
+    return name.split("::")[-1]
+
+
+def load(path):
     out = []
-    for r in rows:
+    for r in _rows(path):
         if r.get("Metric Name") != "gpu__time_duration.sum":
             continue
-        name = r["Kernel Name"]
-        name = re.sub(r"\(.*$", "", name).replace("void ", "").strip()
         v = float(r["Metric Value"].replace(",", ""))
         unit = r.get("Metric Unit", "ns")
         scale = {"ns": 1e-6, "us": 1e-3, "usecond": 1e-3, "ms": 1.0, "msecond": 1.0, "nsecond": 1e-6}.get(unit, 1e-6)
-        out.append((name, v * scale))
+        out.append((kernel_base(r["Kernel Name"]), v * scale))
     return out
 
 
@@ -45,8 +72,59 @@ def summarise(launches):
     return "\n".join(lines)
 
 
-if __name__ == "__main__":
-    launches = load(sys.argv[1])
-    if "--last" in sys.argv:
-        launches = launches[-int(sys.argv[sys.argv.index("--last") + 1]):]
+def dram_bytes(path):
+    """Mean DRAM bytes (read + write) per launch, per kernel."""
+    unit_scale = {"byte": 1.0, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9, "Tbyte": 1e12}
+    per_launch = {}
+    for r in _rows(path):
+        m = r.get("Metric Name")
+        if m not in ("dram__bytes_read.sum", "dram__bytes_write.sum"):
+            continue
+        v = float(r["Metric Value"].replace(",", "")) * unit_scale.get(r.get("Metric Unit", "byte"), 1.0)
+        key = (r["ID"], kernel_base(r["Kernel Name"]))
+        per_launch[key] = per_launch.get(key, 0.0) + v
+    per = {}
+    for (_, name), v in per_launch.items():
+        per.setdefault(name, []).append(v)
+    return {n: sum(v) / len(v) for n, v in per.items()}
+
+
+def csrc_hash():
+    h = hashlib.sha256()
+    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2607_14530_gb300", "csrc", "*"))):
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def main(argv):
+    path = argv[1]
+    if "--traffic" in argv:
+        out = argv[argv.index("--traffic") + 1]
+        wl = argv[argv.index("--workload") + 1]
+        scale = float(argv[argv.index("--scale") + 1])
+        maps = [argv[i + 1].split("=", 1) for i, a in enumerate(argv) if a == "--map"]
+        per = dram_bytes(path)
+        d = {}
+        if os.path.exists(out):
+            with open(out) as f:
+                d = json.load(f)
+        ent = d.setdefault(wl, {})
+        sha = csrc_hash()
+        for name, kern in maps:
+            if kern in per:
+                ent[name] = {"kernel": kern, "dram_bytes_per_launch": per[kern] * scale,
+                             "captured_bytes_per_launch": per[kern], "scale": scale, "csrc_sha": sha}
+        with open(out, "w") as f:
+            json.dump(d, f, indent=1, sort_keys=True)
+        for n, v in sorted(per.items()):
+            print(f"{n:28s} {v / 1e9:10.4f} GB per launch (captured)")
+        return
+    launches = load(path)
+    if "--last" in argv:
+        launches = launches[-int(argv[argv.index("--last") + 1]):]
     print(summarise(launches))
+
+
+if __name__ == "__main__":
+    main(sys.argv)
