@@ -272,15 +272,22 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
     const int ntok = (int)(t1 - t0);
     const int c = blockIdx.x * WSL + 2 * threadIdx.x;
     const bool act = (KS == 2) || c < C;
+    // running pointers of the next token to prefetch (issue() is called once per token, in order)
     const uint16_t* po = out + t0 * C + c;
     const uint16_t* px = xact + t0 * k * C + c;
+    const long long kC = (long long)k * C;
     auto issue = [&](int sl, int tn) {
         if (act && tn < ntok) {
-            cpa4(&R.o[sl][threadIdx.x], po + (long long)tn * C);
+            cpa4(&R.o[sl][threadIdx.x], po);
+            const uint16_t* pj = px;
 #pragma unroll
-            for (int j = 0; j < KM; ++j)
-                if (j < k) cpa4(&R.x[sl][j][threadIdx.x], px + ((long long)tn * k + j) * C);
+            for (int j = 0; j < KM; ++j) {
+                if (j < k) cpa4(&R.x[sl][j][threadIdx.x], pj);
+                pj += C;
+            }
         }
+        po += C;
+        px += kC;
         cpa_commit();
     };
 #pragma unroll
@@ -303,8 +310,9 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
         taps_reg<KW, KS>(d, cw, c, act, tw);
         ring_init<KW>(out, C, c, act, t0, pos0, w);
     }
-    uint16_t* pX = X + t0 * d.N * C + c;
+    uint16_t* pX = X + t0 * d.N * C + c;                              // token rows, advanced per token
     uint16_t* pn = last ? nullptr : xact_next + t0 * k * C + c;
+    const long long NC = (long long)d.N * C;
     __syncthreads();
     const int RU = KW > 0 ? KW : 4;
     for (int tb = 0; tb < ntok; tb += RU) {
@@ -356,11 +364,13 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
                             v = fma2(e.w, uu[3], v);
                         }
                         if (last)
-                            st2(pX + ((long long)tt * d.N + Ish[tt * KM + j]) * C, v);
+                            st2(pX + (long long)Ish[tt * KM + j] * C, v);
                         else
-                            st2(pn + ((long long)tt * k + j) * C, v);
+                            st2(pn + (long long)j * C, v);
                     }
                 }
+                if (last) pX += NC;
+                else pn += kC;
             }
         }
     }
@@ -408,23 +418,32 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
         Ish[q] = (j < k) ? I[(t0 + tt) * k + j] : 0;
     }
     __syncthreads();
+    // running pointers of the next token to prefetch (issue() is called once per token, in order)
     const uint16_t* po = out + t0 * C + c;
     const uint16_t* px = xact + t0 * k * C + c;
     const uint16_t* pX = dX + t0 * d.N * C + c;
     const float* pd = dxact + t0 * k * C + c;
+    const long long kC = (long long)k * C, NC = (long long)d.N * C;
     auto issue = [&](int sl, int tn) {
         if (act && tn < ntok) {
-            cpa4(&R.o[sl][threadIdx.x], po + (long long)tn * C);
+            cpa4(&R.o[sl][threadIdx.x], po);
 #pragma unroll
             for (int j = 0; j < KM; ++j) {
                 if (j >= k) continue;
                 if (last) {
-                    cpa4(&R.x[sl][j][threadIdx.x], px + ((long long)tn * k + j) * C);
-                    cpa4(&R.dn[sl][j][threadIdx.x], pX + ((long long)tn * d.N + Ish[tn * KM + j]) * C);
+                    cpa4(&R.x[sl][j][threadIdx.x], px + (long long)j * C);
+                    cpa4(&R.dn[sl][j][threadIdx.x], pX + (long long)Ish[tn * KM + j] * C);
                 } else {
-                    cpa8(&R.dn[sl][j][threadIdx.x], pd + ((long long)tn * k + j) * C);
+                    cpa8(&R.dn[sl][j][threadIdx.x], pd + (long long)j * C);
                 }
             }
+        }
+        po += C;
+        if (last) {
+            px += kC;
+            pX += NC;
+        } else {
+            pd += kC;
         }
         cpa_commit();
     };
@@ -582,23 +601,29 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
     const int c = blockIdx.x * WSL + 2 * threadIdx.x;
     const bool act = (KS == 2) || c < C;
     __syncthreads();
+    // running pointers: next token to prefetch (issue() is called once per token, in order), the
+    // token whose active gradient is written (last slot), the next d_out row to store
     const uint16_t* po = out + t0 * C + c;
     const uint16_t* pX = dX + t0 * d.N * C + c;
     const float* pd = dn_in + t0 * k * C + c;
     float* pxo = dxact_out + t0 * k * C + c;
     uint16_t* pdo = d_out + t0 * C + c;
+    const long long kC = (long long)k * C, NC = (long long)d.N * C;
     auto issue = [&](int sl, int tn) {
         if (act && tn < ntok) {
-            cpa4(&R.o[sl][threadIdx.x], po + (long long)tn * C);
+            cpa4(&R.o[sl][threadIdx.x], po);
 #pragma unroll
             for (int j = 0; j < KM; ++j) {
                 if (j >= k) continue;
                 if (last)
-                    cpa4(&R.dn[sl][j][threadIdx.x], pX + ((long long)tn * d.N + Ish[tn * KM + j]) * C);
+                    cpa4(&R.dn[sl][j][threadIdx.x], pX + (long long)Ish[tn * KM + j] * C);
                 else
-                    cpa8(&R.dn[sl][j][threadIdx.x], pd + ((long long)tn * k + j) * C);
+                    cpa8(&R.dn[sl][j][threadIdx.x], pd + (long long)j * C);
             }
         }
+        po += C;
+        if (last) pX += NC;
+        else pd += kC;
         cpa_commit();
     };
 #pragma unroll
@@ -682,13 +707,17 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
                             }
 #pragma unroll
                             for (int i = 0; i < KM; ++i)
-                                if (i < k) *reinterpret_cast<float2*>(pxo + ((long long)tt * k + i) * C) = v[i];
+                                if (i < k) *reinterpret_cast<float2*>(pxo + (long long)i * C) = v[i];
+                            pxo += kC;
                         }
                     } else if constexpr (KW > 0) {
                         w[u] = f2z();   // past the sequence end
                     }
                     if constexpr (KW == 0) {
-                        if (tt < n1) st2(pdo + (long long)tt * C, du[0]);
+                        if (tt < n1) {
+                            st2(pdo, du[0]);
+                            pdo += C;
+                        }
                     } else {
                         // conv weight gradient of the run's tokens
                         if (tt < n1) {
@@ -713,7 +742,10 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
                             }
                         }
                         // token tt - (KW - 1) has all its terms (du is zero past the sequence end)
-                        if (tt >= KW - 1) st2(pdo + (long long)(tt - (KW - 1)) * C, pend[(u + 1) % KW]);
+                        if (tt >= KW - 1) {
+                            st2(pdo, pend[(u + 1) % KW]);
+                            pdo += C;
+                        }
                     }
                 }
             }
