@@ -511,7 +511,15 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
                     }
                 }
                 float* dst = wsh + ((size_t)tt * (WT / 32) + warp) * NVP;
-                if constexpr (NV == 16) {
+                if constexpr (KW == 0 && NV == 16) {
+                    // no conv: only P[j][0] = <dXn_j, out> (slots j * 4) carry terms
+                    float v4[KM];
+#pragma unroll
+                    for (int j = 0; j < KM; ++j) v4[j] = v[j * 4];
+                    const float tot = WRed<KM, 16>::run(v4, lane);
+                    constexpr int SH = KM == 4 ? 3 : 2;          // lane >> SH = value index
+                    if ((lane & ((1 << SH) - 1)) == 0) dst[(lane >> SH) * 4] = tot;
+                } else if constexpr (NV == 16) {
                     const float tot = WRed<16, 16>::run(v, lane);
                     if ((lane & 1) == 0) dst[lane >> 1] = tot;
                 } else {
@@ -527,6 +535,7 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
     __syncthreads();
     for (int idx = threadIdx.x; idx < ntok * nv; idx += WT) {
         const int tt = idx / nv, q = idx - tt * nv;
+        if (KW == 0 && NV == 16 && (q & 3) != 0) continue;  // entries without terms (K = 1)
         float sm = 0.f;
 #pragma unroll
         for (int ww = 0; ww < WT / 32; ++ww) sm += wsh[((size_t)tt * (WT / 32) + ww) * NVP + q];
