@@ -587,9 +587,10 @@ xhc_status xhc_post_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
         XHC_CUDA(cudaMemsetAsync(c.W<float>(c.L.dp), 0, (size_t)T32 * d.k * 4, c.st));
         XHC_K("restore", c.st, launch_restore(d, T32, c.xact(0), c.S<int>(c.L.I), X, c.st));
     }
+    const int bslices = wb_bred_slices(d, slot);
     XHC_K("wb_bred", c.st, launch_wb_bred(d, slot, T32, out, cw, dX, c.S<int>(c.L.I), dxact, c.xact(slot),
-                                          c.L.nslice, red, c.st));
-    XHC_K("bwd_coef", c.st, launch_bwd_coef(d, slot, T32, red, c.L.nslice, c.S<float>(c.L.zact[slot]),
+                                          bslices, red, c.st));
+    XHC_K("bwd_coef", c.st, launch_bwd_coef(d, slot, T32, red, bslices, c.S<float>(c.L.zact[slot]),
                              c.S<float>(c.L.rs[slot]), c.S<float>(c.L.p),
                              c.S<float>(c.L.hpost[slot]),
                              (d.K[slot] > 1 && d.gs) ? c.S<double>(c.L.gram[slot]) : nullptr,

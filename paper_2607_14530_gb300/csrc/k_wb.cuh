@@ -778,6 +778,333 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
     }
 }
 
+// ---------------------------------------------------------------------------------------------
+// Write-back kernels of the sublayers without temporal conv (K = 1), 8 channels per thread: no
+// conv ring to keep, so every thread moves 16-byte rows; the next token's rows are loaded into
+// registers while the current one is processed.  A CTA covers W8 channels of a run of tokens.
+
+constexpr int W8 = WT * 8;   // channels per CTA
+
+__device__ __forceinline__ uint4 ld16(const void* p) { return __ldg(reinterpret_cast<const uint4*>(p)); }
+
+// per-token tables shared by the CTA: E[j][0] (write-back coefficient of out), H_res, I
+template <int KM>
+__device__ __forceinline__ void k1_tables(int ntok, long long t0, int k, bool last, const float* emat,
+                                          int estride, const float* hres, const int* I, float* Esh,
+                                          float* Hsh, int* Ish) {
+    for (int idx = threadIdx.x; idx < ntok * KM; idx += WT) {
+        const int tt = idx / KM, j = idx - tt * KM;
+        Esh[idx] = (j < k) ? emat[(t0 + tt) * estride + j * 4] : 0.f;
+        Ish[idx] = (j < k) ? I[(t0 + tt) * k + j] : 0;
+    }
+    if (last)
+        for (int idx = threadIdx.x; idx < ntok * KM * KM; idx += WT) {
+            const int tt = idx / (KM * KM), q = idx - tt * (KM * KM);
+            const int j = q / KM, i = q - j * KM;
+            Hsh[idx] = (j < k && i < k) ? hres[(t0 + tt) * k * k + j * k + i] : 0.f;
+        }
+}
+
+// forward: X_act_new_j = (sum_i H_res[j][i] x_i  |  x_j) + E[j][0] out
+template <int KM>
+__global__ void __launch_bounds__(WT) k_wb_fwd8(Dims d, int slot, int T, int TB,
+                                                const uint16_t* __restrict__ out,
+                                                const float* __restrict__ emat,
+                                                const uint16_t* __restrict__ xact,
+                                                const int* __restrict__ I,
+                                                const float* __restrict__ hres,
+                                                uint16_t* __restrict__ xact_next,
+                                                uint16_t* __restrict__ X) {
+    extern __shared__ __align__(16) unsigned char smu[];
+    float* Esh = reinterpret_cast<float*>(smu);        // [TB][KM]
+    float* Hsh = Esh + TB * KM;                        // [TB][KM][KM]
+    int* Ish = reinterpret_cast<int*>(Hsh + TB * KM * KM);
+    const int k = d.k, C = d.C;
+    const bool last = (slot == d.G - 1);
+    const long long t0 = (long long)blockIdx.y * TB;
+    const int ntok = (int)(min((long long)T, t0 + TB) - t0);
+    k1_tables<KM>(ntok, t0, k, last, emat, TOKMAT, hres, I, Esh, Hsh, Ish);
+    __syncthreads();
+    const int c = blockIdx.x * W8 + threadIdx.x * 8;
+    if (c >= C) return;
+    const long long kC = (long long)k * C, NC = (long long)d.N * C;
+    const uint16_t* po = out + t0 * C + c;
+    const uint16_t* px = xact + t0 * kC + c;
+    uint4 on = ld16(po), xn[KM];
+#pragma unroll
+    for (int j = 0; j < KM; ++j) xn[j] = (j < k) ? ld16(px + j * (long long)C) : make_uint4(0, 0, 0, 0);
+    for (int tt = 0; tt < ntok; ++tt) {
+        const uint4 oc = on;
+        uint4 xc[KM];
+#pragma unroll
+        for (int j = 0; j < KM; ++j) xc[j] = xn[j];
+        po += C;
+        px += kC;
+        if (tt + 1 < ntok) {
+            on = ld16(po);
+#pragma unroll
+            for (int j = 0; j < KM; ++j)
+                if (j < k) xn[j] = ld16(px + j * (long long)C);
+        }
+        const long long t = t0 + tt;
+        float o[8], x[KM][8];
+        unpack8(oc, o);
+#pragma unroll
+        for (int j = 0; j < KM; ++j) unpack8(xc[j], x[j]);
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            if (j >= k) continue;
+            const float e = Esh[tt * KM + j];
+            float v[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                float a = 0.f;
+                if (last) {
+#pragma unroll
+                    for (int i = 0; i < KM; ++i) a = fmaf(Hsh[(tt * KM + j) * KM + i], x[i][q], a);
+                } else {
+                    a = x[j][q];
+                }
+                v[q] = fmaf(e, o[q], a);
+            }
+            uint16_t* dst = last ? X + t * NC + (long long)Ish[tt * KM + j] * C + c
+                                 : xact_next + t * kC + (long long)j * C + c;
+            *reinterpret_cast<uint4*>(dst) = pack8(v);
+        }
+    }
+}
+
+// backward reductions: P[j][0] = <dXn_j, out> (and, last slot, Q[j][i] = <dXn_j, x_i>), one
+// partial per W8-channel slice
+template <int KM>
+__global__ void __launch_bounds__(WT) k_wb_bred8(Dims d, int slot, int T, int TB,
+                                                 const uint16_t* __restrict__ out,
+                                                 const uint16_t* __restrict__ dX,
+                                                 const int* __restrict__ I,
+                                                 const float* __restrict__ dxact,
+                                                 const uint16_t* __restrict__ xact, int nslice,
+                                                 float* __restrict__ red) {
+    constexpr int NQ = KM + KM * KM;                  // P[j][0], then Q[j][i]
+    constexpr int NV = NQ <= 32 ? 32 : 96;            // reduce-scatter width (blocks of 32)
+    extern __shared__ __align__(16) unsigned char smu[];
+    int* Ish = reinterpret_cast<int*>(smu);           // [TB][KM]
+    float* wsh = reinterpret_cast<float*>(Ish + TB * KM);   // [TB][WT/32][NV]
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int k = d.k, C = d.C;
+    const bool last = (slot == d.G - 1);
+    const long long t0 = (long long)blockIdx.y * TB;
+    const int ntok = (int)(min((long long)T, t0 + TB) - t0);
+    for (int idx = threadIdx.x; idx < ntok * KM; idx += WT) {
+        const int tt = idx / KM, j = idx - tt * KM;
+        Ish[idx] = (j < k) ? I[(t0 + tt) * k + j] : 0;
+    }
+    __syncthreads();
+    const int c = blockIdx.x * W8 + threadIdx.x * 8;
+    const bool act = c < C;
+    const long long kC = (long long)k * C, NC = (long long)d.N * C;
+    const uint16_t* po = out + t0 * C + c;
+    const uint16_t* px = xact + t0 * kC + c;
+    const uint16_t* pX = dX + t0 * NC + c;
+    const float* pd = dxact + t0 * kC + c;
+    // next token's rows: out, dXn_j (bf16 rows of dX, or fp32 active gradient), x_j (last)
+    uint4 on = make_uint4(0, 0, 0, 0), dn0[KM], dn1[KM], xn[KM];
+    auto load = [&](int tt) {
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            dn0[j] = make_uint4(0, 0, 0, 0);
+            dn1[j] = dn0[j];
+            xn[j] = dn0[j];
+        }
+        on = dn0[0];
+        if (!act || tt >= ntok) return;
+        on = ld16(po);
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            if (j >= k) continue;
+            if (last) {
+                dn0[j] = ld16(pX + (long long)Ish[tt * KM + j] * C);
+                xn[j] = ld16(px + j * (long long)C);
+            } else {
+                dn0[j] = ld16(pd + j * (long long)C);
+                dn1[j] = ld16(pd + j * (long long)C + 4);
+            }
+        }
+    };
+    load(0);
+    for (int tt = 0; tt < ntok; ++tt) {
+        const uint4 oc = on;
+        uint4 d0[KM], d1[KM], xc[KM];
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            d0[j] = dn0[j];
+            d1[j] = dn1[j];
+            xc[j] = xn[j];
+        }
+        po += C;
+        if (last) {
+            px += kC;
+            pX += NC;
+        } else {
+            pd += kC;
+        }
+        load(tt + 1);
+        float o[8], dn[KM][8];
+        unpack8(oc, o);
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            if (last) {
+                unpack8(d0[j], dn[j]);
+            } else {
+                dn[j][0] = __uint_as_float(d0[j].x); dn[j][1] = __uint_as_float(d0[j].y);
+                dn[j][2] = __uint_as_float(d0[j].z); dn[j][3] = __uint_as_float(d0[j].w);
+                dn[j][4] = __uint_as_float(d1[j].x); dn[j][5] = __uint_as_float(d1[j].y);
+                dn[j][6] = __uint_as_float(d1[j].z); dn[j][7] = __uint_as_float(d1[j].w);
+            }
+        }
+        float v[NV];
+#pragma unroll
+        for (int q = 0; q < NV; ++q) v[q] = 0.f;
+#pragma unroll
+        for (int j = 0; j < KM; ++j)
+#pragma unroll
+            for (int q = 0; q < 8; ++q) v[j] = fmaf(dn[j][q], o[q], v[j]);
+        if (last) {
+            float x[KM][8];
+#pragma unroll
+            for (int i = 0; i < KM; ++i) unpack8(xc[i], x[i]);
+#pragma unroll
+            for (int j = 0; j < KM; ++j)
+#pragma unroll
+                for (int i = 0; i < KM; ++i)
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) v[KM + j * KM + i] = fmaf(dn[j][q], x[i][q], v[KM + j * KM + i]);
+        }
+        float tot[NV / 32];
+        wred32<NV / 32>(v, lane, tot);
+        float* dst = wsh + ((size_t)tt * (WT / 32) + warp) * NV;
+#pragma unroll
+        for (int bb = 0; bb < NV / 32; ++bb) dst[bb * 32 + lane] = tot[bb];
+    }
+    __syncthreads();
+    // red layout of the reverse maps: P[j][a] at j*4 + a, Q[j][i] at KM*4 + j*KM + i
+    const int nq = last ? NQ : KM;
+    for (int idx = threadIdx.x; idx < ntok * nq; idx += WT) {
+        const int tt = idx / nq, q = idx - tt * nq;
+        float sm = 0.f;
+#pragma unroll
+        for (int ww = 0; ww < WT / 32; ++ww) sm += wsh[((size_t)tt * (WT / 32) + ww) * NV + q];
+        const int slotq = q < KM ? q * 4 : KM * 4 + (q - KM);
+        red[((t0 + tt) * nslice + blockIdx.x) * NRED + slotq] = sm;
+    }
+}
+
+// backward apply: d_out = sum_j E[j][0] dXn_j; last slot: dX_act_i = sum_j H_res[j][i] dXn_j
+template <int KM>
+__global__ void __launch_bounds__(WT) k_wb_bapp8(Dims d, int slot, int T, int TB,
+                                                 const uint16_t* __restrict__ dX,
+                                                 const int* __restrict__ I,
+                                                 const float* dn_in,  // may alias dxact_out
+                                                 const float* __restrict__ tokmat,
+                                                 float* dxact_out,
+                                                 uint16_t* __restrict__ d_out) {
+    extern __shared__ __align__(16) unsigned char smu[];
+    float* Esh = reinterpret_cast<float*>(smu);        // [TB][KM]
+    float* Hsh = Esh + TB * KM;                        // [TB][KM][KM]
+    int* Ish = reinterpret_cast<int*>(Hsh + TB * KM * KM);
+    const int k = d.k, C = d.C;
+    const bool last = (slot == d.G - 1);
+    const long long t0 = (long long)blockIdx.y * TB;
+    const int ntok = (int)(min((long long)T, t0 + TB) - t0);
+    for (int idx = threadIdx.x; idx < ntok * KM; idx += WT) {
+        const int tt = idx / KM, j = idx - tt * KM;
+        Esh[idx] = (j < k) ? tokmat[(t0 + tt) * TOKMAT + j * 4] : 0.f;
+        Ish[idx] = (last && j < k) ? I[(t0 + tt) * k + j] : 0;
+    }
+    if (last)
+        for (int idx = threadIdx.x; idx < ntok * KM * KM; idx += WT) {
+            const int tt = idx / (KM * KM), q = idx - tt * (KM * KM);
+            const int j = q / KM, i = q - j * KM;
+            Hsh[idx] = (j < k && i < k) ? tokmat[(t0 + tt) * TOKMAT + 48 + j * 8 + i] : 0.f;
+        }
+    __syncthreads();
+    const int c = blockIdx.x * W8 + threadIdx.x * 8;
+    if (c >= C) return;
+    const long long kC = (long long)k * C, NC = (long long)d.N * C;
+    const uint16_t* pX = dX + t0 * NC + c;
+    const float* pd = dn_in + t0 * kC + c;
+    uint4 dn0[KM], dn1[KM];
+    auto load = [&](int tt) {
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            dn0[j] = make_uint4(0, 0, 0, 0);
+            dn1[j] = dn0[j];
+        }
+        if (tt >= ntok) return;
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            if (j >= k) continue;
+            if (last) {
+                dn0[j] = ld16(pX + (long long)Ish[tt * KM + j] * C);
+            } else {
+                dn0[j] = ld16(pd + j * (long long)C);
+                dn1[j] = ld16(pd + j * (long long)C + 4);
+            }
+        }
+    };
+    load(0);
+    for (int tt = 0; tt < ntok; ++tt) {
+        uint4 d0[KM], d1[KM];
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            d0[j] = dn0[j];
+            d1[j] = dn1[j];
+        }
+        if (last) pX += NC;
+        else pd += kC;
+        load(tt + 1);
+        const long long t = t0 + tt;
+        float dn[KM][8];
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            if (last) {
+                unpack8(d0[j], dn[j]);
+            } else {
+                dn[j][0] = __uint_as_float(d0[j].x); dn[j][1] = __uint_as_float(d0[j].y);
+                dn[j][2] = __uint_as_float(d0[j].z); dn[j][3] = __uint_as_float(d0[j].w);
+                dn[j][4] = __uint_as_float(d1[j].x); dn[j][5] = __uint_as_float(d1[j].y);
+                dn[j][6] = __uint_as_float(d1[j].z); dn[j][7] = __uint_as_float(d1[j].w);
+            }
+        }
+        float g[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) g[q] = 0.f;
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            const float e = Esh[tt * KM + j];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) g[q] = fmaf(e, dn[j][q], g[q]);
+        }
+        *reinterpret_cast<uint4*>(d_out + t * C + c) = pack8(g);
+        if (last) {
+#pragma unroll
+            for (int i = 0; i < KM; ++i) {
+                if (i >= k) continue;
+                float v[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    float a = 0.f;
+#pragma unroll
+                    for (int j = 0; j < KM; ++j) a = fmaf(Hsh[(tt * KM + j) * KM + i], dn[j][q], a);
+                    v[q] = a;
+                }
+                float4* dst = reinterpret_cast<float4*>(dxact_out + t * kC + (long long)i * C + c);
+                dst[0] = make_float4(v[0], v[1], v[2], v[3]);
+                dst[1] = make_float4(v[4], v[5], v[6], v[7]);
+            }
+        }
+    }
+}
+
 inline int kw_of(const Dims& d) {
     const int km = d.kapmax;
     return km <= 4 ? 4 : km <= 8 ? 8 : km <= 12 ? 12 : 16;

@@ -77,6 +77,17 @@ cudaError_t fwd_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs
     return cudaGetLastError();
 }
 
+template <int KM>
+cudaError_t fwd8_kw(const Dims& d, int slot, int T, const uint16_t* out, const float* emat,
+                    const uint16_t* xact, const int* I, const float* hres, uint16_t* xact_next,
+                    uint16_t* X, cudaStream_t st) {
+    const int TB = 32;
+    const size_t sm = (size_t)TB * (KM + KM * KM + KM) * 4;
+    dim3 grid((d.C + W8 - 1) / W8, (T + TB - 1) / TB);
+    k_wb_fwd8<KM><<<grid, WT, sm, st>>>(d, slot, T, TB, out, emat, xact, I, hres, xact_next, X); note_launch();
+    return cudaGetLastError();
+}
+
 }  // namespace
 
 int wb_nslice(int C) { return (C + WSL - 1) / WSL; }
@@ -101,11 +112,10 @@ cudaError_t launch_wb_fwd(const Dims& d, int slot, int T, const uint16_t* out, C
                           const float* hres, uint16_t* xact_next, uint16_t* X, cudaStream_t st) {
     const bool conv = d.K[slot] > 1;
     if (d.k <= 4) {
-        if (!conv && wb_fast(d)) return fwd_kw<4, 0, 2>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st);
-        if (!conv) return fwd_kw<4, 0, 0>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st);
+        if (!conv) return fwd8_kw<4>(d, slot, T, out, emat, xact, I, hres, xact_next, X, st);
         XHC_KW_DISPATCH(d, wb_fast(d), (fwd_kw<4, KWC, KSC>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st)));
     }
-    if (!conv) return fwd_kw<8, 0, 0>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st);
+    if (!conv) return fwd8_kw<8>(d, slot, T, out, emat, xact, I, hres, xact_next, X, st);
     XHC_KW_DISPATCH(d, false, (fwd_kw<8, KWC, KSC>(d, slot, T, out, cw, emat, nslice, xact, I, hres, xact_next, X, st)));
 }
 

@@ -259,7 +259,8 @@ cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, 
                          const int* I, const float* dxact, const float* scal, int scal_ld,
                          uint16_t* dX, int* err, cudaStream_t st);
 int wb_nslice(int C);
-int wb_conv_runs(const Dims& d, int64_t T);  // runs (conv weight-gradient partials) of wb_bapp
+int wb_conv_runs(const Dims& d, int64_t T);
+int wb_bred_slices(const Dims& d, int slot);  // partial-sum slices of wb_bred (and bwd_coef)  // runs (conv weight-gradient partials) of wb_bapp
 cudaError_t launch_wb_gram(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
                            int nslice, float* red, cudaStream_t st);
 cudaError_t launch_wb_coef(const Dims& d, int slot, int T, const float* red, int nslice, const float* p,
