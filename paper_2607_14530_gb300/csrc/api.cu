@@ -346,6 +346,51 @@ xhc_status xhc_saved_layout_of(const xhc_handle* h, int64_t T, xhc_saved_layout*
 
 namespace {
 
+// Side stream of a device (created on first use, kept for the life of the process): work of a
+// call that does not feed the rest of the call (weight gradients, column sums) runs there,
+// forked from and joined back into the caller's stream with events, so it overlaps the
+// bandwidth- or latency-bound kernels of the main chain.  Without a side stream everything runs
+// on the caller's stream.
+static std::mutex g_smu;
+static cudaStream_t g_side[64];
+
+static cudaStream_t side_stream() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> lk(g_smu);
+    if (!g_side[dev]) {
+        cudaStream_t st = nullptr;
+        if (cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking) != cudaSuccess) {
+            cudaGetLastError();
+            return nullptr;
+        }
+        g_side[dev] = st;
+    }
+    return g_side[dev];
+}
+
+// `to` waits for the work enqueued so far on `from` (a fresh event per call: concurrent callers
+// never wait on each other's record)
+static bool stream_after(cudaStream_t to, cudaStream_t from) {
+    cudaEvent_t e;
+    if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return false;
+    bool ok = cudaEventRecord(e, from) == cudaSuccess && cudaStreamWaitEvent(to, e, 0) == cudaSuccess;
+    cudaEventDestroy(e);
+    return ok;
+}
+
+// a stream forked from `main`: the side stream, or `main` itself
+static cudaStream_t fork_from(cudaStream_t main) {
+    cudaStream_t side = side_stream();
+    if (!side || !stream_after(side, main)) return main;
+    return side;
+}
+
+static xhc_status join_into(cudaStream_t main, cudaStream_t side) {
+    if (side == main) return XHC_OK;
+    return stream_after(main, side) ? XHC_OK : XHC_ERR_CUDA;
+}
+
 struct Ctx {
     Dims d;
     Layout L;
@@ -597,6 +642,30 @@ xhc_status xhc_post_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
                              P->alpha_post, P->b_post[slot],
                              P->alpha_res, P->b_res, c.W<float>(c.L.tokmat), c.W<float>(c.L.dz),
                              c.W<float>(c.L.dp), c.W<float>(c.L.tokgrad), c.st));
+    // weight gradient of the post/res projections and the alpha / b column sums need only dZ_act
+    // and the per-token contributions: side stream, overlapping the apply kernel
+    const cudaStream_t sd = fork_from(c.st);
+    if (T32 < 64 || d.k * d.C < 128) {
+        const int ts = std::min(c.L.tsplits, pick_tsplits(d.k * d.C, T32));
+        XHC_K("wgrad_active", sd, launch_wgrad(c.xact(slot), (int64_t)d.k * d.C, d.k * d.C, T32,
+                                               c.W<float>(c.L.dz), n, n, ts, c.W<float>(c.L.wpart),
+                                               act_segs_g(d, g, slot), sd));
+    } else {
+        ProjTcPlan pl = plan_proj_tc(d.k * d.C, T32, n, device_sms(), false);
+        XHC_K("wgrad_tc_active", sd, launch_wgrad_tc(c.xact(slot), T32, d.k * d.C, c.W<float>(c.L.dz), n, n,
+                                                     c.W<uint16_t>(c.L.dzpack), pl, c.W<float>(c.L.wpart),
+                                                     c.W<int>(c.L.err), sd));
+        XHC_K("wgrad_reduce", sd, launch_wgrad_reduce(c.W<float>(c.L.wpart), pl.nseg, d.k * d.C, n,
+                                                      act_segs_g(d, g, slot), sd));
+    }
+    float* tg = c.W<float>(c.L.tokgrad);
+    float* scr = c.W<float>(c.L.colscr);
+    XHC_K("colsum", sd, launch_colsum(tg, T32, NTG, d.k * K, g->b_post[slot], 1, scr, sd));
+    XHC_K("colsum", sd, launch_colsum(tg + d.k * K, T32, NTG, 1, g->alpha_post + slot, 1, scr, sd));
+    if (last) {
+        XHC_K("colsum", sd, launch_colsum(tg + d.k * K + 1, T32, NTG, d.k * d.k, g->b_res, 1, scr, sd));
+        XHC_K("colsum", sd, launch_colsum(tg + d.k * K + 1 + d.k * d.k, T32, NTG, 1, g->alpha_res, 1, scr, sd));
+    }
     // d_out, conv weight-gradient partials and (last slot) the mixed active gradient; the
     // active gradient of earlier slots is read in place and completed by pre_bwd(slot)
     XHC_K("wb_bapp", c.st, launch_wb_bapp(d, slot, T32, out, cw, dX, c.S<int>(c.L.I), dxact,
@@ -606,33 +675,12 @@ xhc_status xhc_post_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
     // dZ_act stays in the workspace: pre_bwd(slot) applies it to dX_act on the tensor cores
     if (!dxa_tc_ok(T32, d.k, d.C, n))
         XHC_K("gemm_dzw", c.st, launch_gemm_dzw(d, T32, c.W<float>(c.L.dz), n, n, wa, d.k * d.C, dxact, c.st));
-    if (T32 < 64 || d.k * d.C < 128) {
-        const int ts = std::min(c.L.tsplits, pick_tsplits(d.k * d.C, T32));
-        XHC_K("wgrad_active", c.st, launch_wgrad(c.xact(slot), (int64_t)d.k * d.C, d.k * d.C, T32,
-                                                 c.W<float>(c.L.dz), n, n, ts, c.W<float>(c.L.wpart),
-                                                 act_segs_g(d, g, slot), c.st));
-    } else {
-        ProjTcPlan pl = plan_proj_tc(d.k * d.C, T32, n, device_sms(), false);
-        XHC_K("wgrad_tc_active", c.st, launch_wgrad_tc(c.xact(slot), T32, d.k * d.C, c.W<float>(c.L.dz), n, n,
-                                                       c.W<uint16_t>(c.L.dzpack), pl, c.W<float>(c.L.wpart),
-                                                       c.W<int>(c.L.err), c.st));
-        XHC_K("wgrad_reduce", c.st, launch_wgrad_reduce(c.W<float>(c.L.wpart), pl.nseg, d.k * d.C, n,
-                                                        act_segs_g(d, g, slot), c.st));
-    }
-    float* tg = c.W<float>(c.L.tokgrad);
-    float* scr = c.W<float>(c.L.colscr);
-    XHC_K("colsum", c.st, launch_colsum(tg, T32, NTG, d.k * K, g->b_post[slot], 1, scr, c.st));
-    XHC_K("colsum", c.st, launch_colsum(tg + d.k * K, T32, NTG, 1, g->alpha_post + slot, 1, scr, c.st));
-    if (last) {
-        XHC_K("colsum", c.st, launch_colsum(tg + d.k * K + 1, T32, NTG, d.k * d.k, g->b_res, 1, scr, c.st));
-        XHC_K("colsum", c.st, launch_colsum(tg + d.k * K + 1 + d.k * d.k, T32, NTG, 1, g->alpha_res, 1, scr, c.st));
-    }
     if (K > 1) {
         ConvGradPtrs gc;
         for (int j = 0; j < 3; ++j) gc.w[j] = (j < d.nconv) ? g->conv_w[slot][j] : nullptr;
         XHC_K("conv_wgrad_reduce", c.st, launch_conv_wgrad_reduce(d, slot, c.W<float>(c.L.cpart), c.L.ntiles, gc, c.st));
     }
-    return XHC_OK;
+    return join_into(c.st, sd);
 }
 
 xhc_status xhc_pre_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
@@ -671,6 +719,31 @@ xhc_status xhc_pre_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
                               c.S<float>(c.L.zfull), c.S<float>(c.L.stats), c.W<float>(c.L.wsum),
                               c.S<int>(c.L.I), c.W<float>(c.L.dp), P->alpha_pre,
                               c.W<float>(c.L.dz), c.W<float>(c.L.tokgrad), c.st));
+    // the full-state weight gradient and the pre-map / router column sums need only dZ and the
+    // per-token contributions: side stream, overlapping the full-state dX
+    const cudaStream_t sd = fork_from(c.st);
+    if (T32 < 64 || d.N * d.C < 128) {
+        const int ts = std::min(c.L.tsplits, pick_tsplits(d.N * d.C, T32));
+        XHC_K("wgrad_full", sd, launch_wgrad(X, (int64_t)d.N * d.C, d.N * d.C, T32, c.W<float>(c.L.dz),
+                                               d.nfull, d.nfull, ts, c.W<float>(c.L.wpart),
+                                               full_segs_g(d, g), sd));
+    } else {
+        const ProjTcPlan& pl = c.L.twf;
+        XHC_K("wgrad_tc_full", sd, launch_wgrad_tc(X, T32, d.N * d.C, c.W<float>(c.L.dz), d.nfull, d.nfull,
+                                                     c.W<uint16_t>(c.L.dzpack), pl, c.W<float>(c.L.wpart),
+                                                     c.W<int>(c.L.err), sd));
+        XHC_K("wgrad_reduce", sd, launch_wgrad_reduce(c.W<float>(c.L.wpart), pl.nseg, d.N * d.C, d.nfull,
+                                                        full_segs_g(d, g), sd));
+    }
+    float* tg = c.W<float>(c.L.tokgrad);
+    float* scr = c.W<float>(c.L.colscr);
+    XHC_K("colsum", sd, launch_colsum(tg + 2, T32, NTG, d.G * d.N, g->b_pre, 1, scr, sd));
+    XHC_K("colsum", sd, launch_colsum(tg + 2 + d.G * d.N, T32, NTG, d.G, g->alpha_pre, 1, scr, sd));
+    if (d.hr) {
+        float* rsum = c.W<float>(c.L.rsum);
+        XHC_K("colsum", sd, launch_colsum(tg + 2 + d.G * d.N + d.G, T32, NTG, d.N, rsum, 0, scr, sd));
+        XHC_K("sub_rows", sd, launch_sub_rows(g->W_r, d.N * d.C, d.N, rsum, sd));
+    }
     const WSegs wf = full_segs(d, P);
     if (dx_tc_ok(T32, d.N, d.C, d.nfull)) {
         XHC_K("dx_tc", c.st, launch_dx_tc(d, T32, c.W<float>(c.L.dz), wf, c.W<uint16_t>(c.L.dz16),
@@ -682,29 +755,7 @@ xhc_status xhc_pre_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
                                               c.S<int>(c.L.I), c.W<float>(c.L.dxact),
                                               c.W<float>(c.L.tokgrad), dX, c.st));
     }
-    if (T32 < 64 || d.N * d.C < 128) {
-        const int ts = std::min(c.L.tsplits, pick_tsplits(d.N * d.C, T32));
-        XHC_K("wgrad_full", c.st, launch_wgrad(X, (int64_t)d.N * d.C, d.N * d.C, T32, c.W<float>(c.L.dz),
-                                               d.nfull, d.nfull, ts, c.W<float>(c.L.wpart),
-                                               full_segs_g(d, g), c.st));
-    } else {
-        const ProjTcPlan& pl = c.L.twf;
-        XHC_K("wgrad_tc_full", c.st, launch_wgrad_tc(X, T32, d.N * d.C, c.W<float>(c.L.dz), d.nfull, d.nfull,
-                                                     c.W<uint16_t>(c.L.dzpack), pl, c.W<float>(c.L.wpart),
-                                                     c.W<int>(c.L.err), c.st));
-        XHC_K("wgrad_reduce", c.st, launch_wgrad_reduce(c.W<float>(c.L.wpart), pl.nseg, d.N * d.C, d.nfull,
-                                                        full_segs_g(d, g), c.st));
-    }
-    float* tg = c.W<float>(c.L.tokgrad);
-    float* scr = c.W<float>(c.L.colscr);
-    XHC_K("colsum", c.st, launch_colsum(tg + 2, T32, NTG, d.G * d.N, g->b_pre, 1, scr, c.st));
-    XHC_K("colsum", c.st, launch_colsum(tg + 2 + d.G * d.N, T32, NTG, d.G, g->alpha_pre, 1, scr, c.st));
-    if (d.hr) {
-        float* rsum = c.W<float>(c.L.rsum);
-        XHC_K("colsum", c.st, launch_colsum(tg + 2 + d.G * d.N + d.G, T32, NTG, d.N, rsum, 0, scr, c.st));
-        XHC_K("sub_rows", c.st, launch_sub_rows(g->W_r, d.N * d.C, d.N, rsum, c.st));
-    }
-    return XHC_OK;
+    return join_into(c.st, sd);
 }
 
 }  // extern "C"
