@@ -26,7 +26,11 @@
  * Ownership and execution: every buffer is allocated and owned by the caller (device memory
  * unless stated).  The library allocates no device memory, never synchronises, and enqueues
  * all work asynchronously on the caller's stream (a cudaStream_t passed as void*; NULL = the
- * legacy default stream).  `saved` (xhc_saved_bytes) carries the group's forward state to its
+ * legacy default stream).  post_bwd and pre_bwd(0) run their weight-gradient and column-sum
+ * kernels on an internal stream of the device (created on first use, one per device), forked
+ * from the caller's stream with an event after the work they depend on and joined back into
+ * it with an event before the call returns: to the caller every call stays ordered on its
+ * stream.  `saved` (xhc_saved_bytes) carries the group's forward state to its
  * backward and must not be touched in between; `workspace` (xhc_workspace_bytes) is scratch that
  * must stay the same buffer across the calls of one group's forward and across those of its
  * backward, and may be reused by other groups between those phases.  Two groups in flight on
