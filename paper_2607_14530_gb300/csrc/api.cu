@@ -180,6 +180,7 @@ Layout make_layout(const Dims& d, int64_t T) {
     L.part = o;
     o = al(o + std::max((size_t)L.splits_full * d.nfull, (size_t)L.splits_act * nact_max) * t * 4);
     L.pstats = o; o = al(o + (size_t)std::max(L.splits_full, L.splits_act) * t * 2 * 4);
+    L.astat = o; o = al(o + t * 2 * 4);
     L.wsum = o; o = al(o + (size_t)d.N * 4);
     L.rsum = o; o = al(o + (size_t)d.N * 4);
     L.base = o; o = al(o + (size_t)(d.G - 1) * t * d.C * 4);
@@ -520,7 +521,8 @@ ConvPtrs conv_of(const Dims& d, const xhc_params* P, int slot) {
 xhc_status active_maps(const Ctx& c, int slot, const xhc_params* P) {
     const Dims& d = c.d;
     const WSegs wa = act_segs(d, P, slot);
-    int splits = c.L.splits_act;
+    int splits = c.L.splits_act, ssplits = c.L.splits_act;
+    float* pstats = c.W<float>(c.L.pstats);
     if (c.T < 128 || d.k * d.C < 64) {
         XHC_K("rowproj_active", c.st, launch_rowproj(c.xact(slot), (int64_t)d.k * d.C, d.k * d.C, c.T, wa,
                                                      d.nact[slot], c.L.splits_act, c.W<float>(c.L.part),
@@ -530,11 +532,14 @@ xhc_status active_maps(const Ctx& c, int slot, const xhc_params* P) {
         splits = pl.nseg;
         XHC_K("pack_w", c.st, launch_pack_w(wa, d.nact[slot], pl.NB, d.k * d.C,
                                             c.W<uint16_t>(c.L.wpack), c.st));
+        // the norm statistics come from the read / input pass that produced x_act
         XHC_K("proj_tc_active", c.st, launch_proj_tc(c.xact(slot), c.T, d.k * d.C, c.W<uint16_t>(c.L.wpack),
-                                                     d.nact[slot], pl, c.W<float>(c.L.part),
-                                                     c.W<float>(c.L.pstats), c.W<int>(c.L.err), c.st));
+                                                     d.nact[slot], pl, c.W<float>(c.L.part), nullptr,
+                                                     c.W<int>(c.L.err), c.st));
+        pstats = c.W<float>(c.L.astat);
+        ssplits = 1;
     }
-    XHC_K("coef_act", c.st, launch_coef_act(d, slot, c.T, c.W<float>(c.L.part), c.W<float>(c.L.pstats),
+    XHC_K("coef_act", c.st, launch_coef_act(d, slot, c.T, c.W<float>(c.L.part), pstats, ssplits,
                              splits, P->alpha_post, P->b_post[slot], P->alpha_res, P->b_res,
                              c.S<float>(c.L.zact[slot]), c.S<float>(c.L.rs[slot]),
                              c.S<float>(c.L.hpost[slot]), c.S<float>(c.L.hres), c.st));
@@ -579,10 +584,10 @@ xhc_status xhc_pre_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
                                   c.S<float>(c.L.zfull), c.S<float>(c.L.stats),
                                   c.S<float>(c.L.hpre), c.S<int>(c.L.I), c.S<float>(c.L.p), c.st));
         XHC_K("read", c.st, launch_read(d, c.T, X, c.S<float>(c.L.hpre), c.S<int>(c.L.I), input,
-                             c.W<float>(c.L.base), c.xact(0), c.st));
+                             c.W<float>(c.L.base), c.xact(0), c.W<float>(c.L.astat), c.st));
     } else {
         XHC_K("input", c.st, launch_input(d, slot, c.T, c.W<float>(c.L.base), c.xact(slot),
-                              c.S<float>(c.L.hpre), c.S<int>(c.L.I), input, c.st));
+                              c.S<float>(c.L.hpre), c.S<int>(c.L.I), input, c.W<float>(c.L.astat), c.st));
     }
     return active_maps(c, slot, P);
 }

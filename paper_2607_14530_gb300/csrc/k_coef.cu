@@ -248,7 +248,7 @@ cudaError_t launch_coef_full(const Dims& d, int T, const float* part, const floa
 
 template <int KM>
 __global__ void k_coef_act(Dims d, int slot, int T, const float* __restrict__ part,
-                           const float* __restrict__ pstats, int splits,
+                           const float* __restrict__ pstats, int ssplits, int splits,
                            const float* __restrict__ alpha_post, const float* __restrict__ b_post,
                            const float* __restrict__ alpha_res, const float* __restrict__ b_res,
                            float* __restrict__ zact, float* __restrict__ rs,
@@ -258,7 +258,7 @@ __global__ void k_coef_act(Dims d, int slot, int T, const float* __restrict__ pa
     const int k = d.k, K = d.K[slot], n = d.nact[slot];
     const bool last = (slot == d.G - 1);
     float s2 = 0.f;
-    for (int q = 0; q < splits; ++q) s2 += pstats[((int64_t)q * T + t) * 2 + 1];
+    for (int q = 0; q < ssplits; ++q) s2 += pstats[((int64_t)q * T + t) * 2 + 1];
     const float r = 1.0f / sqrtf(s2 / (float)(k * d.C) + d.eps);
     rs[t] = r;
     const float ap = alpha_post[slot];
@@ -295,14 +295,14 @@ __global__ void k_coef_act(Dims d, int slot, int T, const float* __restrict__ pa
 }
 
 cudaError_t launch_coef_act(const Dims& d, int slot, int T, const float* part,
-                            const float* pstats, int splits, const float* alpha_post,
+                            const float* pstats, int ssplits, int splits, const float* alpha_post,
                             const float* b_post, const float* alpha_res, const float* b_res,
                             float* zact, float* rs, float* hpost, float* hres, cudaStream_t st) {
     if (d.k <= 4) {
-        k_coef_act<4><<<(T + 127) / 128, 128, 0, st>>>(d, slot, T, part, pstats, splits, alpha_post,
+        k_coef_act<4><<<(T + 127) / 128, 128, 0, st>>>(d, slot, T, part, pstats, ssplits, splits, alpha_post,
                                                         b_post, alpha_res, b_res, zact, rs, hpost, hres); note_launch();
     } else {
-        k_coef_act<8><<<(T + 127) / 128, 128, 0, st>>>(d, slot, T, part, pstats, splits, alpha_post,
+        k_coef_act<8><<<(T + 127) / 128, 128, 0, st>>>(d, slot, T, part, pstats, ssplits, splits, alpha_post,
                                                         b_post, alpha_res, b_res, zact, rs, hpost, hres); note_launch();
     }
     return cudaGetLastError();

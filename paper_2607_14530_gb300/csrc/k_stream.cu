@@ -1,8 +1,11 @@
 // Streaming kernels of the connection op (HBM-bound, fp32 math on bf16 data):
 //   read        second full-state pass: dense read of slot 0 (Eq. dense_read), non-active base
 //               readouts of the later slots (Eq. app_four_sub_base), gather of the active
-//               streams (Alg. 1 Gather)
-//   input       input_t = base_t + sum_j H_pre_t[I_j] x_act_j (Eq. app_active_state_correction)
+//               streams (Alg. 1 Gather), sum of squares of the gathered rows
+//   input       input_t = base_t + sum_j H_pre_t[I_j] x_act_j (Eq. app_active_state_correction),
+//               sum of squares of x_act
+//   (the sums of squares are the norm statistics of the slot's active-state projection, which
+//   then reads its operand only through the tensor-core pipeline)
 //   restore     put the saved entry rows back into X before the backward
 //   conv_wgrad_reduce  sum of the per-run conv weight-gradient partials
 //   dinput_act  dense-read backward on the active streams (and dH_pre of the active streams)
@@ -17,6 +20,20 @@ static int chunk_threads(int C) {
 }
 
 // ---------------------------------------------------------------------------------------------
+// sum over the block (blockDim a multiple of 32, at most 256 threads); the total is valid in
+// thread 0.  Fixed order: deterministic.
+__device__ __forceinline__ float block_sum(float v, float* sh) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if ((threadIdx.x & 31) == 0) sh[threadIdx.x >> 5] = v;
+    __syncthreads();
+    float r = 0.f;
+    if (threadIdx.x == 0)
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) r += sh[w];
+    return r;
+}
+
+// ---------------------------------------------------------------------------------------------
 // read: one block per token, threads over 8-channel chunks.
 
 __global__ void __launch_bounds__(256) k_read(Dims d, int T, const uint16_t* __restrict__ X,
@@ -24,8 +41,10 @@ __global__ void __launch_bounds__(256) k_read(Dims d, int T, const uint16_t* __r
                                               const int* __restrict__ I,
                                               uint16_t* __restrict__ input0,
                                               float* __restrict__ base,
-                                              uint16_t* __restrict__ xact0) {
+                                              uint16_t* __restrict__ xact0,
+                                              float* __restrict__ astat) {
     __shared__ float sh[4 * MAXN];
+    __shared__ float red[8];
     __shared__ int slotmap[MAXN];
     const int t = blockIdx.x;
     const int N = d.N, G = d.G, C = d.C;
@@ -38,6 +57,7 @@ __global__ void __launch_bounds__(256) k_read(Dims d, int T, const uint16_t* __r
     }
     __syncthreads();
     const uint16_t* xt = X + (int64_t)t * N * C;
+    float ss = 0.f;  // sum of squares of the gathered active rows (their projection's norm)
     for (int c8 = threadIdx.x; c8 < C / 8; c8 += blockDim.x) {
         float acc[4][8];
 #pragma unroll
@@ -71,6 +91,8 @@ __global__ void __launch_bounds__(256) k_read(Dims d, int T, const uint16_t* __r
                     }
                 } else {
                     *reinterpret_cast<uint4*>(xact0 + ((int64_t)t * d.k + j) * C + c8 * 8) = ub[ii];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) ss = fmaf(x[e], x[e], ss);
                 }
             }
         }
@@ -84,11 +106,16 @@ __global__ void __launch_bounds__(256) k_read(Dims d, int T, const uint16_t* __r
             }
         }
     }
+    ss = block_sum(ss, red);
+    if (threadIdx.x == 0) {
+        astat[(int64_t)t * 2 + 0] = 0.f;
+        astat[(int64_t)t * 2 + 1] = ss;
+    }
 }
 
 cudaError_t launch_read(const Dims& d, int T, const uint16_t* X, const float* hpre, const int* I,
-                        uint16_t* input0, float* base, uint16_t* xact0, cudaStream_t st) {
-    k_read<<<T, chunk_threads(d.C), 0, st>>>(d, T, X, hpre, I, input0, base, xact0); note_launch();
+                        uint16_t* input0, float* base, uint16_t* xact0, float* astat, cudaStream_t st) {
+    k_read<<<T, chunk_threads(d.C), 0, st>>>(d, T, X, hpre, I, input0, base, xact0, astat); note_launch();
     return cudaGetLastError();
 }
 
@@ -100,12 +127,15 @@ __global__ void __launch_bounds__(256) k_input(Dims d, int slot, int T,
                                                const uint16_t* __restrict__ xact,
                                                const float* __restrict__ hpre,
                                                const int* __restrict__ I,
-                                               uint16_t* __restrict__ input) {
+                                               uint16_t* __restrict__ input,
+                                               float* __restrict__ astat) {
     __shared__ float hj[MAXK];
+    __shared__ float red[8];
     const int t = blockIdx.x, C = d.C;
     if (threadIdx.x < d.k)
         hj[threadIdx.x] = hpre[((int64_t)t * d.G + slot) * d.N + I[(int64_t)t * d.k + threadIdx.x]];
     __syncthreads();
+    float ss = 0.f;  // sum of squares of the active state (its projection's norm)
     for (int c8 = threadIdx.x; c8 < C / 8; c8 += blockDim.x) {
         const float* bp = base + ((int64_t)(slot - 1) * T + t) * C + c8 * 8;
         const float4 b0 = *reinterpret_cast<const float4*>(bp);
@@ -116,15 +146,23 @@ __global__ void __launch_bounds__(256) k_input(Dims d, int slot, int T,
             float x[8];
             unpack8(u, x);
 #pragma unroll
-            for (int e = 0; e < 8; ++e) acc[e] = fmaf(hj[j], x[e], acc[e]);
+            for (int e = 0; e < 8; ++e) {
+                acc[e] = fmaf(hj[j], x[e], acc[e]);
+                ss = fmaf(x[e], x[e], ss);
+            }
         }
         *reinterpret_cast<uint4*>(input + (int64_t)t * C + c8 * 8) = pack8(acc);
+    }
+    ss = block_sum(ss, red);
+    if (threadIdx.x == 0) {
+        astat[(int64_t)t * 2 + 0] = 0.f;
+        astat[(int64_t)t * 2 + 1] = ss;
     }
 }
 
 cudaError_t launch_input(const Dims& d, int slot, int T, const float* base, const uint16_t* xact,
-                         const float* hpre, const int* I, uint16_t* input, cudaStream_t st) {
-    k_input<<<T, chunk_threads(d.C), 0, st>>>(d, slot, T, base, xact, hpre, I, input); note_launch();
+                         const float* hpre, const int* I, uint16_t* input, float* astat, cudaStream_t st) {
+    k_input<<<T, chunk_threads(d.C), 0, st>>>(d, slot, T, base, xact, hpre, I, input, astat); note_launch();
     return cudaGetLastError();
 }
 

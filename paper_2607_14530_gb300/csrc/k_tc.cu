@@ -145,7 +145,7 @@ struct ProjTcArgs {
     int stages;         // smem ring depth
     int kps;            // k-blocks of 64 per stage (projections; 1 for the weight gradients)
     float* part;        // [nseg][T][nfull]
-    float* pstats;      // [nseg][T][2]
+    float* pstats;      // [nseg][T][2] row sums / sums of squares of A; null: not computed
     int* err;           // set to a nonzero code when a wait gives up
 };
 
@@ -294,7 +294,11 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
         while (g < g1 && ok) {
             const int m = (int)(g / a.KB);
             const long long gend = min(g1, (long long)(m + 1) * a.KB);
-            float s1 = 0.f, s2 = 0.f;
+            // row sums in packed pairs, four independent accumulators each (short dependency
+            // chains, half the instructions of scalar sums)
+            float2 a1[4], a2[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) a1[e] = a2[e] = make_float2(0.f, 0.f);
             for (; g < gend; ++g, ++it) {
                 const int s = (int)(it % STAGES);
                 const uint32_t ph = (uint32_t)((it / STAGES) & 1);
@@ -303,20 +307,24 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                     ok = false;
                     break;
                 }
-                if (!A_MN) {
+                if (!A_MN && a.pstats) {
                     // row r of the A tile: 128 bytes, 16-byte chunks permuted by the swizzle (the
                     // sum over the row does not depend on the order)
                     for (int p2 = 0; p2 < KPS; ++p2) {
                         const uint4* row = reinterpret_cast<const uint4*>(smem + (size_t)s * STAGE +
                                                                           p2 * BM * BK * 2 + r * 128);
+                        uint4 v[8];
+#pragma unroll
+                        for (int q = 0; q < 8; ++q) v[q] = row[q];
 #pragma unroll
                         for (int q = 0; q < 8; ++q) {
-                            float f[8];
-                            unpack8(row[q], f);
+                            const uint32_t w[4] = {v[q].x, v[q].y, v[q].z, v[q].w};
 #pragma unroll
-                            for (int e = 0; e < 8; ++e) {
-                                s1 += f[e];
-                                s2 = fmaf(f[e], f[e], s2);
+                            for (int e = 0; e < 4; ++e) {
+                                const float2 f = make_float2(__uint_as_float(w[e] << 16),
+                                                             __uint_as_float(w[e] & 0xffff0000u));
+                                a1[e] = __fadd2_rn(a1[e], f);
+                                a2[e] = __ffma2_rn(f, f, a2[e]);
                             }
                         }
                     }
@@ -348,7 +356,9 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                     for (int q = 0; q < n; ++q) dst[o0 + q] = hi[q] + lo[q];
                 }
             }
-            if (!A_MN && t < a.T) {
+            if (!A_MN && a.pstats && t < a.T) {
+                const float s1 = (a1[0].x + a1[0].y) + (a1[1].x + a1[1].y) + (a1[2].x + a1[2].y) + (a1[3].x + a1[3].y);
+                const float s2 = (a2[0].x + a2[0].y) + (a2[1].x + a2[1].y) + (a2[2].x + a2[2].y) + (a2[3].x + a2[3].y);
                 a.pstats[((long long)j * a.T + t) * 2 + 0] = s1;
                 a.pstats[((long long)j * a.T + t) * 2 + 1] = s2;
             }
@@ -485,8 +495,10 @@ cudaError_t launch_proj_tc(const uint16_t* X, int T, int K, const uint16_t* Wpac
         return cudaErrorInvalidValue;
     cudaError_t e = cudaMemsetAsync(part, 0, (size_t)p.nseg * T * nfull * sizeof(float), st);
     if (e != cudaSuccess) return e;
-    e = cudaMemsetAsync(pstats, 0, (size_t)p.nseg * T * 2 * sizeof(float), st);
-    if (e != cudaSuccess) return e;
+    if (pstats) {
+        e = cudaMemsetAsync(pstats, 0, (size_t)p.nseg * T * 2 * sizeof(float), st);
+        if (e != cudaSuccess) return e;
+    }
     const size_t sm = proj_tc_smem(p);
     e = cudaFuncSetAttribute((const void*)k_proj_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;

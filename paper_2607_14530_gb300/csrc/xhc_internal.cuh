@@ -84,6 +84,8 @@ struct Layout {
     size_t wpack;           // bf16 [NB][N*C]: hi / lo rows of the full-state projection weight
     size_t part;            // f32 [splits][T][nmax] projection split-K partials
     size_t pstats;          // f32 [splits][T][2]
+    size_t astat;           // f32 [T][2]: row statistics of the active state being mapped (sum
+                            // of squares at 1; the sum at 0 is not used and left 0)
     size_t wsum;            // f32 [N]: column sums of W_r
     size_t rsum;            // f32 [N]: sum_t mu_t dZ_r[t] (router mean-term gradient)
     size_t base;            // f32 [G-1][T][C]: non-active base readouts of slots 1..G-1
@@ -240,6 +242,7 @@ void note_launch();  // counts every kernel launch of the library
 cudaError_t launch_rowproj(const uint16_t* A, int64_t lda, int K, int T, const WSegs& W, int n,
                            int splits, float* part, float* pstats, cudaStream_t st);
 cudaError_t launch_pack_w(const WSegs& W, int nfull, int NB, int K, uint16_t* Wpack, cudaStream_t st);
+// pstats null: no row statistics (the caller has them from the kernel that wrote X)
 cudaError_t launch_proj_tc(const uint16_t* X, int T, int K, const uint16_t* Wpack, int nfull,
                            const ProjTcPlan& p, float* part, float* pstats, int* err,
                            cudaStream_t st);
@@ -285,13 +288,13 @@ cudaError_t launch_coef_full(const Dims& d, int T, const float* part, const floa
                              const float* b_pre, float* zfull, float* stats, float* hpre,
                              int* I, float* p, cudaStream_t st);
 cudaError_t launch_coef_act(const Dims& d, int slot, int T, const float* part,
-                            const float* pstats, int splits, const float* alpha_post,
+                            const float* pstats, int ssplits, int splits, const float* alpha_post,
                             const float* b_post, const float* alpha_res, const float* b_res,
                             float* zact, float* rs, float* hpost, float* hres, cudaStream_t st);
 cudaError_t launch_read(const Dims& d, int T, const uint16_t* X, const float* hpre, const int* I,
-                        uint16_t* input0, float* base, uint16_t* xact0, cudaStream_t st);
+                        uint16_t* input0, float* base, uint16_t* xact0, float* astat, cudaStream_t st);
 cudaError_t launch_input(const Dims& d, int slot, int T, const float* base, const uint16_t* xact,
-                         const float* hpre, const int* I, uint16_t* input, cudaStream_t st);
+                         const float* hpre, const int* I, uint16_t* input, float* astat, cudaStream_t st);
 cudaError_t launch_restore(const Dims& d, int T, const uint16_t* xact0, const int* I,
                            uint16_t* X, cudaStream_t st);
 cudaError_t launch_bwd_coef(const Dims& d, int slot, int T, const float* red, int nslice,
