@@ -180,7 +180,7 @@ Layout make_layout(const Dims& d, int64_t T) {
     L.part = o;
     o = al(o + std::max((size_t)L.splits_full * d.nfull, (size_t)L.splits_act * nact_max) * t * 4);
     L.pstats = o; o = al(o + (size_t)std::max(L.splits_full, L.splits_act) * t * 2 * 4);
-    L.astat = o; o = al(o + t * 2 * 4);
+    L.astat = o; o = al(o + (size_t)stream_warps(d.C) * t * 2 * 4);
     L.wsum = o; o = al(o + (size_t)d.N * 4);
     L.rsum = o; o = al(o + (size_t)d.N * 4);
     L.base = o; o = al(o + (size_t)(d.G - 1) * t * d.C * 4);
@@ -537,7 +537,7 @@ xhc_status active_maps(const Ctx& c, int slot, const xhc_params* P) {
                                                      d.nact[slot], pl, c.W<float>(c.L.part), nullptr,
                                                      c.W<int>(c.L.err), c.st));
         pstats = c.W<float>(c.L.astat);
-        ssplits = 1;
+        ssplits = stream_warps(d.C);
     }
     XHC_K("coef_act", c.st, launch_coef_act(d, slot, c.T, c.W<float>(c.L.part), pstats, ssplits,
                              splits, P->alpha_post, P->b_post[slot], P->alpha_res, P->b_res,

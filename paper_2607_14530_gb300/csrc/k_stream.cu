@@ -20,18 +20,15 @@ static int chunk_threads(int C) {
 }
 
 // ---------------------------------------------------------------------------------------------
-// sum over the block (blockDim a multiple of 32, at most 256 threads); the total is valid in
-// thread 0.  Fixed order: deterministic.
-__device__ __forceinline__ float block_sum(float v, float* sh) {
+// the block's warps each store their partial of a per-token sum: slot w of [warps][T][2], entry 1
+// (no block barrier, so the block retires as soon as its stores are issued)
+__device__ __forceinline__ void warp_partial(float v, float* __restrict__ dst, int T, int t) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    if ((threadIdx.x & 31) == 0) sh[threadIdx.x >> 5] = v;
-    __syncthreads();
-    float r = 0.f;
-    if (threadIdx.x == 0)
-        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) r += sh[w];
-    return r;
+    if ((threadIdx.x & 31) == 0) dst[((int64_t)(threadIdx.x >> 5) * T + t) * 2 + 1] = v;
 }
+
+int stream_warps(int C) { return chunk_threads(C) / 32; }
 
 // ---------------------------------------------------------------------------------------------
 // read: one block per token, threads over 8-channel chunks.
@@ -44,7 +41,6 @@ __global__ void __launch_bounds__(256) k_read(Dims d, int T, const uint16_t* __r
                                               uint16_t* __restrict__ xact0,
                                               float* __restrict__ astat) {
     __shared__ float sh[4 * MAXN];
-    __shared__ float red[8];
     __shared__ int slotmap[MAXN];
     const int t = blockIdx.x;
     const int N = d.N, G = d.G, C = d.C;
@@ -106,11 +102,7 @@ __global__ void __launch_bounds__(256) k_read(Dims d, int T, const uint16_t* __r
             }
         }
     }
-    ss = block_sum(ss, red);
-    if (threadIdx.x == 0) {
-        astat[(int64_t)t * 2 + 0] = 0.f;
-        astat[(int64_t)t * 2 + 1] = ss;
-    }
+    warp_partial(ss, astat, T, t);
 }
 
 cudaError_t launch_read(const Dims& d, int T, const uint16_t* X, const float* hpre, const int* I,
@@ -130,7 +122,6 @@ __global__ void __launch_bounds__(256) k_input(Dims d, int slot, int T,
                                                uint16_t* __restrict__ input,
                                                float* __restrict__ astat) {
     __shared__ float hj[MAXK];
-    __shared__ float red[8];
     const int t = blockIdx.x, C = d.C;
     if (threadIdx.x < d.k)
         hj[threadIdx.x] = hpre[((int64_t)t * d.G + slot) * d.N + I[(int64_t)t * d.k + threadIdx.x]];
@@ -153,11 +144,7 @@ __global__ void __launch_bounds__(256) k_input(Dims d, int slot, int T,
         }
         *reinterpret_cast<uint4*>(input + (int64_t)t * C + c8 * 8) = pack8(acc);
     }
-    ss = block_sum(ss, red);
-    if (threadIdx.x == 0) {
-        astat[(int64_t)t * 2 + 0] = 0.f;
-        astat[(int64_t)t * 2 + 1] = ss;
-    }
+    warp_partial(ss, astat, T, t);
 }
 
 cudaError_t launch_input(const Dims& d, int slot, int T, const float* base, const uint16_t* xact,

@@ -84,8 +84,8 @@ struct Layout {
     size_t wpack;           // bf16 [NB][N*C]: hi / lo rows of the full-state projection weight
     size_t part;            // f32 [splits][T][nmax] projection split-K partials
     size_t pstats;          // f32 [splits][T][2]
-    size_t astat;           // f32 [T][2]: row statistics of the active state being mapped (sum
-                            // of squares at 1; the sum at 0 is not used and left 0)
+    size_t astat;           // f32 [stream_warps(C)][T][2]: per-warp partial sums of squares (at 1;
+                            // 0 is not written) of the active state being mapped
     size_t wsum;            // f32 [N]: column sums of W_r
     size_t rsum;            // f32 [N]: sum_t mu_t dZ_r[t] (router mean-term gradient)
     size_t base;            // f32 [G-1][T][C]: non-active base readouts of slots 1..G-1
@@ -291,6 +291,7 @@ cudaError_t launch_coef_act(const Dims& d, int slot, int T, const float* part,
                             const float* pstats, int ssplits, int splits, const float* alpha_post,
                             const float* b_post, const float* alpha_res, const float* b_res,
                             float* zact, float* rs, float* hpost, float* hres, cudaStream_t st);
+int stream_warps(int C);  // warps per block of the one-block-per-token stream kernels
 cudaError_t launch_read(const Dims& d, int T, const uint16_t* X, const float* hpre, const int* I,
                         uint16_t* input0, float* base, uint16_t* xact0, float* astat, cudaStream_t st);
 cudaError_t launch_input(const Dims& d, int slot, int T, const float* base, const uint16_t* xact,
