@@ -722,8 +722,7 @@ xhc_status xhc_pre_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
         XHC_K("colsum", c.st, launch_colsum(P->W_r, d.N * d.C, d.N, d.N, c.W<float>(c.L.wsum), 0,
                                c.W<float>(c.L.colscr), c.st));
     if (join_into(c.st, sa) != XHC_OK) return XHC_ERR_CUDA;
-    XHC_K("full_dots", c.st, launch_full_dots(d, T32, X, dinput, c.S<int>(c.L.I), c.S<float>(c.L.hpre), dX,
-                                              c.W<float>(c.L.dhpre), c.st));
+    XHC_K("full_dots", c.st, launch_full_dots(d, T32, X, dinput, c.S<int>(c.L.I), c.W<float>(c.L.dhpre), c.st));
     XHC_K("full_coef", c.st, launch_full_coef(d, T32, c.W<float>(c.L.dhpre), c.S<float>(c.L.hpre),
                               c.S<float>(c.L.zfull), c.S<float>(c.L.stats), c.W<float>(c.L.wsum),
                               c.S<int>(c.L.I), c.W<float>(c.L.dp), P->alpha_pre,
@@ -754,7 +753,7 @@ xhc_status xhc_pre_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
         XHC_K("sub_rows", sd, launch_sub_rows(g->W_r, d.N * d.C, d.N, rsum, sd));
     }
     const WSegs wf = full_segs(d, P);
-    if (dx_tc_ok(T32, d.N, d.C, d.nfull)) {
+    if (dx_tc_ok(T32, d.N, d.C, d.nfull, d.G)) {
         XHC_K("dx_tc", c.st, launch_dx_tc(d, T32, c.W<float>(c.L.dz), wf, c.W<uint16_t>(c.L.dz16),
                                           c.W<uint16_t>(c.L.w16), X, dinput, c.S<float>(c.L.hpre),
                                           c.S<int>(c.L.I), c.W<float>(c.L.dxact), c.W<float>(c.L.tokgrad),

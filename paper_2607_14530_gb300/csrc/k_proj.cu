@@ -242,8 +242,9 @@ cudaError_t launch_gemm_dzw(const Dims& d, int T, const float* dz, int ldz, int 
 
 // ---------------------------------------------------------------------------------------------
 // full_dx: dX[t][e] = base(t, e) + sum_o dz[t][o] W[e][o] + a_t + b_t * x[t][e], e = i*C + c,
-// base = dX_act[t][j][c] if stream i is active slot j, else dX[t][e] (which already holds the
-// dense-read gradient, added by full_dots)
+// base = dX_act[t][j][c] if stream i is active slot j, else dX[t][e] plus the dense-read
+// gradient sum_q H_pre[t][q][i] d_input_q[t][c] (Eq. dense_read reversed; din holds the G
+// d_input copies [G][T][C])
 
 __global__ void __launch_bounds__(256) k_full_dx(Dims d, int T, const float* __restrict__ dz,
                                                  WSegs W, const uint16_t* __restrict__ X,
@@ -307,6 +308,14 @@ __global__ void __launch_bounds__(256) k_full_dx(Dims d, int T, const float* __r
             const uint2 u = *reinterpret_cast<const uint2*>(dX + (int64_t)t * E + e);
             v[0] = __uint_as_float(u.x << 16); v[1] = __uint_as_float(u.x & 0xffff0000u);
             v[2] = __uint_as_float(u.y << 16); v[3] = __uint_as_float(u.y & 0xffff0000u);
+            for (int q = 0; q < d.G; ++q) {
+                const float h = hpre[((int64_t)t * d.G + q) * d.N + i];
+                const uint2 g = *reinterpret_cast<const uint2*>(din + ((int64_t)q * T + t) * d.C + c);
+                v[0] = fmaf(h, __uint_as_float(g.x << 16), v[0]);
+                v[1] = fmaf(h, __uint_as_float(g.x & 0xffff0000u), v[1]);
+                v[2] = fmaf(h, __uint_as_float(g.y << 16), v[2]);
+                v[3] = fmaf(h, __uint_as_float(g.y & 0xffff0000u), v[3]);
+            }
         }
         const float a = scal[(int64_t)t * NTG + 0], b = scal[(int64_t)t * NTG + 1];
         const uint2 xu = *reinterpret_cast<const uint2*>(X + (int64_t)t * E + e);

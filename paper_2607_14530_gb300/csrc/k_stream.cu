@@ -281,21 +281,19 @@ cudaError_t launch_dinput_act(const Dims& d, int slot, int T, int add_dx, const 
 }
 
 // ---------------------------------------------------------------------------------------------
-// full_dots: for the non-active streams i, dH_pre[t][q][i] = <x_i, d_input_q> and the dense-read
-// gradient dX[t][i] += sum_q H_pre[t][q][i] d_input_q (Eq. dense_read reversed).  One CTA per
-// token: the token's G d_input rows are staged in shared memory, then each warp takes whole
-// non-active streams (warp-level reductions only, no block barrier per stream).
+// full_dots: for the non-active streams i, dH_pre[t][q][i] = <x_i, d_input_q> (Eq. dense_read
+// reversed; the dense-read gradient itself, dX[t][i] += sum_q H_pre[t][q][i] d_input_q, is added
+// by the full-state dX kernel).  One CTA per token: the token's G d_input rows are staged in
+// shared memory, then each warp takes whole non-active streams (warp-level reductions only, no
+// block barrier per stream).
 
 __global__ void __launch_bounds__(256) k_full_dots(Dims d, int T, const uint16_t* __restrict__ X,
                                                    const uint16_t* __restrict__ dinput,
                                                    const int* __restrict__ I,
-                                                   const float* __restrict__ hpre,
-                                                   uint16_t* __restrict__ dX,
                                                    float* __restrict__ dhpre) {
     extern __shared__ __align__(16) uint16_t din[];   // [G][C]
     __shared__ int list[MAXN];
     __shared__ int nlist;
-    __shared__ float hs[4 * MAXN];
     const int t = blockIdx.x, C = d.C, G = d.G;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int nw = blockDim.x >> 5;
@@ -309,7 +307,6 @@ __global__ void __launch_bounds__(256) k_full_dots(Dims d, int T, const uint16_t
         }
         nlist = n;
     }
-    for (int q = threadIdx.x; q < G * d.N; q += blockDim.x) hs[q] = hpre[(int64_t)t * G * d.N + q];
     for (int idx = threadIdx.x; idx < G * C / 8; idx += blockDim.x) {
         const int q = idx / (C / 8), c8 = idx - q * (C / 8);
         reinterpret_cast<uint4*>(din)[idx] =
@@ -319,40 +316,29 @@ __global__ void __launch_bounds__(256) k_full_dots(Dims d, int T, const uint16_t
     for (int li = warp; li < nlist; li += nw) {
         const int i = list[li];
         float acc[4] = {0.f, 0.f, 0.f, 0.f};
-        float h[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) h[q] = (q < G) ? hs[q * d.N + i] : 0.f;
         const int64_t row = ((int64_t)t * d.N + i) * C;
-        // 4 chunks per lane per step: their 8 reads are issued before any is used
+        // 4 chunks per lane per step: their reads are issued before any is used
         for (int c0 = lane; c0 < C / 8; c0 += 128) {
-            uint4 xr[4], dr[4];
+            uint4 xr[4];
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 const int c8 = c0 + 32 * u;
-                if (c8 < C / 8) {
-                    xr[u] = __ldg(reinterpret_cast<const uint4*>(X + row + c8 * 8));
-                    dr[u] = *reinterpret_cast<const uint4*>(dX + row + c8 * 8);
-                }
+                if (c8 < C / 8) xr[u] = __ldg(reinterpret_cast<const uint4*>(X + row + c8 * 8));
             }
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 const int c8 = c0 + 32 * u;
                 if (c8 >= C / 8) continue;
-                float x[8], dx[8];
+                float x[8];
                 unpack8(xr[u], x);
-                unpack8(dr[u], dx);
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
                     if (q >= G) continue;
                     float g[8];
                     unpack8(reinterpret_cast<const uint4*>(din + q * C)[c8], g);
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        acc[q] = fmaf(x[e], g[e], acc[q]);
-                        dx[e] = fmaf(h[q], g[e], dx[e]);
-                    }
+                    for (int e = 0; e < 8; ++e) acc[q] = fmaf(x[e], g[e], acc[q]);
                 }
-                *reinterpret_cast<uint4*>(dX + row + c8 * 8) = pack8(dx);
             }
         }
 #pragma unroll
@@ -364,15 +350,14 @@ __global__ void __launch_bounds__(256) k_full_dots(Dims d, int T, const uint16_t
 }
 
 cudaError_t launch_full_dots(const Dims& d, int T, const uint16_t* X, const uint16_t* dinput,
-                             const int* I, const float* hpre, uint16_t* dX, float* dhpre,
-                             cudaStream_t st) {
+                             const int* I, float* dhpre, cudaStream_t st) {
     const size_t sm = (size_t)d.G * d.C * 2;
     if (sm > 48 * 1024) {
         cudaError_t e = cudaFuncSetAttribute((const void*)k_full_dots, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)sm);
         if (e != cudaSuccess) return e;
     }
-    k_full_dots<<<T, 256, sm, st>>>(d, T, X, dinput, I, hpre, dX, dhpre); note_launch();
+    k_full_dots<<<T, 256, sm, st>>>(d, T, X, dinput, I, dhpre); note_launch();
     return cudaGetLastError();
 }
 

@@ -133,6 +133,19 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
     for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// TMEM -> registers, 32 lanes x 8 columns (wait in the same statement, as above)
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, float* v) {
+    uint32_t r[8];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];\n"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7])
+        : "r"(taddr));
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
+}
+
 struct ProjTcArgs {
     int T, KB;          // tokens, k-blocks per tile
     int MT;             // M tiles
@@ -585,9 +598,9 @@ int device_sms() { return num_sms(); }
 //   dX[t][i*C + c] = base + sum_o dZ[t][o] W[i*C + c][o] + a_t + b_t x[t][i*C + c]
 //   base = dX_act[t][j][c]                                  if stream i is active slot j
 //        = dX[t][i*C + c] + sum_q H_pre[t][q][i] d_input_q[t][c]   otherwise
-// Tiles of 128 tokens x 128 channels of one stream; MMA K = nfull (dZ and W in bf16: this term
-// is a small share of dX, whose storage is bf16).  Persistent CTAs take tiles with stride P, the
-// stream index fastest, so the d_input tile of a (token, channel) block is reused from L2.
+// MMA K = nfull (dZ and W in bf16: this term is a small share of dX, whose storage is bf16); the
+// tiling is described at the kernel (k_dxf_tc).  The same machinery with "streams" = the k active
+// slots updates dX_act in the backward of each slot's pre-map (k_dx_tc<true>).
 
 namespace {
 
@@ -605,6 +618,7 @@ __device__ __forceinline__ uint4 ld_stream(const void* p) {
 
 struct DxArgs {
     int T, C, N, k, G;
+    int m;                // full-state epilogue: fixed streams 0..m-1 (active on every token)
     int slot;             // active epilogue: slot of the pre-map
     int NH;               // active epilogue: streams of the H_pre rows
     float* dxa;           // active epilogue: dX_act [T][k][C] fp32, updated in place
@@ -912,128 +926,175 @@ __device__ __forceinline__ bool named_bar_or(int id, int nthreads, bool p) {
     return r != 0;
 }
 
-constexpr int DXF_TILE = 2 * BM * 64 * 2;   // X (or dX) tile: two 64-channel boxes, 32 KB
+constexpr int DG_BN = 64;                    // channels of a full-state dX tile
+constexpr int DG_TILE = BM * DG_BN * 2;      // one 128 x 64 bf16 box, 16 KB
 
+// Full-state dX, grouped by column block: a block is 128 tokens x 64 channels; its N stream tiles
+// are processed in turn by one CTA, which stages the G d_input rows of the block in shared memory
+// once for all of them (the dense-read gradient of the non-active rows).  Streams m..N-1 come
+// first and the fixed (always active, no d_input) streams 0..m-1 last, so the d_input buffer is
+// released, and the next block's rows loaded, while the last tiles of a block are finished.
+// Per tile: MMA 128 x 64 x nfull (A = the block's dZ rows, B = the stream's W rows), TMA-staged X
+// and dX tiles, the result written over the X tile and TMA-stored into dX.
 __global__ void __launch_bounds__(DX_THREADS, 1)
 k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-         const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmD, DxArgs a) {
+         const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmD,
+         const __grid_constant__ CUtensorMap tmG, DxArgs a) {
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    const uint32_t A_BYTES = (uint32_t)a.nkb * BM * BK * 2;
-    const uint32_t B_BYTES = (uint32_t)a.nkb * DX_BN * BK * 2;
-    const uint32_t OPS = A_BYTES + B_BYTES;
-    unsigned char* epi = smem + OPS;                 // [2 groups][X tile | dX tile]
-    uint64_t* bars = reinterpret_cast<uint64_t*>(epi + 2 * 2 * DXF_TILE);
-    // [0] ops full, [1] ops empty, [2,4) tmem full, [4,6) tmem empty, [6,8) epi full, [8,10) epi empty
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 10);
+    const uint32_t A_BYTES = (uint32_t)a.nkb * BM * BK * 2;      // dZ rows of the token tile
+    const uint32_t B_BYTES = (uint32_t)a.nkb * DG_BN * BK * 2;   // W rows of one stream's block
+    unsigned char* sA = smem;
+    unsigned char* sB = sA + A_BYTES;                // [2 stages]
+    unsigned char* sG = sB + 2 * B_BYTES;            // [G][128 tokens][64 channels]
+    unsigned char* sE = sG + (size_t)a.G * DG_TILE;  // [2 groups][X tile | dX tile]
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sE + 2 * 2 * DG_TILE);
+    // [0] A full [1] A empty [2,4) B full [4,6) B empty [6] G full [7] G empty
+    // [8,10) TMEM full [10,12) TMEM empty [12,14) epi full [14,16) epi empty
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
     volatile int* s_abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
         *s_abort = 0;
         mbar_init(smem_u32(&bars[0]), 1);
         mbar_init(smem_u32(&bars[1]), 1);
+        mbar_init(smem_u32(&bars[6]), 1);
+        mbar_init(smem_u32(&bars[7]), 2);
         for (int g = 0; g < 2; ++g) {
             mbar_init(smem_u32(&bars[2 + g]), 1);
-            mbar_init(smem_u32(&bars[4 + g]), DX_EW / 2);
-            mbar_init(smem_u32(&bars[6 + g]), 1);
+            mbar_init(smem_u32(&bars[4 + g]), 1);
             mbar_init(smem_u32(&bars[8 + g]), 1);
+            mbar_init(smem_u32(&bars[10 + g]), DX_EW / 2);
+            mbar_init(smem_u32(&bars[12 + g]), 1);
+            mbar_init(smem_u32(&bars[14 + g]), 1);
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                         smem_u32(tmem_slot)), "r"(256u) : "memory");
+                         smem_u32(tmem_slot)), "r"(128u) : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    const long long nloc = (a.ntiles > blockIdx.x) ? (a.ntiles - 1 - blockIdx.x) / a.P + 1 : 0;
+    const int N = a.N;
+    const int ndin = N - a.m;   // leading tiles of a block that may read d_input (streams m..N-1)
+    const long long nblk = (a.ntiles > blockIdx.x) ? (a.ntiles - 1 - blockIdx.x) / a.P + 1 : 0;
+    const long long nloc = nblk * N;
+    // local tile n: block n / N of this CTA, position p in the block, stream (p + m) mod N
+    auto decode = [&](long long n, int& p, int& tt, int& cb, int& i) {
+        const long long b = n / N;
+        p = (int)(n - b * N);
+        const long long block = blockIdx.x + b * a.P;
+        tt = (int)(block / a.CT);
+        cb = (int)(block - (long long)tt * a.CT);
+        i = p + a.m;
+        if (i >= N) i -= N;
+    };
 
     if (warp == 0) {
         if (lane == 0) {
             for (long long n = 0; n < nloc; ++n) {
                 if (*s_abort) break;
-                const long long tile = blockIdx.x + n * a.P;
-                const int i = (int)(tile % a.N);
-                const long long rest = tile / a.N;
-                const int ct = (int)(rest % a.CT), tt = (int)(rest / a.CT);
-                if (n >= 1 && !mbar_wait(smem_u32(&bars[1]), (uint32_t)((n - 1) & 1))) {
-                    atomicExch(a.err, 21);
+                int p, tt, cb, i;
+                decode(n, p, tt, cb, i);
+                const long long blk = n / N;
+                if (p == 0) {
+                    if (blk >= 1 && !mbar_wait(smem_u32(&bars[1]), (uint32_t)((blk - 1) & 1))) {
+                        atomicExch(a.err, 31);
+                        *s_abort = 1;
+                        break;
+                    }
+                    const uint32_t fa = smem_u32(&bars[0]);
+                    mbar_expect_tx(fa, A_BYTES);
+                    for (int kb = 0; kb < a.nkb; ++kb)
+                        tma_load_2d(smem_u32(sA + kb * BM * BK * 2), &tmA, kb * BK, tt * BM, fa);
+                }
+                const int s = (int)(n & 1);
+                if (n >= 2 && !mbar_wait(smem_u32(&bars[4 + s]), (uint32_t)(((n >> 1) - 1) & 1))) {
+                    atomicExch(a.err, 32);
                     *s_abort = 1;
                     break;
                 }
-                const uint32_t full = smem_u32(&bars[0]);
-                mbar_expect_tx(full, OPS);
-                for (int kb = 0; kb < a.nkb; ++kb) {
-                    tma_load_2d(smem_u32(smem + kb * BM * BK * 2), &tmA, kb * BK, tt * BM, full);
-                    tma_load_2d(smem_u32(smem + A_BYTES + kb * DX_BN * BK * 2), &tmB, kb * BK,
-                                i * a.C + ct * DX_BN, full);
-                }
-                const int g = (int)(n & 1);
-                if (n >= 2 && !mbar_wait(smem_u32(&bars[8 + g]), (uint32_t)(((n >> 1) - 1) & 1))) {
-                    atomicExch(a.err, 22);
+                const uint32_t fb = smem_u32(&bars[2 + s]);
+                mbar_expect_tx(fb, B_BYTES);
+                for (int kb = 0; kb < a.nkb; ++kb)
+                    tma_load_2d(smem_u32(sB + s * B_BYTES + kb * DG_BN * BK * 2), &tmB, kb * BK,
+                                i * a.C + cb * DG_BN, fb);
+                if (n >= 2 && !mbar_wait(smem_u32(&bars[14 + s]), (uint32_t)(((n >> 1) - 1) & 1))) {
+                    atomicExch(a.err, 33);
                     *s_abort = 1;
                     break;
                 }
-                const uint32_t ef = smem_u32(&bars[6 + g]);
-                mbar_expect_tx(ef, 2 * DXF_TILE);
-                unsigned char* xt = epi + (size_t)g * 2 * DXF_TILE;
-                for (int h = 0; h < 2; ++h) {
-                    const int x = i * a.C + ct * DX_BN + h * 64;
-                    tma_load_2d(smem_u32(xt + h * (DXF_TILE / 2)), &tmX, x, tt * BM, ef);
-                    tma_load_2d(smem_u32(xt + DXF_TILE + h * (DXF_TILE / 2)), &tmD, x, tt * BM, ef);
+                const uint32_t fe = smem_u32(&bars[12 + s]);
+                mbar_expect_tx(fe, 2 * DG_TILE);
+                unsigned char* xt = sE + (size_t)s * 2 * DG_TILE;
+                tma_load_2d(smem_u32(xt), &tmX, i * a.C + cb * DG_BN, tt * BM, fe);
+                tma_load_2d(smem_u32(xt + DG_TILE), &tmD, i * a.C + cb * DG_BN, tt * BM, fe);
+                if (p == 0) {
+                    if (blk >= 1 && !mbar_wait(smem_u32(&bars[7]), (uint32_t)((blk - 1) & 1))) {
+                        atomicExch(a.err, 34);
+                        *s_abort = 1;
+                        break;
+                    }
+                    const uint32_t fg = smem_u32(&bars[6]);
+                    mbar_expect_tx(fg, (uint32_t)a.G * DG_TILE);
+                    for (int q = 0; q < a.G; ++q)
+                        tma_load_2d(smem_u32(sG + q * DG_TILE), &tmG, cb * DG_BN, q * a.T + tt * BM, fg);
                 }
             }
         }
     } else if (warp == 1) {
         if (lane == 0) {
-            const uint32_t idesc = idesc_bf16(BM, DX_BN);
+            const uint32_t idesc = idesc_bf16(BM, DG_BN);
             for (long long n = 0; n < nloc; ++n) {
+                const long long blk = n / N;
+                const int p = (int)(n - blk * N);
                 const int s = (int)(n & 1);
-                if (!mbar_wait(smem_u32(&bars[0]), (uint32_t)(n & 1))) {
-                    atomicExch(a.err, 23);
-                    *s_abort = 1;
-                    break;
-                }
-                if (n >= 2 && !mbar_wait(smem_u32(&bars[4 + s]), (uint32_t)(((n >> 1) - 1) & 1))) {
-                    atomicExch(a.err, 24);
+                bool ok = (p != 0) || mbar_wait(smem_u32(&bars[0]), (uint32_t)(blk & 1));
+                ok = ok && mbar_wait(smem_u32(&bars[2 + s]), (uint32_t)((n >> 1) & 1));
+                ok = ok && (n < 2 || mbar_wait(smem_u32(&bars[10 + s]), (uint32_t)(((n >> 1) - 1) & 1)));
+                if (!ok) {
+                    atomicExch(a.err, 35);
                     *s_abort = 1;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t abase = smem_u32(smem);
-                const uint32_t bbase = abase + A_BYTES;
+                const uint32_t abase = smem_u32(sA);
+                const uint32_t bbase = smem_u32(sB + s * B_BYTES);
                 for (int ks = 0; ks < a.ksteps; ++ks) {
                     const int kb = ks >> 2, kk = ks & 3;
-                    mma_bf16(tmem + (uint32_t)(s * DX_BN), sw128_desc(abase + kb * BM * BK * 2 + kk * 32),
-                             sw128_desc(bbase + kb * DX_BN * BK * 2 + kk * 32), idesc, ks > 0 ? 1u : 0u);
+                    mma_bf16(tmem + (uint32_t)(s * DG_BN), sw128_desc(abase + kb * BM * BK * 2 + kk * 32),
+                             sw128_desc(bbase + kb * DG_BN * BK * 2 + kk * 32), idesc, ks > 0 ? 1u : 0u);
                 }
-                mma_commit(smem_u32(&bars[1]));       // operands consumed
-                mma_commit(smem_u32(&bars[2 + s]));   // accumulator ready
+                mma_commit(smem_u32(&bars[4 + s]));              // B stage consumed
+                mma_commit(smem_u32(&bars[8 + s]));              // accumulator ready
+                if (p == N - 1) mma_commit(smem_u32(&bars[1]));  // the block's A rows consumed
             }
         }
     } else {
         // group g = tiles n = g mod 2 (TMEM buffer g, epilogue stage g); in the group, warp w owns
-        // the TMEM lane quarter warp % 4 (rows) and the 64-channel box (w % 8) / 4
+        // the TMEM lane quarter warp % 4 (rows) and the 32-channel half (w % 8) / 4
         const int ew = warp - 2;
         const int grp = ew >> 3;
         const int quarter = warp & 3;
-        const int box = (ew & 7) >> 2;
+        const int half = (ew & 7) >> 2;
         const int r = quarter * 32 + lane;          // tile row
         const bool leader = (ew & 7) == 0 && lane == 0;
-        unsigned char* xt = epi + (size_t)grp * 2 * DXF_TILE;
-        unsigned char* xrow = xt + box * (DXF_TILE / 2) + r * 128;                // this row, X box
-        const unsigned char* drow = xt + DXF_TILE + box * (DXF_TILE / 2) + r * 128; // dX box
-        const int sw = r & 7;                                                     // 128B swizzle
+        unsigned char* xt = sE + (size_t)grp * 2 * DG_TILE;
+        unsigned char* xrow = xt + r * 128;                       // this row of the X tile
+        const unsigned char* drow = xt + DG_TILE + r * 128;       // of the dX tile
+        const unsigned char* grow = sG + r * 128;                 // of the d_input rows
+        const int sw = r & 7;                                     // 128B swizzle
         bool stored = false;
         for (long long n = grp; n < nloc; n += 2) {
-            const long long tile = blockIdx.x + n * a.P;
-            const int i = (int)(tile % a.N);
-            const long long rest = tile / a.N;
-            const int ct = (int)(rest % a.CT), tt = (int)(rest / a.CT);
+            int p, tt, cb, i;
+            decode(n, p, tt, cb, i);
+            const long long blk = n / N;
+            const bool usesg = p < ndin;
             const int t = tt * BM + r;
             int j = -1;
             float sa = 0.f, sb = 0.f;
@@ -1043,69 +1104,83 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
                 sa = a.scal[(long long)t * a.scal_ld + 0];
                 sb = a.scal[(long long)t * a.scal_ld + 1];
             }
-            // fp32 base of an active row: 16 channels (two chunks) per step, each step's reads
-            // issued one step ahead, the first before the waits
             const bool arow = (j >= 0) && (t < a.T);
-            const float* brow = a.dxact + ((long long)t * a.k + (j < 0 ? 0 : j)) * a.C + ct * DX_BN + box * 64;
-            uint4 pfa[4], pfb[4];
-            auto prefetch = [&](int step, uint4 (&dst)[4]) {
-                if (arow) {
+            float hq[4];
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) dst[e] = ld_stream(brow + step * 16 + e * 4);
+            for (int q = 0; q < 4; ++q)
+                hq[q] = (usesg && !arow && t < a.T && q < a.G) ? a.hpre[((long long)t * a.G + q) * N + i] : 0.f;
+            // an active row's fp32 base, 8 channels per chunk, read one chunk ahead (the first
+            // before the waits)
+            const float* brow = a.dxact + ((long long)t * a.k + (j < 0 ? 0 : j)) * a.C + cb * DG_BN + half * 32;
+            uint4 pfa[2], pfb[2];
+            auto prefetch = [&](int c4, uint4 (&dst)[2]) {
+                if (arow) {
+                    dst[0] = ld_stream(brow + c4 * 8);
+                    dst[1] = ld_stream(brow + c4 * 8 + 4);
                 }
             };
             prefetch(0, pfa);
-            bool ok = mbar_wait(smem_u32(&bars[6 + grp]), (uint32_t)((n >> 1) & 1));
-            ok = ok && mbar_wait(smem_u32(&bars[2 + grp]), (uint32_t)((n >> 1) & 1));
+            bool ok = mbar_wait(smem_u32(&bars[12 + grp]), (uint32_t)((n >> 1) & 1));
+            ok = ok && mbar_wait(smem_u32(&bars[8 + grp]), (uint32_t)((n >> 1) & 1));
+            ok = ok && (!usesg || mbar_wait(smem_u32(&bars[6]), (uint32_t)(blk & 1)));
             if (!ok) {
-                atomicExch(a.err, 25);
+                atomicExch(a.err, 36);
                 *s_abort = 1;
             } else {
                 tc_fence_after();
-                const uint32_t tl = tmem + (uint32_t)(grp * DX_BN + box * 64) + ((uint32_t)(quarter * 32) << 16);
-                auto step_body = [&](int step, const uint4 (&pf)[4]) {
-                    float acc[16];
-                    tmem_ld16(tl + (uint32_t)(step * 16), acc);
+                const uint32_t tl = tmem + (uint32_t)(grp * DG_BN + half * 32) + ((uint32_t)(quarter * 32) << 16);
+                auto chunk = [&](int c4, const uint4 (&pf)[2]) {
+                    float acc[8];
+                    tmem_ld8(tl + (uint32_t)(c4 * 8), acc);
+                    const int ph = ((half * 4 + c4) ^ sw) * 16;
+                    float x[8], v[8];
+                    unpack8(*reinterpret_cast<const uint4*>(xrow + ph), x);
+                    if (arow) {
+                        v[0] = __uint_as_float(pf[0].x); v[1] = __uint_as_float(pf[0].y);
+                        v[2] = __uint_as_float(pf[0].z); v[3] = __uint_as_float(pf[0].w);
+                        v[4] = __uint_as_float(pf[1].x); v[5] = __uint_as_float(pf[1].y);
+                        v[6] = __uint_as_float(pf[1].z); v[7] = __uint_as_float(pf[1].w);
+                    } else {
+                        unpack8(*reinterpret_cast<const uint4*>(drow + ph), v);
+                        if (usesg) {
 #pragma unroll
-                    for (int cc = 0; cc < 2; ++cc) {
-                        const int q = step * 2 + cc;               // logical 16-byte chunk
-                        const int ph = (q ^ sw) * 16;
-                        float x[8], v[8];
-                        unpack8(*reinterpret_cast<const uint4*>(xrow + ph), x);
-                        if (arow) {
-                            const uint4 b0 = pf[cc * 2], b1 = pf[cc * 2 + 1];
-                            v[0] = __uint_as_float(b0.x); v[1] = __uint_as_float(b0.y);
-                            v[2] = __uint_as_float(b0.z); v[3] = __uint_as_float(b0.w);
-                            v[4] = __uint_as_float(b1.x); v[5] = __uint_as_float(b1.y);
-                            v[6] = __uint_as_float(b1.z); v[7] = __uint_as_float(b1.w);
-                        } else {
-                            unpack8(*reinterpret_cast<const uint4*>(drow + ph), v);
+                            for (int q = 0; q < 4; ++q) {
+                                if (q < a.G) {
+                                    float g[8];
+                                    unpack8(*reinterpret_cast<const uint4*>(grow + q * DG_TILE + ph), g);
+#pragma unroll
+                                    for (int e = 0; e < 8; ++e) v[e] = fmaf(hq[q], g[e], v[e]);
+                                }
+                            }
                         }
-                        float o[8];
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) o[e] = v[e] + acc[cc * 8 + e] + sa + sb * x[e];
-                        *reinterpret_cast<uint4*>(xrow + ph) = pack8(o);
                     }
+                    float o[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) o[e] = v[e] + acc[e] + sa + sb * x[e];
+                    *reinterpret_cast<uint4*>(xrow + ph) = pack8(o);
                 };
                 prefetch(1, pfb);
-                step_body(0, pfa);
+                chunk(0, pfa);
                 prefetch(2, pfa);
-                step_body(1, pfb);
+                chunk(1, pfb);
                 prefetch(3, pfb);
-                step_body(2, pfa);
-                step_body(3, pfb);
+                chunk(2, pfa);
+                chunk(3, pfb);
                 tc_fence_before();
             }
             __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&bars[4 + grp]));  // TMEM buffer free
-            fence_async_smem();                                     // results visible to TMA
+            if (lane == 0) mbar_arrive(smem_u32(&bars[10 + grp]));  // TMEM buffer free
+            fence_async_smem();                                      // results visible to TMA
             if (named_bar_or(1 + grp, (DX_EW / 2) * 32, *s_abort != 0)) break;  // same decision in the group
             if (leader) {
-                for (int h = 0; h < 2; ++h)
-                    tma_store_2d(&tmD, smem_u32(xt + h * (DXF_TILE / 2)), i * a.C + ct * DX_BN + h * 64, tt * BM);
+                // the group's last reader of this block's d_input rows (or, when it has none of the
+                // block's d_input tiles, its first tile of the block) releases them: one arrival
+                // per group and block
+                if ((usesg && p + 2 >= ndin) || (!usesg && p < 2)) mbar_arrive(smem_u32(&bars[7]));
+                tma_store_2d(&tmD, smem_u32(xt), i * a.C + cb * DG_BN, tt * BM);
                 bulk_commit();
-                bulk_wait_read0();                                  // the stage may be reloaded
-                mbar_arrive(smem_u32(&bars[8 + grp]));
+                bulk_wait_read0();                                   // the stage may be reloaded
+                mbar_arrive(smem_u32(&bars[14 + grp]));
                 stored = true;
             }
         }
@@ -1115,7 +1190,7 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
     __syncthreads();
     if (warp == 1) {
         tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(256u)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(128u)
                      : "memory");
     }
 }
@@ -1201,9 +1276,8 @@ cudaError_t launch_dxa_tc(const Dims& d, int slot, int T, const float* dzs, int 
     return cudaGetLastError();
 }
 
-bool dx_tc_ok(int T, int N, int C, int nfull) {
-    (void)N;
-    return T >= BM && C % DX_BN == 0 && nfull <= 2 * BK;
+bool dx_tc_ok(int T, int N, int C, int nfull, int G) {
+    return T >= BM && C % DG_BN == 0 && nfull <= 2 * BK && N >= 2 && G >= 1 && G <= 4;
 }
 
 cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, uint16_t* dz16,
@@ -1221,27 +1295,29 @@ cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, 
     k_pack_rows<<<(unsigned)((tot + 255) / 256), 256, 0, st>>>(W, n, NC, ld, w16); note_launch();
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    CUtensorMap ma, mb;
+    CUtensorMap ma, mb, mx, md, mg;
     if (!make_map_box(&ma, dz16, (uint64_t)n, (uint64_t)T, BK, BM, (uint64_t)ld * 2)) return cudaErrorInvalidValue;
-    if (!make_map_box(&mb, w16, (uint64_t)n, (uint64_t)NC, BK, DX_BN, (uint64_t)ld * 2)) return cudaErrorInvalidValue;
+    if (!make_map_box(&mb, w16, (uint64_t)n, (uint64_t)NC, BK, DG_BN, (uint64_t)ld * 2)) return cudaErrorInvalidValue;
+    if (!make_map_box(&mx, X, (uint64_t)NC, (uint64_t)T, DG_BN, BM)) return cudaErrorInvalidValue;
+    if (!make_map_box(&md, dX, (uint64_t)NC, (uint64_t)T, DG_BN, BM)) return cudaErrorInvalidValue;
+    // the G d_input copies [G][T][C] as one [G T][C] matrix (rows of a token tile past T read the
+    // next copy's rows or zeros; those rows are never stored)
+    if (!make_map_box(&mg, dinput, (uint64_t)d.C, (uint64_t)d.G * T, DG_BN, BM)) return cudaErrorInvalidValue;
     DxArgs a;
     memset(&a, 0, sizeof(a));
-    a.T = T; a.C = d.C; a.N = d.N; a.k = d.k; a.G = d.G;
+    a.T = T; a.C = d.C; a.N = d.N; a.k = d.k; a.G = d.G; a.m = d.m;
     a.nkb = (n + BK - 1) / BK;
     a.ksteps = (n + 15) / 16;
     a.TT = (T + BM - 1) / BM;
-    a.CT = d.C / DX_BN;
-    a.ntiles = (long long)a.TT * a.CT * d.N;
+    a.CT = d.C / DG_BN;
+    a.ntiles = (long long)a.TT * a.CT;   // column blocks, N tiles each
     a.P = (int)std::min<long long>(num_sms(), a.ntiles);
     a.X = X; a.dX = dX; a.dinput = dinput; a.hpre = hpre; a.I = I; a.dxact = dxact;
     a.scal = scal; a.scal_ld = scal_ld; a.err = err;
-    CUtensorMap mx, md;
-    if (!make_map_box(&mx, X, (uint64_t)NC, (uint64_t)T, 64, BM)) return cudaErrorInvalidValue;
-    if (!make_map_box(&md, dX, (uint64_t)NC, (uint64_t)T, 64, BM)) return cudaErrorInvalidValue;
-    const size_t sm = (size_t)a.nkb * (BM + DX_BN) * BK * 2 + 4 * (size_t)DXF_TILE + 128 + 1024;
+    const size_t sm = (size_t)a.nkb * (BM + 2 * DG_BN) * BK * 2 + (size_t)(d.G + 4) * DG_TILE + 256 + 1024;
     e = cudaFuncSetAttribute((const void*)k_dxf_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
-    k_dxf_tc<<<a.P, DX_THREADS, sm, st>>>(ma, mb, mx, md, a); note_launch();
+    k_dxf_tc<<<a.P, DX_THREADS, sm, st>>>(ma, mb, mx, md, mg, a); note_launch();
     return cudaGetLastError();
 }
 

@@ -249,7 +249,7 @@ cudaError_t launch_proj_tc(const uint16_t* X, int T, int K, const uint16_t* Wpac
 cudaError_t launch_wgrad_tc(const uint16_t* A, int T, int E, const float* dz, int ldz, int n,
                             uint16_t* dzpack, const ProjTcPlan& p, float* part, int* err,
                             cudaStream_t st);
-bool dx_tc_ok(int T, int N, int C, int nfull);
+bool dx_tc_ok(int T, int N, int C, int nfull, int G);
 bool dxa_tc_ok(int T, int k, int C, int nact);
 // dX_act += dZ_act W_act^T (three-term bf16 split on the tensor cores) + H_pre[slot][I_j] d_input
 //           - cx x_act (the write-back's own term, cx per token in tokmat)
@@ -314,8 +314,7 @@ cudaError_t launch_dinput_act(const Dims& d, int slot, int T, int add_dx, const 
                               float* dxact, float* dhpre, uint16_t* dinput_copy,
                               const float* tokmat, cudaStream_t st);
 cudaError_t launch_full_dots(const Dims& d, int T, const uint16_t* X, const uint16_t* dinput,
-                             const int* I, const float* hpre, uint16_t* dX, float* dhpre,
-                             cudaStream_t st);
+                             const int* I, float* dhpre, cudaStream_t st);
 cudaError_t launch_full_coef(const Dims& d, int T, const float* dhpre, const float* hpre,
                              const float* zfull, const float* stats, const float* wsum,
                              const int* I, const float* dp, const float* alpha_pre, float* dz,
