@@ -283,29 +283,36 @@ cudaError_t launch_dinput_act(const Dims& d, int slot, int T, int add_dx, const 
 // ---------------------------------------------------------------------------------------------
 // full_dots: for the non-active streams i, dH_pre[t][q][i] = <x_i, d_input_q> (Eq. dense_read
 // reversed; the dense-read gradient itself, dX[t][i] += sum_q H_pre[t][q][i] d_input_q, is added
-// by the full-state dX kernel).  One CTA per token: the token's G d_input rows are staged in
-// shared memory, then each warp takes whole non-active streams (warp-level reductions only, no
-// block barrier per stream).
+// by the full-state dX kernel).  One CTA per token with one warp per non-active stream (there are
+// N - k of them on every token: the k active streams are distinct); the token's G d_input rows
+// are staged in shared memory while each warp's first X reads are in flight.
 
-__global__ void __launch_bounds__(256) k_full_dots(Dims d, int T, const uint16_t* __restrict__ X,
-                                                   const uint16_t* __restrict__ dinput,
-                                                   const int* __restrict__ I,
-                                                   float* __restrict__ dhpre) {
+__global__ void __launch_bounds__(1024) k_full_dots(Dims d, int T, const uint16_t* __restrict__ X,
+                                                    const uint16_t* __restrict__ dinput,
+                                                    const int* __restrict__ I,
+                                                    float* __restrict__ dhpre) {
     extern __shared__ __align__(16) uint16_t din[];   // [G][C]
-    __shared__ int list[MAXN];
-    __shared__ int nlist;
     const int t = blockIdx.x, C = d.C, G = d.G;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int nw = blockDim.x >> 5;
-    if (threadIdx.x == 0) {
-        int n = 0;
-        for (int i = 0; i < d.N; ++i) {
-            bool a = false;
-            for (int q = 0; q < d.k; ++q)
-                if (I[(int64_t)t * d.k + q] == i) a = true;
-            if (!a) list[n++] = i;
+    // this warp's stream: the warp-th stream that is not active on token t
+    uint32_t act = 0u;
+    for (int q = 0; q < d.k; ++q) act |= 1u << I[(int64_t)t * d.k + q];
+    int i = -1;
+    for (int s = 0, cnt = 0; s < d.N; ++s)
+        if (!(act & (1u << s))) {
+            if (cnt == warp) {
+                i = s;
+                break;
+            }
+            ++cnt;
         }
-        nlist = n;
+    const int64_t row = ((int64_t)t * d.N + (i < 0 ? 0 : i)) * C;
+    // the first 4 chunks per lane, read before the staging barrier
+    uint4 xr[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const int c8 = lane + 32 * u;
+        if (i >= 0 && c8 < C / 8) xr[u] = __ldg(reinterpret_cast<const uint4*>(X + row + c8 * 8));
     }
     for (int idx = threadIdx.x; idx < G * C / 8; idx += blockDim.x) {
         const int q = idx / (C / 8), c8 = idx - q * (C / 8);
@@ -313,51 +320,50 @@ __global__ void __launch_bounds__(256) k_full_dots(Dims d, int T, const uint16_t
             *reinterpret_cast<const uint4*>(dinput + ((int64_t)q * T + t) * C + c8 * 8);
     }
     __syncthreads();
-    for (int li = warp; li < nlist; li += nw) {
-        const int i = list[li];
-        float acc[4] = {0.f, 0.f, 0.f, 0.f};
-        const int64_t row = ((int64_t)t * d.N + i) * C;
-        // 4 chunks per lane per step: their reads are issued before any is used
-        for (int c0 = lane; c0 < C / 8; c0 += 128) {
-            uint4 xr[4];
+    if (i < 0) return;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int c0 = lane; c0 < C / 8; c0 += 128) {
+        if (c0 != lane) {
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 const int c8 = c0 + 32 * u;
                 if (c8 < C / 8) xr[u] = __ldg(reinterpret_cast<const uint4*>(X + row + c8 * 8));
             }
+        }
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int c8 = c0 + 32 * u;
-                if (c8 >= C / 8) continue;
-                float x[8];
-                unpack8(xr[u], x);
+        for (int u = 0; u < 4; ++u) {
+            const int c8 = c0 + 32 * u;
+            if (c8 >= C / 8) continue;
+            float x[8];
+            unpack8(xr[u], x);
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    if (q >= G) continue;
-                    float g[8];
-                    unpack8(reinterpret_cast<const uint4*>(din + q * C)[c8], g);
+            for (int q = 0; q < 4; ++q) {
+                if (q >= G) continue;
+                float g[8];
+                unpack8(reinterpret_cast<const uint4*>(din + q * C)[c8], g);
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) acc[q] = fmaf(x[e], g[e], acc[q]);
-                }
+                for (int e = 0; e < 8; ++e) acc[q] = fmaf(x[e], g[e], acc[q]);
             }
         }
+    }
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const float v = warp_sum(acc[q]);
-            if (lane == 0 && q < G) dhpre[((int64_t)t * G + q) * d.N + i] = v;
-        }
+    for (int q = 0; q < 4; ++q) {
+        const float v = warp_sum(acc[q]);
+        if (lane == 0 && q < G) dhpre[((int64_t)t * G + q) * d.N + i] = v;
     }
 }
 
 cudaError_t launch_full_dots(const Dims& d, int T, const uint16_t* X, const uint16_t* dinput,
                              const int* I, float* dhpre, cudaStream_t st) {
+    const int nw = d.N - d.k;   // non-active streams per token
+    if (nw <= 0) return cudaSuccess;
     const size_t sm = (size_t)d.G * d.C * 2;
     if (sm > 48 * 1024) {
         cudaError_t e = cudaFuncSetAttribute((const void*)k_full_dots, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)sm);
         if (e != cudaSuccess) return e;
     }
-    k_full_dots<<<T, 256, sm, st>>>(d, T, X, dinput, I, dhpre); note_launch();
+    k_full_dots<<<T, 32 * nw, sm, st>>>(d, T, X, dinput, I, dhpre); note_launch();
     return cudaGetLastError();
 }
 

@@ -1029,11 +1029,12 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
                     *s_abort = 1;
                     break;
                 }
+                const bool need_dx = p < ndin;   // a fixed stream's tile: every row takes the fp32 base
                 const uint32_t fe = smem_u32(&bars[12 + s]);
-                mbar_expect_tx(fe, 2 * DG_TILE);
+                mbar_expect_tx(fe, need_dx ? 2 * DG_TILE : DG_TILE);
                 unsigned char* xt = sE + (size_t)s * 2 * DG_TILE;
                 tma_load_2d(smem_u32(xt), &tmX, i * a.C + cb * DG_BN, tt * BM, fe);
-                tma_load_2d(smem_u32(xt + DG_TILE), &tmD, i * a.C + cb * DG_BN, tt * BM, fe);
+                if (need_dx) tma_load_2d(smem_u32(xt + DG_TILE), &tmD, i * a.C + cb * DG_BN, tt * BM, fe);
                 if (p == 0) {
                     if (blk >= 1 && !mbar_wait(smem_u32(&bars[7]), (uint32_t)((blk - 1) & 1))) {
                         atomicExch(a.err, 34);
