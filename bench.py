@@ -87,10 +87,10 @@ def kernel_model(cfg, T):
     # tensor-core projection: X read once; the packed weight streams from L2
     add("proj_tc", X + T * nfull * f32, 2.0 * T * N * C * nb, "hbm")
     add("coef_full", T * nfull * f32 + T * (G * N + 2 * k) * f32)
-    add("read", X + row + (G - 1) * T * C * f32 + xa)
+    add("read", X + row + (G - 1) * row + xa)
     for t in range(G):
         if t > 0:
-            add("input", T * C * f32 + xa + row)
+            add("input", row + xa + row)
         add("pack_w", k * C * nact[t] * f32 + 2 * nact[t] * k * C * b16)
         add("proj_tc_active", xa + T * nact[t] * f32, 2.0 * T * k * C * 2 * nact[t], "hbm")
         add("coef_act", T * nact[t] * f32 * 2)
@@ -120,11 +120,12 @@ def kernel_model(cfg, T):
         add("dxa_tc", 2 * xa32 + xa + row + 3 * T * nact[t] * b16, 2.0 * T * k * C * 3 * nact[t], "hbm")
     if hr:
         add("colsum", N * C * N * f32)
-    # dH_pre of the inactive streams and their dense-read gradient (dX rows read and written)
-    add("full_dots", 3 * T * (N - k) * C * b16 + G * row)
+    # dH_pre of the inactive streams: their X rows and the G d_input rows read
+    add("full_dots", T * (N - k) * C * b16 + G * row)
     add("full_coef", T * (nfull + G * N) * f32)
-    # tensor-core dX: X read, inactive dX rows read, active-row gradient read, dX written
-    add("dx_tc", X + T * (N - k) * C * b16 + xa32 + X, 2.0 * T * N * C * nfull, "hbm")
+    # tensor-core dX: X read, inactive dX rows read, active-row gradient read, the G d_input rows
+    # read once per column block (dense-read gradient of the inactive rows), dX written
+    add("dx_tc", X + T * (N - k) * C * b16 + xa32 + G * row + X, 2.0 * T * N * C * nfull, "hbm")
     add("wgrad_tc_full", X + T * nfull * f32 + 2 * T * nfull * b16 + N * C * nfull * f32,
         2.0 * T * N * C * 2 * nfull, "hbm")
     add("wgrad_reduce", 2 * N * C * nfull * f32)

@@ -183,7 +183,7 @@ Layout make_layout(const Dims& d, int64_t T) {
     L.astat = o; o = al(o + (size_t)stream_warps(d.C) * t * 2 * 4);
     L.wsum = o; o = al(o + (size_t)d.N * 4);
     L.rsum = o; o = al(o + (size_t)d.N * 4);
-    L.base = o; o = al(o + (size_t)(d.G - 1) * t * d.C * 4);
+    L.base = o; o = al(o + (size_t)(d.G - 1) * t * d.C * 2);
     L.red = o; o = al(o + t * L.nslice * NRED * 4);
     L.dxact = o; o = al(o + t * d.k * d.C * 4);
     L.dinput = o; o = al(o + (size_t)d.G * t * d.C * 2);
@@ -584,9 +584,9 @@ xhc_status xhc_pre_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
                                   c.S<float>(c.L.zfull), c.S<float>(c.L.stats),
                                   c.S<float>(c.L.hpre), c.S<int>(c.L.I), c.S<float>(c.L.p), c.st));
         XHC_K("read", c.st, launch_read(d, c.T, X, c.S<float>(c.L.hpre), c.S<int>(c.L.I), input,
-                             c.W<float>(c.L.base), c.xact(0), c.W<float>(c.L.astat), c.st));
+                             c.W<uint16_t>(c.L.base), c.xact(0), c.W<float>(c.L.astat), c.st));
     } else {
-        XHC_K("input", c.st, launch_input(d, slot, c.T, c.W<float>(c.L.base), c.xact(slot),
+        XHC_K("input", c.st, launch_input(d, slot, c.T, c.W<uint16_t>(c.L.base), c.xact(slot),
                               c.S<float>(c.L.hpre), c.S<int>(c.L.I), input, c.W<float>(c.L.astat), c.st));
     }
     return active_maps(c, slot, P);

@@ -1,7 +1,8 @@
 // Streaming kernels of the connection op (HBM-bound, fp32 math on bf16 data):
 //   read        second full-state pass: dense read of slot 0 (Eq. dense_read), non-active base
-//               readouts of the later slots (Eq. app_four_sub_base), gather of the active
-//               streams (Alg. 1 Gather), sum of squares of the gathered rows
+//               readouts of the later slots (Eq. app_four_sub_base; stored in bf16, as the
+//               paper's traffic model stores them), gather of the active streams (Alg. 1
+//               Gather), sum of squares of the gathered rows
 //   input       input_t = base_t + sum_j H_pre_t[I_j] x_act_j (Eq. app_active_state_correction),
 //               sum of squares of x_act
 //   (the sums of squares are the norm statistics of the slot's active-state projection, which
@@ -37,13 +38,21 @@ __global__ void __launch_bounds__(256) k_read(Dims d, int T, const uint16_t* __r
                                               const float* __restrict__ hpre,
                                               const int* __restrict__ I,
                                               uint16_t* __restrict__ input0,
-                                              float* __restrict__ base,
+                                              uint16_t* __restrict__ base,
                                               uint16_t* __restrict__ xact0,
                                               float* __restrict__ astat) {
     __shared__ float sh[4 * MAXN];
     __shared__ int slotmap[MAXN];
     const int t = blockIdx.x;
     const int N = d.N, G = d.G, C = d.C;
+    const uint16_t* xt = X + (int64_t)t * N * C;
+    // the first 8 streams of this thread's first chunk are read before the coefficient set-up
+    uint4 ub[8];
+    if (threadIdx.x < C / 8) {
+#pragma unroll
+        for (int ii = 0; ii < 8; ++ii)
+            if (ii < N) ub[ii] = __ldg(reinterpret_cast<const uint4*>(xt + (int64_t)ii * C + threadIdx.x * 8));
+    }
     for (int q = threadIdx.x; q < G * N; q += blockDim.x) sh[q] = hpre[(int64_t)t * G * N + q];
     for (int i = threadIdx.x; i < N; i += blockDim.x) {
         int j = -1;
@@ -52,7 +61,6 @@ __global__ void __launch_bounds__(256) k_read(Dims d, int T, const uint16_t* __r
         slotmap[i] = j;
     }
     __syncthreads();
-    const uint16_t* xt = X + (int64_t)t * N * C;
     float ss = 0.f;  // sum of squares of the gathered active rows (their projection's norm)
     for (int c8 = threadIdx.x; c8 < C / 8; c8 += blockDim.x) {
         float acc[4][8];
@@ -62,10 +70,11 @@ __global__ void __launch_bounds__(256) k_read(Dims d, int T, const uint16_t* __r
             for (int e = 0; e < 8; ++e) acc[q][e] = 0.f;
         // streams in blocks of 8: the block's 8 reads are issued before any is used
         for (int i0 = 0; i0 < N; i0 += 8) {
-            uint4 ub[8];
+            if (i0 != 0 || c8 != (int)threadIdx.x) {
 #pragma unroll
-            for (int ii = 0; ii < 8; ++ii)
-                if (i0 + ii < N) ub[ii] = __ldg(reinterpret_cast<const uint4*>(xt + (int64_t)(i0 + ii) * C + c8 * 8));
+                for (int ii = 0; ii < 8; ++ii)
+                    if (i0 + ii < N) ub[ii] = __ldg(reinterpret_cast<const uint4*>(xt + (int64_t)(i0 + ii) * C + c8 * 8));
+            }
 #pragma unroll
             for (int ii = 0; ii < 8; ++ii) {
                 const int i = i0 + ii;
@@ -94,19 +103,15 @@ __global__ void __launch_bounds__(256) k_read(Dims d, int T, const uint16_t* __r
         }
         *reinterpret_cast<uint4*>(input0 + (int64_t)t * C + c8 * 8) = pack8(acc[0]);
 #pragma unroll
-        for (int q = 1; q < 4; ++q) {
-            if (q < G) {
-                float* bp = base + ((int64_t)(q - 1) * T + t) * C + c8 * 8;
-                *reinterpret_cast<float4*>(bp) = make_float4(acc[q][0], acc[q][1], acc[q][2], acc[q][3]);
-                *reinterpret_cast<float4*>(bp + 4) = make_float4(acc[q][4], acc[q][5], acc[q][6], acc[q][7]);
-            }
-        }
+        for (int q = 1; q < 4; ++q)
+            if (q < G)
+                *reinterpret_cast<uint4*>(base + ((int64_t)(q - 1) * T + t) * C + c8 * 8) = pack8(acc[q]);
     }
     warp_partial(ss, astat, T, t);
 }
 
 cudaError_t launch_read(const Dims& d, int T, const uint16_t* X, const float* hpre, const int* I,
-                        uint16_t* input0, float* base, uint16_t* xact0, float* astat, cudaStream_t st) {
+                        uint16_t* input0, uint16_t* base, uint16_t* xact0, float* astat, cudaStream_t st) {
     k_read<<<T, chunk_threads(d.C), 0, st>>>(d, T, X, hpre, I, input0, base, xact0, astat); note_launch();
     return cudaGetLastError();
 }
@@ -114,28 +119,39 @@ cudaError_t launch_read(const Dims& d, int T, const uint16_t* X, const float* hp
 // ---------------------------------------------------------------------------------------------
 // input: slots >= 1
 
+template <int KM>
 __global__ void __launch_bounds__(256) k_input(Dims d, int slot, int T,
-                                               const float* __restrict__ base,
+                                               const uint16_t* __restrict__ base,
                                                const uint16_t* __restrict__ xact,
                                                const float* __restrict__ hpre,
                                                const int* __restrict__ I,
                                                uint16_t* __restrict__ input,
                                                float* __restrict__ astat) {
     __shared__ float hj[MAXK];
-    const int t = blockIdx.x, C = d.C;
-    if (threadIdx.x < d.k)
-        hj[threadIdx.x] = hpre[((int64_t)t * d.G + slot) * d.N + I[(int64_t)t * d.k + threadIdx.x]];
+    const int t = blockIdx.x, C = d.C, k = d.k;
+    // the reads of this thread's first chunk (base row, k active rows) are issued before the
+    // coefficient set-up and its barrier
+    uint4 bb, xx[KM];
+    auto load = [&](int c8) {
+        bb = *reinterpret_cast<const uint4*>(base + ((int64_t)(slot - 1) * T + t) * C + c8 * 8);
+#pragma unroll
+        for (int j = 0; j < KM; ++j)
+            if (j < k) xx[j] = *reinterpret_cast<const uint4*>(xact + ((int64_t)t * k + j) * C + c8 * 8);
+    };
+    if ((int)threadIdx.x < C / 8) load(threadIdx.x);
+    if (threadIdx.x < k)
+        hj[threadIdx.x] = hpre[((int64_t)t * d.G + slot) * d.N + I[(int64_t)t * k + threadIdx.x]];
     __syncthreads();
     float ss = 0.f;  // sum of squares of the active state (its projection's norm)
     for (int c8 = threadIdx.x; c8 < C / 8; c8 += blockDim.x) {
-        const float* bp = base + ((int64_t)(slot - 1) * T + t) * C + c8 * 8;
-        const float4 b0 = *reinterpret_cast<const float4*>(bp);
-        const float4 b1 = *reinterpret_cast<const float4*>(bp + 4);
-        float acc[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
-        for (int j = 0; j < d.k; ++j) {
-            const uint4 u = *reinterpret_cast<const uint4*>(xact + ((int64_t)t * d.k + j) * C + c8 * 8);
+        if (c8 != (int)threadIdx.x) load(c8);
+        float acc[8];
+        unpack8(bb, acc);
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            if (j >= k) break;
             float x[8];
-            unpack8(u, x);
+            unpack8(xx[j], x);
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
                 acc[e] = fmaf(hj[j], x[e], acc[e]);
@@ -147,9 +163,13 @@ __global__ void __launch_bounds__(256) k_input(Dims d, int slot, int T,
     warp_partial(ss, astat, T, t);
 }
 
-cudaError_t launch_input(const Dims& d, int slot, int T, const float* base, const uint16_t* xact,
+cudaError_t launch_input(const Dims& d, int slot, int T, const uint16_t* base, const uint16_t* xact,
                          const float* hpre, const int* I, uint16_t* input, float* astat, cudaStream_t st) {
-    k_input<<<T, chunk_threads(d.C), 0, st>>>(d, slot, T, base, xact, hpre, I, input, astat); note_launch();
+    if (d.k <= 4) {
+        k_input<4><<<T, chunk_threads(d.C), 0, st>>>(d, slot, T, base, xact, hpre, I, input, astat); note_launch();
+    } else {
+        k_input<8><<<T, chunk_threads(d.C), 0, st>>>(d, slot, T, base, xact, hpre, I, input, astat); note_launch();
+    }
     return cudaGetLastError();
 }
 

@@ -88,7 +88,7 @@ struct Layout {
                             // 0 is not written) of the active state being mapped
     size_t wsum;            // f32 [N]: column sums of W_r
     size_t rsum;            // f32 [N]: sum_t mu_t dZ_r[t] (router mean-term gradient)
-    size_t base;            // f32 [G-1][T][C]: non-active base readouts of slots 1..G-1
+    size_t base;            // bf16 [G-1][T][C]: non-active base readouts of slots 1..G-1
     size_t red;             // f32 [T][nslice][NRED]: per-slice reduction partials
     size_t dxact;           // f32 [T][k][C]: active-state gradient
     size_t dinput;          // bf16 [G][T][C]: copies of d_input
@@ -293,8 +293,8 @@ cudaError_t launch_coef_act(const Dims& d, int slot, int T, const float* part,
                             float* zact, float* rs, float* hpost, float* hres, cudaStream_t st);
 int stream_warps(int C);  // warps per block of the one-block-per-token stream kernels
 cudaError_t launch_read(const Dims& d, int T, const uint16_t* X, const float* hpre, const int* I,
-                        uint16_t* input0, float* base, uint16_t* xact0, float* astat, cudaStream_t st);
-cudaError_t launch_input(const Dims& d, int slot, int T, const float* base, const uint16_t* xact,
+                        uint16_t* input0, uint16_t* base, uint16_t* xact0, float* astat, cudaStream_t st);
+cudaError_t launch_input(const Dims& d, int slot, int T, const uint16_t* base, const uint16_t* xact,
                          const float* hpre, const int* I, uint16_t* input, float* astat, cudaStream_t st);
 cudaError_t launch_restore(const Dims& d, int T, const uint16_t* xact0, const int* I,
                            uint16_t* X, cudaStream_t st);
