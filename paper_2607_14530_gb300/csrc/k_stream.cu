@@ -34,7 +34,7 @@ int stream_warps(int C) { return chunk_threads(C) / 32; }
 // ---------------------------------------------------------------------------------------------
 // read: one block per token, threads over 8-channel chunks.
 
-__global__ void __launch_bounds__(256) k_read(Dims d, int T, const uint16_t* __restrict__ X,
+__global__ void __launch_bounds__(256, 3) k_read(Dims d, int T, const uint16_t* __restrict__ X,
                                               const float* __restrict__ hpre,
                                               const int* __restrict__ I,
                                               uint16_t* __restrict__ input0,
@@ -127,10 +127,11 @@ __global__ void __launch_bounds__(256) k_input(Dims d, int slot, int T,
                                                const int* __restrict__ I,
                                                uint16_t* __restrict__ input,
                                                float* __restrict__ astat) {
-    __shared__ float hj[MAXK];
     const int t = blockIdx.x, C = d.C, k = d.k;
+    const int lane = threadIdx.x & 31;
     // the reads of this thread's first chunk (base row, k active rows) are issued before the
-    // coefficient set-up and its barrier
+    // coefficients, which every warp fetches for itself (lanes j < k, then broadcast: no block
+    // barrier)
     uint4 bb, xx[KM];
     auto load = [&](int c8) {
         bb = *reinterpret_cast<const uint4*>(base + ((int64_t)(slot - 1) * T + t) * C + c8 * 8);
@@ -139,9 +140,11 @@ __global__ void __launch_bounds__(256) k_input(Dims d, int slot, int T,
             if (j < k) xx[j] = *reinterpret_cast<const uint4*>(xact + ((int64_t)t * k + j) * C + c8 * 8);
     };
     if ((int)threadIdx.x < C / 8) load(threadIdx.x);
-    if (threadIdx.x < k)
-        hj[threadIdx.x] = hpre[((int64_t)t * d.G + slot) * d.N + I[(int64_t)t * k + threadIdx.x]];
-    __syncthreads();
+    float hl = 0.f;
+    if (lane < k) hl = hpre[((int64_t)t * d.G + slot) * d.N + I[(int64_t)t * k + lane]];
+    float hj[KM];
+#pragma unroll
+    for (int j = 0; j < KM; ++j) hj[j] = __shfl_sync(0xffffffffu, hl, j);
     float ss = 0.f;  // sum of squares of the active state (its projection's norm)
     for (int c8 = threadIdx.x; c8 < C / 8; c8 += blockDim.x) {
         if (c8 != (int)threadIdx.x) load(c8);
