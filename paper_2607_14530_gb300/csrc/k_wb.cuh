@@ -877,7 +877,7 @@ __global__ void __launch_bounds__(WT) k_wb_fwd8(Dims d, int slot, int T, int TB,
 // backward reductions: P[j][0] = <dXn_j, out> (and, last slot, Q[j][i] = <dXn_j, x_i>), one
 // partial per W8-channel slice
 template <int KM>
-__global__ void __launch_bounds__(WT) k_wb_bred8(Dims d, int slot, int T, int TB,
+__global__ void __launch_bounds__(WT, 4) k_wb_bred8(Dims d, int slot, int T, int TB,
                                                  const uint16_t* __restrict__ out,
                                                  const uint16_t* __restrict__ dX,
                                                  const int* __restrict__ I,
