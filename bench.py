@@ -53,6 +53,10 @@ def workloads():
 # every input read once, every output written once; flops of the contractions)
 
 
+# side-stream kernels forked at the same point as a main-stream kernel and overlapping it
+OVERLAP = {"dxa_tc": ("dinput_act",)}
+
+
 def kernel_model(cfg, T):
     N, k, C, G = cfg.N, cfg.k, cfg.C, cfg.G
     hr = cfg.m < cfg.k
@@ -409,6 +413,15 @@ def run_xhc(args, wl_name):
         roof = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": hbm_peak,
                 "unit": "GB/s", "frac": achieved / hbm_peak, "peak_source": f"{peak_src} hbm_gbs"}
     roof["traffic"] = ncu_traffic(dom, wl_name)
+    # kernels the library launches on its side stream at the same point, which finish inside the
+    # dominant kernel's event window and share its HBM bandwidth: their bytes over that window
+    part = [n for n in OVERLAP.get(dom, ()) if n in per and n in model and per[n][1] <= tot]
+    if part and roof["bound"] == "hbm":
+        wb = mm["bytes"] / launches_per_step + sum(model[n]["bytes"] / model[n]["launches"] for n in part)
+        roof["concurrent"] = {"kernels": part, "window_gbs": wb / secs / 1e9,
+                              "window_frac": wb / secs / 1e9 / hbm_peak,
+                              "note": "side-stream kernels running inside this kernel's launch window; "
+                                      "achieved / frac above count this kernel's bytes only"}
 
     step_bytes = sum(v["bytes"] for v in model.values())
     hbm = {"model_bytes_per_step": step_bytes, "achieved_gbs": step_bytes / (ms_step / 1000.0) / 1e9,
