@@ -253,6 +253,19 @@ def ncu_traffic(kernel, workload):
     return e.get("dram_bytes_per_launch")
 
 
+def job_rate(ms_local, tokens_per_rank, steps, world, device=None):
+    """(slowest rank's ms, whole-job tokens/s): every rank processes its own tokens_per_rank per
+    step (weak scaling, no data-path collective); the timed region is the max over ranks."""
+    ms = float(ms_local)
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        t = torch.tensor([ms], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    return ms, world * tokens_per_rank * steps / (ms / 1000.0)
+
+
 def oracle_step(cfg, X, outs, dX, dins, P):
     """One fp64 oracle fwd+bwd on CPU tensors (the oracle as it stands)."""
     import torch
@@ -366,13 +379,8 @@ def run_xhc(args, wl_name):
     launches = xhc.launch_count() - n0
     xhc.trace_enable(False)
     ck = clocks.stop()
-    ms = e0.elapsed_time(e1)
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms, value = job_rate(e0.elapsed_time(e1), T, args.steps, world, dev)
     ms_step = ms / args.steps
-    value = world * T * args.steps / (ms / 1000.0)
 
     # per-kernel device time over the timed region
     recs = xhc.trace_records()
@@ -521,12 +529,8 @@ def run_xhc(args, wl_name):
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         run(ksteps, a, b)
         torch.cuda.synchronize()
-        ems = a.elapsed_time(b)
-        if world > 1:
-            t = torch.tensor([ems], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ems = float(t.item())
-        line["e2e"] = {"value": world * T * ksteps / (ems / 1000.0), "unit": "tokens/s",
+        ems, evalue = job_rate(a.elapsed_time(b), T, ksteps, world, dev)
+        line["e2e"] = {"value": evalue, "unit": "tokens/s",
                        "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": ksteps,
                        "pipelined": "copy-in of step i+1 and copy-out of step i overlap step i+1's compute"}
 
