@@ -193,6 +193,33 @@ xhc_status xhc_post_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
                         uint16_t* X, const uint16_t* out, void* saved, void* workspace,
                         void* stream);
 
+/* Decoding: one new token per sequence.
+ *
+ * The op is token-parallel except for the causal conv of the MLP slots (Eq. aug, Sec. 3.3.4),
+ * which reads the R = max(kappa) - 1 previous `out` rows of the token's sequence.  For decoding
+ * those rows live in a per-sequence ring owned by the caller, one per conv slot: ring [B][R][C]
+ * bf16, row (s mod R) holding out[s] of position s.  pos [B] int64 (device) is the position of
+ * each sequence's current token.  A decode step of a group is, for slot = 0..G-1,
+ * xhc_pre_fwd(slot, T = B) then xhc_post_fwd_decode(slot, B); use a handle whose seq_len is 0
+ * (or divides B): the conv history comes from the ring, not from the call's tokens.
+ *
+ * xhc_ring_bytes: size of one conv slot's ring for B sequences (0 without a conv).
+ * xhc_ring_fill: after a prefill of B sequences of S tokens each (rows b*S .. b*S+S-1 of `out`,
+ *   the slot's sublayer output), stores each sequence's last min(S, R) rows in its ring; the
+ *   caller then sets pos[b] = S.  Rows the conv will not read are left as they are.
+ * xhc_post_fwd_decode: xhc_post_fwd for B tokens, token b at position pos[b] of sequence b, with
+ *   the conv history read from `ring` (null for a slot without a conv); afterwards the token's
+ *   out row is stored in its ring row, and the group's last slot advances pos by one.  Same
+ *   saved / workspace contract as xhc_post_fwd with T = B.  Errors: XHC_ERR_INVALID_ARG for a
+ *   null ring on a conv slot, null pos, B <= 0; XHC_ERR_ALIGNMENT for pointers not 16-byte
+ *   aligned. */
+xhc_status xhc_ring_bytes(const xhc_handle* h, int64_t B, size_t* bytes);
+xhc_status xhc_ring_fill(const xhc_handle* h, int64_t B, int64_t S, const uint16_t* out, void* ring,
+                         void* stream);
+xhc_status xhc_post_fwd_decode(const xhc_handle* h, int slot, int64_t B, const xhc_params* P,
+                               uint16_t* X, const uint16_t* out, void* ring, int64_t* pos,
+                               void* saved, void* workspace, void* stream);
+
 /* Backward of post_fwd(slot).  Reads dX (slot G-1: the gradient w.r.t. the group output) or the
  * workspace-held active gradient, leaves the post/res map-logit gradient in the workspace for
  * pre_bwd(slot), writes d_out [T, C] (= dL/d out, including the paths through

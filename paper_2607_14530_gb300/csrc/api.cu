@@ -615,6 +615,50 @@ xhc_status xhc_post_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
     return XHC_OK;
 }
 
+xhc_status xhc_ring_bytes(const xhc_handle* h, int64_t B, size_t* bytes) {
+    if (!h || !bytes || B <= 0) return XHC_ERR_INVALID_ARG;
+    const Dims& d = h->h.d;
+    *bytes = d.nconv > 0 ? (size_t)B * (d.kapmax - 1) * d.C * 2 : 0;
+    return XHC_OK;
+}
+
+xhc_status xhc_ring_fill(const xhc_handle* h, int64_t B, int64_t S, const uint16_t* out, void* ring,
+                         void* stream) {
+    if (!h || !out || !ring || B <= 0 || S <= 0 || B * S > ((int64_t)1 << 30)) return XHC_ERR_INVALID_ARG;
+    if (!aligned16(out) || !aligned16(ring)) return XHC_ERR_ALIGNMENT;
+    const Dims& d = h->h.d;
+    if (d.nconv == 0) return XHC_OK;
+    if (launch_ring_fill(d, (int)B, (int)S, out, (uint16_t*)ring, (cudaStream_t)stream) != cudaSuccess)
+        return XHC_ERR_CUDA;
+    return XHC_OK;
+}
+
+xhc_status xhc_post_fwd_decode(const xhc_handle* h, int slot, int64_t B, const xhc_params* P,
+                               uint16_t* X, const uint16_t* out, void* ring, int64_t* pos,
+                               void* saved, void* workspace, void* stream) {
+    Ctx c;
+    xhc_status s = common_check(h, slot, B, saved, workspace, c, stream);
+    if (s != XHC_OK) return s;
+    const Dims& d = c.d;
+    const bool conv = d.K[slot] > 1;
+    if (!X || !out || !pos || (conv && !ring) || !params_ok(d, P, slot, false)) return XHC_ERR_INVALID_ARG;
+    if (!aligned16(X) || !aligned16(out) || (ring && !aligned16(ring))) return XHC_ERR_ALIGNMENT;
+    const ConvPtrs cw = conv_of(d, P, slot);
+    const bool last = (slot == d.G - 1);
+    long long* ps = reinterpret_cast<long long*>(pos);
+    uint16_t* rg = static_cast<uint16_t*>(ring);
+    if (conv && d.gs)
+        XHC_K("dec_gram", c.st, launch_dec_gram(d, slot, c.T, out, cw, rg, ps, c.W<float>(c.L.red), c.st));
+    XHC_K("wb_coef", c.st, launch_wb_coef(d, slot, c.T, c.W<float>(c.L.red), 1, c.S<float>(c.L.p),
+                                          c.S<float>(c.L.hpost[slot]),
+                                          (conv && d.gs) ? c.S<double>(c.L.gram[slot]) : nullptr,
+                                          c.W<float>(c.L.tokmat), c.st));
+    XHC_K("dec_fwd", c.st, launch_dec_fwd(d, slot, c.T, out, cw, rg, ps, c.W<float>(c.L.tokmat),
+                                          c.xact(slot), c.S<int>(c.L.I), c.S<float>(c.L.hres),
+                                          last ? nullptr : c.xact(slot + 1), X, c.st));
+    return XHC_OK;
+}
+
 xhc_status xhc_post_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
                         uint16_t* X, uint16_t* dX, const uint16_t* out, uint16_t* d_out,
                         const xhc_grads* g, void* saved, void* workspace, void* stream) {

@@ -1,0 +1,203 @@
+// Decode: the write-back of a conv slot for one new token per sequence.
+//
+// In decoding, token t of the call is the next token of its own sequence b = t, at position
+// pos[t] of that sequence.  The causal conv of Eq. aug (Sec. 3.3.4: g_j[s] = sum_{i < kappa_j}
+// w_j[i] out[s - i], zero before the sequence start) needs the R = max(kappa) - 1 previous `out`
+// rows of the sequence, which no longer exist as a contiguous [T][C] buffer: they are kept in a
+// per-sequence ring [B][R][C] bf16 (row (s mod R) holds out[s]).  The kernels below are the
+// decode forms of the Gram reduction and of the write-back (Eq. gs, Eq. sparse_write_delta,
+// Eq. sparse_write): one CTA per token, threads over channel pairs, the conv read from the ring
+// plus the token's own `out` row.  The write-back stores the token's `out` into its ring row
+// afterwards, and the group's last slot advances pos.
+#include <algorithm>
+
+#include "xhc_internal.cuh"
+
+namespace xhc {
+namespace {
+
+__device__ __forceinline__ float2 ldp(const uint16_t* p) {
+    const uint32_t u = *reinterpret_cast<const uint32_t*>(p);
+    return make_float2(__uint_as_float(u << 16), __uint_as_float(u & 0xffff0000u));
+}
+
+// the write-back components of channels (c, c + 1) of token t: u_0 = out, u_{1+j} = g_j
+__device__ __forceinline__ void dec_components(const Dims& d, int slot, int t, int c,
+                                               const uint16_t* __restrict__ out, ConvPtrs cw,
+                                               const uint16_t* __restrict__ ring, long long pos,
+                                               float2 (&u)[4]) {
+    const int C = d.C, R = d.kapmax - 1;
+    const float2 o = ldp(out + (long long)t * C + c);
+    u[0] = o;
+    u[1] = u[2] = u[3] = make_float2(0.f, 0.f);
+    if (d.K[slot] <= 1) return;
+    for (int j = 0; j < d.nconv; ++j) {
+        float2 g = make_float2(0.f, 0.f);
+        for (int i = 0; i < d.kap[j]; ++i) {
+            const long long s = pos - i;                       // position of the tap's token
+            if (s < 0) break;                                  // before the sequence start: zero
+            const float2 v = (i == 0) ? o : ldp(ring + ((long long)t * R + (int)(s % R)) * C + c);
+            const float2 w = make_float2(cw.w[j][(size_t)i * C + c], cw.w[j][(size_t)i * C + c + 1]);
+            g.x = fmaf(w.x, v.x, g.x);
+            g.y = fmaf(w.y, v.y, g.y);
+        }
+        u[1 + j] = g;
+    }
+}
+
+// Gram matrix of the components of each token (lower triangle, the order of the prefill's
+// reduction), into reduction slice 0
+__global__ void __launch_bounds__(256) k_dec_gram(Dims d, int slot, const uint16_t* __restrict__ out,
+                                                  ConvPtrs cw, const uint16_t* __restrict__ ring,
+                                                  const long long* __restrict__ pos,
+                                                  float* __restrict__ red) {
+    __shared__ float sh[8][NGRAM];
+    const int t = blockIdx.x, K = d.K[slot];
+    const long long p = pos[t];
+    float v[NGRAM];
+#pragma unroll
+    for (int q = 0; q < NGRAM; ++q) v[q] = 0.f;
+    for (int c = 2 * threadIdx.x; c < d.C; c += 2 * blockDim.x) {
+        float2 u[4];
+        dec_components(d, slot, t, c, out, cw, ring, p, u);
+        int q = 0;
+#pragma unroll
+        for (int a = 0; a < 4; ++a)
+#pragma unroll
+            for (int b = 0; b <= a; ++b, ++q)
+                if (a < K) v[q] = fmaf(u[a].x, u[b].x, fmaf(u[a].y, u[b].y, v[q]));
+    }
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+    for (int q = 0; q < NGRAM; ++q) {
+        float x = v[q];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+        if (lane == 0) sh[warp][q] = x;
+    }
+    __syncthreads();
+    if (threadIdx.x < NGRAM) {
+        float s = 0.f;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) s += sh[w][threadIdx.x];
+        red[(long long)t * NRED + threadIdx.x] = s;
+    }
+}
+
+// X_act_new_j = (H_res x_act)_j (last slot) or x_act_j, + sum_a E[j][a] u_a; the last slot
+// scatters into the state rows I_j, the others write the next slot's active state.  Then the
+// token's out row goes into its ring row (each thread its own channels, after its last read of
+// them), and the last slot advances the token's position.
+__global__ void __launch_bounds__(256) k_dec_fwd(Dims d, int slot, const uint16_t* __restrict__ out,
+                                                 ConvPtrs cw, uint16_t* __restrict__ ring,
+                                                 long long* __restrict__ pos,
+                                                 const float* __restrict__ emat,
+                                                 const uint16_t* __restrict__ xact,
+                                                 const int* __restrict__ I,
+                                                 const float* __restrict__ hres,
+                                                 uint16_t* __restrict__ xact_next,
+                                                 uint16_t* __restrict__ X) {
+    const int t = blockIdx.x, C = d.C, k = d.k, R = d.kapmax - 1;
+    const bool last = (slot == d.G - 1);
+    const bool conv = d.K[slot] > 1;
+    const long long p = pos[t];
+    const float* E = emat + (long long)t * TOKMAT;
+    for (int c = 2 * threadIdx.x; c < C; c += 2 * blockDim.x) {
+        float2 u[4];
+        dec_components(d, slot, t, c, out, cw, ring, p, u);
+        float2 x[MAXK];
+#pragma unroll
+        for (int j = 0; j < MAXK; ++j)
+            x[j] = (j < k) ? ldp(xact + ((long long)t * k + j) * C + c) : make_float2(0.f, 0.f);
+#pragma unroll
+        for (int j = 0; j < MAXK; ++j) {
+            if (j >= k) break;
+            float2 v;
+            if (last) {
+                v = make_float2(0.f, 0.f);
+#pragma unroll
+                for (int i = 0; i < MAXK; ++i) {
+                    if (i >= k) break;
+                    const float h = hres[((long long)t * k + j) * k + i];
+                    v.x = fmaf(h, x[i].x, v.x);
+                    v.y = fmaf(h, x[i].y, v.y);
+                }
+            } else {
+                v = x[j];
+            }
+#pragma unroll
+            for (int a = 0; a < 4; ++a) {
+                const float e = E[j * 4 + a];
+                v.x = fmaf(e, u[a].x, v.x);
+                v.y = fmaf(e, u[a].y, v.y);
+            }
+            uint16_t* dst = last ? X + ((long long)t * d.N + I[(long long)t * k + j]) * C + c
+                                 : xact_next + ((long long)t * k + j) * C + c;
+            *reinterpret_cast<uint32_t*>(dst) = pack2(v.x, v.y);
+        }
+        if (conv && R > 0)
+            *reinterpret_cast<uint32_t*>(ring + ((long long)t * R + (int)(p % R)) * C + c) =
+                *reinterpret_cast<const uint32_t*>(out + (long long)t * C + c);
+    }
+}
+
+// the last slot advances every token's position (after every CTA of the write-back is done:
+// a separate launch)
+__global__ void k_pos_advance(long long* __restrict__ pos, int B) {
+    const int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b < B) pos[b] += 1;
+}
+
+// ring rows from a prefill: sequence b of S tokens (rows b*S .. b*S + S - 1 of out) leaves its
+// last min(S, R) rows in ring rows (s mod R)
+__global__ void k_ring_fill(const uint16_t* __restrict__ out, int B, int S, int C, int R,
+                            uint16_t* __restrict__ ring) {
+    const long long n = (long long)B * R * (C / 8);
+    for (long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x; idx < n;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const int c8 = (int)(idx % (C / 8));
+        const long long r = idx / (C / 8);
+        const int lag = (int)(r % R) + 1;           // 1..R: token S - lag
+        const int b = (int)(r / R);
+        const long long s = (long long)S - lag;
+        if (s < 0) continue;
+        *reinterpret_cast<uint4*>(ring + ((long long)b * R + (int)(s % R)) * C + c8 * 8) =
+            *reinterpret_cast<const uint4*>(out + ((long long)b * S + s) * C + c8 * 8);
+    }
+}
+
+int dec_threads(int C) {
+    int th = ((C / 2 + 31) / 32) * 32;
+    return th > 256 ? 256 : (th < 32 ? 32 : th);
+}
+
+}  // namespace
+
+cudaError_t launch_dec_gram(const Dims& d, int slot, int B, const uint16_t* out, ConvPtrs cw,
+                            const uint16_t* ring, const long long* pos, float* red, cudaStream_t st) {
+    k_dec_gram<<<B, dec_threads(d.C), 0, st>>>(d, slot, out, cw, ring, pos, red); note_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_dec_fwd(const Dims& d, int slot, int B, const uint16_t* out, ConvPtrs cw,
+                           uint16_t* ring, long long* pos, const float* emat, const uint16_t* xact,
+                           const int* I, const float* hres, uint16_t* xact_next, uint16_t* X,
+                           cudaStream_t st) {
+    k_dec_fwd<<<B, dec_threads(d.C), 0, st>>>(d, slot, out, cw, ring, pos, emat, xact, I, hres,
+                                              xact_next, X); note_launch();
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess || slot != d.G - 1) return e;
+    k_pos_advance<<<(B + 255) / 256, 256, 0, st>>>(pos, B); note_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_ring_fill(const Dims& d, int B, int S, const uint16_t* out, uint16_t* ring,
+                             cudaStream_t st) {
+    const int R = d.kapmax - 1;
+    if (R <= 0) return cudaSuccess;
+    const long long n = (long long)B * R * (d.C / 8);
+    const int blocks = (int)std::min<long long>((n + 255) / 256, 4096);
+    k_ring_fill<<<blocks, 256, 0, st>>>(out, B, S, d.C, R, ring); note_launch();
+    return cudaGetLastError();
+}
+
+}  // namespace xhc

@@ -264,6 +264,15 @@ cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, 
 int wb_nslice(int C);
 int wb_conv_runs(const Dims& d, int64_t T);
 int wb_bred_slices(const Dims& d, int slot);  // partial-sum slices of wb_bred (and bwd_coef)  // runs (conv weight-gradient partials) of wb_bapp
+// decode (one token per sequence, conv history in a per-sequence ring of max(kappa) - 1 rows)
+cudaError_t launch_dec_gram(const Dims& d, int slot, int B, const uint16_t* out, ConvPtrs cw,
+                            const uint16_t* ring, const long long* pos, float* red, cudaStream_t st);
+cudaError_t launch_dec_fwd(const Dims& d, int slot, int B, const uint16_t* out, ConvPtrs cw,
+                           uint16_t* ring, long long* pos, const float* emat, const uint16_t* xact,
+                           const int* I, const float* hres, uint16_t* xact_next, uint16_t* X,
+                           cudaStream_t st);
+cudaError_t launch_ring_fill(const Dims& d, int B, int S, const uint16_t* out, uint16_t* ring,
+                             cudaStream_t st);
 cudaError_t launch_wb_gram(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
                            int nslice, float* red, cudaStream_t st);
 cudaError_t launch_wb_coef(const Dims& d, int slot, int T, const float* red, int nslice, const float* p,

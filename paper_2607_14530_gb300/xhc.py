@@ -77,6 +77,9 @@ def lib() -> ctypes.CDLL:
         L.xhc_pre_bwd.argtypes = [vp, ctypes.c_int, i64, P, vp, vp, vp, P, vp, vp, vp]
         L.xhc_saved_layout_of.argtypes = [vp, i64, ctypes.POINTER(_SavedLayout)]
         L.xhc_route_noalloc.argtypes = [vp, i64, P, vp, vp, vp, vp, vp]
+        L.xhc_ring_bytes.argtypes = [vp, i64, ctypes.POINTER(sz)]
+        L.xhc_ring_fill.argtypes = [vp, i64, i64, vp, vp, vp]
+        L.xhc_post_fwd_decode.argtypes = [vp, ctypes.c_int, i64, P, vp, vp, vp, vp, vp, vp, vp]
         L.xhc_workspace_error.argtypes = [vp, ctypes.POINTER(ctypes.c_int), ctypes.c_int]
         L.xhc_trace_enable.argtypes = [ctypes.c_int]
         L.xhc_trace_count.restype = ctypes.c_int
@@ -346,6 +349,45 @@ class Group:
         for t in range(self.cfg.G):
             self.pre_fwd(t, pp, X, inputs[t], saved, ws, stream)
             self.post_fwd(t, pp, X, outs[t], saved, ws, stream)
+        return inputs
+
+    # ---- decoding: one new token per sequence (see xhc_post_fwd_decode) ----
+
+    def ring_bytes(self, B: int) -> int:
+        n = ctypes.c_size_t()
+        _check(lib().xhc_ring_bytes(self._h, B, ctypes.byref(n)), "xhc_ring_bytes")
+        return n.value
+
+    def alloc_rings(self, B: int, device="cuda") -> list:
+        """One conv-history ring per slot (None for a slot without a conv)."""
+        n = self.ring_bytes(B)
+        return [torch.zeros(n, dtype=torch.uint8, device=device) if (n and self.cfg.K(t) > 1) else None
+                for t in range(self.cfg.G)]
+
+    def ring_fill(self, B: int, S: int, out, ring, stream=None):
+        """After a prefill of B sequences of S tokens: the last rows of each sequence's `out`."""
+        _check(lib().xhc_ring_fill(self._h, B, S, _bf16(out, "out"), _ptr(ring), _stream(stream)),
+               "xhc_ring_fill")
+
+    def post_fwd_decode(self, slot, P, X, out, ring, pos, saved, ws, stream=None):
+        B = X.shape[0]
+        pp = P if isinstance(P, _Params) else self.params(P)
+        if pos.dtype != torch.int64 or not pos.is_cuda or not pos.is_contiguous():
+            raise XhcError("pos must be a contiguous int64 CUDA tensor")
+        _check(lib().xhc_post_fwd_decode(self._h, slot, B, ctypes.byref(pp), _bf16(X, "X"), _bf16(out, "out"),
+                                         _ptr(ring), _ptr(pos), _ptr(saved), _ptr(ws), _stream(stream)),
+               f"xhc_post_fwd_decode({slot})")
+
+    def forward_decode(self, P, X, outs, rings, pos, saved, ws, inputs=None, stream=None):
+        """One decode step of the group: X [B, N, C] (token b = next token of sequence b, at
+        position pos[b]) updated in place; pos advanced by one.  Returns the inputs."""
+        B, C = X.shape[0], self.cfg.C
+        if inputs is None:
+            inputs = [torch.empty(B, C, dtype=torch.bfloat16, device=X.device) for _ in range(self.cfg.G)]
+        pp = self.params(P)
+        for t in range(self.cfg.G):
+            self.pre_fwd(t, pp, X, inputs[t], saved, ws, stream)
+            self.post_fwd_decode(t, pp, X, outs[t], rings[t], pos, saved, ws, stream)
         return inputs
 
     def backward(self, P, X, dX, outs, d_inputs, grads, saved, ws, d_outs=None, stream=None):
