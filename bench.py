@@ -550,6 +550,102 @@ def run_xhc(args, wl_name):
         dist.destroy_process_group()
 
 
+def run_decode(args, wl_name):
+    """Inference legs (not part of the default line): forward-only prefill of the workload, and
+    decode steps (one new token per sequence, conv history in rings) for a batch of sequences,
+    eagerly and as a captured CUDA graph of one step.  One JSON line."""
+    import torch
+    from paper_2607_14530_gb300 import build, synth, xhc
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    build.build()
+    xhc.lib()
+    desc, cfg, T = workloads()[wl_name]
+    if args.tokens:
+        T = args.tokens
+    seed = 1234
+    P = {n: v.to(dev) for n, v in synth.params(cfg.param_shapes(), seed).items()}
+    stream = torch.cuda.current_stream()
+
+    def timed(fn, k):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(k):
+            fn()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / k
+
+    # prefill: the forward of the whole workload (sequences of seq_len tokens)
+    g = xhc.Group(cfg)
+    X = synth.normal_bf16_on((T, cfg.N, cfg.C), seed, dev)
+    outs = [synth.normal_bf16_on((T, cfg.C), seed + 101 + t, dev) for t in range(cfg.G)]
+    saved, ws = g.alloc(T, device=dev)
+    inputs = [torch.empty(T, cfg.C, dtype=torch.bfloat16, device=dev) for _ in range(cfg.G)]
+    X0 = X.clone()
+
+    def prefill():
+        X.copy_(X0)
+        g.forward(P, X, outs, saved, ws, inputs=inputs)
+
+    copy_ms = timed(lambda: X.copy_(X0), args.steps)
+    pre_ms = timed(prefill, args.steps) - copy_ms
+    del saved, ws, X, X0, inputs
+    torch.cuda.empty_cache()
+
+    # decode: B sequences, one token each per step
+    B = args.decode_batch
+    gd = xhc.Group(type(cfg).flash(cfg.N, cfg.k, cfg.m, cfg.C, cfg.G, seq_len=0) if cfg.G > 1 else cfg)
+    Xd = synth.normal_bf16_on((B, cfg.N, cfg.C), seed + 3, dev)
+    outs_d = [synth.normal_bf16_on((B, cfg.C), seed + 301 + t, dev) for t in range(cfg.G)]
+    saved_d, ws_d = gd.alloc(B, device=dev)
+    rings = gd.alloc_rings(B, device=dev)
+    pos = torch.full((B,), 4096, dtype=torch.int64, device=dev)
+    ins_d = [torch.empty(B, cfg.C, dtype=torch.bfloat16, device=dev) for _ in range(cfg.G)]
+
+    def dstep():
+        gd.forward_decode(P, Xd, outs_d, rings, pos, saved_d, ws_d, inputs=ins_d)
+
+    eager_ms = timed(dstep, args.steps)
+    n0 = xhc.launch_count()
+    xhc.trace_enable(True)
+    dstep()
+    torch.cuda.synchronize()
+    launches = xhc.launch_count() - n0
+    per = {}
+    for name, t_ms in xhc.trace_records():
+        per[name] = per.get(name, 0.0) + t_ms
+    xhc.trace_enable(False)
+    top = sorted(per.items(), key=lambda kv: -kv[1])[:6]
+    graph_ms = None
+    try:
+        graph = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream()
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):
+            dstep()
+        stream.wait_stream(side)
+        torch.cuda.synchronize()
+        with torch.cuda.graph(graph):
+            dstep()
+        graph_ms = timed(graph.replay, args.steps)
+    except Exception as e:  # capture not possible on this stack: eager numbers only
+        graph_ms = f"not captured: {type(e).__name__}"
+    line = {"metric": "inference: prefill and decode tokens/s", "unit": "tokens/s",
+            "prefill": {"workload": desc, "tokens": T, "ms": pre_ms, "value": T / (pre_ms / 1000.0)},
+            "decode": {"batch": B, "launches_per_step": launches, "eager_ms": eager_ms,
+                       "top_calls_ms": [[n, round(t, 4)] for n, t in top],
+                       "eager_value": B / (eager_ms / 1000.0),
+                       "graph_ms": graph_ms,
+                       "graph_value": (B / (graph_ms / 1000.0)) if isinstance(graph_ms, float) else None},
+            "steps": args.steps, "dtype": "f32", "data": "synthetic"}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -563,11 +659,16 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--kernels-out", default="")
+    ap.add_argument("--mode", default="train", choices=["train", "inference"],
+                    help="inference: forward-only prefill and decode legs (a separate line)")
+    ap.add_argument("--decode-batch", type=int, default=256)
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "xhc":
         args.warmup = 3
     if args.impl == "reference":
         run_reference(args, args.workload)
+    elif args.mode == "inference":
+        run_decode(args, args.workload)
     else:
         run_xhc(args, args.workload)
 

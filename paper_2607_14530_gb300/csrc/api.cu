@@ -517,6 +517,9 @@ ConvPtrs conv_of(const Dims& d, const xhc_params* P, int slot) {
     return c;
 }
 
+// above this many split-K partial slots the coefficient kernels get them pre-summed
+constexpr int SLOT_SUM_MIN = 8;
+
 // Active-state mapping generation of one slot (Eq. param_post, Eq. param_res).
 xhc_status active_maps(const Ctx& c, int slot, const xhc_params* P) {
     const Dims& d = c.d;
@@ -538,6 +541,14 @@ xhc_status active_maps(const Ctx& c, int slot, const xhc_params* P) {
                                                      c.W<int>(c.L.err), c.st));
         pstats = c.W<float>(c.L.astat);
         ssplits = stream_warps(d.C);
+    }
+    if (splits > SLOT_SUM_MIN) {
+        XHC_K("slot_sum", c.st, launch_slot_sum(c.W<float>(c.L.part), splits, (long long)c.T * d.nact[slot], c.st));
+        splits = 1;
+    }
+    if (ssplits > SLOT_SUM_MIN && pstats == c.W<float>(c.L.pstats)) {
+        XHC_K("slot_sum", c.st, launch_slot_sum(pstats, ssplits, (long long)c.T * 2, c.st));
+        ssplits = 1;
     }
     XHC_K("coef_act", c.st, launch_coef_act(d, slot, c.T, c.W<float>(c.L.part), pstats, ssplits,
                              splits, P->alpha_post, P->b_post[slot], P->alpha_res, P->b_res,
@@ -578,6 +589,12 @@ xhc_status xhc_pre_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
         XHC_K("proj_tc", c.st, launch_proj_tc(X, c.T, d.N * d.C, c.W<uint16_t>(c.L.wpack), d.nfull,
                                               c.L.tc, c.W<float>(c.L.part), c.W<float>(c.L.pstats),
                                               c.W<int>(c.L.err), c.st));
+        }
+        if (fsplits > SLOT_SUM_MIN) {
+            // few tokens, many split-K slots: summed in parallel first
+            XHC_K("slot_sum", c.st, launch_slot_sum(c.W<float>(c.L.part), fsplits, (long long)c.T * d.nfull, c.st));
+            XHC_K("slot_sum", c.st, launch_slot_sum(c.W<float>(c.L.pstats), fsplits, (long long)c.T * 2, c.st));
+            fsplits = 1;
         }
         XHC_K("coef_full", c.st, launch_coef_full(d, c.T, c.W<float>(c.L.part), c.W<float>(c.L.pstats),
                                   fsplits, c.W<float>(c.L.wsum), P->alpha_pre, P->b_pre,
@@ -649,7 +666,7 @@ xhc_status xhc_post_fwd_decode(const xhc_handle* h, int slot, int64_t B, const x
     uint16_t* rg = static_cast<uint16_t*>(ring);
     if (conv && d.gs)
         XHC_K("dec_gram", c.st, launch_dec_gram(d, slot, c.T, out, cw, rg, ps, c.W<float>(c.L.red), c.st));
-    XHC_K("wb_coef", c.st, launch_wb_coef(d, slot, c.T, c.W<float>(c.L.red), 1, c.S<float>(c.L.p),
+    XHC_K("wb_coef", c.st, launch_wb_coef(d, slot, c.T, c.W<float>(c.L.red), dec_nslice(d.C), c.S<float>(c.L.p),
                                           c.S<float>(c.L.hpost[slot]),
                                           (conv && d.gs) ? c.S<double>(c.L.gram[slot]) : nullptr,
                                           c.W<float>(c.L.tokmat), c.st));

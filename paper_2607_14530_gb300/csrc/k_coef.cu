@@ -7,6 +7,8 @@
 //              write-back contraction (Eq. sparse_write_delta)
 //   full_coef  reverse of coef_full (norm corrections, pre-map sigmoid, router through the
 //              selected routed scores only)
+#include <algorithm>
+
 #include "xhc_internal.cuh"
 
 namespace xhc {
@@ -169,6 +171,27 @@ __device__ void sinkhorn_bwd(const float (&M)[KM][KM], int k, int iters, int L, 
     for (int a = 0; a < KM; ++a)
 #pragma unroll
         for (int b = 0; b < KM; ++b) dM[a][b] = (a < k && b < k) ? dA[a][b] * A0[a][b] : 0.f;
+}
+
+// ---------------------------------------------------------------------------------------------
+// slot_sum: x[e] = sum_q x[q * n + e] over the split-K partial slots, in slot order (the order
+// in which the coefficient kernels sum them, so a summed buffer read as one slot gives the same
+// bits), into slot 0.  Used when there are many slots (few tokens): one thread per element
+// instead of one thread per token walking every slot.
+
+__global__ void k_slot_sum(float* __restrict__ x, int nslots, long long n) {
+    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < n;
+         e += (long long)gridDim.x * blockDim.x) {
+        float s = 0.f;
+        for (int q = 0; q < nslots; ++q) s += x[(long long)q * n + e];
+        x[e] = s;
+    }
+}
+
+cudaError_t launch_slot_sum(float* x, int nslots, long long n, cudaStream_t st) {
+    const int blocks = (int)std::min<long long>((n + 255) / 256, 4096);
+    k_slot_sum<<<blocks, 256, 0, st>>>(x, nslots, n); note_launch();
+    return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------------------------------------

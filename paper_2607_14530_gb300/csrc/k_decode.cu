@@ -6,9 +6,9 @@
 // rows of the sequence, which no longer exist as a contiguous [T][C] buffer: they are kept in a
 // per-sequence ring [B][R][C] bf16 (row (s mod R) holds out[s]).  The kernels below are the
 // decode forms of the Gram reduction and of the write-back (Eq. gs, Eq. sparse_write_delta,
-// Eq. sparse_write): one CTA per token, threads over channel pairs, the conv read from the ring
-// plus the token's own `out` row.  The write-back stores the token's `out` into its ring row
-// afterwards, and the group's last slot advances pos.
+// Eq. sparse_write): CTAs over (256-channel slice, 16 tokens), one channel pair per thread, the
+// conv read from the ring plus the token's own `out` row.  The write-back stores the token's
+// `out` into its ring row afterwards, and the group's last slot advances pos.
 #include <algorithm>
 
 #include "xhc_internal.cuh"
@@ -31,12 +31,15 @@ __device__ __forceinline__ void dec_components(const Dims& d, int slot, int t, i
     u[0] = o;
     u[1] = u[2] = u[3] = make_float2(0.f, 0.f);
     if (d.K[slot] <= 1) return;
+    const int r0 = (int)(pos % R);                             // ring row of position pos
+    const uint16_t* rt = ring + (long long)t * R * C + c;
     for (int j = 0; j < d.nconv; ++j) {
         float2 g = make_float2(0.f, 0.f);
         for (int i = 0; i < d.kap[j]; ++i) {
-            const long long s = pos - i;                       // position of the tap's token
-            if (s < 0) break;                                  // before the sequence start: zero
-            const float2 v = (i == 0) ? o : ldp(ring + ((long long)t * R + (int)(s % R)) * C + c);
+            if (pos - i < 0) break;                            // before the sequence start: zero
+            int r = r0 - i;                                    // row of position pos - i
+            if (r < 0) r += R;
+            const float2 v = (i == 0) ? o : ldp(rt + (long long)r * C);
             const float2 w = make_float2(cw.w[j][(size_t)i * C + c], cw.w[j][(size_t)i * C + c + 1]);
             g.x = fmaf(w.x, v.x, g.x);
             g.y = fmaf(w.y, v.y, g.y);
@@ -45,63 +48,80 @@ __device__ __forceinline__ void dec_components(const Dims& d, int slot, int t, i
     }
 }
 
+// Both kernels: CTA (slice, block) takes the 256 channels of slice `slice` (one pair per
+// thread) for DT consecutive tokens, so the conv taps of its channels are read once per CTA and
+// reused from L1 for the following tokens.
+constexpr int DT = 16;
+constexpr int DTH = 128;
+
 // Gram matrix of the components of each token (lower triangle, the order of the prefill's
-// reduction), into reduction slice 0
-__global__ void __launch_bounds__(256) k_dec_gram(Dims d, int slot, const uint16_t* __restrict__ out,
+// reduction), partial over the CTA's channel slice: red[t][slice][q]
+__global__ void __launch_bounds__(DTH) k_dec_gram(Dims d, int slot, int B, const uint16_t* __restrict__ out,
                                                   ConvPtrs cw, const uint16_t* __restrict__ ring,
-                                                  const long long* __restrict__ pos,
+                                                  const long long* __restrict__ pos, int nslice,
                                                   float* __restrict__ red) {
-    __shared__ float sh[8][NGRAM];
-    const int t = blockIdx.x, K = d.K[slot];
-    const long long p = pos[t];
-    float v[NGRAM];
-#pragma unroll
-    for (int q = 0; q < NGRAM; ++q) v[q] = 0.f;
-    for (int c = 2 * threadIdx.x; c < d.C; c += 2 * blockDim.x) {
-        float2 u[4];
-        dec_components(d, slot, t, c, out, cw, ring, p, u);
-        int q = 0;
-#pragma unroll
-        for (int a = 0; a < 4; ++a)
-#pragma unroll
-            for (int b = 0; b <= a; ++b, ++q)
-                if (a < K) v[q] = fmaf(u[a].x, u[b].x, fmaf(u[a].y, u[b].y, v[q]));
-    }
+    __shared__ float sh[DTH / 32][NGRAM];
+    const int slice = blockIdx.x, K = d.K[slot];
+    const int c = slice * 2 * DTH + 2 * threadIdx.x;
+    const bool act = c < d.C;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int tt = 0; tt < DT; ++tt) {
+        const int t = blockIdx.y * DT + tt;
+        if (t >= B) break;
+        float v[NGRAM];
 #pragma unroll
-    for (int q = 0; q < NGRAM; ++q) {
-        float x = v[q];
+        for (int q = 0; q < NGRAM; ++q) v[q] = 0.f;
+        if (act) {
+            float2 u[4];
+            dec_components(d, slot, t, c, out, cw, ring, pos[t], u);
+            int q = 0;
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-        if (lane == 0) sh[warp][q] = x;
-    }
-    __syncthreads();
-    if (threadIdx.x < NGRAM) {
-        float s = 0.f;
-        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) s += sh[w][threadIdx.x];
-        red[(long long)t * NRED + threadIdx.x] = s;
+            for (int a = 0; a < 4; ++a)
+#pragma unroll
+                for (int b = 0; b <= a; ++b, ++q)
+                    if (a < K) v[q] = fmaf(u[a].x, u[b].x, u[a].y * u[b].y);
+        }
+#pragma unroll
+        for (int q = 0; q < NGRAM; ++q) {
+            float x = v[q];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+            if (lane == 0) sh[warp][q] = x;
+        }
+        __syncthreads();
+        if (threadIdx.x < NGRAM) {
+            float s2 = 0.f;
+#pragma unroll
+            for (int w = 0; w < DTH / 32; ++w) s2 += sh[w][threadIdx.x];
+            red[((long long)t * nslice + slice) * NRED + threadIdx.x] = s2;
+        }
+        __syncthreads();
     }
 }
 
 // X_act_new_j = (H_res x_act)_j (last slot) or x_act_j, + sum_a E[j][a] u_a; the last slot
 // scatters into the state rows I_j, the others write the next slot's active state.  Then the
 // token's out row goes into its ring row (each thread its own channels, after its last read of
-// them), and the last slot advances the token's position.
-__global__ void __launch_bounds__(256) k_dec_fwd(Dims d, int slot, const uint16_t* __restrict__ out,
+// them).
+__global__ void __launch_bounds__(DTH) k_dec_fwd(Dims d, int slot, int B, const uint16_t* __restrict__ out,
                                                  ConvPtrs cw, uint16_t* __restrict__ ring,
-                                                 long long* __restrict__ pos,
+                                                 const long long* __restrict__ pos,
                                                  const float* __restrict__ emat,
                                                  const uint16_t* __restrict__ xact,
                                                  const int* __restrict__ I,
                                                  const float* __restrict__ hres,
                                                  uint16_t* __restrict__ xact_next,
                                                  uint16_t* __restrict__ X) {
-    const int t = blockIdx.x, C = d.C, k = d.k, R = d.kapmax - 1;
+    const int C = d.C, k = d.k, R = d.kapmax - 1;
     const bool last = (slot == d.G - 1);
     const bool conv = d.K[slot] > 1;
-    const long long p = pos[t];
-    const float* E = emat + (long long)t * TOKMAT;
-    for (int c = 2 * threadIdx.x; c < C; c += 2 * blockDim.x) {
+    const int c = blockIdx.x * 2 * DTH + 2 * threadIdx.x;
+    if (c >= C) return;
+    for (int tt = 0; tt < DT; ++tt) {
+        const int t = blockIdx.y * DT + tt;
+        if (t >= B) break;
+        const long long p = pos[t];
+        const float* E = emat + (long long)t * TOKMAT;
         float2 u[4];
         dec_components(d, slot, t, c, out, cw, ring, p, u);
         float2 x[MAXK];
@@ -165,25 +185,26 @@ __global__ void k_ring_fill(const uint16_t* __restrict__ out, int B, int S, int 
     }
 }
 
-int dec_threads(int C) {
-    int th = ((C / 2 + 31) / 32) * 32;
-    return th > 256 ? 256 : (th < 32 ? 32 : th);
-}
+int dec_slices(int C) { return (C + 2 * DTH - 1) / (2 * DTH); }
 
 }  // namespace
 
 cudaError_t launch_dec_gram(const Dims& d, int slot, int B, const uint16_t* out, ConvPtrs cw,
                             const uint16_t* ring, const long long* pos, float* red, cudaStream_t st) {
-    k_dec_gram<<<B, dec_threads(d.C), 0, st>>>(d, slot, out, cw, ring, pos, red); note_launch();
+    const dim3 grid(dec_slices(d.C), (B + DT - 1) / DT);
+    k_dec_gram<<<grid, DTH, 0, st>>>(d, slot, B, out, cw, ring, pos, dec_slices(d.C), red); note_launch();
     return cudaGetLastError();
 }
+
+int dec_nslice(int C) { return dec_slices(C); }
 
 cudaError_t launch_dec_fwd(const Dims& d, int slot, int B, const uint16_t* out, ConvPtrs cw,
                            uint16_t* ring, long long* pos, const float* emat, const uint16_t* xact,
                            const int* I, const float* hres, uint16_t* xact_next, uint16_t* X,
                            cudaStream_t st) {
-    k_dec_fwd<<<B, dec_threads(d.C), 0, st>>>(d, slot, out, cw, ring, pos, emat, xact, I, hres,
-                                              xact_next, X); note_launch();
+    const dim3 grid(dec_slices(d.C), (B + DT - 1) / DT);
+    k_dec_fwd<<<grid, DTH, 0, st>>>(d, slot, B, out, cw, ring, pos, emat, xact, I, hres, xact_next,
+                                    X); note_launch();
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess || slot != d.G - 1) return e;
     k_pos_advance<<<(B + 255) / 256, 256, 0, st>>>(pos, B); note_launch();

@@ -273,6 +273,7 @@ cudaError_t launch_dec_fwd(const Dims& d, int slot, int B, const uint16_t* out, 
                            cudaStream_t st);
 cudaError_t launch_ring_fill(const Dims& d, int B, int S, const uint16_t* out, uint16_t* ring,
                              cudaStream_t st);
+int dec_nslice(int C);  // channel slices (partial Gram slots) of the decode Gram reduction
 cudaError_t launch_wb_gram(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
                            int nslice, float* red, cudaStream_t st);
 cudaError_t launch_wb_coef(const Dims& d, int slot, int T, const float* red, int nslice, const float* p,
@@ -292,6 +293,8 @@ cudaError_t launch_wgrad_reduce(const float* wpart, int splits, int E, int n, co
 cudaError_t launch_colsum(const float* in, int rows, int ld, int n, float* out, int accumulate,
                           float* scratch, cudaStream_t st);
 cudaError_t launch_sub_rows(float* G, int rows, int n, const float* v, cudaStream_t st);
+// sum of split-K partial slots into slot 0, in slot order ([nslots][n] -> [n])
+cudaError_t launch_slot_sum(float* x, int nslots, long long n, cudaStream_t st);
 cudaError_t launch_coef_full(const Dims& d, int T, const float* part, const float* pstats,
                              int splits, const float* wsum, const float* alpha_pre,
                              const float* b_pre, float* zfull, float* stats, float* hpre,
