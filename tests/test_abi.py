@@ -116,6 +116,16 @@ def test_entry_points_validate_on_host(L):
     Gd.W_post[0] = None
     assert L.xhc_post_bwd(h, 0, 64, ctypes.byref(P), Xp, addr[30], inp, addr[31], ctypes.byref(Gd),
                           sv, ws, None) == INVALID
+    # decode entry points: sizes, and validation before any launch
+    sz = ctypes.c_size_t()
+    assert L.xhc_ring_bytes(h, 4, ctypes.byref(sz)) == 0 and sz.value == 4 * 11 * 64 * 2
+    assert L.xhc_ring_bytes(h, 0, ctypes.byref(sz)) == INVALID
+    ring, pos = addr[33], addr[34]
+    assert L.xhc_post_fwd_decode(h, 0, 64, ctypes.byref(P), Xp, inp, None, pos, sv, ws, None) == INVALID
+    assert L.xhc_post_fwd_decode(h, 0, 64, ctypes.byref(P), Xp, inp, ring, None, sv, ws, None) == INVALID
+    assert L.xhc_post_fwd_decode(h, 0, 64, ctypes.byref(P), Xp, inp, ring + 4, pos, sv, ws, None) == ALIGN
+    assert L.xhc_ring_fill(h, 4, 0, inp, ring, None) == INVALID
+    assert L.xhc_ring_fill(h, 4, 16, inp + 2, ring, None) == ALIGN
     # sequence length must divide T
     g2 = X.Group(X.Config.full(8, 4, 2, 64, True, seq_len=48))
     assert L.xhc_pre_fwd(g2._h, 0, 64, ctypes.byref(P), Xp, inp, sv, ws, None) == INVALID
