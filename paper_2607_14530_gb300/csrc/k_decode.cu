@@ -6,7 +6,7 @@
 // rows of the sequence, which no longer exist as a contiguous [T][C] buffer: they are kept in a
 // per-sequence ring [B][R][C] bf16 (row (s mod R) holds out[s]).  The kernels below are the
 // decode forms of the Gram reduction and of the write-back (Eq. gs, Eq. sparse_write_delta,
-// Eq. sparse_write): CTAs over (256-channel slice, 16 tokens), one channel pair per thread, the
+// Eq. sparse_write): CTAs over (256-channel slice, 4 tokens), one channel pair per thread, the
 // conv read from the ring plus the token's own `out` row.  The write-back stores the token's
 // `out` into its ring row afterwards, and the group's last slot advances pos.
 #include <algorithm>
@@ -51,7 +51,7 @@ __device__ __forceinline__ void dec_components(const Dims& d, int slot, int t, i
 // Both kernels: CTA (slice, block) takes the 256 channels of slice `slice` (one pair per
 // thread) for DT consecutive tokens, so the conv taps of its channels are read once per CTA and
 // reused from L1 for the following tokens.
-constexpr int DT = 16;
+constexpr int DT = 4;
 constexpr int DTH = 128;
 
 // Gram matrix of the components of each token (lower triangle, the order of the prefill's
