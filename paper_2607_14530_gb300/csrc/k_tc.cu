@@ -638,10 +638,11 @@ struct DxArgs {
     int* err;
 };
 
-// ACT = false: full-state dX epilogue (streams i of N, tiles of one stream).
-// ACT = true : active-state epilogue, "streams" are the k active slots j:
+// ACT = true (the instantiated form): active-state epilogue, "streams" are the k active slots j:
 //              dX_act[t][j][c] += acc + H_pre[t][slot][I_j] d_input[t][c] - cx_t x_act[t][j][c]
 //              (X = x_act of the slot, scal = the per-token matrices with cx at 112).
+// ACT = false: a full-state epilogue over the N streams; not instantiated (the full-state dX is
+// k_dxf_tc, which also adds the dense-read gradient of the non-active rows).
 template <bool ACT>
 __global__ void __launch_bounds__(DX_THREADS, 1)
 k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, DxArgs a) {
@@ -895,13 +896,8 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
 }
 
 // ---------------------------------------------------------------------------------------------
-// Full-state dX with TMA-staged epilogue tiles.  Per tile (128 tokens x 128 channels of stream i):
-// the producer loads the MMA operands (one stage) and, into the epilogue stage of the tile's
-// warp group, the X and dX tiles of the stream (two 64-channel boxes each, 128-byte swizzle);
-// the epilogue warps read their row from TMEM (row per lane) and from the staged tiles, write
-// the bf16 result over the X tile, and one thread of the group stores the tile with TMA.  Rows
-// of active streams take their base from dX_act (fp32) with plain loads; the dX tile supplies
-// the base of the other rows.
+// TMA store, bulk-group and proxy-fence helpers of the full-state dX kernel below, and a named
+// barrier that also ORs a flag over the participating threads.
 
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, uint32_t src, int x, int y) {
     asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
