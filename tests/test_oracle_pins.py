@@ -206,6 +206,26 @@ def test_conv_delta_shift_causality_and_sequence_reset():
     assert torch.allclose(base[t], ref, atol=1e-14)
 
 
+@pytest.mark.parametrize("cfg", [O.flash(5, 3, 1, 8, 4, conv_k=(2, 3)), O.full(4, 2, 1, 6, True, conv_k=(3,))],
+                         ids=["flash4", "fullM"])
+def test_forward_of_a_sequence_prefix_is_the_prefix_of_the_forward(cfg):
+    # tokens interact only through the causal conv: the forward of the first L' tokens of a
+    # sequence equals the first L' rows of the forward of the whole sequence (what decoding one
+    # token at a time relies on); with sequence starts every L, sequences are independent too
+    L, Lp, nseq = 9, 5, 2
+    P = _params(cfg, 11)
+    Xw, outs_w = _inputs(cfg, nseq * L, 12)
+    cw = O.Config(**{**cfg.__dict__, "seq_len": L})
+    cp = O.Config(**{**cfg.__dict__, "seq_len": Lp})
+    Xo_w, ins_w, aux_w = O.forward(cw, P, Xw, outs_w)
+    rows = torch.cat([torch.arange(b * L, b * L + Lp) for b in range(nseq)])
+    Xo_p, ins_p, aux_p = O.forward(cp, P, Xw[rows], [o[rows] for o in outs_w])
+    assert torch.allclose(Xo_p, Xo_w[rows], rtol=0, atol=1e-12)
+    for t in range(cfg.G):
+        assert torch.allclose(ins_p[t], ins_w[t][rows], rtol=0, atol=1e-12)
+    assert torch.equal(aux_p["I"], aux_w["I"][rows])
+
+
 # ---------------------------------------------------------------------------------------------
 # routing, sparse write-back and the whole group against the brute-force oracle
 
