@@ -142,7 +142,9 @@ typedef struct xhc_handle xhc_handle;
 /* Validate *cfg and create a handle (host memory only).  XHC_ERR_INVALID_ARG for values the
  * paper's method cannot take (e.g. m > k), XHC_ERR_UNSUPPORTED for values beyond the limits
  * above, or for a variant whose structure does not match (MHC needs k = m = N, G = 1, no MLP
- * augmentation; FULL needs G = 1; FLASH needs G in {2, 4} with slots alternating A, M). */
+ * augmentation; FULL needs G = 1; FLASH needs G in {2, 4} with slots alternating A, M: the MLP
+ * slots' bits set in mlp_mask, the attention slots' bits optional -- set, they give the
+ * attention-side temporal augmentation of App. "Additional Ablation Studies"). */
 xhc_status xhc_create(const xhc_config* cfg, xhc_handle** out);
 void xhc_destroy(xhc_handle* h);
 

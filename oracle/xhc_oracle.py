@@ -27,7 +27,7 @@ Sources (section / equation labels of the paper):
   App. A       20 Sinkhorn iterations, row-sum clamp, alpha initialised to 0.01
   App. C       per-layer parameter counts (Eq. xhc_params, Eq. mhc_params)
 
-Readings where the paper is silent (each also listed in the design doc):
+Readings where the paper is silent (the same readings are used by the kernels):
   eps_norm = 1e-5 for every LayerNorm / RMSNorm (the backbone RMSNorm epsilon, App. A table);
   no affine weights in those norms; LayerNorm variance is the population variance nu - mu^2;
   FixedIdx = streams 0..m-1; routed streams are taken by score descending, ties to the lower
@@ -168,6 +168,25 @@ def to_oracle_params(flat: dict, cfg: Config, requires_grad: bool = False) -> di
 # building blocks
 
 
+def bf16_other_neighbor(v: torch.Tensor, r: torch.Tensor) -> torch.Tensor:
+    """The bf16 value next to r on the side of v, where r is v rounded to bf16 (r itself where
+    v == r exactly).  Together r and this value bracket v: they are the two roundings that an
+    evaluation of v with an error across the midpoint between them can produce."""
+    bits = r.to(torch.bfloat16).view(torch.int16).to(torch.int32) & 0xFFFF
+    neg = (bits >> 15) == 1
+    mag = bits & 0x7FFF
+    up = v > r                                    # the neighbour lies towards +infinity
+    away = torch.where(neg, ~up, up)              # ... i.e. away from zero in magnitude
+    mag2 = torch.where(away, mag + 1, mag - 1)
+    bits2 = torch.where(neg, mag2 | 0x8000, mag2)
+    zero = mag == 0                               # r = +-0: smallest subnormal of v's sign
+    bits2 = torch.where(zero, torch.where(v < 0, torch.full_like(bits, 0x8001),
+                                          torch.full_like(bits, 0x0001)), bits2)
+    bits2 = torch.where(v == r, bits, bits2)
+    out = (bits2 - ((bits2 >> 15) << 16)).to(torch.int16).view(torch.bfloat16)
+    return out.to(v.dtype)
+
+
 def rnd(x: torch.Tensor, on: bool) -> torch.Tensor:
     """Round to bf16 storage (round-to-nearest-even); identity in the backward."""
     if not on:
@@ -226,12 +245,17 @@ def augment(cfg: Config, out: torch.Tensor, conv_ws: list, T: int) -> list:
     return [out] + gs
 
 
-def router_scores(cfg: Config, x: torch.Tensor, W_r: torch.Tensor) -> torch.Tensor:
-    """s = sigmoid(LN(flatten X) W_r) (Eq. router).  x: [T, N*C]."""
+def router_logits(cfg: Config, x: torch.Tensor, W_r: torch.Tensor) -> torch.Tensor:
+    """LN(flatten X) W_r, the argument of the sigmoid in Eq. router.  x: [T, N*C]."""
     mu = x.mean(dim=1, keepdim=True)
     nu = (x * x).mean(dim=1, keepdim=True)
     x_ln = (x - mu) / torch.sqrt(nu - mu * mu + cfg.eps_norm)
-    return torch.sigmoid(x_ln @ W_r)
+    return x_ln @ W_r
+
+
+def router_scores(cfg: Config, x: torch.Tensor, W_r: torch.Tensor) -> torch.Tensor:
+    """s = sigmoid(LN(flatten X) W_r) (Eq. router).  x: [T, N*C]."""
+    return torch.sigmoid(router_logits(cfg, x, W_r))
 
 
 def route(cfg: Config, s: torch.Tensor | None, T: int):
@@ -273,6 +297,11 @@ def forward(cfg: Config, P: dict, X: torch.Tensor, outs: list, *, round_bf16: bo
     sublayer output of slot t (out^(t) = F_t(input^(t)) in the paper; here an input of the op).
     Returns (X_out, inputs, aux): the state after the group, the G sublayer inputs, and a dict
     of intermediates (s, H_pre, I, p, H_post, H_res, the active state before every slot).
+
+    For the tests, aux also holds, for every slot t >= 1 of a group, the active state entering
+    slot t before its bf16 rounding (``pre[t]``) and the sum of the magnitudes of the terms that
+    make it up (``mag[t]``: |X_act| plus p_j sum_r |H_post[j][r]| times the summed magnitudes of
+    out and of the raw conv components), which bounds the error of any evaluation of that sum.
     """
     T, N, C = X.shape
     k, G, eps = cfg.k, cfg.G, cfg.eps_norm
@@ -292,6 +321,7 @@ def forward(cfg: Config, P: dict, X: torch.Tensor, outs: list, *, round_bf16: bo
     X_act = X[rows, I]                              # Gather(X, I): [T, k, C]
     X_cur = X
     inputs, H_post_all, X_act_all = [], [], []
+    pre, mag = {}, {}
     H_res = None
     for t in range(G):
         X_act_all.append(X_act)
@@ -322,10 +352,20 @@ def forward(cfg: Config, P: dict, X: torch.Tensor, outs: list, *, round_bf16: bo
             mixed = torch.einsum("tji,tic->tjc", H_res, X_act)   # H_res X_act
         else:
             mixed = X_act                                         # Eq. flash_attn_update
-        X_act = rnd(mixed + delta, round_bf16)                    # Eq. sparse_write
+        new = mixed + delta                                       # Eq. sparse_write
+        if t < G - 1:
+            # magnitudes of the terms of the next slot's active state (test bookkeeping only)
+            raw = [outs[t]] + ([causal_dwconv(outs[t], P[f"conv_w.{t}.{j}"], cfg.S(T))
+                                for j in range(len(cfg.conv_k))] if K > 1 else [])
+            mu = sum(c.detach().abs() for c in raw)                   # [T, C]
+            hp = (p.detach().abs() * H_post.detach().abs().sum(dim=2))  # [T, k]
+            pre[t + 1] = new.detach()
+            mag[t + 1] = mixed.detach().abs() + hp[:, :, None] * mu[:, None, :]
+        X_act = rnd(new, round_bf16)
         X_cur = torch.index_put(X_cur, (rows, I), X_act)          # Scatter: inactive rows unchanged
 
-    aux = dict(s=s, I=I, p=p, H_pre=H_pre, H_post=H_post_all, H_res=H_res, X_act=X_act_all)
+    aux = dict(s=s, I=I, p=p, H_pre=H_pre, H_post=H_post_all, H_res=H_res, X_act=X_act_all,
+               pre=pre, mag=mag)
     return X_cur, inputs, aux
 
 

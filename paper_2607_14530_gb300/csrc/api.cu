@@ -208,10 +208,6 @@ Layout make_layout(const Dims& d, int64_t T) {
 
 using namespace xhc;
 
-struct xhc_handle {
-    Handle h;
-};
-
 static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
 extern "C" {
@@ -299,8 +295,11 @@ xhc_status xhc_create(const xhc_config* cfg, xhc_handle** out) {
             break;
         case XHC_FLASH: {
             if (c.group != 2 && c.group != 4) return XHC_ERR_INVALID_ARG;
-            const int want = (c.group == 2) ? 0x2 : 0xA;  // slots A, M (, A, M)
-            if (c.mlp_mask != want) return XHC_ERR_INVALID_ARG;
+            // slots A, M (, A, M): the MLP slots carry the temporal augmentation; the attention
+            // slots may carry it too (the attention-side ablation of App. "Additional Ablation
+            // Studies")
+            const int want = (c.group == 2) ? 0x2 : 0xA;
+            if ((c.mlp_mask & want) != want) return XHC_ERR_INVALID_ARG;
             break;
         }
     }

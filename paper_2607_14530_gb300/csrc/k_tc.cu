@@ -133,6 +133,23 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
     for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// registers -> TMEM (32 lanes x 16 columns); the caller waits with tmem_st_wait before the
+// values are read again
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const float* v) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
+        ::"r"(taddr), "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+          "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+          "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+          "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+          "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+          "r"(__float_as_uint(v[15]))
+        : "memory");
+}
+__device__ __forceinline__ void tmem_st_wait() {
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
 // TMEM -> registers, 32 lanes x 8 columns (wait in the same statement, as above)
 __device__ __forceinline__ void tmem_ld8(uint32_t taddr, float* v) {
     uint32_t r[8];
@@ -144,6 +161,20 @@ __device__ __forceinline__ void tmem_ld8(uint32_t taddr, float* v) {
         : "r"(taddr));
 #pragma unroll
     for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// The tensor cores' fp32 accumulation loses accuracy in proportion to the length of the chain of
+// MMAs accumulated in one TMEM accumulator (measured: about 7e-8 of the result per 64-element
+// k-block, systematic rather than random, so ~6e-5 over the ~860 k-blocks a CTA covers at
+// K = 65536).  The accumulator is therefore restarted every SUB_K k-elements (a sub-segment);
+// the epilogue adds the sub-segments' results in fp32 (round to nearest) into a running sum kept
+// in TMEM columns [NB, NB + nfull), and writes the piece's partial once, as before.
+constexpr int SUB_K = 1024;
+
+// TMEM columns of one CTA: the accumulator (NB) and the running sum (nfull), a power of two
+__host__ __device__ inline uint32_t proj_tc_cols(int NB, int nfull) {
+    const int need = NB + nfull;
+    return need <= 32 ? 32u : need <= 64 ? 64u : need <= 128 ? 128u : need <= 256 ? 256u : 512u;
 }
 
 struct ProjTcArgs {
@@ -188,7 +219,9 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int c = blockIdx.x;
     const long long g0 = range_start(a.W, a.P, c), g1 = range_start(a.W, a.P, c + 1);
-    const uint32_t ncols = (a.NB <= 256) ? 256u : 512u;
+    const uint32_t ncols = proj_tc_cols(a.NB, a.nfull);
+    // k-block groups (g units) per sub-segment
+    const int SUBG = max(1, SUB_K / (BK * KPS));
 
     if (threadIdx.x == 0) {
         s_abort = 0;
@@ -254,7 +287,8 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
             long long g = g0;
             while (g < g1) {
                 const int m = (int)(g / a.KB);
-                const long long gend = min(g1, (long long)(m + 1) * a.KB);
+                const long long sub_end = (long long)m * a.KB + ((g - (long long)m * a.KB) / SUBG + 1) * SUBG;
+                const long long gend = min(min(g1, (long long)(m + 1) * a.KB), sub_end);
                 if (seg > 0 && !mbar_wait(smem_u32(&bars[2 * STAGES + 1]), (uint32_t)((seg - 1) & 1))) {
                     atomicExch(a.err, 2);
                     s_abort = 1;
@@ -304,14 +338,20 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
         int seg = 0;
         long long g = g0;
         bool ok = true;
+        // row sums in packed pairs, four independent accumulators each (short dependency chains,
+        // half the instructions of scalar sums), over the whole piece (tile x this CTA's range)
+        float2 a1[4], a2[4];
         while (g < g1 && ok) {
             const int m = (int)(g / a.KB);
-            const long long gend = min(g1, (long long)(m + 1) * a.KB);
-            // row sums in packed pairs, four independent accumulators each (short dependency
-            // chains, half the instructions of scalar sums)
-            float2 a1[4], a2[4];
+            const long long piece_end = min(g1, (long long)(m + 1) * a.KB);
+            const long long sub_end = (long long)m * a.KB + ((g - (long long)m * a.KB) / SUBG + 1) * SUBG;
+            const long long gend = min(piece_end, sub_end);
+            const bool first_sub = (g == max(g0, (long long)m * a.KB));
+            const bool last_sub = (gend == piece_end);
+            if (first_sub) {
 #pragma unroll
-            for (int e = 0; e < 4; ++e) a1[e] = a2[e] = make_float2(0.f, 0.f);
+                for (int e = 0; e < 4; ++e) a1[e] = a2[e] = make_float2(0.f, 0.f);
+            }
             for (; g < gend; ++g, ++it) {
                 const int s = (int)(it % STAGES);
                 const uint32_t ph = (uint32_t)((it / STAGES) & 1);
@@ -359,17 +399,31 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
             const int t = m * BM + r;
             float* dst = a.part + ((long long)j * a.T + t) * a.nfull;
             const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
-            // hi columns [0, nfull), lo columns [nfull, 2 nfull)
+            // hi columns [0, nfull), lo columns [nfull, 2 nfull); running sum of the piece's
+            // sub-segments at [NB, NB + nfull)
             for (int o0 = 0; o0 < a.nfull; o0 += 16) {
-                float hi[16], lo[16];
+                float hi[16], lo[16], sum[16];
                 tmem_ld16(tl + (uint32_t)o0, hi);
                 tmem_ld16(tl + (uint32_t)(a.nfull + o0), lo);
-                if (t < a.T) {
+                if (first_sub) {
+#pragma unroll
+                    for (int q = 0; q < 16; ++q) sum[q] = hi[q] + lo[q];
+                } else {
+                    tmem_ld16(tl + (uint32_t)(a.NB + o0), sum);
+#pragma unroll
+                    for (int q = 0; q < 16; ++q) sum[q] += hi[q] + lo[q];
+                }
+                if (!last_sub) {
+                    tmem_st16(tl + (uint32_t)(a.NB + o0), sum);
+                } else if (t < a.T) {
                     const int n = min(16, a.nfull - o0);
-                    for (int q = 0; q < n; ++q) dst[o0 + q] = hi[q] + lo[q];
+#pragma unroll
+                    for (int q = 0; q < 16; ++q)
+                        if (q < n) dst[o0 + q] = sum[q];
                 }
             }
-            if (!A_MN && a.pstats && t < a.T) {
+            if (!last_sub) tmem_st_wait();
+            if (last_sub && !A_MN && a.pstats && t < a.T) {
                 const float s1 = (a1[0].x + a1[0].y) + (a1[1].x + a1[1].y) + (a1[2].x + a1[2].y) + (a1[3].x + a1[3].y);
                 const float s2 = (a2[0].x + a2[0].y) + (a2[1].x + a2[1].y) + (a2[2].x + a2[2].y) + (a2[3].x + a2[3].y);
                 a.pstats[((long long)j * a.T + t) * 2 + 0] = s1;
@@ -479,7 +533,9 @@ ProjTcPlan plan_proj_tc(int T, int K, int nfull, int nsm, bool proj) {
     p.MT = (T + BM - 1) / BM;
     p.W = (long long)p.KB * p.MT;
     p.nchunk = p.NB > 256 ? 2 : 1;
-    p.ctas = (p.NB <= 256 && proj_tc_stages_for(p.NB, p.kps, 2) >= 2) ? 2 : 1;
+    // two CTAs per SM need both rings in shared memory and both TMEM allocations (accumulator and
+    // running sum) within half of the SM's 512 columns
+    p.ctas = (proj_tc_cols(p.NB, nfull) <= 256 && proj_tc_stages_for(p.NB, p.kps, 2) >= 2) ? 2 : 1;
     const int sms = p.ctas * (nsm > 0 ? nsm : 148);
     long long P = std::min<long long>(sms, std::max<long long>(1, p.W / 4));
     p.P = (int)P;

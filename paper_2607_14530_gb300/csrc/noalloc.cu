@@ -29,11 +29,6 @@ size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 using namespace xhc;
 
-// same definition as in api.cu
-struct xhc_handle {
-    Handle h;
-};
-
 extern "C" xhc_status xhc_route_noalloc(const xhc_handle* hh, int64_t T, const xhc_params* P,
                                         const uint16_t* X, int32_t* I, float* p, float* hpre,
                                         void* stream) {

@@ -129,6 +129,15 @@ struct Handle {
     Dims d;
 };
 
+}  // namespace xhc
+
+// The opaque handle of the C ABI (include/xhc.h), defined once for every translation unit.
+struct xhc_handle {
+    xhc::Handle h;
+};
+
+namespace xhc {
+
 Layout make_layout(const Dims& d, int64_t T);
 Dims make_dims(const xhc_config& c);
 

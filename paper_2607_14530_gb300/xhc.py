@@ -149,8 +149,10 @@ class Config:
         return Config(FULL, N, k, m, C, 1, 1 if mlp else 0, **kw)
 
     @staticmethod
-    def flash(N, k, m, C, G, **kw):
-        return Config(FLASH, N, k, m, C, G, 0x2 if G == 2 else 0xA, **kw)
+    def flash(N, k, m, C, G, attn_tfa=False, **kw):
+        """xHC-Flash group, slots A, M (, A, M); attn_tfa also augments the attention slots."""
+        mask = (0x2 if G == 2 else 0xA) | ((0x1 if G == 2 else 0x5) if attn_tfa else 0)
+        return Config(FLASH, N, k, m, C, G, mask, **kw)
 
     @property
     def has_router(self):

@@ -130,3 +130,17 @@ def test_entry_points_validate_on_host(L):
     g2 = X.Group(X.Config.full(8, 4, 2, 64, True, seq_len=48))
     assert L.xhc_pre_fwd(g2._h, 0, 64, ctypes.byref(P), Xp, inp, sv, ws, None) == INVALID
     assert L.xhc_status_string(3) == b"pointer not 16-byte aligned"
+
+
+def test_route_noalloc_rejects_oversized_T(L):
+    """xhc_route_noalloc checks T against its fixed scratch array on the host, before any device
+    work (the pointers below are never dereferenced)."""
+    g = X.Group(X.Config.flash(32, 4, 2, 4096, 4))
+    T = 1 << 20
+    P = X._Params()
+    for i in range(4):
+        P.W_pre[i] = 0x7f0000000000 + 4096 * i
+    P.W_r, P.alpha_pre, P.b_pre = 0x7f0000100000, 0x7f0000200000, 0x7f0000300000
+    addr = 0x7f0001000000
+    st = L.xhc_route_noalloc(g._h, T, ctypes.byref(P), addr, addr, addr, addr, None)
+    assert st == UNSUPPORTED

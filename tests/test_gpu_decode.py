@@ -9,11 +9,10 @@ padding before the sequence start."""
 import pytest
 import torch
 
-from oracle import xhc_oracle as O
 from paper_2607_14530_gb300 import synth
 from paper_2607_14530_gb300.xhc import Config, Group
 
-from xhc_cases import F64, TIE_MARGIN, assert_bf16_close, assert_f32_close, oracle_cfg, run_oracle
+from xhc_cases import assert_bf16_close, assert_f32_close, flash_bases, run_oracle, tie_free
 
 pytestmark = pytest.mark.gpu
 
@@ -34,19 +33,18 @@ def _cfg(N, k, m, C, G, S, **kw):
 def test_decode_matches_the_whole_sequence_forward(N, k, m, C, G, B, S):
     L = S + ND
     cfg_o = _cfg(N, k, m, C, G, L)
-    ocfg = oracle_cfg(cfg_o)
     # seeded whole sequences without a routing near-tie (the oracle decides)
     for attempt in range(50):
         seed = 7 + 1000 * attempt
         inp = synth.group_inputs(B * L, N, C, G, seed)
         P = synth.params(cfg_o.param_shapes(), seed)
-        sc = O.router_scores(ocfg, inp["X"].to(F64).reshape(B * L, -1), P["W_r"].to(F64))
-        if bool((O.routing_margin(ocfg, sc) > TIE_MARGIN).all()):
+        if bool(tie_free(cfg_o, inp["X"], P["W_r"]).all()):
             break
     else:
         raise RuntimeError("no tie-free draw")
     ref = run_oracle(cfg_o, inp, P)
     aux = ref["aux"]
+    bases = flash_bases(cfg_o, inp["X"], aux)
 
     pre_rows = torch.cat([torch.arange(b * L, b * L + S) for b in range(B)])
 
@@ -89,7 +87,8 @@ def test_decode_matches_the_whole_sequence_forward(N, k, m, C, G, B, S):
         if not torch.equal(co["I"].cpu().long(), aux["I"][r]):
             errors.append(f"{tag}: routing differs")
         for t in range(G):
-            chk(assert_bf16_close, ins[t], ref["inputs"][t][r], f"{tag} input[{t}]")
+            chk(assert_bf16_close, ins[t], ref["inputs"][t][r], f"{tag} input[{t}]",
+                None if bases[t] is None else bases[t][r])
             chk(assert_f32_close, co["hpost"][t].cpu(), aux["H_post"][t][r], f"{tag} H_post[{t}]")
         chk(assert_f32_close, co["hres"].cpu(), aux["H_res"][r], f"{tag} H_res")
         chk(assert_bf16_close, X, ref["X"][r], f"{tag} X_out")

@@ -297,6 +297,32 @@ def test_routed_scores_sorted_and_maximal():
         assert torch.equal(p[t, :2], torch.ones(2, dtype=F64))
 
 
+def test_routing_margin_hand_computed_gaps():
+    """routing_margin decides which seeds the parity suite uses (a selection is unique only
+    when the routed scores that TopK separates differ): the smallest gap between consecutive
+    non-fixed scores among the k - m + 1 largest, computed here by hand."""
+    cfg = O.full(5, 3, 1, 8, False)  # m = 1 fixed, k - m = 2 routed out of streams 1..4
+    s = torch.tensor([[0.99, 0.10, 0.50, 0.45, 0.20],   # sorted routed: .50 .45 .20 .10 -> gaps .05, .25
+                      [0.01, 0.70, 0.30, 0.60, 0.65],   # .70 .65 .60 -> gaps .05, .05
+                      [0.50, 0.40, 0.40, 0.90, 0.10],   # .90 .40 .40 -> gaps .50, 0 (a tie)
+                      [0.50, 0.80, 0.20, 0.30, 0.10]],  # .80 .30 .20 -> gaps .50, .10
+                     dtype=F64)
+    got = O.routing_margin(cfg, s)
+    want = torch.tensor([0.05, 0.05, 0.0, 0.10], dtype=F64)
+    assert torch.allclose(got, want, atol=1e-15, rtol=0), got
+    # the fixed stream's score never enters (stream 0 is fixed whatever its score)
+    s2 = s.clone()
+    s2[:, 0] = 0.475
+    assert torch.equal(O.routing_margin(cfg, s2), got)
+    # k - m + 1 larger than the routed candidates: every candidate counts (N = 3, m = 1, k = 3)
+    cfg3 = O.full(3, 3, 1, 8, False)
+    assert torch.allclose(O.routing_margin(cfg3, torch.tensor([[0.3, 0.8, 0.5]], dtype=F64)),
+                          torch.tensor([0.3], dtype=F64), atol=1e-15, rtol=0)
+    # nothing to choose: no router (k = m), or a single routed candidate
+    assert math.isinf(float(O.routing_margin(O.full(4, 2, 2, 8, False), s[:, :4])[0]))
+    assert math.isinf(float(O.routing_margin(O.full(2, 2, 1, 8, False), s[:, :2])[0]))
+
+
 # ---------------------------------------------------------------------------------------------
 # xHC-Flash dense-read reuse is exact (App. E.1, E.2, E.3)
 
@@ -422,3 +448,49 @@ def test_traffic_model_reproduces_table():
         assert r + w == row["total"], (row, r, w)
         if "read" in row:
             assert (r, w) == (row["read"], row["write"])
+
+
+# ---------------------------------------------------------------------------------------------
+# bf16 rounding bookkeeping used by the parity tests
+
+
+def test_bf16_other_neighbor_hand_values():
+    """Spacing of bf16 is 2^-7 on [1, 2) and 2^-8 on [1/2, 1); the smallest subnormal is 2^-133."""
+    v = torch.tensor([1 + 0.3 * 2 ** -7, 1 - 0.3 * 2 ** -8, -(1 + 0.3 * 2 ** -7), -(1 - 0.3 * 2 ** -8),
+                      3e-41, -3e-41, 1.5, 0.0], dtype=F64)
+    r = v.to(torch.bfloat16).to(F64)
+    want = torch.tensor([1 + 2 ** -7, 1 - 2 ** -8, -(1 + 2 ** -7), -(1 - 2 ** -8),
+                         2.0 ** -133, -(2.0 ** -133), 1.5, 0.0], dtype=F64)
+    assert torch.equal(r[:4].abs(), torch.ones(4, dtype=F64))
+    assert torch.equal(O.bf16_other_neighbor(v, r), want)
+
+
+def test_bf16_other_neighbor_brackets_random_values():
+    g = torch.Generator().manual_seed(7)
+    v = torch.randn(20000, generator=g, dtype=F64) * torch.exp2(torch.randint(-20, 20, (20000,), generator=g)).to(F64)
+    r = v.to(torch.bfloat16).to(F64)
+    o = O.bf16_other_neighbor(v, r)
+    assert torch.equal(o.to(torch.bfloat16).to(F64), o)           # representable
+    lo, hi = torch.minimum(r, o), torch.maximum(r, o)
+    exact = v == r
+    assert bool(((lo <= v) & (v <= hi))[~exact].all())              # brackets v
+    # adjacent: the midpoint rounds to one of the two (no bf16 value strictly between)
+    mid = (0.5 * (r + o)).to(torch.bfloat16).to(F64)
+    assert bool(((mid == r) | (mid == o))[~exact].all())
+    assert bool(((v - r).abs() <= (v - o).abs())[~exact].all())     # r is the nearer one
+
+
+def test_prerounding_bookkeeping():
+    """pre[t] rounds to the active state entering slot t (Eq. sparse_write, Eq. flash_attn_update)
+    and mag[t] bounds |pre[t]| (triangle inequality over the terms it sums)."""
+    cfg = O.flash(6, 3, 1, 16, 4, conv_k=(2, 3))
+    T = 10
+    P = _params(cfg, 21, alpha=0.1, w_std=0.2)
+    X, outs = _inputs(cfg, T, 21)
+    X = X.to(torch.bfloat16).to(F64)
+    outs = [o.to(torch.bfloat16).to(F64) for o in outs]
+    _, _, aux = O.forward(cfg, P, X, outs)
+    assert sorted(aux["pre"]) == [1, 2, 3]
+    for t in range(1, 4):
+        assert torch.equal(O.rnd(aux["pre"][t], True), aux["X_act"][t])
+        assert bool((aux["mag"][t] >= aux["pre"][t].abs() * (1 - 1e-12)).all())
