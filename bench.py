@@ -144,20 +144,14 @@ def kernel_model(cfg, T):
 def paper_forward_bytes_per_token(cfg):
     """Forward traffic of Table overhead_analysis for this group, bytes per token."""
     from paper_2607_14530_gb300 import traffic
-    N, k = cfg.N, cfg.k
-    if cfg.variant == 0:
-        r, w = traffic.paper_model("mhc", N)
-        per_group_C = (r + w)
-    elif cfg.G == 4:
-        r, w = traffic.paper_model("flash4", N, k)
-        per_group_C = 4 * (r + w)
-    elif cfg.G == 2:
-        r, w = traffic.paper_model("flash2", N, k)
-        per_group_C = 2 * (r + w)
-    else:
-        r, w = traffic.paper_model("xhc", N, k)
-        per_group_C = r + w
-    return per_group_C * cfg.C * 2
+    return traffic.forward_model("mhc" if cfg.variant == 0 else "xhc", cfg.N, cfg.k, cfg.G) * cfg.C * 2
+
+
+def model_bytes_per_token(cfg):
+    """(forward, backward) algorithmic bytes per token of one group: the paper's forward
+    accounting and the backward model of traffic.backward_model (bf16 = 2 bytes)."""
+    from paper_2607_14530_gb300 import traffic
+    return paper_forward_bytes_per_token(cfg), traffic.backward_model(cfg.N, cfg.k, cfg.G) * cfg.C * 2
 
 
 # ---------------------------------------------------------------------------------------------
@@ -251,6 +245,20 @@ def ncu_traffic(kernel, workload):
     if not e or e.get("csrc_sha") != csrc_hash():
         return None
     return e.get("dram_bytes_per_launch")
+
+
+def ncu_forward_bytes(workload):
+    """Measured forward DRAM bytes per token (ncu, the forward kernels of one group) from the
+    committed summary, if it was taken on the current kernel sources; else None."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    e = d.get(workload, {}).get("_forward")
+    if not e or e.get("csrc_sha") != csrc_hash():
+        return None
+    return e.get("dram_bytes_per_token")
 
 
 def job_rate(ms_local, tokens_per_rank, steps, world, device=None):
@@ -432,9 +440,39 @@ def run_xhc(args, wl_name):
                                       "achieved / frac above count this kernel's bytes only"}
 
     step_bytes = sum(v["bytes"] for v in model.values())
-    hbm = {"model_bytes_per_step": step_bytes, "achieved_gbs": step_bytes / (ms_step / 1000.0) / 1e9,
-           "frac_of_measured_peak": step_bytes / (ms_step / 1000.0) / 1e9 / hbm_peak,
-           "paper_fwd_bytes_per_token": paper_forward_bytes_per_token(cfg)}
+    fb, bb = model_bytes_per_token(cfg)
+    alg = (fb + bb) * T
+    hbm = {"kernel_model_bytes_per_step": step_bytes,
+           "kernel_model_gbs": step_bytes / (ms_step / 1000.0) / 1e9,
+           "kernel_model_frac": step_bytes / (ms_step / 1000.0) / 1e9 / hbm_peak,
+           "algorithmic_bytes_per_step": alg,
+           "algorithmic_gbs": alg / (ms_step / 1000.0) / 1e9,
+           "algorithmic_frac": alg / (ms_step / 1000.0) / 1e9 / hbm_peak,
+           "algorithmic_model": "paper forward accounting (Table overhead_analysis) + traffic.backward_model, "
+                                "bf16, per group per token: fwd %.0f B + bwd %.0f B" % (fb, bb),
+           "paper_fwd_bytes_per_token": fb}
+
+    # forward only (prefill-style: pre_fwd / post_fwd of every slot), same inputs, CUDA events
+    def fwd_step():
+        g.forward(P, X, outs, saved, ws, inputs=inputs)
+
+    for _ in range(2):
+        fwd_step()
+    torch.cuda.synchronize()
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    f0.record(stream)
+    for _ in range(args.steps):
+        fwd_step()
+    f1.record(stream)
+    torch.cuda.synchronize()
+    fms, fvalue = job_rate(f0.elapsed_time(f1), T, args.steps, world, dev)
+    fwd = {"tokens_per_s": fvalue, "ms_per_step": fms / args.steps,
+           "algorithmic_frac": fb * T / (fms / args.steps / 1000.0) / 1e9 / hbm_peak}
+    dram = ncu_forward_bytes(wl_name)
+    if dram is not None:
+        fwd["dram_bytes_per_token"] = dram
+        fwd["dram_vs_paper_model"] = dram / fb
+        fwd["gate"] = "<= 1.2 x the paper's forward model"
 
     line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
@@ -443,7 +481,7 @@ def run_xhc(args, wl_name):
             "config": {"workload": desc, "tokens": T, "storage": "bf16 state, fp32 params/coefficients",
                        "l2": "inputs larger than L2 (state alone is %.1f GiB), no flush" % (T * cfg.N * cfg.C * 2 / 2**30),
                        "parallelism": "replicas" if world > 1 else "1 GPU"},
-            "roofline": roof, "hbm": hbm, "gpu_launches": launches, "clocks": ck}
+            "roofline": roof, "hbm": hbm, "fwd": fwd, "gpu_launches": launches, "clocks": ck}
 
     if args.kernels_out and rank == 0:
         with open(args.kernels_out, "w") as f:

@@ -1329,8 +1329,18 @@ cudaError_t launch_dxa_tc(const Dims& d, int slot, int T, const float* dzs, int 
     return cudaGetLastError();
 }
 
+// shared memory of k_dxf_tc: the token tile's dZ rows and two stages of W rows (nkb k-blocks
+// each), the G d_input tiles and two X | dX tile pairs, barriers, alignment slack
+static size_t dxf_smem(int nfull, int G) {
+    const int nkb = (nfull + BK - 1) / BK;
+    return (size_t)nkb * (BM + 2 * DG_BN) * BK * 2 + (size_t)(G + 4) * DG_TILE + 256 + 1024;
+}
+
+// up to three k-blocks (nfull <= 192: N = 32 with a router and four pre-maps) fit the 227 KB a
+// block may use
 bool dx_tc_ok(int T, int N, int C, int nfull, int G) {
-    return T >= BM && C % DG_BN == 0 && nfull <= 2 * BK && N >= 2 && G >= 1 && G <= 4;
+    return T >= BM && C % DG_BN == 0 && nfull <= 3 * BK && N >= 2 && G >= 1 && G <= 4 &&
+           dxf_smem(nfull, G) <= 232448;
 }
 
 cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, uint16_t* dz16,
@@ -1367,7 +1377,7 @@ cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, 
     a.P = (int)std::min<long long>(num_sms(), a.ntiles);
     a.X = X; a.dX = dX; a.dinput = dinput; a.hpre = hpre; a.I = I; a.dxact = dxact;
     a.scal = scal; a.scal_ld = scal_ld; a.err = err;
-    const size_t sm = (size_t)a.nkb * (BM + 2 * DG_BN) * BK * 2 + (size_t)(d.G + 4) * DG_TILE + 256 + 1024;
+    const size_t sm = dxf_smem(n, d.G);
     e = cudaFuncSetAttribute((const void*)k_dxf_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
     k_dxf_tc<<<a.P, DX_THREADS, sm, st>>>(ma, mb, mx, md, mg, a); note_launch();

@@ -42,3 +42,32 @@ def paper_model(method: str, N: int, k: int = 4, K_r: int = 4, n_conv: int = 3):
         W = 4 + k + k + 4 * k + 4 * k + 2 * n_conv + 3
         return R / 4.0, W / 4.0
     raise ValueError(method)
+
+
+def backward_model(N: int, k: int, G: int) -> float:
+    """Elements (units of C) a group's backward must move at least, per token; the paper gives no
+    backward count, so this is the build's own model, counted the way the paper counts the
+    forward (bf16 state, every stored tensor read or written once, coefficients excluded):
+      3N       the entry state X read once, dX read (gradient of the group output) and written
+      (G-1)k   the active state entering each slot t >= 1, read back from the forward
+      2(G-1)k  the gradient of that state handed from slot t to slot t-1 (bf16 write + read)
+      3G       per slot: d_input read, the sublayer output read (write-back components), d_out
+               written
+    An fp32 active gradient, partial sums or any other intermediate an implementation chooses
+    counts as overhead against this model, not as algorithmic traffic."""
+    return float(3 * N + (G - 1) * k + 2 * (G - 1) * k + 3 * G)
+
+
+def forward_model(variant: str, N: int, k: int, G: int) -> float:
+    """The paper's forward accounting for one group, units of C per token (Table
+    overhead_analysis; per-sublayer averages times the group's sublayers)."""
+    if variant == "mhc":
+        r, w = paper_model("mhc", N)
+        return r + w
+    if G == 4:
+        r, w = paper_model("flash4", N, k)
+    elif G == 2:
+        r, w = paper_model("flash2", N, k)
+    else:
+        r, w = paper_model("xhc", N, k)
+    return G * (r + w)
