@@ -282,7 +282,8 @@ def oracle_step(cfg, X, outs, dX, dins, P):
                     mlp=tuple(bool((cfg.mlp_mask >> t) & 1) for t in range(cfg.G)),
                     conv_k=tuple(cfg.conv_k), gram_schmidt=cfg.gram_schmidt,
                     sinkhorn_iters=cfg.sinkhorn_iters, eps_norm=cfg.eps_norm,
-                    eps_gs=(cfg.eps_gs if cfg.eps_gs > 0 else None), seq_len=cfg.seq_len)
+                    eps_gs=(cfg.eps_gs if cfg.eps_gs > 0 else None), seq_len=cfg.seq_len,
+                    router=cfg.router, dense_read=not cfg.sparse_read)
     f64 = torch.float64
     P64 = {n: v.to(f64) for n, v in P.items()}
     O.backward(ocfg, P64, X.to(f64), [o.to(f64) for o in outs], dX.to(f64), [d.to(f64) for d in dins])

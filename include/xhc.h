@@ -93,6 +93,10 @@ typedef struct {
     float eps_norm;            /* LayerNorm / RMSNorm epsilon (1e-5)                          */
     float eps_gs;              /* Gram-Schmidt denominator epsilon; <= 0 means 1e-6 * C        */
     int seq_len;               /* S: the conv never crosses a sequence start; 0 means T       */
+    int router;                /* 0: sigmoid scores (Eq. router); 1: softmax over the N       */
+                               /*    logits (the softmax-router ablation, Table ablation (11)) */
+    int sparse_read;           /* 0: dense read of all N streams (Eq. dense_read); 1: read     */
+                               /*    only the k active streams (Table ablation (6), (7))      */
 } xhc_config;
 
 /* Device pointers to the fp32 parameters of one group (Sec. 3.3.4, Sec. 5.2).

@@ -50,12 +50,17 @@ def forward(cfg, P, X, outs, round_bf16=True):
         # router
         if m < k:
             sd = math.sqrt(nu - mu * mu + eps)
-            s = []
+            zs = []
             for o in range(N):
                 z = 0.0
                 for e in range(n):
                     z += (x[e] - mu) / sd * P["W_r"][e][o]
-                s.append(_sig(z))
+                zs.append(z)
+            if getattr(cfg, "router", "sigmoid") == "softmax":
+                den = sum(math.exp(z) for z in zs)
+                s = [math.exp(z) / den for z in zs]
+            else:
+                s = [_sig(z) for z in zs]
             best, best_sum = None, None
             for sub in itertools.combinations(range(m, N), k - m):
                 tot = sum(s[i] for i in sub)
@@ -80,11 +85,14 @@ def forward(cfg, P, X, outs, round_bf16=True):
             Hpre.append(h)
         state = [[X[t][i][c] for c in range(C)] for i in range(N)]
         for q in range(G):
-            # dense read over every stream of the current state
+            # dense read over every stream of the current state (only the active ones in the
+            # sparse-read ablation)
+            dense = getattr(cfg, "dense_read", True)
             for c in range(C):
                 acc = 0.0
                 for i in range(N):
-                    acc += Hpre[q][i] * state[i][c]
+                    if dense or i in I:
+                        acc += Hpre[q][i] * state[i][c]
                 inputs[q][t][c] = _round(acc, round_bf16)
             act = [state[I[j]] for j in range(k)]
             xa = [act[j][c] for j in range(k) for c in range(C)]

@@ -75,6 +75,8 @@ class Config:
     eps_norm: float = 1e-5
     eps_gs: float | None = None
     seq_len: int = 0
+    router: str = "sigmoid"     # "softmax": the softmax-router ablation (Table ablation, row 11)
+    dense_read: bool = True     # False: read only the active streams (Table ablation, rows 6-7)
 
     @property
     def has_router(self) -> bool:
@@ -254,8 +256,13 @@ def router_logits(cfg: Config, x: torch.Tensor, W_r: torch.Tensor) -> torch.Tens
 
 
 def router_scores(cfg: Config, x: torch.Tensor, W_r: torch.Tensor) -> torch.Tensor:
-    """s = sigmoid(LN(flatten X) W_r) (Eq. router).  x: [T, N*C]."""
-    return torch.sigmoid(router_logits(cfg, x, W_r))
+    """s = sigmoid(LN(flatten X) W_r) (Eq. router).  x: [T, N*C].  With the softmax-router
+    ablation (Sec. 4, Table ablation row 11) the sigmoid is replaced by a softmax over the N
+    logits of the token (the fixed streams' logits included, as the projection produces all N)."""
+    z = router_logits(cfg, x, W_r)
+    if cfg.router == "softmax":
+        return torch.softmax(z, dim=1)
+    return torch.sigmoid(z)
 
 
 def route(cfg: Config, s: torch.Tensor | None, T: int):
@@ -319,6 +326,11 @@ def forward(cfg: Config, P: dict, X: torch.Tensor, outs: list, *, round_bf16: bo
 
     rows = torch.arange(T)[:, None].expand(T, k)
     X_act = X[rows, I]                              # Gather(X, I): [T, k, C]
+    # read mask: every stream (Eq. dense_read), or only the active ones (sparse-read ablation)
+    read = torch.ones(T, N, dtype=X.dtype)
+    if not cfg.dense_read:
+        read = torch.zeros(T, N, dtype=X.dtype)
+        read[rows, I] = 1.0
     X_cur = X
     inputs, H_post_all, X_act_all = [], [], []
     pre, mag = {}, {}
@@ -326,7 +338,7 @@ def forward(cfg: Config, P: dict, X: torch.Tensor, outs: list, *, round_bf16: bo
     for t in range(G):
         X_act_all.append(X_act)
         # Dense read of the current full state (Eq. dense_read).
-        inputs.append(rnd(torch.einsum("ti,tic->tc", H_pre[t], X_cur), round_bf16))
+        inputs.append(rnd(torch.einsum("ti,tic->tc", H_pre[t] * read, X_cur), round_bf16))
 
         # Post- and residual maps from the RMSNorm-normalised current active state
         # (Eq. param_post, Eq. param_res with the App. A row clamp).

@@ -103,6 +103,8 @@ Dims make_dims(const xhc_config& c) {
         d.kapmax = std::max(d.kapmax, d.kap[j]);
         d.kapsum += d.kap[j];
     }
+    d.softmax = c.router == 1 ? 1 : 0;
+    d.dense = c.sparse_read ? 0 : 1;
     for (int t = 0; t < 4; ++t) {
         const bool mlp = (t < d.G) && ((c.mlp_mask >> t) & 1) && c.n_conv > 0;
         d.K[t] = mlp ? 1 + c.n_conv : 1;
@@ -212,7 +214,7 @@ static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
 extern "C" {
 
-int xhc_version(void) { return 100; }
+int xhc_version(void) { return 200; }
 
 xhc_status xhc_trace_enable(int on) {
     std::lock_guard<std::mutex> lk(g_tmu);
@@ -274,7 +276,8 @@ xhc_status xhc_create(const xhc_config* cfg, xhc_handle** out) {
     const xhc_config& c = *cfg;
     if (c.N < 1 || c.k < 1 || c.m < 0 || c.m > c.k || c.k > c.N || c.C < 1 || c.group < 1 ||
         c.n_conv < 0 || c.n_conv > XHC_MAX_CONV || c.sinkhorn_iters < 0 || !(c.eps_norm > 0.f) ||
-        c.seq_len < 0 || c.variant < XHC_MHC || c.variant > XHC_FLASH)
+        c.seq_len < 0 || c.variant < XHC_MHC || c.variant > XHC_FLASH || c.router < 0 ||
+        c.router > 1 || c.sparse_read < 0 || c.sparse_read > 1)
         return XHC_ERR_INVALID_ARG;
     if (c.group > XHC_MAX_GROUP) return XHC_ERR_UNSUPPORTED;
     if (c.mlp_mask & ~((1 << c.group) - 1)) return XHC_ERR_INVALID_ARG;

@@ -231,14 +231,23 @@ __global__ void k_coef_full(Dims d, int T, const float* __restrict__ part,
         }
     }
     // Eq. router_topk: fixed streams 0..m-1 (p = 1), then TopK over i >= m by router logit
-    // (sigmoid is monotone), descending, ties to the lower stream index.
+    // (sigmoid and softmax are both monotone in the logit), descending, ties to the lower
+    // stream index.
     for (int j = 0; j < d.m; ++j) {
         I[(int64_t)t * d.k + j] = j;
         p[(int64_t)t * d.k + j] = 1.0f;
     }
     if (d.hr) {
         const float lstd = 1.0f / sqrtf(nu - mu * mu + d.eps);
-        for (int i = 0; i < d.N; ++i) zr[i] = (zr[i] - mu * wsum[i]) * lstd;
+        float zmax = -INFINITY;
+        for (int i = 0; i < d.N; ++i) {
+            zr[i] = (zr[i] - mu * wsum[i]) * lstd;
+            zmax = fmaxf(zmax, zr[i]);
+        }
+        // softmax router: s_i = exp(z_i) / sum over all N logits (the fixed streams' included)
+        float den = 0.f;
+        if (d.softmax)
+            for (int i = 0; i < d.N; ++i) den += expf(zr[i] - zmax);
         uint32_t taken = 0u;
         for (int j = d.m; j < d.k; ++j) {
             int best = -1;
@@ -252,7 +261,7 @@ __global__ void k_coef_full(Dims d, int T, const float* __restrict__ part,
             }
             taken |= 1u << best;
             I[(int64_t)t * d.k + j] = best;
-            p[(int64_t)t * d.k + j] = sigm(bv);
+            p[(int64_t)t * d.k + j] = d.softmax ? expf(bv - zmax) / den : sigm(bv);
         }
     }
 }
@@ -554,15 +563,43 @@ __global__ void k_full_coef(Dims d, int T, const float* __restrict__ dhpre,
             dzt[i] = 0.f;
             tg[2 + G * N + G + i] = 0.f;
         }
-        for (int j = d.m; j < d.k; ++j) {
-            const int i = I[(int64_t)t * d.k + j];
-            const float zc = zf[i] - mu * wsum[i];
-            const float s = sigm(zc * lstd);
-            const float dzr = dp[(int64_t)t * d.k + j] * s * (1.0f - s);
-            dzt[i] = dzr * lstd;
-            tg[2 + G * N + G + i] = mu * dzr * lstd;
-            dmu -= dzr * lstd * wsum[i];
-            dlstd += dzr * zc;
+        if (!d.softmax) {
+            // sigmoid scores: only the selected routed streams' logits receive a gradient
+            for (int j = d.m; j < d.k; ++j) {
+                const int i = I[(int64_t)t * d.k + j];
+                const float zc = zf[i] - mu * wsum[i];
+                const float s = sigm(zc * lstd);
+                const float dzr = dp[(int64_t)t * d.k + j] * s * (1.0f - s);
+                dzt[i] = dzr * lstd;
+                tg[2 + G * N + G + i] = mu * dzr * lstd;
+                dmu -= dzr * lstd * wsum[i];
+                dlstd += dzr * zc;
+            }
+        } else {
+            // softmax scores s = softmax(z): dz_l = s_l (g_l - sum_j dp_j s_{I_j}), g_l = dp_j
+            // where l = I_j is a selected routed stream, 0 elsewhere; every logit receives one
+            float zmax = -INFINITY;
+            for (int i = 0; i < N; ++i) zmax = fmaxf(zmax, (zf[i] - mu * wsum[i]) * lstd);
+            float den = 0.f;
+            for (int i = 0; i < N; ++i) den += expf((zf[i] - mu * wsum[i]) * lstd - zmax);
+            float gs[MAXN];
+            for (int i = 0; i < N; ++i) gs[i] = 0.f;
+            float dot = 0.f;
+            for (int j = d.m; j < d.k; ++j) {
+                const int i = I[(int64_t)t * d.k + j];
+                const float s = expf((zf[i] - mu * wsum[i]) * lstd - zmax) / den;
+                gs[i] = dp[(int64_t)t * d.k + j];
+                dot += gs[i] * s;
+            }
+            for (int i = 0; i < N; ++i) {
+                const float zc = zf[i] - mu * wsum[i];
+                const float s = expf(zc * lstd - zmax) / den;
+                const float dzr = s * (gs[i] - dot);
+                dzt[i] = dzr * lstd;
+                tg[2 + G * N + G + i] = mu * dzr * lstd;
+                dmu -= dzr * lstd * wsum[i];
+                dlstd += dzr * zc;
+            }
         }
         const float l3 = lstd * lstd * lstd;
         dnu += -0.5f * dlstd * l3;

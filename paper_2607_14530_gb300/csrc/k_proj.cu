@@ -308,7 +308,7 @@ __global__ void __launch_bounds__(256) k_full_dx(Dims d, int T, const float* __r
             const uint2 u = *reinterpret_cast<const uint2*>(dX + (int64_t)t * E + e);
             v[0] = __uint_as_float(u.x << 16); v[1] = __uint_as_float(u.x & 0xffff0000u);
             v[2] = __uint_as_float(u.y << 16); v[3] = __uint_as_float(u.y & 0xffff0000u);
-            for (int q = 0; q < d.G; ++q) {
+            for (int q = 0; q < (d.dense ? d.G : 0); ++q) {   // sparse-read ablation: none
                 const float h = hpre[((int64_t)t * d.G + q) * d.N + i];
                 const uint2 g = *reinterpret_cast<const uint2*>(din + ((int64_t)q * T + t) * d.C + c);
                 v[0] = fmaf(h, __uint_as_float(g.x << 16), v[0]);

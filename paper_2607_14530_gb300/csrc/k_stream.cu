@@ -82,16 +82,19 @@ __global__ void __launch_bounds__(256, 3) k_read(Dims d, int T, const uint16_t* 
                 float x[8];
                 unpack8(ub[ii], x);
                 const int j = slotmap[i];
-                const float h0 = sh[i];
+                // sparse-read ablation: the non-active streams are not read
+                const float h0 = (j >= 0 || d.dense) ? sh[i] : 0.f;
 #pragma unroll
                 for (int e = 0; e < 8; ++e) acc[0][e] = fmaf(h0, x[e], acc[0][e]);
                 if (j < 0) {
+                    if (d.dense) {
 #pragma unroll
-                    for (int q = 1; q < 4; ++q) {
-                        if (q < G) {
-                            const float h = sh[q * N + i];
+                        for (int q = 1; q < 4; ++q) {
+                            if (q < G) {
+                                const float h = sh[q * N + i];
 #pragma unroll
-                            for (int e = 0; e < 8; ++e) acc[q][e] = fmaf(h, x[e], acc[q][e]);
+                                for (int e = 0; e < 8; ++e) acc[q][e] = fmaf(h, x[e], acc[q][e]);
+                            }
                         }
                     }
                 } else {
@@ -329,6 +332,12 @@ __global__ void __launch_bounds__(1024) k_full_dots(Dims d, int T, const uint16_
             }
             ++cnt;
         }
+    if (!d.dense) {
+        // sparse-read ablation: the non-active streams are not read, so their dH_pre is zero
+        if (i >= 0 && lane == 0)
+            for (int q = 0; q < G; ++q) dhpre[((int64_t)t * G + q) * d.N + i] = 0.f;
+        return;
+    }
     const int64_t row = ((int64_t)t * d.N + (i < 0 ? 0 : i)) * C;
     // the first 4 chunks per lane, read before the staging barrier
     uint4 xr[4];

@@ -675,6 +675,7 @@ __device__ __forceinline__ uint4 ld_stream(const void* p) {
 struct DxArgs {
     int T, C, N, k, G;
     int m;                // full-state epilogue: fixed streams 0..m-1 (active on every token)
+    int dense;            // full-state epilogue: 0 = sparse-read ablation (no dense-read term)
     int slot;             // active epilogue: slot of the pre-map
     int NH;               // active epilogue: streams of the H_pre rows
     float* dxa;           // active epilogue: dX_act [T][k][C] fp32, updated in place
@@ -1161,7 +1162,7 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
             float hq[4];
 #pragma unroll
             for (int q = 0; q < 4; ++q)
-                hq[q] = (usesg && !arow && t < a.T && q < a.G) ? a.hpre[((long long)t * a.G + q) * N + i] : 0.f;
+                hq[q] = (a.dense && usesg && !arow && t < a.T && q < a.G) ? a.hpre[((long long)t * a.G + q) * N + i] : 0.f;
             // an active row's fp32 base, 8 channels per chunk, read one chunk ahead (the first
             // before the waits)
             const float* brow = a.dxact + ((long long)t * a.k + (j < 0 ? 0 : j)) * a.C + cb * DG_BN + half * 32;
@@ -1368,7 +1369,7 @@ cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, 
     if (!make_map_box(&mg, dinput, (uint64_t)d.C, (uint64_t)d.G * T, DG_BN, BM)) return cudaErrorInvalidValue;
     DxArgs a;
     memset(&a, 0, sizeof(a));
-    a.T = T; a.C = d.C; a.N = d.N; a.k = d.k; a.G = d.G; a.m = d.m;
+    a.T = T; a.C = d.C; a.N = d.N; a.k = d.k; a.G = d.G; a.m = d.m; a.dense = d.dense;
     a.nkb = (n + BK - 1) / BK;
     a.ksteps = (n + 15) / 16;
     a.TT = (T + BM - 1) / BM;

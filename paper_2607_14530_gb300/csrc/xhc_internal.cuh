@@ -32,6 +32,8 @@ struct Dims {
     int kapsum;          // sum of kernel sizes
     int K[4];            // write-back components per slot
     int nact[4];         // active projection width per slot: k*K_t (+ k*k for the last slot)
+    int softmax;         // router scores: 0 sigmoid (Eq. router), 1 softmax over the N logits
+    int dense;           // 1: dense read of all N streams (Eq. dense_read); 0: active streams only
 };
 
 // Column segments of a projection weight: column o of the logical [rows, n] matrix lives in

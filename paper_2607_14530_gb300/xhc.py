@@ -27,7 +27,8 @@ class _Config(ctypes.Structure):
                 ("mlp_mask", ctypes.c_int), ("n_conv", ctypes.c_int),
                 ("conv_k", ctypes.c_int * MAX_CONV), ("gram_schmidt", ctypes.c_int),
                 ("sinkhorn_iters", ctypes.c_int), ("eps_norm", ctypes.c_float),
-                ("eps_gs", ctypes.c_float), ("seq_len", ctypes.c_int)]
+                ("eps_gs", ctypes.c_float), ("seq_len", ctypes.c_int), ("router", ctypes.c_int),
+                ("sparse_read", ctypes.c_int)]
 
 
 _P = ctypes.c_void_p
@@ -139,6 +140,8 @@ class Config:
     eps_norm: float = 1e-5
     eps_gs: float = 0.0
     seq_len: int = 0
+    router: str = "sigmoid"        # or "softmax" (the softmax-router ablation)
+    sparse_read: bool = False      # read only the k active streams (the sparse-read ablation)
 
     @staticmethod
     def mhc(N, C, **kw):
@@ -194,6 +197,8 @@ class Config:
         c.eps_norm = self.eps_norm
         c.eps_gs = self.eps_gs
         c.seq_len = self.seq_len
+        c.router = {"sigmoid": 0, "softmax": 1}[self.router]
+        c.sparse_read = 1 if self.sparse_read else 0
         return c
 
 

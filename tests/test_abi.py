@@ -28,7 +28,7 @@ def test_exports_every_declared_function(L):
     assert len(names) >= 10, names
     for n in names:
         assert hasattr(L, n), f"{n} not exported"
-    assert L.xhc_version() == 100
+    assert L.xhc_version() == 200
 
 
 def _create(cfg):
@@ -46,6 +46,19 @@ def test_create_accepts_paper_configs(L):
     assert _create(X.Config.flash(16, 4, 2, 4096, 4)) == OK
     assert _create(X.Config.flash(16, 4, 2, 4096, 2)) == OK
     assert _create(X.Config.flash(32, 4, 2, 4096, 4)) == OK
+    # ablations: softmax router, sparse read, attention-side temporal augmentation
+    assert _create(X.Config.full(16, 4, 2, 2048, True, router="softmax")) == OK
+    assert _create(X.Config.full(16, 4, 0, 2048, False, sparse_read=True)) == OK
+    assert _create(X.Config.flash(16, 4, 2, 4096, 4, attn_tfa=True)) == OK
+
+
+def test_create_rejects_unknown_ablation_codes(L):
+    c = X.Config.full(16, 4, 2, 256, True)._c()
+    for field, bad in (("router", 2), ("router", -1), ("sparse_read", 2)):
+        cc = X._Config.from_buffer_copy(c)
+        setattr(cc, field, bad)
+        h = ctypes.c_void_p()
+        assert L.xhc_create(ctypes.byref(cc), ctypes.byref(h)) == INVALID, field
 
 
 @pytest.mark.parametrize("cfg,want", [

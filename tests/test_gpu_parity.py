@@ -45,6 +45,12 @@ CASES = {
     # attention-side temporal augmentation (App. "Additional Ablation Studies")
     "flash4_attn_tfa": (Config.flash(16, 4, 2, 256, 4, attn_tfa=True, seq_len=128), 512, {}),
     "flash2_attn_tfa": (Config.flash(16, 4, 2, 256, 2, attn_tfa=True, seq_len=128), 256, {}),
+    # Table ablation: softmax router (11); no dense read (7); no dense read and no fixed stream (6)
+    "fullM_softmax_router": (Config.full(16, 4, 2, 256, True, seq_len=128, router="softmax"), 256, {}),
+    "fullM_sparse_read": (Config.full(16, 4, 2, 256, True, seq_len=128, sparse_read=True), 256, {}),
+    "fullA_sparse_read_m0": (Config.full(16, 4, 0, 256, False, sparse_read=True), 200, {}),
+    "flash4_softmax_sparse": (Config.flash(16, 4, 2, 256, 4, seq_len=128, router="softmax",
+                                           sparse_read=True), 256, {}),
 }
 
 

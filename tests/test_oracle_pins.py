@@ -239,10 +239,21 @@ CFGS = [
     O.flash(5, 3, 1, 8, 2, conv_k=(2, 3)),
     O.flash(5, 3, 1, 8, 4, seq_len=3, conv_k=(2, 3)),
     O.flash(4, 2, 1, 6, 4, conv_k=(2, 3), gram_schmidt=False),
+    # ablations of Table ablation: softmax router (11), no dense read (7), neither dense read
+    # nor fixed streams (6)
+    O.full(5, 3, 1, 8, True, seq_len=3, conv_k=(2, 3), router="softmax"),
+    O.full(5, 3, 1, 8, False, dense_read=False),
+    O.full(5, 3, 0, 6, True, conv_k=(2,), dense_read=False),
+    O.flash(5, 3, 1, 8, 4, seq_len=3, conv_k=(2, 3), router="softmax", dense_read=False),
 ]
 
 
-@pytest.mark.parametrize("cfg", CFGS, ids=lambda c: f"N{c.N}k{c.k}m{c.m}G{c.G}{''.join('M' if x else 'A' for x in c.mlp)}")
+def _cid(c):
+    tag = f"N{c.N}k{c.k}m{c.m}G{c.G}{''.join('M' if x else 'A' for x in c.mlp)}"
+    return tag + ("-softmax" if c.router == "softmax" else "") + ("-sparse" if not c.dense_read else "")
+
+
+@pytest.mark.parametrize("cfg", CFGS, ids=_cid)
 @pytest.mark.parametrize("rounding", [False, True])
 def test_group_matches_brute_force(cfg, rounding):
     T = 6
@@ -358,7 +369,9 @@ def test_flash_corrected_inputs_equal_full_dense_reads(G):
     O.full(4, 3, 1, 6, False),
     O.mhc(3, 8),
     O.flash(5, 3, 1, 8, 4, seq_len=3, conv_k=(2, 3)),
-], ids=["fullM", "fullA", "mhc", "flash4"])
+    O.full(4, 2, 1, 8, True, seq_len=3, conv_k=(2, 3), router="softmax"),
+    O.flash(5, 3, 0, 8, 4, seq_len=3, conv_k=(2, 3), dense_read=False),
+], ids=["fullM", "fullA", "mhc", "flash4", "fullM-softmax", "flash4-sparse-m0"])
 def test_backward_matches_central_differences(cfg):
     T = 6
     P = _params(cfg, 1)
@@ -494,3 +507,21 @@ def test_prerounding_bookkeeping():
     for t in range(1, 4):
         assert torch.equal(O.rnd(aux["pre"][t], True), aux["X_act"][t])
         assert bool((aux["mag"][t] >= aux["pre"][t].abs() * (1 - 1e-12)).all())
+
+
+def test_softmax_router_scores_and_sparse_read_closed_forms():
+    """Softmax router (Table ablation row 11): the N scores of a token sum to 1 and order the
+    streams like the sigmoid scores (both monotone in the logit).  Sparse read (rows 6-7): the
+    sublayer input is the pre-map-weighted sum of the active streams only."""
+    cfg = O.full(6, 3, 1, 8, False, router="softmax", dense_read=False)
+    T = 7
+    P = _params(cfg, 31)
+    X, outs = _inputs(cfg, T, 31)
+    Xo, ins, aux = O.forward(cfg, P, X, outs, round_bf16=False)
+    s = aux["s"]
+    assert torch.allclose(s.sum(1), torch.ones(T, dtype=F64), atol=1e-14, rtol=0)
+    sig = O.router_scores(O.full(6, 3, 1, 8, False), X.reshape(T, -1), P["W_r"])
+    assert torch.equal(torch.argsort(s, dim=1), torch.argsort(sig, dim=1))
+    I = aux["I"]
+    want = torch.einsum("tj,tjc->tc", aux["H_pre"][0].gather(1, I), X[torch.arange(T)[:, None], I])
+    assert torch.allclose(ins[0], want, atol=1e-13, rtol=0)

@@ -49,7 +49,8 @@ def oracle_cfg(cfg: Config) -> O.Config:
                     mlp=tuple(bool((cfg.mlp_mask >> t) & 1) for t in range(cfg.G)),
                     conv_k=tuple(cfg.conv_k), gram_schmidt=cfg.gram_schmidt,
                     sinkhorn_iters=cfg.sinkhorn_iters, eps_norm=cfg.eps_norm,
-                    eps_gs=(cfg.eps_gs if cfg.eps_gs > 0 else None), seq_len=cfg.seq_len)
+                    eps_gs=(cfg.eps_gs if cfg.eps_gs > 0 else None), seq_len=cfg.seq_len,
+                    router=cfg.router, dense_read=not cfg.sparse_read)
 
 
 def tie_free(cfg: Config, X: torch.Tensor, W_r: torch.Tensor) -> torch.Tensor:
