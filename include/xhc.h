@@ -246,6 +246,43 @@ xhc_status xhc_pre_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
                        const uint16_t* X, const uint16_t* d_input, uint16_t* dX,
                        const xhc_grads* grads, void* saved, void* workspace, void* stream);
 
+/* Sequence split (context parallelism, chunked prefill).
+ *
+ * A sequence may be cut into consecutive chunks that are processed by separate calls (on separate
+ * GPUs, or one after the other).  Every step of the op is token-local except the causal conv of
+ * the temporal augmentation (conv formula of Sec. 3.3.4), which reads the R = max(kappa) - 1
+ * sublayer outputs before each token; for the first tokens of a chunk those belong to the previous
+ * chunk.  They travel as a halo: [B][R][C] bf16 per conv slot, row r of sequence b holding `out`
+ * at position r - R relative to the chunk's first token (zero rows where that position is before
+ * the sequence start; B = T / seq_len sequences in the call, each a chunk).
+ *
+ * xhc_halo_bytes: bytes of one slot's halo for B sequences (0 without a conv); its gradient
+ *   d_halo is the same shape in fp32 (twice the bytes).
+ * xhc_halo_fill: from a chunk's sublayer output `out` (B sequences of S tokens), the halo the
+ *   next chunk needs: halo[b][r] = out[b*S + S - R + r] (zero where S - R + r < 0).
+ * xhc_post_fwd_halo: xhc_post_fwd with the conv history of every sequence's first tokens read
+ *   from `halo` (null = a sequence start; ignored on slots without a conv).
+ * xhc_post_bwd_halo: xhc_post_bwd of such a call; the conv weight gradient includes the halo's
+ *   terms, and d_halo [B][R][C] fp32 (required with a halo on a conv slot, else
+ *   XHC_ERR_INVALID_ARG) receives the gradient w.r.t. the halo rows, which belongs to the
+ *   previous chunk's d_out.
+ * xhc_halo_add: on the previous chunk, d_out[b*S + S - R + r] += d_halo[b][r] (the sum rounded
+ *   once to bf16); run after its own xhc_post_bwd(slot), before its sublayer's backward.
+ * The parameter gradients of the chunks add up (accumulate into the same buffers, or all-reduce
+ * them across the GPUs that hold the chunks).  Same ownership and error rules as above. */
+xhc_status xhc_halo_bytes(const xhc_handle* h, int64_t B, size_t* bytes);
+xhc_status xhc_halo_fill(const xhc_handle* h, int64_t B, int64_t S, const uint16_t* out, void* halo,
+                         void* stream);
+xhc_status xhc_post_fwd_halo(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
+                             uint16_t* X, const uint16_t* out, const uint16_t* halo, void* saved,
+                             void* workspace, void* stream);
+xhc_status xhc_post_bwd_halo(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
+                             uint16_t* X, uint16_t* dX, const uint16_t* out, uint16_t* d_out,
+                             const xhc_grads* grads, const uint16_t* halo, float* d_halo,
+                             void* saved, void* workspace, void* stream);
+xhc_status xhc_halo_add(const xhc_handle* h, int64_t B, int64_t S, uint16_t* d_out,
+                        const float* d_halo, void* stream);
+
 /* Routing and pre-maps for callers that cannot allocate device memory.
  *
  * The paper has no counterpart: this is a deployment convenience.  Some callers cannot provide

@@ -211,9 +211,17 @@ def row_clamp(H: torch.Tensor) -> torch.Tensor:
     return H / torch.where(s > 1.0, s, torch.ones_like(s))
 
 
-def causal_dwconv(out: torch.Tensor, w: torch.Tensor, S: int) -> torch.Tensor:
+def causal_dwconv(out: torch.Tensor, w: torch.Tensor, S: int, hist: torch.Tensor | None = None) -> torch.Tensor:
     """g[t] = sum_{i=0}^{kappa-1} w[i] * out[t-i] channel-wise (Sec. 3.3.4), zero before the
-    start of each length-S sequence.  out: [T, C], w: [kappa, C]."""
+    start of each length-S sequence.  out: [T, C], w: [kappa, C].
+
+    ``hist`` [B, R, C] (B = T / S): the R outputs that precede each of the B sequences, when the
+    call holds a later chunk of longer sequences (sequence split); out[t - i] before the chunk's
+    first token is then hist[b][R + (t - i) - b S] (zero before that)."""
+    if hist is not None:
+        B, R, C = hist.shape
+        ext = torch.cat([hist, out.reshape(B, S, C)], dim=1).reshape(B * (R + S), C)
+        return causal_dwconv(ext, w, R + S).reshape(B, R + S, C)[:, R:].reshape(B * S, C)
     T = out.shape[0]
     pos = torch.arange(T) % S
     g = torch.zeros_like(out)
@@ -238,10 +246,11 @@ def gram_schmidt(out: torch.Tensor, gs: list, eps: float) -> list:
     return v
 
 
-def augment(cfg: Config, out: torch.Tensor, conv_ws: list, T: int) -> list:
-    """out_aug of Eq. aug (after Eq. gs when enabled): K_r = r + 1 components, each [T, C]."""
+def augment(cfg: Config, out: torch.Tensor, conv_ws: list, T: int, hist: torch.Tensor | None = None) -> list:
+    """out_aug of Eq. aug (after Eq. gs when enabled): K_r = r + 1 components, each [T, C].
+    ``hist``: the outputs preceding each sequence of a later chunk (see causal_dwconv)."""
     S = cfg.S(T)
-    gs = [causal_dwconv(out, w, S) for w in conv_ws]
+    gs = [causal_dwconv(out, w, S, hist) for w in conv_ws]
     if cfg.gram_schmidt:
         return gram_schmidt(out, gs, cfg.gs_eps())
     return [out] + gs
@@ -297,13 +306,16 @@ def routing_margin(cfg: Config, s: torch.Tensor) -> torch.Tensor:
 # forward / backward of one group
 
 
-def forward(cfg: Config, P: dict, X: torch.Tensor, outs: list, *, round_bf16: bool = True):
+def forward(cfg: Config, P: dict, X: torch.Tensor, outs: list, *, round_bf16: bool = True,
+            halos: list | None = None):
     """One connection-op group: Alg. 1 (G = 1) or Alg. 2 / App. E.2 (G = 2, 4).
 
     X: [T, N, C] float64 holding the entry state; outs[t]: [T, C] float64, the caller's
     sublayer output of slot t (out^(t) = F_t(input^(t)) in the paper; here an input of the op).
     Returns (X_out, inputs, aux): the state after the group, the G sublayer inputs, and a dict
     of intermediates (s, H_pre, I, p, H_post, H_res, the active state before every slot).
+    ``halos[t]`` ([B, R, C] or None): for a call holding a later chunk of its sequences, the
+    sublayer outputs of slot t that precede each sequence (read by the causal conv only).
 
     For the tests, aux also holds, for every slot t >= 1 of a group, the active state entering
     slot t before its bf16 rounding (``pre[t]``) and the sum of the magnitudes of the terms that
@@ -350,8 +362,9 @@ def forward(cfg: Config, P: dict, X: torch.Tensor, outs: list, *, round_bf16: bo
         H_post_all.append(H_post)
 
         # Write-back components (Eq. aug + Eq. gs for MLP slots, out itself otherwise).
+        hist = None if halos is None else halos[t]
         if K > 1:
-            comps = augment(cfg, outs[t], [P[f"conv_w.{t}.{j}"] for j in range(len(cfg.conv_k))], T)
+            comps = augment(cfg, outs[t], [P[f"conv_w.{t}.{j}"] for j in range(len(cfg.conv_k))], T, hist)
         else:
             comps = [outs[t]]
         out_aug = torch.stack(comps, dim=1)                       # [T, K, C]
@@ -367,7 +380,7 @@ def forward(cfg: Config, P: dict, X: torch.Tensor, outs: list, *, round_bf16: bo
         new = mixed + delta                                       # Eq. sparse_write
         if t < G - 1:
             # magnitudes of the terms of the next slot's active state (test bookkeeping only)
-            raw = [outs[t]] + ([causal_dwconv(outs[t], P[f"conv_w.{t}.{j}"], cfg.S(T))
+            raw = [outs[t]] + ([causal_dwconv(outs[t], P[f"conv_w.{t}.{j}"], cfg.S(T), hist)
                                 for j in range(len(cfg.conv_k))] if K > 1 else [])
             mu = sum(c.detach().abs() for c in raw)                   # [T, C]
             hp = (p.detach().abs() * H_post.detach().abs().sum(dim=2))  # [T, k]
@@ -382,25 +395,41 @@ def forward(cfg: Config, P: dict, X: torch.Tensor, outs: list, *, round_bf16: bo
 
 
 def backward(cfg: Config, P: dict, X: torch.Tensor, outs: list, dX_out: torch.Tensor,
-             d_inputs: list, *, round_bf16: bool = True):
+             d_inputs: list, *, round_bf16: bool = True, halos: list | None = None):
     """Reverse mode of :func:`forward` for the loss L = <X_out, dX_out> + sum_t <input_t, d_input_t>.
 
     Returns (dX, d_outs, dP): the gradient w.r.t. the entry state, each sublayer output and every
     parameter (flat names as in :func:`param_shapes`).  No gradient flows through the TopK
     selection or the fixed p = 1 (Eq. router_topk); routing gradients reach W_r only through the
-    selected routed scores p_j."""
+    selected routed scores p_j.
+
+    With ``halos`` (see :func:`forward`) a fourth value is returned: the gradient w.r.t. every
+    halo (None where the slot has none), which belongs to the previous chunk's sublayer outputs."""
     Xl = X.detach().clone().requires_grad_(True)
     outl = [o.detach().clone().requires_grad_(True) for o in outs]
     Pl = {n: v.detach().clone().requires_grad_(True) for n, v in P.items()}
-    Xo, inputs, _ = forward(cfg, Pl, Xl, outl, round_bf16=round_bf16)
+    hl = None if halos is None else [None if h is None else h.detach().clone().requires_grad_(True)
+                                     for h in halos]
+    Xo, inputs, _ = forward(cfg, Pl, Xl, outl, round_bf16=round_bf16, halos=hl)
     L = (Xo * dX_out).sum()
     for inp, d in zip(inputs, d_inputs):
         L = L + (inp * d).sum()
     names = list(Pl)
-    grads = torch.autograd.grad(L, [Xl] + outl + [Pl[n] for n in names], allow_unused=True)
+    hx = [] if hl is None else [h for h in hl if h is not None]
+    grads = torch.autograd.grad(L, [Xl] + outl + [Pl[n] for n in names] + hx, allow_unused=True)
     dX = grads[0]
     d_outs = list(grads[1:1 + len(outl)])
     dP = {}
-    for n, g in zip(names, grads[1 + len(outl):]):
+    nP = 1 + len(outl) + len(names)
+    for n, g in zip(names, grads[1 + len(outl):nP]):
         dP[n] = g if g is not None else torch.zeros_like(Pl[n])
-    return dX, d_outs, dP
+    if hl is None:
+        return dX, d_outs, dP
+    dh, i = [], nP
+    for h in hl:
+        if h is None:
+            dh.append(None)
+        else:
+            dh.append(grads[i] if grads[i] is not None else torch.zeros_like(h))
+            i += 1
+    return dX, d_outs, dP, dh

@@ -516,6 +516,8 @@ WSegsOut act_segs_g(const Dims& d, const xhc_grads* g, int slot) {
 ConvPtrs conv_of(const Dims& d, const xhc_params* P, int slot) {
     ConvPtrs c;
     for (int j = 0; j < 3; ++j) c.w[j] = (j < d.nconv && d.K[slot] > 1) ? P->conv_w[slot][j] : nullptr;
+    c.halo = nullptr;
+    c.dhalo = nullptr;
     return c;
 }
 
@@ -611,16 +613,21 @@ xhc_status xhc_pre_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
     return active_maps(c, slot, P);
 }
 
-xhc_status xhc_post_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
-                        uint16_t* X, const uint16_t* out, void* saved, void* workspace,
-                        void* stream) {
+}  // extern "C"
+
+namespace {
+
+xhc_status post_fwd_impl(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
+                         uint16_t* X, const uint16_t* out, const uint16_t* halo, void* saved,
+                         void* workspace, void* stream) {
     Ctx c;
     xhc_status s = common_check(h, slot, T, saved, workspace, c, stream);
     if (s != XHC_OK) return s;
     if (!X || !out || !params_ok(c.d, P, slot, false)) return XHC_ERR_INVALID_ARG;
-    if (!aligned16(X) || !aligned16(out)) return XHC_ERR_ALIGNMENT;
+    if (!aligned16(X) || !aligned16(out) || (halo && !aligned16(halo))) return XHC_ERR_ALIGNMENT;
     const Dims& d = c.d;
-    const ConvPtrs cw = conv_of(d, P, slot);
+    ConvPtrs cw = conv_of(d, P, slot);
+    if (d.K[slot] > 1) cw.halo = halo;
     if (d.K[slot] > 1 && d.gs)
         XHC_K("wb_gram", c.st, launch_wb_gram(d, slot, c.T, out, cw, c.L.nslice, c.W<float>(c.L.red), c.st));
     const bool last = (slot == d.G - 1);
@@ -631,6 +638,47 @@ xhc_status xhc_post_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
     XHC_K("wb_fwd", c.st, launch_wb_fwd(d, slot, c.T, out, cw, c.W<float>(c.L.tokmat), c.L.nslice,
                                         c.xact(slot), c.S<int>(c.L.I), c.S<float>(c.L.hres),
                                         last ? nullptr : c.xact(slot + 1), X, c.st));
+    return XHC_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+xhc_status xhc_post_fwd(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
+                        uint16_t* X, const uint16_t* out, void* saved, void* workspace,
+                        void* stream) {
+    return post_fwd_impl(h, slot, T, P, X, out, nullptr, saved, workspace, stream);
+}
+
+xhc_status xhc_post_fwd_halo(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
+                             uint16_t* X, const uint16_t* out, const uint16_t* halo, void* saved,
+                             void* workspace, void* stream) {
+    return post_fwd_impl(h, slot, T, P, X, out, halo, saved, workspace, stream);
+}
+
+xhc_status xhc_halo_bytes(const xhc_handle* h, int64_t B, size_t* bytes) {
+    if (!h || !bytes || B <= 0) return XHC_ERR_INVALID_ARG;
+    const Dims& d = h->h.d;
+    *bytes = d.nconv > 0 ? (size_t)B * (d.kapmax - 1) * d.C * 2 : 0;
+    return XHC_OK;
+}
+
+xhc_status xhc_halo_fill(const xhc_handle* h, int64_t B, int64_t S, const uint16_t* out, void* halo,
+                         void* stream) {
+    if (!h || !out || !halo || B <= 0 || S <= 0 || B * S > ((int64_t)1 << 30)) return XHC_ERR_INVALID_ARG;
+    if (!aligned16(out) || !aligned16(halo)) return XHC_ERR_ALIGNMENT;
+    const cudaError_t e = launch_halo_fill(h->h.d, (int)B, (int)S, out, (uint16_t*)halo, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, __LINE__);
+    return XHC_OK;
+}
+
+xhc_status xhc_halo_add(const xhc_handle* h, int64_t B, int64_t S, uint16_t* d_out, const float* d_halo,
+                        void* stream) {
+    if (!h || !d_out || !d_halo || B <= 0 || S <= 0 || B * S > ((int64_t)1 << 30)) return XHC_ERR_INVALID_ARG;
+    if (!aligned16(d_out) || !aligned16(d_halo)) return XHC_ERR_ALIGNMENT;
+    const cudaError_t e = launch_halo_add(h->h.d, (int)B, (int)S, d_out, d_halo, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, __LINE__);
     return XHC_OK;
 }
 
@@ -678,21 +726,31 @@ xhc_status xhc_post_fwd_decode(const xhc_handle* h, int slot, int64_t B, const x
     return XHC_OK;
 }
 
-xhc_status xhc_post_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
-                        uint16_t* X, uint16_t* dX, const uint16_t* out, uint16_t* d_out,
-                        const xhc_grads* g, void* saved, void* workspace, void* stream) {
+}  // extern "C"
+
+namespace {
+
+xhc_status post_bwd_impl(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
+                         uint16_t* X, uint16_t* dX, const uint16_t* out, uint16_t* d_out,
+                         const xhc_grads* g, const uint16_t* halo, float* d_halo, void* saved,
+                         void* workspace, void* stream) {
     Ctx c;
     xhc_status s = common_check(h, slot, T, saved, workspace, c, stream);
     if (s != XHC_OK) return s;
     if (!X || !dX || !out || !d_out || !params_ok(c.d, P, slot, false) ||
         !grads_ok(c.d, g, slot, false))
         return XHC_ERR_INVALID_ARG;
-    if (!aligned16(X) || !aligned16(dX) || !aligned16(out) || !aligned16(d_out))
+    if (!aligned16(X) || !aligned16(dX) || !aligned16(out) || !aligned16(d_out) ||
+        (halo && !aligned16(halo)) || (d_halo && !aligned16(d_halo)))
         return XHC_ERR_ALIGNMENT;
     const Dims& d = c.d;
     const int T32 = c.T;
     const bool last = (slot == d.G - 1);
-    const ConvPtrs cw = conv_of(d, P, slot);
+    ConvPtrs cw = conv_of(d, P, slot);
+    if (d.K[slot] > 1) {
+        cw.halo = halo;
+        cw.dhalo = d_halo;
+    }
     const int K = d.K[slot], n = d.nact[slot];
     float* red = c.W<float>(c.L.red);
     float* dxact = c.W<float>(c.L.dxact);
@@ -749,6 +807,26 @@ xhc_status xhc_post_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_para
         XHC_K("conv_wgrad_reduce", c.st, launch_conv_wgrad_reduce(d, slot, c.W<float>(c.L.cpart), c.L.ntiles, gc, c.st));
     }
     return join_into(c.st, sd);
+}
+
+}  // namespace
+
+extern "C" {
+
+xhc_status xhc_post_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
+                        uint16_t* X, uint16_t* dX, const uint16_t* out, uint16_t* d_out,
+                        const xhc_grads* g, void* saved, void* workspace, void* stream) {
+    return post_bwd_impl(h, slot, T, P, X, dX, out, d_out, g, nullptr, nullptr, saved, workspace, stream);
+}
+
+xhc_status xhc_post_bwd_halo(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,
+                             uint16_t* X, uint16_t* dX, const uint16_t* out, uint16_t* d_out,
+                             const xhc_grads* g, const uint16_t* halo, float* d_halo, void* saved,
+                             void* workspace, void* stream) {
+    // a slot with a conv and a halo must return the halo's gradient
+    if (h && slot >= 0 && slot < h->h.d.G && h->h.d.K[slot] > 1 && halo && !d_halo)
+        return XHC_ERR_INVALID_ARG;
+    return post_bwd_impl(h, slot, T, P, X, dX, out, d_out, g, halo, d_halo, saved, workspace, stream);
 }
 
 xhc_status xhc_pre_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_params* P,

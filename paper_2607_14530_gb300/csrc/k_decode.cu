@@ -185,6 +185,44 @@ __global__ void k_ring_fill(const uint16_t* __restrict__ out, int B, int S, int 
     }
 }
 
+// halo rows for the next chunk of B sequences of S tokens: halo[b][r] = out of position
+// S - R + r of sequence b (zero where that position is before the sequence start)
+__global__ void k_halo_fill(const uint16_t* __restrict__ out, int B, int S, int C, int R,
+                            uint16_t* __restrict__ halo) {
+    const long long n = (long long)B * R * (C / 8);
+    for (long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x; idx < n;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const int c8 = (int)(idx % (C / 8));
+        const long long br = idx / (C / 8);
+        const int r = (int)(br % R);
+        const long long b = br / R;
+        const long long s = (long long)S - R + r;
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (s >= 0) v = *reinterpret_cast<const uint4*>(out + (b * S + s) * C + c8 * 8);
+        *reinterpret_cast<uint4*>(halo + br * C + c8 * 8) = v;
+    }
+}
+
+// the gradient of a chunk's halo rows, returned to the chunk that produced them: d_out of
+// position S - R + r of sequence b += d_halo[b][r] (in fp32, one bf16 rounding)
+__global__ void k_halo_add(uint16_t* __restrict__ d_out, int B, int S, int C, int R,
+                           const float* __restrict__ dhalo) {
+    const long long n = (long long)B * R * (C / 2);
+    for (long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x; idx < n;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const int c2 = (int)(idx % (C / 2));
+        const long long br = idx / (C / 2);
+        const int r = (int)(br % R);
+        const long long b = br / R;
+        const long long s = (long long)S - R + r;
+        if (s < 0) continue;
+        uint32_t* p = reinterpret_cast<uint32_t*>(d_out + (b * S + s) * C + c2 * 2);
+        const float2 g = *reinterpret_cast<const float2*>(dhalo + br * C + c2 * 2);
+        const uint32_t u = *p;
+        *p = pack2(__uint_as_float(u << 16) + g.x, __uint_as_float(u & 0xffff0000u) + g.y);
+    }
+}
+
 int dec_slices(int C) { return (C + 2 * DTH - 1) / (2 * DTH); }
 
 }  // namespace
@@ -218,6 +256,26 @@ cudaError_t launch_ring_fill(const Dims& d, int B, int S, const uint16_t* out, u
     const long long n = (long long)B * R * (d.C / 8);
     const int blocks = (int)std::min<long long>((n + 255) / 256, 4096);
     k_ring_fill<<<blocks, 256, 0, st>>>(out, B, S, d.C, R, ring); note_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_halo_fill(const Dims& d, int B, int S, const uint16_t* out, uint16_t* halo,
+                             cudaStream_t st) {
+    const int R = d.kapmax - 1;
+    if (R <= 0) return cudaSuccess;
+    const long long n = (long long)B * R * (d.C / 8);
+    const int blocks = (int)std::min<long long>((n + 255) / 256, 4096);
+    k_halo_fill<<<blocks, 256, 0, st>>>(out, B, S, d.C, R, halo); note_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_halo_add(const Dims& d, int B, int S, uint16_t* d_out, const float* dhalo,
+                            cudaStream_t st) {
+    const int R = d.kapmax - 1;
+    if (R <= 0) return cudaSuccess;
+    const long long n = (long long)B * R * (d.C / 2);
+    const int blocks = (int)std::min<long long>((n + 255) / 256, 4096);
+    k_halo_add<<<blocks, 256, 0, st>>>(d_out, B, S, d.C, R, dhalo); note_launch();
     return cudaGetLastError();
 }
 

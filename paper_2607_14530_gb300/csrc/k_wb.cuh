@@ -113,13 +113,25 @@ __device__ __forceinline__ void taps_reg(const Dims& d, const ConvPtrs& cw, int 
 }
 
 // ring w[s] = out[t] for t - t0 = s (mod KW); prepares the run starting at t0, whose position in
-// its sequence is pos0: values before the sequence start are zero
+// its sequence is pos0: values before the sequence start come from the call's halo rows of the
+// sequence (the previous chunk's last outputs), or are zero without a halo
 template <int KW>
-__device__ __forceinline__ void ring_init(const uint16_t* out, int C, int c, bool act, long long t0,
-                                          int pos0, float2 (&w)[KW]) {
+__device__ __forceinline__ void ring_init(const Dims& d, const ConvPtrs& cw, const uint16_t* out, int c,
+                                          bool act, long long t0, int pos0, float2 (&w)[KW]) {
+    const int C = d.C, R = d.kapmax - 1;
+    const long long seq = (t0 - pos0) / d.S;
     w[0] = f2z();
 #pragma unroll
-    for (int i = 1; i < KW; ++i) w[KW - i] = (act && i <= pos0) ? ld2(out + (t0 - i) * C + c) : f2z();
+    for (int i = 1; i < KW; ++i) {
+        float2 v = f2z();
+        if (act && i <= pos0) {
+            v = ld2(out + (t0 - i) * C + c);
+        } else if (act && cw.halo != nullptr) {
+            const int r = R + pos0 - i;   // halo row of position pos0 - i < 0
+            if (r >= 0) v = ld2(cw.halo + (seq * R + r) * C + c);
+        }
+        w[KW - i] = v;
+    }
 }
 
 // g_j = sum_i tw[j][i] out[t - i], with out[t - i] at ring slot (U - i) mod KW
@@ -191,7 +203,7 @@ __global__ void __launch_bounds__(WT) k_wb_gram(Dims d, int slot, int T, int TB,
     const int nq = K * (K + 1) / 2;
     float2 tw[3][KW], w[KW];
     taps_reg<KW, KS>(d, cw, c, act, tw);
-    ring_init<KW>(out, C, c, act, t0, pos0, w);
+    ring_init<KW>(d, cw, out, c, act, t0, pos0, w);
     const uint16_t* po = out + t0 * C + c;
     // the out values of the next block of KW tokens are loaded while this block is processed
     uint32_t ob[KW];
@@ -308,7 +320,7 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
     float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
     if constexpr (KW > 0) {
         taps_reg<KW, KS>(d, cw, c, act, tw);
-        ring_init<KW>(out, C, c, act, t0, pos0, w);
+        ring_init<KW>(d, cw, out, c, act, t0, pos0, w);
     }
     uint16_t* pX = X + t0 * d.N * C + c;                              // token rows, advanced per token
     uint16_t* pn = last ? nullptr : xact_next + t0 * k * C + c;
@@ -452,7 +464,7 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
     float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
     if constexpr (KW > 0) {
         taps_reg<KW, KS>(d, cw, c, act, tw);
-        ring_init<KW>(out, C, c, act, t0, pos0, w);
+        ring_init<KW>(d, cw, out, c, act, t0, pos0, w);
     }
     const int RU = KW > 0 ? KW : 4;
     for (int tb = 0; tb < ntok; tb += RU) {
@@ -641,7 +653,7 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
     float2 acc[3][KW > 0 ? KW : 1];
     if constexpr (KW > 0) {
         taps_reg<KW, KS>(d, cw, c, act, tw);
-        ring_init<KW>(out, C, c, act, t0, pos0, w);
+        ring_init<KW>(d, cw, out, c, act, t0, pos0, w);
 #pragma unroll
         for (int s = 0; s < KW; ++s) pend[s] = f2z();
 #pragma unroll
@@ -738,6 +750,15 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
                                     const float2 o = w[(u - i + KW) % KW];
                                     acc[j][i] = ffma2(du[1 + j], o, acc[j][i]);
                                 }
+                        }
+                        // positions before the sequence start (a call on a later chunk of its
+                        // sequences): slot u held the complete gradient of halo position
+                        // u - KW, whose last term came from token u - 1
+                        if (cw.dhalo != nullptr && pos0 == 0 && tt >= 1 && tt < KW) {
+                            const int r = d.kapmax - 1 + tt - KW;
+                            if (r >= 0)
+                                *reinterpret_cast<float2*>(
+                                    cw.dhalo + (((t0 / d.S) * (d.kapmax - 1) + r) * C + c)) = pend[u];
                         }
                         // d_out[t - i] += w_j[i] du_{1+j}[t]
                         pend[u] = du[0];

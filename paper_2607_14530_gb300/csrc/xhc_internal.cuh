@@ -118,9 +118,14 @@ constexpr int NRED = 112;    // per-token reduction slots (>= k*K + k*k + K*K)
 constexpr int TOKMAT = 176;  // E[k][4] + D[4][4] + Hres[k][k] + dX_act mix + scalars (k<=8)
 constexpr int NTG = 208;     // per-token alpha/b gradient contributions
 
-// Conv taps of one MLP slot (by value into kernels): w[j] is [kappa_j, C].
+// Conv taps of one MLP slot (by value into kernels): w[j] is [kappa_j, C].  For a call on a
+// later chunk of its sequences (sequence split), halo [B][R][C] bf16 holds the R = max(kappa) - 1
+// sublayer outputs preceding each sequence of the call (null: none, zero padding as at a
+// sequence start) and dhalo [B][R][C] fp32 receives their gradient (backward apply only).
 struct ConvPtrs {
     const float* w[3];
+    const uint16_t* halo;
+    float* dhalo;
 };
 struct ConvGradPtrs {
     float* w[3];
@@ -285,6 +290,11 @@ cudaError_t launch_dec_fwd(const Dims& d, int slot, int B, const uint16_t* out, 
 cudaError_t launch_ring_fill(const Dims& d, int B, int S, const uint16_t* out, uint16_t* ring,
                              cudaStream_t st);
 int dec_nslice(int C);  // channel slices (partial Gram slots) of the decode Gram reduction
+// sequence split: the halo rows a chunk passes to the next, and the return of their gradient
+cudaError_t launch_halo_fill(const Dims& d, int B, int S, const uint16_t* out, uint16_t* halo,
+                             cudaStream_t st);
+cudaError_t launch_halo_add(const Dims& d, int B, int S, uint16_t* d_out, const float* dhalo,
+                            cudaStream_t st);
 cudaError_t launch_wb_gram(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
                            int nslice, float* red, cudaStream_t st);
 cudaError_t launch_wb_coef(const Dims& d, int slot, int T, const float* red, int nslice, const float* p,

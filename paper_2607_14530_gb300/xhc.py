@@ -81,6 +81,11 @@ def lib() -> ctypes.CDLL:
         L.xhc_ring_bytes.argtypes = [vp, i64, ctypes.POINTER(sz)]
         L.xhc_ring_fill.argtypes = [vp, i64, i64, vp, vp, vp]
         L.xhc_post_fwd_decode.argtypes = [vp, ctypes.c_int, i64, P, vp, vp, vp, vp, vp, vp, vp]
+        L.xhc_halo_bytes.argtypes = [vp, i64, ctypes.POINTER(sz)]
+        L.xhc_halo_fill.argtypes = [vp, i64, i64, vp, vp, vp]
+        L.xhc_halo_add.argtypes = [vp, i64, i64, vp, vp, vp]
+        L.xhc_post_fwd_halo.argtypes = [vp, ctypes.c_int, i64, P, vp, vp, vp, vp, vp, vp]
+        L.xhc_post_bwd_halo.argtypes = [vp, ctypes.c_int, i64, P, vp, vp, vp, vp, P, vp, vp, vp, vp, vp]
         L.xhc_workspace_error.argtypes = [vp, ctypes.POINTER(ctypes.c_int), ctypes.c_int]
         L.xhc_trace_enable.argtypes = [ctypes.c_int]
         L.xhc_trace_count.restype = ctypes.c_int
@@ -323,19 +328,58 @@ class Group:
         _check(lib().xhc_pre_fwd(self._h, slot, T, ctypes.byref(pp), _bf16(X, "X"), _bf16(inp, "input"),
                                  _ptr(saved), _ptr(ws), _stream(stream)), f"xhc_pre_fwd({slot})")
 
-    def post_fwd(self, slot, P, X, out, saved, ws, stream=None):
+    def post_fwd(self, slot, P, X, out, saved, ws, stream=None, halo=None):
+        """xhc_post_fwd; with ``halo`` (bf16 [B, R, C], see halo_fill) xhc_post_fwd_halo."""
         T = X.shape[0]
         pp = P if isinstance(P, _Params) else self.params(P)
-        _check(lib().xhc_post_fwd(self._h, slot, T, ctypes.byref(pp), _bf16(X, "X"), _bf16(out, "out"),
-                                  _ptr(saved), _ptr(ws), _stream(stream)), f"xhc_post_fwd({slot})")
+        if halo is None:
+            _check(lib().xhc_post_fwd(self._h, slot, T, ctypes.byref(pp), _bf16(X, "X"), _bf16(out, "out"),
+                                      _ptr(saved), _ptr(ws), _stream(stream)), f"xhc_post_fwd({slot})")
+        else:
+            _check(lib().xhc_post_fwd_halo(self._h, slot, T, ctypes.byref(pp), _bf16(X, "X"),
+                                           _bf16(out, "out"), _bf16(halo, "halo"), _ptr(saved), _ptr(ws),
+                                           _stream(stream)), f"xhc_post_fwd_halo({slot})")
 
-    def post_bwd(self, slot, P, X, dX, out, d_out, grads, saved, ws, stream=None):
+    def post_bwd(self, slot, P, X, dX, out, d_out, grads, saved, ws, stream=None, halo=None,
+                 d_halo=None):
+        """xhc_post_bwd; with ``halo`` xhc_post_bwd_halo, writing the halo's gradient into
+        ``d_halo`` (fp32 [B, R, C])."""
         T = X.shape[0]
         pp = P if isinstance(P, _Params) else self.params(P)
         gg = grads if isinstance(grads, _Params) else self.params(grads)
-        _check(lib().xhc_post_bwd(self._h, slot, T, ctypes.byref(pp), _bf16(X, "X"), _bf16(dX, "dX"),
-                                  _bf16(out, "out"), _bf16(d_out, "d_out"), ctypes.byref(gg),
-                                  _ptr(saved), _ptr(ws), _stream(stream)), f"xhc_post_bwd({slot})")
+        if halo is None:
+            _check(lib().xhc_post_bwd(self._h, slot, T, ctypes.byref(pp), _bf16(X, "X"), _bf16(dX, "dX"),
+                                      _bf16(out, "out"), _bf16(d_out, "d_out"), ctypes.byref(gg),
+                                      _ptr(saved), _ptr(ws), _stream(stream)), f"xhc_post_bwd({slot})")
+        else:
+            if d_halo is None or d_halo.dtype != torch.float32 or not d_halo.is_cuda or not d_halo.is_contiguous():
+                raise XhcError("d_halo must be a contiguous fp32 CUDA tensor")
+            _check(lib().xhc_post_bwd_halo(self._h, slot, T, ctypes.byref(pp), _bf16(X, "X"), _bf16(dX, "dX"),
+                                           _bf16(out, "out"), _bf16(d_out, "d_out"), ctypes.byref(gg),
+                                           _bf16(halo, "halo"), _ptr(d_halo), _ptr(saved), _ptr(ws),
+                                           _stream(stream)), f"xhc_post_bwd_halo({slot})")
+
+    # ---- sequence split: halo rows between consecutive chunks of the same sequences ----
+
+    def halo_rows(self) -> int:
+        """R = max(kappa) - 1 (0 without a conv)."""
+        return max(self.cfg.conv_k) - 1 if self.cfg.conv_k else 0
+
+    def halo_fill(self, B: int, S: int, out, halo=None, stream=None):
+        """The halo [B, R, C] bf16 that the next chunk of these B sequences (S tokens each here)
+        needs from this chunk's sublayer output ``out``."""
+        if halo is None:
+            halo = torch.empty(B, self.halo_rows(), self.cfg.C, dtype=torch.bfloat16, device=out.device)
+        _check(lib().xhc_halo_fill(self._h, B, S, _bf16(out, "out"), _bf16(halo, "halo"), _stream(stream)),
+               "xhc_halo_fill")
+        return halo
+
+    def halo_add(self, B: int, S: int, d_out, d_halo, stream=None):
+        """d_out of this chunk's last R tokens += the next chunk's d_halo (fp32 [B, R, C])."""
+        if d_halo.dtype != torch.float32 or not d_halo.is_cuda or not d_halo.is_contiguous():
+            raise XhcError("d_halo must be a contiguous fp32 CUDA tensor")
+        _check(lib().xhc_halo_add(self._h, B, S, _bf16(d_out, "d_out"), _ptr(d_halo), _stream(stream)),
+               "xhc_halo_add")
 
     def pre_bwd(self, slot, P, X, d_input, dX, grads, saved, ws, stream=None):
         T = X.shape[0]

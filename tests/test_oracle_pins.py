@@ -525,3 +525,48 @@ def test_softmax_router_scores_and_sparse_read_closed_forms():
     I = aux["I"]
     want = torch.einsum("tj,tjc->tc", aux["H_pre"][0].gather(1, I), X[torch.arange(T)[:, None], I])
     assert torch.allclose(ins[0], want, atol=1e-13, rtol=0)
+
+
+@pytest.mark.parametrize("cfg", [O.full(5, 3, 1, 8, True, conv_k=(2, 4)),
+                                 O.flash(5, 3, 1, 8, 4, conv_k=(2, 3, 4))], ids=["fullM", "flash4"])
+def test_sequence_split_with_halo_equals_unsplit(cfg):
+    """Cutting each sequence into two chunks: the second chunk's forward with the first chunk's
+    last R = max(kappa) - 1 outputs as its halo equals the unsplit forward on those tokens; in the
+    backward, the first chunk's d_out plus the second chunk's halo gradient equals the unsplit
+    d_out, and the parameter gradients of the chunks add up to the unsplit ones."""
+    B, S1, S2 = 2, 5, 4
+    S = S1 + S2
+    T = B * S
+    R = max(cfg.conv_k) - 1
+    P = _params(cfg, 41, alpha=0.3)
+    X, outs = _inputs(cfg, T, 41)
+    g = torch.Generator().manual_seed(42)
+    dXo = torch.randn(X.shape, generator=g, dtype=F64)
+    dins = [torch.randn(T, cfg.C, generator=g, dtype=F64) for _ in range(cfg.G)]
+    full = O.Config(**{**cfg.__dict__, "seq_len": S})
+    Xo, ins, _ = O.forward(full, P, X, outs, round_bf16=False)
+    dX, dout, dP = O.backward(full, P, X, outs, dXo, dins, round_bf16=False)
+
+    def rows(lo, hi):
+        return torch.cat([torch.arange(b * S + lo, b * S + hi) for b in range(B)])
+
+    r1, r2 = rows(0, S1), rows(S1, S)
+    c1 = O.Config(**{**cfg.__dict__, "seq_len": S1})
+    c2 = O.Config(**{**cfg.__dict__, "seq_len": S2})
+    halos = [outs[t].reshape(B, S, cfg.C)[:, S1 - R:S1] for t in range(cfg.G)]
+    X2o, ins2, _ = O.forward(c2, P, X[r2], [o[r2] for o in outs], round_bf16=False, halos=halos)
+    assert torch.allclose(X2o, Xo[r2], atol=1e-12, rtol=0)
+    for t in range(cfg.G):
+        assert torch.allclose(ins2[t], ins[t][r2], atol=1e-12, rtol=0)
+    dX1, dout1, dP1 = O.backward(c1, P, X[r1], [o[r1] for o in outs], dXo[r1], [d[r1] for d in dins],
+                                 round_bf16=False)
+    dX2, dout2, dP2, dh = O.backward(c2, P, X[r2], [o[r2] for o in outs], dXo[r2], [d[r2] for d in dins],
+                                     round_bf16=False, halos=halos)
+    assert torch.allclose(dX1, dX[r1], atol=1e-12, rtol=0) and torch.allclose(dX2, dX[r2], atol=1e-12, rtol=0)
+    for t in range(cfg.G):
+        d1 = dout1[t].reshape(B, S1, cfg.C).clone()
+        d1[:, S1 - R:] += dh[t]
+        assert torch.allclose(d1.reshape(-1, cfg.C), dout[t][r1], atol=1e-12, rtol=0)
+        assert torch.allclose(dout2[t], dout[t][r2], atol=1e-12, rtol=0)
+    for n in dP:
+        assert torch.allclose(dP1[n] + dP2[n], dP[n], atol=1e-11, rtol=1e-12), n
