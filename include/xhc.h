@@ -283,6 +283,19 @@ xhc_status xhc_post_bwd_halo(const xhc_handle* h, int slot, int64_t T, const xhc
 xhc_status xhc_halo_add(const xhc_handle* h, int64_t B, int64_t S, uint16_t* d_out,
                         const float* d_halo, void* stream);
 
+/* Model glue around a stack of groups (App. A, "Final Stream Reduction"):
+ * xhc_stream_expand: X[t][i] = hidden[t] for the N streams of every token ([T, C] -> [T, N, C]
+ *   bf16): the expanded state entering the first group (the paper does not state the
+ *   initialisation; N copies of the embedding output is the HC convention).  It is also the
+ *   backward of xhc_stream_sum (the gradient of a sum reaches every term).
+ * xhc_stream_sum: y[t] = sum_i X[t][i] ([T, N, C] -> [T, C], fp32 sum, bf16 store): the N
+ *   streams reduced to one hidden vector before the final RMSNorm and unembedding.  It is also
+ *   the backward of xhc_stream_expand.
+ * N and C come from the handle; same ownership and error rules as above. */
+xhc_status xhc_stream_expand(const xhc_handle* h, int64_t T, const uint16_t* hidden, uint16_t* X,
+                             void* stream);
+xhc_status xhc_stream_sum(const xhc_handle* h, int64_t T, const uint16_t* X, uint16_t* y, void* stream);
+
 /* Routing and pre-maps for callers that cannot allocate device memory.
  *
  * The paper has no counterpart: this is a deployment convenience.  Some callers cannot provide

@@ -311,7 +311,8 @@ def forward(cfg: Config, P: dict, X: torch.Tensor, outs: list, *, round_bf16: bo
     """One connection-op group: Alg. 1 (G = 1) or Alg. 2 / App. E.2 (G = 2, 4).
 
     X: [T, N, C] float64 holding the entry state; outs[t]: [T, C] float64, the caller's
-    sublayer output of slot t (out^(t) = F_t(input^(t)) in the paper; here an input of the op).
+    sublayer output of slot t (out^(t) = F_t(input^(t)) in the paper; here an input of the op),
+    or a callable F_t applied to the slot's input (to compose groups with sublayers, Alg. 1).
     Returns (X_out, inputs, aux): the state after the group, the G sublayer inputs, and a dict
     of intermediates (s, H_pre, I, p, H_post, H_res, the active state before every slot).
     ``halos[t]`` ([B, R, C] or None): for a call holding a later chunk of its sequences, the
@@ -363,10 +364,11 @@ def forward(cfg: Config, P: dict, X: torch.Tensor, outs: list, *, round_bf16: bo
 
         # Write-back components (Eq. aug + Eq. gs for MLP slots, out itself otherwise).
         hist = None if halos is None else halos[t]
+        o_t = outs[t](inputs[t]) if callable(outs[t]) else outs[t]
         if K > 1:
-            comps = augment(cfg, outs[t], [P[f"conv_w.{t}.{j}"] for j in range(len(cfg.conv_k))], T, hist)
+            comps = augment(cfg, o_t, [P[f"conv_w.{t}.{j}"] for j in range(len(cfg.conv_k))], T, hist)
         else:
-            comps = [outs[t]]
+            comps = [o_t]
         out_aug = torch.stack(comps, dim=1)                       # [T, K, C]
         delta = p[:, :, None] * torch.einsum("tjr,trc->tjc", H_post, out_aug)  # Eq. sparse_write_delta
 
@@ -380,7 +382,7 @@ def forward(cfg: Config, P: dict, X: torch.Tensor, outs: list, *, round_bf16: bo
         new = mixed + delta                                       # Eq. sparse_write
         if t < G - 1:
             # magnitudes of the terms of the next slot's active state (test bookkeeping only)
-            raw = [outs[t]] + ([causal_dwconv(outs[t], P[f"conv_w.{t}.{j}"], cfg.S(T), hist)
+            raw = [o_t] + ([causal_dwconv(o_t, P[f"conv_w.{t}.{j}"], cfg.S(T), hist)
                                 for j in range(len(cfg.conv_k))] if K > 1 else [])
             mu = sum(c.detach().abs() for c in raw)                   # [T, C]
             hp = (p.detach().abs() * H_post.detach().abs().sum(dim=2))  # [T, k]

@@ -682,6 +682,25 @@ xhc_status xhc_halo_add(const xhc_handle* h, int64_t B, int64_t S, uint16_t* d_o
     return XHC_OK;
 }
 
+xhc_status xhc_stream_expand(const xhc_handle* h, int64_t T, const uint16_t* hidden, uint16_t* X,
+                             void* stream) {
+    if (!h || !hidden || !X || T <= 0 || T > ((int64_t)1 << 30)) return XHC_ERR_INVALID_ARG;
+    if (!aligned16(hidden) || !aligned16(X)) return XHC_ERR_ALIGNMENT;
+    const Dims& d = h->h.d;
+    const cudaError_t e = launch_stream_bcast((int)T, d.N, d.C, hidden, X, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, __LINE__);
+    return XHC_OK;
+}
+
+xhc_status xhc_stream_sum(const xhc_handle* h, int64_t T, const uint16_t* X, uint16_t* y, void* stream) {
+    if (!h || !X || !y || T <= 0 || T > ((int64_t)1 << 30)) return XHC_ERR_INVALID_ARG;
+    if (!aligned16(X) || !aligned16(y)) return XHC_ERR_ALIGNMENT;
+    const Dims& d = h->h.d;
+    const cudaError_t e = launch_stream_sum((int)T, d.N, d.C, X, y, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, __LINE__);
+    return XHC_OK;
+}
+
 xhc_status xhc_ring_bytes(const xhc_handle* h, int64_t B, size_t* bytes) {
     if (!h || !bytes || B <= 0) return XHC_ERR_INVALID_ARG;
     const Dims& d = h->h.d;

@@ -399,4 +399,43 @@ cudaError_t launch_full_dots(const Dims& d, int T, const uint16_t* X, const uint
     return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------------------------------------
+// model glue: stream expansion and the final stream sum, one CTA per token, 16-byte accesses
+
+// X[t][i] = h[t] for every stream i (N copies; also the backward of the stream sum)
+__global__ void __launch_bounds__(256) k_stream_bcast(int T, int N, int C, const uint16_t* __restrict__ h,
+                                                      uint16_t* __restrict__ X) {
+    const long long t = blockIdx.x;
+    for (int c8 = threadIdx.x; c8 < C / 8; c8 += blockDim.x) {
+        const uint4 v = *reinterpret_cast<const uint4*>(h + t * C + c8 * 8);
+        for (int i = 0; i < N; ++i) *reinterpret_cast<uint4*>(X + (t * N + i) * C + c8 * 8) = v;
+    }
+}
+
+// y[t] = sum_i X[t][i] in fp32, stored bf16 (also the backward of the expansion)
+__global__ void __launch_bounds__(256) k_stream_sum(int T, int N, int C, const uint16_t* __restrict__ X,
+                                                    uint16_t* __restrict__ y) {
+    const long long t = blockIdx.x;
+    for (int c8 = threadIdx.x; c8 < C / 8; c8 += blockDim.x) {
+        float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        for (int i = 0; i < N; ++i) {
+            float x[8];
+            unpack8(*reinterpret_cast<const uint4*>(X + (t * N + i) * C + c8 * 8), x);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc[e] += x[e];
+        }
+        *reinterpret_cast<uint4*>(y + t * C + c8 * 8) = pack8(acc);
+    }
+}
+
+cudaError_t launch_stream_bcast(int T, int N, int C, const uint16_t* h, uint16_t* X, cudaStream_t st) {
+    k_stream_bcast<<<T, chunk_threads(C), 0, st>>>(T, N, C, h, X); note_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_stream_sum(int T, int N, int C, const uint16_t* X, uint16_t* y, cudaStream_t st) {
+    k_stream_sum<<<T, chunk_threads(C), 0, st>>>(T, N, C, X, y); note_launch();
+    return cudaGetLastError();
+}
+
 }  // namespace xhc

@@ -572,7 +572,10 @@ struct ARing {
     uint2 dn[PD][KM][WT];
 };
 
-template <int KM, int KW, int KS>
+// HALO: the variant for a call on a later chunk of its sequences, which also returns the
+// gradient of the halo rows (cw.dhalo); compiled only for the generic tap set (KS = 0), so the
+// common variants carry none of its registers
+template <int KM, int KW, int KS, bool HALO = false>
 __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int TB,
                                                    const uint16_t* __restrict__ out, ConvPtrs cw,
                                                    const uint16_t* __restrict__ dX,
@@ -661,7 +664,11 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
 #pragma unroll
             for (int i = 0; i < KW; ++i) acc[j][i] = f2z();
     }
+    // the halo gradient (a call on a later chunk): rows of this sequence, this channel pair
+    float* dhalo_row = (HALO && KW > 0 && cw.dhalo != nullptr && pos0 == 0)
+                           ? cw.dhalo + (t0 / d.S) * (d.kapmax - 1) * C + c : nullptr;
     for (int tb = 0; tb < nloop; tb += RU) {
+        const bool first_blk = HALO && (tb == 0) && dhalo_row != nullptr;
 #pragma unroll
         for (int u = 0; u < RU; ++u) {
             const int tt = tb + u;
@@ -752,13 +759,13 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
                                 }
                         }
                         // positions before the sequence start (a call on a later chunk of its
-                        // sequences): slot u held the complete gradient of halo position
-                        // u - KW, whose last term came from token u - 1
-                        if (cw.dhalo != nullptr && pos0 == 0 && tt >= 1 && tt < KW) {
-                            const int r = d.kapmax - 1 + tt - KW;
-                            if (r >= 0)
-                                *reinterpret_cast<float2*>(
-                                    cw.dhalo + (((t0 / d.S) * (d.kapmax - 1) + r) * C + c)) = pend[u];
+                        // sequences): in the first block of tokens, slot u held the complete
+                        // gradient of halo position u - KW, whose last term came from token u - 1
+                        if constexpr (HALO) {
+                            if (u >= 1 && first_blk) {
+                                const int r = d.kapmax - 1 + u - KW;
+                                if (r >= 0) *reinterpret_cast<float2*>(dhalo_row + (long long)r * C) = pend[u];
+                            }
                         }
                         // d_out[t - i] += w_j[i] du_{1+j}[t]
                         pend[u] = du[0];

@@ -290,6 +290,9 @@ cudaError_t launch_dec_fwd(const Dims& d, int slot, int B, const uint16_t* out, 
 cudaError_t launch_ring_fill(const Dims& d, int B, int S, const uint16_t* out, uint16_t* ring,
                              cudaStream_t st);
 int dec_nslice(int C);  // channel slices (partial Gram slots) of the decode Gram reduction
+// model glue: N copies of a hidden vector per token, and the sum of the N streams
+cudaError_t launch_stream_bcast(int T, int N, int C, const uint16_t* h, uint16_t* X, cudaStream_t st);
+cudaError_t launch_stream_sum(int T, int N, int C, const uint16_t* X, uint16_t* y, cudaStream_t st);
 // sequence split: the halo rows a chunk passes to the next, and the return of their gradient
 cudaError_t launch_halo_fill(const Dims& d, int B, int S, const uint16_t* out, uint16_t* halo,
                              cudaStream_t st);

@@ -81,6 +81,8 @@ def lib() -> ctypes.CDLL:
         L.xhc_ring_bytes.argtypes = [vp, i64, ctypes.POINTER(sz)]
         L.xhc_ring_fill.argtypes = [vp, i64, i64, vp, vp, vp]
         L.xhc_post_fwd_decode.argtypes = [vp, ctypes.c_int, i64, P, vp, vp, vp, vp, vp, vp, vp]
+        L.xhc_stream_expand.argtypes = [vp, i64, vp, vp, vp]
+        L.xhc_stream_sum.argtypes = [vp, i64, vp, vp, vp]
         L.xhc_halo_bytes.argtypes = [vp, i64, ctypes.POINTER(sz)]
         L.xhc_halo_fill.argtypes = [vp, i64, i64, vp, vp, vp]
         L.xhc_halo_add.argtypes = [vp, i64, i64, vp, vp, vp]
@@ -358,6 +360,26 @@ class Group:
                                            _bf16(out, "out"), _bf16(d_out, "d_out"), ctypes.byref(gg),
                                            _bf16(halo, "halo"), _ptr(d_halo), _ptr(saved), _ptr(ws),
                                            _stream(stream)), f"xhc_post_bwd_halo({slot})")
+
+    # ---- model glue ----
+
+    def stream_expand(self, hidden, X=None, stream=None):
+        """[T, C] -> [T, N, C]: N copies of every token's hidden vector (xhc_stream_expand)."""
+        T = hidden.shape[0]
+        if X is None:
+            X = torch.empty(T, self.cfg.N, self.cfg.C, dtype=torch.bfloat16, device=hidden.device)
+        _check(lib().xhc_stream_expand(self._h, T, _bf16(hidden, "hidden"), _bf16(X, "X"), _stream(stream)),
+               "xhc_stream_expand")
+        return X
+
+    def stream_sum(self, X, y=None, stream=None):
+        """[T, N, C] -> [T, C]: the sum of the N streams of every token (xhc_stream_sum)."""
+        T = X.shape[0]
+        if y is None:
+            y = torch.empty(T, self.cfg.C, dtype=torch.bfloat16, device=X.device)
+        _check(lib().xhc_stream_sum(self._h, T, _bf16(X, "X"), _bf16(y, "y"), _stream(stream)),
+               "xhc_stream_sum")
+        return y
 
     # ---- sequence split: halo rows between consecutive chunks of the same sequences ----
 

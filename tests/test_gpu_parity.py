@@ -51,6 +51,9 @@ CASES = {
     "fullA_sparse_read_m0": (Config.full(16, 4, 0, 256, False, sparse_read=True), 200, {}),
     "flash4_softmax_sparse": (Config.flash(16, 4, 2, 256, 4, seq_len=128, router="softmax",
                                            sparse_read=True), 256, {}),
+    # every active stream fixed (m = k < N): no router
+    "fullM_m_eq_k": (Config.full(8, 4, 4, 128, True, seq_len=64), 128, {}),
+    "flash4_m_eq_k": (Config.flash(8, 4, 4, 128, 4, seq_len=64), 128, {}),
 }
 
 

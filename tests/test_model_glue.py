@@ -1,0 +1,108 @@
+"""Autograd wiring of the model glue (paper_2607_14530_gb300.model) on CPU, with a stand-in for
+the library's calls: the slot order of the forward (pre_fwd(t), sublayer t, post_fwd(t)) and of
+the backward (post_bwd(t), the sublayer's backward, pre_bwd(t), in reverse slot order and reverse
+group order), and the gradients that reach the embedding, the sublayers' parameters and the
+group's parameters.  The stand-in's arithmetic is simple and mirrored by a plain-autograd
+re-implementation; the library's own arithmetic is checked on the GPU (tests/test_gpu_model.py)."""
+import torch
+from torch import nn
+
+from paper_2607_14530_gb300 import model as M
+from paper_2607_14530_gb300.xhc import Config
+
+
+class FakeGroup:
+    """pre_fwd: input = mean over streams; post_fwd: every stream += a * out (a = W_post.t[0,0]);
+    the backward calls are the exact reverses; bf16 storage as in the library."""
+
+    def __init__(self, cfg, log, tag):
+        self.cfg, self.log, self.tag = cfg, log, tag
+
+    def params(self, P):
+        return P
+
+    def alloc(self, T, device="cpu"):
+        return None, None
+
+    def stream_expand(self, h, X=None):
+        return h[:, None, :].expand(h.shape[0], self.cfg.N, h.shape[1]).contiguous()
+
+    def stream_sum(self, X, y=None):
+        return X.float().sum(1).to(torch.bfloat16)
+
+    def pre_fwd(self, t, P, X, inp, saved, ws):
+        self.log.append((self.tag, "pre_fwd", t))
+        inp.copy_(X.float().mean(1).to(torch.bfloat16))
+
+    def post_fwd(self, t, P, X, out, saved, ws):
+        self.log.append((self.tag, "post_fwd", t))
+        a = P[f"W_post.{t}"][0, 0]
+        X.copy_((X.float() + a * out.float()[:, None, :]).to(torch.bfloat16))
+
+    def post_bwd(self, t, P, X, dX, out, d_out, gg, saved, ws):
+        self.log.append((self.tag, "post_bwd", t))
+        a = P[f"W_post.{t}"][0, 0]
+        X.copy_((X.float() - a * out.float()[:, None, :]).to(torch.bfloat16))   # restore the entry state
+        d_out.copy_((a * dX.float().sum(1)).to(torch.bfloat16))
+        gg[f"W_post.{t}"][0, 0] += (dX.float().sum(1) * out.float()).sum()
+
+    def pre_bwd(self, t, P, X, d_in, dX, gg, saved, ws):
+        self.log.append((self.tag, "pre_bwd", t))
+        dX.copy_((dX.float() + d_in.float()[:, None, :] / self.cfg.N).to(torch.bfloat16))
+
+
+class Scale(nn.Module):
+    def __init__(self, v, log, tag):
+        super().__init__()
+        self.s = nn.Parameter(torch.tensor(float(v)))
+        self.log, self.tag = log, tag
+
+    def forward(self, x):
+        self.log.append((self.tag, "sublayer", 0))
+        y = x.float() * self.s
+        y.register_hook(lambda g: self.log.append((self.tag, "sublayer_bwd", 0)))
+        return y
+
+
+def test_group_chain_call_order_and_gradients():
+    cfg = Config.flash(4, 2, 1, 8, 2, seq_len=3)
+    log = []
+    stack = M.XhcStack(cfg, 2, lambda l, t: Scale(0.5 if t == 0 else 2.0, log, (l, t)))
+    for l, grp in enumerate(stack.groups):
+        grp.g = FakeGroup(cfg, log, l)
+        with torch.no_grad():
+            for t in range(cfg.G):
+                getattr(grp, f"W_post_{t}")[0, 0] = 0.25 * (1 + l + t)
+    T = 6
+    g = torch.Generator().manual_seed(0)
+    h = torch.randn(T, cfg.C, generator=g).to(torch.bfloat16).requires_grad_(True)
+    dy = torch.randn(T, cfg.C, generator=g)
+    y = stack(h)
+    (y.float() * dy).sum().backward()
+
+    # order: forward group by group, slot by slot; backward in reverse, sublayer backward between
+    fwd = [e for e in log if e[1] in ("pre_fwd", "post_fwd")]
+    assert fwd == [(l, k, t) for l in range(2) for t in range(2) for k in ("pre_fwd", "post_fwd")]
+    bwd = [e for e in log if e[1] in ("post_bwd", "pre_bwd", "sublayer_bwd")]
+    want = []
+    for l in (1, 0):
+        for t in (1, 0):
+            want += [(l, "post_bwd", t), ((l, t), "sublayer_bwd", 0), (l, "pre_bwd", t)]
+    assert bwd == want, bwd
+
+    # gradients against the same arithmetic written with plain autograd (fp32, bf16 storage
+    # treated as the identity, as the stand-in's backward does)
+    h2 = h.detach().float().requires_grad_(True)
+    a = [[torch.tensor(0.25 * (1 + l + t), requires_grad=True) for t in range(2)] for l in range(2)]
+    s = [[torch.tensor(0.5 if t == 0 else 2.0, requires_grad=True) for t in range(2)] for l in range(2)]
+    X = h2[:, None, :].expand(T, cfg.N, cfg.C)
+    for l in range(2):
+        for t in range(2):
+            out = X.mean(1) * s[l][t]
+            X = X + a[l][t] * out[:, None, :]
+    (X.sum(1) * dy).sum().backward()
+    assert torch.allclose(h.grad.float(), h2.grad, rtol=2e-2, atol=2e-2)
+    for l, grp in enumerate(stack.groups):
+        for t in range(2):
+            assert torch.allclose(grp.sublayers[t].s.grad, s[l][t].grad, rtol=2e-2), (l, t)
+            assert torch.allclose(getattr(grp, f"W_post_{t}").grad[0, 0], a[l][t].grad, rtol=2e-2), (l, t)
