@@ -65,7 +65,7 @@ typedef enum {
     XHC_ERR_UNSUPPORTED = 2, /* valid per the paper but outside the limits listed above     */
     XHC_ERR_ALIGNMENT = 3,   /* a pointer is not 16-byte aligned                            */
     XHC_ERR_CUDA = 4,        /* a CUDA launch or query failed                               */
-    XHC_ERR_TIMEOUT = 5      /* reserved: a bounded device-side wait gave up                */
+    XHC_ERR_TIMEOUT = 5      /* a bounded device-side wait gave up (xhc_workspace_error)    */
 } xhc_status;
 
 typedef enum {
@@ -326,11 +326,25 @@ xhc_status xhc_trace_enable(int on);
 int xhc_trace_count(void);
 xhc_status xhc_trace_record(int i, const char** name, float* ms);
 
-/* Device error word of a workspace: kernels with bounded waits (the tensor-core projection) set
- * it to a nonzero code instead of waiting forever, and return.  Synchronous (a device-to-host
- * copy).  *code receives the word; returns XHC_ERR_TIMEOUT if it is nonzero; clear != 0 resets
- * it.  A fresh workspace must be zeroed once before first use (e.g. cudaMemset). */
+/* Device error word of a workspace: kernels with bounded waits (the tensor-core kernels) set it
+ * to a nonzero code instead of waiting forever, and return; a launch whose wait gave up leaves
+ * its outputs undefined, and the CUDA context stays usable.  Synchronous (a device-to-host copy).
+ * *code receives the word (the number of the wait that gave up); returns XHC_ERR_TIMEOUT if it is
+ * nonzero; clear != 0 resets it.  A fresh workspace must be zeroed once before first use (e.g.
+ * cudaMemset). */
 xhc_status xhc_workspace_error(const void* workspace, int* code, int clear);
+
+/* Test hooks for the bounded waits (process-wide, host side; not for production use).
+ * XHC_DEBUG_WAIT_LIMIT_NS: the limit of every bounded device wait of later launches, in ns
+ *   (0 = the default of about 4 s).
+ * XHC_DEBUG_FORCE_TIMEOUT: value != 0 makes the next full-state projection launch (xhc_pre_fwd
+ *   of slot 0 on the tensor cores) wait, before it issues any copy or MMA, for a release that
+ *   nothing triggers, so that every wait of that launch runs out: it sets the workspace's error
+ *   word and returns without touching its outputs.  One-shot.
+ * Returns XHC_ERR_INVALID_ARG for an unknown `what` or a negative limit. */
+#define XHC_DEBUG_WAIT_LIMIT_NS 1
+#define XHC_DEBUG_FORCE_TIMEOUT 2
+xhc_status xhc_debug_set(int what, int64_t value);
 
 /* Number of kernels the library has launched since it was loaded. */
 uint64_t xhc_launch_count(void);

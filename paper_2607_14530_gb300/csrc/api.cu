@@ -15,6 +15,15 @@ namespace xhc {
 static std::atomic<unsigned long long> g_launches{0};
 void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
+// ---- test hooks -----------------------------------------------------------------------------
+static std::atomic<unsigned long long> g_wait_ns{0};   // 0: the default limit (~4 s)
+static std::atomic<int> g_force_timeout{0};
+uint64_t debug_wait_ns() {
+    const unsigned long long v = g_wait_ns.load();
+    return v ? (uint64_t)v : 4000000000ull;
+}
+int debug_take_force_timeout() { return g_force_timeout.exchange(0); }
+
 struct TraceRec {
     const char* name;
     cudaEvent_t a, b;
@@ -244,6 +253,19 @@ xhc_status xhc_trace_record(int i, const char** name, float* ms) {
 }
 
 uint64_t xhc_launch_count(void) { return (uint64_t)g_launches.load(); }
+
+xhc_status xhc_debug_set(int what, int64_t value) {
+    switch (what) {
+        case XHC_DEBUG_WAIT_LIMIT_NS:
+            if (value < 0) return XHC_ERR_INVALID_ARG;
+            g_wait_ns.store((unsigned long long)value);
+            return XHC_OK;
+        case XHC_DEBUG_FORCE_TIMEOUT:
+            g_force_timeout.store(value ? 1 : 0);
+            return XHC_OK;
+    }
+    return XHC_ERR_INVALID_ARG;
+}
 
 xhc_status xhc_workspace_error(const void* workspace, int* code, int clear) {
     if (!workspace || !code) return XHC_ERR_INVALID_ARG;

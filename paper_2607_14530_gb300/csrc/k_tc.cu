@@ -23,7 +23,7 @@ constexpr int BM = 128;        // tokens per tile (MMA M)
 constexpr int BK = 64;         // k-elements per stage (128 bytes of bf16 = one swizzle row)
 constexpr int MAXSTAGES = 8;
 constexpr int NTHREADS = 192;  // warp 0 TMA, warp 1 MMA + TMEM, warps 2..5 statistics + epilogue
-constexpr uint64_t WAIT_NS = 4000000000ull;  // give up a wait after ~4 s
+constexpr uint64_t WAIT_NS = 4000000000ull;  // give up a wait after ~4 s (default limit)
 // a waiting thread may be suspended up to this long per try (it resumes as soon as the phase
 // completes); fewer polls leave the shared-memory pipe to the TMA writes and the epilogues
 constexpr uint32_t WAIT_HINT_NS = 20000;
@@ -41,8 +41,8 @@ __device__ __forceinline__ void mbar_expect_tx(uint32_t a, uint32_t bytes) {
 __device__ __forceinline__ void mbar_arrive(uint32_t a) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(a) : "memory");
 }
-// Bounded wait on a phase of an mbarrier: false once ~4 s (global timer) have passed.
-__device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity) {
+// Bounded wait on a phase of an mbarrier: false once `limit` ns (global timer) have passed.
+__device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity, uint64_t limit) {
     uint64_t t0 = 0;
     for (uint32_t it = 0;; ++it) {
         uint32_t ok;
@@ -55,7 +55,7 @@ __device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity) {
             uint64_t now;
             asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(now));
             if (t0 == 0) t0 = now;
-            else if (now - t0 > WAIT_NS) return false;
+            else if (now - t0 > limit) return false;
         }
     }
 }
@@ -188,6 +188,8 @@ struct ProjTcArgs {
     int nseg;           // partial slots per tile
     int stages;         // smem ring depth
     int kps;            // k-blocks of 64 per stage (projections; 1 for the weight gradients)
+    uint64_t wait_ns;   // limit of every bounded wait
+    int force_timeout;  // test hook: wait for a release that nothing triggers (see below)
     float* part;        // [nseg][T][nfull]
     float* pstats;      // [nseg][T][2] row sums / sums of squares of A; null: not computed
     int* err;           // set to a nonzero code when a wait gives up
@@ -249,11 +251,19 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
     if (warp == 0) {
         // ---------------- TMA producer ----------------
         if (lane == 0) {
+            // test hook (xhc_debug_set, XHC_DEBUG_FORCE_TIMEOUT): before anything is issued, wait
+            // for the first release of stage 0, which needs the MMA of a load that was never
+            // issued.  The waits of every role then run out with no TMA load and no MMA in
+            // flight, and the kernel takes its abort path: error word set, TMEM freed, return.
+            if (a.force_timeout && g0 < g1 && !mbar_wait(smem_u32(&bars[STAGES]), 0u, a.wait_ns)) {
+                atomicExch(a.err, 6);
+                s_abort = 1;
+            }
             long long it = 0;
-            for (long long g = g0; g < g1; ++g, ++it) {
+            for (long long g = g0; g < g1 && !*(volatile int*)&s_abort; ++g, ++it) {
                 const int s = (int)(it % STAGES);
                 const uint32_t ph = (uint32_t)((it / STAGES) & 1);
-                if (it >= STAGES && !mbar_wait(smem_u32(&bars[STAGES + s]), ph ^ 1)) {
+                if (it >= STAGES && !mbar_wait(smem_u32(&bars[STAGES + s]), ph ^ 1, a.wait_ns)) {
                     atomicExch(a.err, 1);
                     s_abort = 1;
                     break;
@@ -289,7 +299,7 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                 const int m = (int)(g / a.KB);
                 const long long sub_end = (long long)m * a.KB + ((g - (long long)m * a.KB) / SUBG + 1) * SUBG;
                 const long long gend = min(min(g1, (long long)(m + 1) * a.KB), sub_end);
-                if (seg > 0 && !mbar_wait(smem_u32(&bars[2 * STAGES + 1]), (uint32_t)((seg - 1) & 1))) {
+                if (seg > 0 && !mbar_wait(smem_u32(&bars[2 * STAGES + 1]), (uint32_t)((seg - 1) & 1), a.wait_ns)) {
                     atomicExch(a.err, 2);
                     s_abort = 1;
                     break;
@@ -299,7 +309,7 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                 for (; g < gend; ++g, ++it) {
                     const int s = (int)(it % STAGES);
                     const uint32_t ph = (uint32_t)((it / STAGES) & 1);
-                    if (!mbar_wait(smem_u32(&bars[s]), ph)) {
+                    if (!mbar_wait(smem_u32(&bars[s]), ph, a.wait_ns)) {
                         atomicExch(a.err, 3);
                         s_abort = 1;
                         break;
@@ -355,7 +365,7 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
             for (; g < gend; ++g, ++it) {
                 const int s = (int)(it % STAGES);
                 const uint32_t ph = (uint32_t)((it / STAGES) & 1);
-                if (!mbar_wait(smem_u32(&bars[s]), ph)) {
+                if (!mbar_wait(smem_u32(&bars[s]), ph, a.wait_ns)) {
                     atomicExch(a.err, 4);
                     ok = false;
                     break;
@@ -391,7 +401,7 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
             while (c0 > 0 && range_start(a.W, a.P, c0) > (long long)m * a.KB) --c0;
             while (range_start(a.W, a.P, c0 + 1) <= (long long)m * a.KB) ++c0;
             const int j = c - c0;
-            if (!mbar_wait(smem_u32(&bars[2 * STAGES]), (uint32_t)(seg & 1))) {
+            if (!mbar_wait(smem_u32(&bars[2 * STAGES]), (uint32_t)(seg & 1), a.wait_ns)) {
                 atomicExch(a.err, 5);
                 break;
             }
@@ -587,6 +597,8 @@ cudaError_t launch_proj_tc(const uint16_t* X, int T, int K, const uint16_t* Wpac
     a.part = part;
     a.pstats = pstats;
     a.err = err;
+    a.wait_ns = debug_wait_ns();
+    a.force_timeout = debug_take_force_timeout();
     k_proj_tc<false><<<p.P, NTHREADS, sm, st>>>(ma, mb, a); note_launch();
     return cudaGetLastError();
 }
@@ -642,6 +654,8 @@ cudaError_t launch_wgrad_tc(const uint16_t* A, int T, int E, const float* dz, in
     a.part = part;
     a.pstats = nullptr;
     a.err = err;
+    a.wait_ns = debug_wait_ns();
+    a.force_timeout = 0;
     k_proj_tc<true><<<p.P, NTHREADS, sm, st>>>(ma, mb, a); note_launch();
     return cudaGetLastError();
 }
@@ -693,6 +707,7 @@ struct DxArgs {
     const float* scal;
     int scal_ld;
     int* err;
+    uint64_t wait_ns;     // limit of every bounded wait
 };
 
 // ACT = true (the instantiated form): active-state epilogue, "streams" are the k active slots j:
@@ -743,7 +758,7 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
                 const long long rest = tile / a.N;
                 const int ct = (int)(rest % a.CT), tt = (int)(rest / a.CT);
                 const int s = (int)(n & nsh);
-                if (n >= NS && !mbar_wait(smem_u32(&bars[2 + s]), (uint32_t)(((n >> nsh) - 1) & 1))) {
+                if (n >= NS && !mbar_wait(smem_u32(&bars[2 + s]), (uint32_t)(((n >> nsh) - 1) & 1), a.wait_ns)) {
                     atomicExch(a.err, 11);
                     break;
                 }
@@ -763,11 +778,11 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
             for (long long n = 0; n < nloc; ++n) {
                 const int s = (int)(n & 1);        // TMEM buffer
                 const int os = (int)(n & nsh);     // operand stage
-                if (!mbar_wait(smem_u32(&bars[os]), (uint32_t)((n >> nsh) & 1))) {
+                if (!mbar_wait(smem_u32(&bars[os]), (uint32_t)((n >> nsh) & 1), a.wait_ns)) {
                     atomicExch(a.err, 12);
                     break;
                 }
-                if (n >= 2 && !mbar_wait(smem_u32(&bars[6 + s]), (uint32_t)(((n >> 1) - 1) & 1))) {
+                if (n >= 2 && !mbar_wait(smem_u32(&bars[6 + s]), (uint32_t)(((n >> 1) - 1) & 1), a.wait_ns)) {
                     atomicExch(a.err, 13);
                     break;
                 }
@@ -866,7 +881,7 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
                 load_pass(0);
                 load_pass(1);
                 if (hh == 0) {
-                    if (!mbar_wait(smem_u32(&bars[4 + s]), (uint32_t)((n >> 1) & 1))) {
+                    if (!mbar_wait(smem_u32(&bars[4 + s]), (uint32_t)((n >> 1) & 1), a.wait_ns)) {
                         atomicExch(a.err, 14);
                         ok = false;
                         break;
@@ -1056,7 +1071,7 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
                 decode(n, p, tt, cb, i);
                 const long long blk = n / N;
                 if (p == 0) {
-                    if (blk >= 1 && !mbar_wait(smem_u32(&bars[1]), (uint32_t)((blk - 1) & 1))) {
+                    if (blk >= 1 && !mbar_wait(smem_u32(&bars[1]), (uint32_t)((blk - 1) & 1), a.wait_ns)) {
                         atomicExch(a.err, 31);
                         *s_abort = 1;
                         break;
@@ -1067,7 +1082,7 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
                         tma_load_2d(smem_u32(sA + kb * BM * BK * 2), &tmA, kb * BK, tt * BM, fa);
                 }
                 const int s = (int)(n & 1);
-                if (n >= 2 && !mbar_wait(smem_u32(&bars[4 + s]), (uint32_t)(((n >> 1) - 1) & 1))) {
+                if (n >= 2 && !mbar_wait(smem_u32(&bars[4 + s]), (uint32_t)(((n >> 1) - 1) & 1), a.wait_ns)) {
                     atomicExch(a.err, 32);
                     *s_abort = 1;
                     break;
@@ -1077,7 +1092,7 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
                 for (int kb = 0; kb < a.nkb; ++kb)
                     tma_load_2d(smem_u32(sB + s * B_BYTES + kb * DG_BN * BK * 2), &tmB, kb * BK,
                                 i * a.C + cb * DG_BN, fb);
-                if (n >= 2 && !mbar_wait(smem_u32(&bars[14 + s]), (uint32_t)(((n >> 1) - 1) & 1))) {
+                if (n >= 2 && !mbar_wait(smem_u32(&bars[14 + s]), (uint32_t)(((n >> 1) - 1) & 1), a.wait_ns)) {
                     atomicExch(a.err, 33);
                     *s_abort = 1;
                     break;
@@ -1089,7 +1104,7 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
                 tma_load_2d(smem_u32(xt), &tmX, i * a.C + cb * DG_BN, tt * BM, fe);
                 if (need_dx) tma_load_2d(smem_u32(xt + DG_TILE), &tmD, i * a.C + cb * DG_BN, tt * BM, fe);
                 if (p == 0) {
-                    if (blk >= 1 && !mbar_wait(smem_u32(&bars[7]), (uint32_t)((blk - 1) & 1))) {
+                    if (blk >= 1 && !mbar_wait(smem_u32(&bars[7]), (uint32_t)((blk - 1) & 1), a.wait_ns)) {
                         atomicExch(a.err, 34);
                         *s_abort = 1;
                         break;
@@ -1108,9 +1123,9 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
                 const long long blk = n / N;
                 const int p = (int)(n - blk * N);
                 const int s = (int)(n & 1);
-                bool ok = (p != 0) || mbar_wait(smem_u32(&bars[0]), (uint32_t)(blk & 1));
-                ok = ok && mbar_wait(smem_u32(&bars[2 + s]), (uint32_t)((n >> 1) & 1));
-                ok = ok && (n < 2 || mbar_wait(smem_u32(&bars[10 + s]), (uint32_t)(((n >> 1) - 1) & 1)));
+                bool ok = (p != 0) || mbar_wait(smem_u32(&bars[0]), (uint32_t)(blk & 1), a.wait_ns);
+                ok = ok && mbar_wait(smem_u32(&bars[2 + s]), (uint32_t)((n >> 1) & 1), a.wait_ns);
+                ok = ok && (n < 2 || mbar_wait(smem_u32(&bars[10 + s]), (uint32_t)(((n >> 1) - 1) & 1), a.wait_ns));
                 if (!ok) {
                     atomicExch(a.err, 35);
                     *s_abort = 1;
@@ -1174,9 +1189,9 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
                 }
             };
             prefetch(0, pfa);
-            bool ok = mbar_wait(smem_u32(&bars[12 + grp]), (uint32_t)((n >> 1) & 1));
-            ok = ok && mbar_wait(smem_u32(&bars[8 + grp]), (uint32_t)((n >> 1) & 1));
-            ok = ok && (!usesg || mbar_wait(smem_u32(&bars[6]), (uint32_t)(blk & 1)));
+            bool ok = mbar_wait(smem_u32(&bars[12 + grp]), (uint32_t)((n >> 1) & 1), a.wait_ns);
+            ok = ok && mbar_wait(smem_u32(&bars[8 + grp]), (uint32_t)((n >> 1) & 1), a.wait_ns);
+            ok = ok && (!usesg || mbar_wait(smem_u32(&bars[6]), (uint32_t)(blk & 1), a.wait_ns));
             if (!ok) {
                 atomicExch(a.err, 36);
                 *s_abort = 1;
@@ -1318,6 +1333,7 @@ cudaError_t launch_dxa_tc(const Dims& d, int slot, int T, const float* dzs, int 
     a.N = d.k;  // tile "streams" are the active slots
     a.NH = d.N;
     a.dinput = d_input; a.hpre = hpre; a.I = I; a.dxa = dxact; a.err = err;
+    a.wait_ns = debug_wait_ns();
     a.X = xact; a.scal = tokmat; a.scal_ld = TOKMAT;
     // one operand stage (the MMA of a tile is short next to its epilogue): the shared memory
     // left over is L1 for the epilogue's in-flight reads
@@ -1378,6 +1394,7 @@ cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, 
     a.P = (int)std::min<long long>(num_sms(), a.ntiles);
     a.X = X; a.dX = dX; a.dinput = dinput; a.hpre = hpre; a.I = I; a.dxact = dxact;
     a.scal = scal; a.scal_ld = scal_ld; a.err = err;
+    a.wait_ns = debug_wait_ns();
     const size_t sm = dxf_smem(n, d.G);
     e = cudaFuncSetAttribute((const void*)k_dxf_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;

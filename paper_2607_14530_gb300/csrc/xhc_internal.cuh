@@ -251,6 +251,10 @@ __device__ inline void gs_coef_bwd(const double (&G)[MAXCOMP][MAXCOMP], int K,
 // launch accounting and tracing (host side)
 
 void note_launch();  // counts every kernel launch of the library
+// test hooks (xhc_debug_set): the limit of the bounded device waits, and a one-shot request that
+// the next full-state projection time out before it issues any copy
+uint64_t debug_wait_ns();
+int debug_take_force_timeout();
 
 // ---------------------------------------------------------------------------------------------
 // launchers (each returns cudaGetLastError() after enqueueing)

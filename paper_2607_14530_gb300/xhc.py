@@ -89,6 +89,7 @@ def lib() -> ctypes.CDLL:
         L.xhc_post_fwd_halo.argtypes = [vp, ctypes.c_int, i64, P, vp, vp, vp, vp, vp, vp]
         L.xhc_post_bwd_halo.argtypes = [vp, ctypes.c_int, i64, P, vp, vp, vp, vp, P, vp, vp, vp, vp, vp]
         L.xhc_workspace_error.argtypes = [vp, ctypes.POINTER(ctypes.c_int), ctypes.c_int]
+        L.xhc_debug_set.argtypes = [ctypes.c_int, i64]
         L.xhc_trace_enable.argtypes = [ctypes.c_int]
         L.xhc_trace_count.restype = ctypes.c_int
         L.xhc_trace_record.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_char_p),
@@ -124,6 +125,18 @@ def trace_records() -> list:
         _check(L.xhc_trace_record(i, ctypes.byref(name), ctypes.byref(ms)), "xhc_trace_record")
         out.append((name.value.decode(), float(ms.value)))
     return out
+
+
+def debug_wait_limit_ns(ns: int) -> None:
+    """Limit of the library's bounded device waits for later launches (0: the default ~4 s).
+    A test hook (xhc_debug_set)."""
+    _check(lib().xhc_debug_set(1, int(ns)), "xhc_debug_set")
+
+
+def debug_force_timeout() -> None:
+    """Make the next tensor-core full-state projection time out before it issues any work (a
+    test hook for the bounded-wait abort path; xhc_debug_set)."""
+    _check(lib().xhc_debug_set(2, 1), "xhc_debug_set")
 
 
 def launch_count() -> int:

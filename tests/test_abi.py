@@ -157,3 +157,10 @@ def test_route_noalloc_rejects_oversized_T(L):
     addr = 0x7f0001000000
     st = L.xhc_route_noalloc(g._h, T, ctypes.byref(P), addr, addr, addr, addr, None)
     assert st == UNSUPPORTED
+
+
+def test_debug_hook_argument_checks(L):
+    assert L.xhc_debug_set(1, -5) == INVALID
+    assert L.xhc_debug_set(99, 0) == INVALID
+    assert L.xhc_debug_set(1, 0) == OK
+    assert L.xhc_debug_set(2, 0) == OK
