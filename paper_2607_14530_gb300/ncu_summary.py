@@ -16,7 +16,10 @@ DRAM traffic (``--metrics dram__bytes_read.sum,dram__bytes_write.sum --csv``)::
 writes, for every trace name NAME mapped to a kernel, the mean DRAM bytes (read + write) per
 launch of that kernel times S (the ratio of the benchmark's token count to the captured one:
 every kernel's traffic is linear in the tokens), tagged with the hash of the kernel sources, so
-that ``bench.py`` reports it only while the sources are unchanged.
+that ``bench.py`` reports it only while the sources are unchanged.  With ``--forward TOKENS``
+(the capture holding exactly one fwd+bwd step of TOKENS tokens, from its first launch) it also
+stores, under ``_forward``, the measured forward DRAM bytes per token of one group: the launches
+before the step's first ``k_restore`` (the backward's first kernel), divided by TOKENS.
 """
 from __future__ import annotations
 
@@ -89,6 +92,30 @@ def dram_bytes(path):
     return {n: sum(v) / len(v) for n, v in per.items()}
 
 
+def dram_launches(path):
+    """[(launch id, kernel, DRAM bytes read + written)] in launch order."""
+    unit_scale = {"byte": 1.0, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9, "Tbyte": 1e12}
+    per = {}
+    for r in _rows(path):
+        if r.get("Metric Name") not in ("dram__bytes_read.sum", "dram__bytes_write.sum"):
+            continue
+        v = float(r["Metric Value"].replace(",", "")) * unit_scale.get(r.get("Metric Unit", "byte"), 1.0)
+        key = (int(r["ID"]), kernel_base(r["Kernel Name"]))
+        per[key] = per.get(key, 0.0) + v
+    return [(i, n, v) for (i, n), v in sorted(per.items())]
+
+
+def forward_bytes(path):
+    """(DRAM bytes of the launches before the first k_restore, number of those launches)."""
+    tot, n = 0.0, 0
+    for _, name, v in dram_launches(path):
+        if name == "k_restore":
+            return tot, n
+        tot += v
+        n += 1
+    raise ValueError("no k_restore launch in the capture: it must hold a whole fwd+bwd step")
+
+
 def csrc_hash():
     h = hashlib.sha256()
     for f in sorted(glob.glob(os.path.join(ROOT, "paper_2607_14530_gb300", "csrc", "*"))):
@@ -115,6 +142,12 @@ def main(argv):
             if kern in per:
                 ent[name] = {"kernel": kern, "dram_bytes_per_launch": per[kern] * scale,
                              "captured_bytes_per_launch": per[kern], "scale": scale, "csrc_sha": sha}
+        if "--forward" in argv:
+            toks = int(argv[argv.index("--forward") + 1])
+            fb, nl = forward_bytes(path)
+            ent["_forward"] = {"dram_bytes_per_token": fb / toks, "captured_tokens": toks,
+                               "launches": nl, "csrc_sha": sha}
+            print(f"forward: {fb / 1e9:.4f} GB over {nl} launches = {fb / toks:.0f} bytes per token")
         with open(out, "w") as f:
             json.dump(d, f, indent=1, sort_keys=True)
         for n, v in sorted(per.items()):
