@@ -107,10 +107,16 @@ def kernel_model(cfg, T):
         dxn = xa if last else xa32
         if last:
             add("restore", 2 * xa)
-        add("wb_bred", row + dxn + (xa if last else 0))
+        if Ks[t] == 1:
+            # one pass: out, dXn (and x_act on the last slot) read; d_out and, on the last slot,
+            # the mixed active gradient written
+            add("wb_b8", row + dxn + (xa if last else 0) + row + (xa32 if last else 0))
+        else:
+            add("wb_bred", row + dxn + (xa if last else 0))
         add("bwd_coef", T * nact[t] * f32 * 2)
-        # out, dXn read; d_out written; last slot writes the mixed active gradient; conv partials
-        add("wb_bapp", row + dxn + row + (xa32 if last else 0) + (cpart if Ks[t] > 1 else 0))
+        if Ks[t] > 1:
+            # out, dXn read; d_out written; last slot writes the mixed active gradient; conv partials
+            add("wb_bapp", row + dxn + row + (xa32 if last else 0) + cpart)
         add("wgrad_tc_active", xa + T * nact[t] * f32 + 2 * T * nact[t] * b16 + k * C * nact[t] * f32,
             2.0 * T * k * C * 2 * nact[t], "hbm")
         add("wgrad_reduce", 2 * k * C * nact[t] * f32)

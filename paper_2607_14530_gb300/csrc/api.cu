@@ -800,8 +800,15 @@ xhc_status post_bwd_impl(const xhc_handle* h, int slot, int64_t T, const xhc_par
         XHC_K("restore", c.st, launch_restore(d, T32, c.xact(0), c.S<int>(c.L.I), X, c.st));
     }
     const int bslices = wb_bred_slices(d, slot);
-    XHC_K("wb_bred", c.st, launch_wb_bred(d, slot, T32, out, cw, dX, c.S<int>(c.L.I), dxact, c.xact(slot),
-                                          bslices, red, c.st));
+    if (K == 1) {
+        // no conv: reductions and apply in one pass (the apply coefficients are forward values)
+        XHC_K("wb_b8", c.st, launch_wb_b8(d, slot, T32, out, dX, c.S<int>(c.L.I), c.S<float>(c.L.p),
+                                          c.S<float>(c.L.hpost[slot]), c.S<float>(c.L.hres), dxact, dxact,
+                                          c.xact(slot), bslices, red, d_out, c.st));
+    } else {
+        XHC_K("wb_bred", c.st, launch_wb_bred(d, slot, T32, out, cw, dX, c.S<int>(c.L.I), dxact, c.xact(slot),
+                                              bslices, red, c.st));
+    }
     XHC_K("bwd_coef", c.st, launch_bwd_coef(d, slot, T32, red, bslices, c.S<float>(c.L.zact[slot]),
                              c.S<float>(c.L.rs[slot]), c.S<float>(c.L.p),
                              c.S<float>(c.L.hpost[slot]),
@@ -835,9 +842,10 @@ xhc_status post_bwd_impl(const xhc_handle* h, int slot, int64_t T, const xhc_par
     }
     // d_out, conv weight-gradient partials and (last slot) the mixed active gradient; the
     // active gradient of earlier slots is read in place and completed by pre_bwd(slot)
-    XHC_K("wb_bapp", c.st, launch_wb_bapp(d, slot, T32, out, cw, dX, c.S<int>(c.L.I), dxact,
-                                          c.W<float>(c.L.tokmat), dxact, d_out,
-                                          c.W<float>(c.L.cpart), c.st));
+    if (K > 1)
+        XHC_K("wb_bapp", c.st, launch_wb_bapp(d, slot, T32, out, cw, dX, c.S<int>(c.L.I), dxact,
+                                              c.W<float>(c.L.tokmat), dxact, d_out,
+                                              c.W<float>(c.L.cpart), c.st));
     const WSegs wa = act_segs(d, P, slot);
     // dZ_act stays in the workspace: pre_bwd(slot) applies it to dX_act on the tensor cores
     if (!dxa_tc_ok(T32, d.k, d.C, n))

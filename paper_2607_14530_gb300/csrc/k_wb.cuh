@@ -1133,6 +1133,178 @@ __global__ void __launch_bounds__(WT) k_wb_bapp8(Dims d, int slot, int T, int TB
     }
 }
 
+// Backward of a slot without conv (K = 1) in one pass: the apply coefficients of such a slot
+// are forward quantities (E[j][0] = p_j H_post[j], and on the last slot the forward H_res), so
+// the reductions P[j][0] = <dXn_j, out> (last slot: Q[j][i] = <dXn_j, x_i>) and the apply
+// d_out = sum_j E[j][0] dXn_j (last slot: dX_act_i = sum_j H_res[j][i] dXn_j) read dXn once.
+// Partial sums per W8-channel slice in the layout of k_wb_bred8.
+template <int KM>
+__global__ void __launch_bounds__(WT, 4) k_wb_b8(Dims d, int slot, int T, int TB,
+                                              const uint16_t* __restrict__ out,
+                                              const uint16_t* __restrict__ dX,
+                                              const int* __restrict__ I,
+                                              const float* __restrict__ p,
+                                              const float* __restrict__ hpost,
+                                              const float* __restrict__ hres,
+                                              const float* dxact,   // read (earlier slots)
+                                              float* dxact_out,     // written (last slot)
+                                              const uint16_t* __restrict__ xact, int nslice,
+                                              float* __restrict__ red,
+                                              uint16_t* __restrict__ d_out) {
+    constexpr int NQ = KM + KM * KM;                  // P[j][0], then Q[j][i]
+    constexpr int NV = NQ <= 32 ? 32 : 96;            // reduce-scatter width (blocks of 32)
+    extern __shared__ __align__(16) unsigned char smu[];
+    int* Ish = reinterpret_cast<int*>(smu);                  // [TB][KM]
+    float* Esh = reinterpret_cast<float*>(Ish + TB * KM);    // [TB][KM]
+    float* Hsh = Esh + TB * KM;                              // [TB][KM][KM] (last slot)
+    float* wsh = Hsh + TB * KM * KM;                         // [TB][WT/32][NV]
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int k = d.k, C = d.C;
+    const bool last = (slot == d.G - 1);
+    const long long t0 = (long long)blockIdx.y * TB;
+    const int ntok = (int)(min((long long)T, t0 + TB) - t0);
+    for (int idx = threadIdx.x; idx < ntok * KM; idx += WT) {
+        const int tt = idx / KM, j = idx - tt * KM;
+        const long long tj = (t0 + tt) * k + j;
+        Ish[idx] = (j < k) ? I[tj] : 0;
+        Esh[idx] = (j < k) ? p[tj] * hpost[tj] : 0.f;
+    }
+    if (last)
+        for (int idx = threadIdx.x; idx < ntok * KM * KM; idx += WT) {
+            const int tt = idx / (KM * KM), q = idx - tt * (KM * KM);
+            const int j = q / KM, i = q - j * KM;
+            Hsh[idx] = (j < k && i < k) ? hres[(t0 + tt) * k * k + j * k + i] : 0.f;
+        }
+    __syncthreads();
+    const int c = blockIdx.x * W8 + threadIdx.x * 8;
+    const bool act = c < C;
+    const long long kC = (long long)k * C, NC = (long long)d.N * C;
+    const uint16_t* po = out + t0 * C + c;
+    const uint16_t* px = xact + t0 * kC + c;
+    const uint16_t* pX = dX + t0 * NC + c;
+    const float* pd = dxact + t0 * kC + c;
+    // next token's rows: out, dXn_j (bf16 rows of dX, or fp32 active gradient), x_j (last)
+    uint4 on = make_uint4(0, 0, 0, 0), dn0[KM], dn1[KM], xn[KM];
+    auto load = [&](int tt) {
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            dn0[j] = make_uint4(0, 0, 0, 0);
+            dn1[j] = dn0[j];
+            xn[j] = dn0[j];
+        }
+        on = dn0[0];
+        if (!act || tt >= ntok) return;
+        on = ld16(po);
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            if (j >= k) continue;
+            if (last) {
+                dn0[j] = ld16(pX + (long long)Ish[tt * KM + j] * C);
+                xn[j] = ld16(px + j * (long long)C);
+            } else {
+                dn0[j] = ld16(pd + j * (long long)C);
+                dn1[j] = ld16(pd + j * (long long)C + 4);
+            }
+        }
+    };
+    load(0);
+    for (int tt = 0; tt < ntok; ++tt) {
+        const uint4 oc = on;
+        uint4 d0[KM], d1[KM], xc[KM];
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            d0[j] = dn0[j];
+            d1[j] = dn1[j];
+            xc[j] = xn[j];
+        }
+        po += C;
+        if (last) {
+            px += kC;
+            pX += NC;
+        } else {
+            pd += kC;
+        }
+        load(tt + 1);
+        const long long t = t0 + tt;
+        float o[8], dn[KM][8];
+        unpack8(oc, o);
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            if (last) {
+                unpack8(d0[j], dn[j]);
+            } else {
+                dn[j][0] = __uint_as_float(d0[j].x); dn[j][1] = __uint_as_float(d0[j].y);
+                dn[j][2] = __uint_as_float(d0[j].z); dn[j][3] = __uint_as_float(d0[j].w);
+                dn[j][4] = __uint_as_float(d1[j].x); dn[j][5] = __uint_as_float(d1[j].y);
+                dn[j][6] = __uint_as_float(d1[j].z); dn[j][7] = __uint_as_float(d1[j].w);
+            }
+        }
+        float v[NV];
+#pragma unroll
+        for (int q = 0; q < NV; ++q) v[q] = 0.f;
+#pragma unroll
+        for (int j = 0; j < KM; ++j)
+#pragma unroll
+            for (int q = 0; q < 8; ++q) v[j] = fmaf(dn[j][q], o[q], v[j]);
+        if (last) {
+            float x[KM][8];
+#pragma unroll
+            for (int i = 0; i < KM; ++i) unpack8(xc[i], x[i]);
+#pragma unroll
+            for (int j = 0; j < KM; ++j)
+#pragma unroll
+                for (int i = 0; i < KM; ++i)
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) v[KM + j * KM + i] = fmaf(dn[j][q], x[i][q], v[KM + j * KM + i]);
+        }
+        if (act) {
+            // apply: d_out = sum_j E[j][0] dXn_j, and the mixed active gradient of the last slot
+            float g[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) g[q] = 0.f;
+#pragma unroll
+            for (int j = 0; j < KM; ++j) {
+                const float e = Esh[tt * KM + j];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) g[q] = fmaf(e, dn[j][q], g[q]);
+            }
+            *reinterpret_cast<uint4*>(d_out + t * C + c) = pack8(g);
+            if (last) {
+#pragma unroll
+                for (int i = 0; i < KM; ++i) {
+                    if (i >= k) continue;
+                    float w[8];
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) {
+                        float a = 0.f;
+#pragma unroll
+                        for (int j = 0; j < KM; ++j) a = fmaf(Hsh[(tt * KM + j) * KM + i], dn[j][q], a);
+                        w[q] = a;
+                    }
+                    float4* dst = reinterpret_cast<float4*>(dxact_out + t * kC + (long long)i * C + c);
+                    dst[0] = make_float4(w[0], w[1], w[2], w[3]);
+                    dst[1] = make_float4(w[4], w[5], w[6], w[7]);
+                }
+            }
+        }
+        float tot[NV / 32];
+        wred32<NV / 32>(v, lane, tot);
+        float* dst = wsh + ((size_t)tt * (WT / 32) + warp) * NV;
+#pragma unroll
+        for (int bb = 0; bb < NV / 32; ++bb) dst[bb * 32 + lane] = tot[bb];
+    }
+    __syncthreads();
+    const int nq = last ? NQ : KM;
+    for (int idx = threadIdx.x; idx < ntok * nq; idx += WT) {
+        const int tt = idx / nq, q = idx - tt * nq;
+        float sm = 0.f;
+#pragma unroll
+        for (int ww = 0; ww < WT / 32; ++ww) sm += wsh[((size_t)tt * (WT / 32) + ww) * NV + q];
+        const int slotq = q < KM ? q * 4 : KM * 4 + (q - KM);
+        red[((t0 + tt) * nslice + blockIdx.x) * NRED + slotq] = sm;
+    }
+}
+
 inline int kw_of(const Dims& d) {
     const int km = d.kapmax;
     return km <= 4 ? 4 : km <= 8 ? 8 : km <= 12 ? 12 : 16;

@@ -33,6 +33,23 @@ cudaError_t bred8_kw(const Dims& d, int slot, int T, const uint16_t* out, const 
     return cudaGetLastError();
 }
 
+template <int KM>
+cudaError_t b8_kw(const Dims& d, int slot, int T, const uint16_t* out, const uint16_t* dX, const int* I,
+                  const float* p, const float* hpost, const float* hres, const float* dxact,
+                  float* dxact_out, const uint16_t* xact, int nslice, float* red, uint16_t* d_out,
+                  cudaStream_t st) {
+    constexpr int NQ = KM + KM * KM;
+    constexpr int NV = NQ <= 32 ? 32 : 96;
+    const int TB = 32;
+    const size_t sm = (size_t)TB * (2 * KM + KM * KM) * 4 + (size_t)TB * (WT / 32) * NV * 4;
+    cudaError_t e = smem_attr((const void*)k_wb_b8<KM>, sm);
+    if (e != cudaSuccess) return e;
+    dim3 grid((d.C + W8 - 1) / W8, (T + TB - 1) / TB);
+    k_wb_b8<KM><<<grid, WT, sm, st>>>(d, slot, T, TB, out, dX, I, p, hpost, hres, dxact, dxact_out, xact,
+                                      nslice, red, d_out); note_launch();
+    return cudaGetLastError();
+}
+
 }  // namespace
 
 // slices (partial sums per token) of the backward reductions of a slot
@@ -60,6 +77,17 @@ cudaError_t launch_wb_bred(const Dims& d, int slot, int T, const uint16_t* out, 
     if (last) XHC_BRED(8, 96, false);
     XHC_BRED(8, 32, false);
 #undef XHC_BRED
+}
+
+// backward reductions and apply of a slot without conv (K = 1), in one pass over dXn
+cudaError_t launch_wb_b8(const Dims& d, int slot, int T, const uint16_t* out, const uint16_t* dX,
+                         const int* I, const float* p, const float* hpost, const float* hres,
+                         const float* dxact, float* dxact_out, const uint16_t* xact, int nslice,
+                         float* red, uint16_t* d_out, cudaStream_t st) {
+    if (d.K[slot] != 1) return cudaErrorInvalidValue;
+    if (d.k <= 4)
+        return b8_kw<4>(d, slot, T, out, dX, I, p, hpost, hres, dxact, dxact_out, xact, nslice, red, d_out, st);
+    return b8_kw<8>(d, slot, T, out, dX, I, p, hpost, hres, dxact, dxact_out, xact, nslice, red, d_out, st);
 }
 
 }  // namespace xhc

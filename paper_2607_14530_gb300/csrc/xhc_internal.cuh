@@ -312,6 +312,10 @@ cudaError_t launch_wb_fwd(const Dims& d, int slot, int T, const uint16_t* out, C
 cudaError_t launch_wb_bred(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
                            const uint16_t* dX, const int* I, const float* dxact,
                            const uint16_t* xact, int nslice, float* red, cudaStream_t st);
+cudaError_t launch_wb_b8(const Dims& d, int slot, int T, const uint16_t* out, const uint16_t* dX,
+                         const int* I, const float* p, const float* hpost, const float* hres,
+                         const float* dxact, float* dxact_out, const uint16_t* xact, int nslice,
+                         float* red, uint16_t* d_out, cudaStream_t st);
 cudaError_t launch_wb_bapp(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
                            const uint16_t* dX, const int* I, const float* dn_in,
                            const float* tokmat, float* dxact_out, uint16_t* d_out, float* cpart,
