@@ -151,6 +151,56 @@ __device__ __forceinline__ void conv_ring(const float2 (&tw)[3][KW], const float
     }
 }
 
+// Block ring of the forward write-back, the backward reductions and the backward apply: the
+// token loop is unrolled by UB tokens only (a 12-token body does not fit the instruction cache),
+// and the ring holds the KW + UB - 1 values a block needs: for the block of tokens tb..tb+UB-1,
+// slot KW - 1 + u - i holds out[tb + u - i] (i < KW).  After a block the ring moves by UB slots.
+constexpr int UB = 4;
+
+template <int KW>
+__device__ __forceinline__ void ring_init_b(const Dims& d, const ConvPtrs& cw, const uint16_t* out, int c,
+                                            bool act, long long t0, int pos0, float2 (&w)[KW + UB - 1]) {
+    const int C = d.C, R = d.kapmax - 1;
+    const long long seq = (t0 - pos0) / d.S;
+#pragma unroll
+    for (int s = 0; s < KW + UB - 1; ++s) w[s] = f2z();
+#pragma unroll
+    for (int i = 1; i < KW; ++i) {
+        float2 v = f2z();
+        if (act && i <= pos0) {
+            v = ld2(out + (t0 - i) * C + c);
+        } else if (act && cw.halo != nullptr) {
+            const int r = R + pos0 - i;   // halo row of position pos0 - i < 0
+            if (r >= 0) v = ld2(cw.halo + (seq * R + r) * C + c);
+        }
+        w[KW - 1 - i] = v;
+    }
+}
+
+// g_j = sum_i tw[j][i] out[t - i] for token t = tb + u of the block
+template <int KW, int KS>
+__device__ __forceinline__ void conv_blk(const float2 (&tw)[3][KW], const float2 (&w)[KW + UB - 1], int u,
+                                         float2 (&g)[3]) {
+#pragma unroll
+    for (int j = 0; j < 3; ++j) g[j] = f2z();
+#pragma unroll
+    for (int i = 0; i < KW; ++i) {
+        const float2 o = w[KW - 1 + u - i];
+#pragma unroll
+        for (int j = 0; j < 3; ++j) {
+            if (i >= ntap<KW, KS>(j)) continue;
+            g[j] = ffma2(tw[j][i], o, g[j]);
+        }
+    }
+}
+
+// move a block ring on by UB tokens
+template <int KW>
+__device__ __forceinline__ void ring_shift(float2 (&w)[KW + UB - 1]) {
+#pragma unroll
+    for (int q = 0; q + 1 < KW; ++q) w[q] = w[q + UB];
+}
+
 // Reduce-scatter of V values (power of two, <= 32) over the warp: every lane returns the total
 // of value index lane >> (5 - log2 V).
 template <int V, int O>
@@ -317,16 +367,16 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
         const int tt = idx / KM, j = idx - tt * KM;
         Ish[idx] = (j < k) ? I[(t0 + tt) * k + j] : 0;
     }
-    float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
+    float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW + UB - 1 : 1];
     if constexpr (KW > 0) {
         taps_reg<KW, KS>(d, cw, c, act, tw);
-        ring_init<KW>(d, cw, out, c, act, t0, pos0, w);
+        ring_init_b<KW>(d, cw, out, c, act, t0, pos0, w);
     }
     uint16_t* pX = X + t0 * d.N * C + c;                              // token rows, advanced per token
     uint16_t* pn = last ? nullptr : xact_next + t0 * k * C + c;
     const long long NC = (long long)d.N * C;
     __syncthreads();
-    const int RU = KW > 0 ? KW : 4;
+    constexpr int RU = UB;
     for (int tb = 0; tb < ntok; tb += RU) {
 #pragma unroll
         for (int u = 0; u < RU; ++u) {
@@ -339,9 +389,9 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
                     const float2 o = u2f2(R.o[sl][threadIdx.x]);
                     float2 uu[4] = {o, f2z(), f2z(), f2z()};
                     if constexpr (KW > 0) {
-                        w[u] = o;
+                        w[KW - 1 + u] = o;
                         float2 g[3];
-                        conv_ring<KW, KS>(tw, w, u, g);
+                        conv_blk<KW, KS>(tw, w, u, g);
                         uu[1] = g[0];
                         uu[2] = g[1];
                         uu[3] = g[2];
@@ -385,6 +435,7 @@ __global__ void __launch_bounds__(WT) k_wb_fwd(Dims d, int slot, int T, int TB,
                 else pn += kC;
             }
         }
+        if constexpr (KW > 0) ring_shift<KW>(w);
     }
     cpa_wait<0>();
 }
@@ -461,12 +512,12 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
     };
 #pragma unroll
     for (int q = 0; q < PD - 1; ++q) issue(q, q);
-    float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1];
+    float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW + UB - 1 : 1];
     if constexpr (KW > 0) {
         taps_reg<KW, KS>(d, cw, c, act, tw);
-        ring_init<KW>(d, cw, out, c, act, t0, pos0, w);
+        ring_init_b<KW>(d, cw, out, c, act, t0, pos0, w);
     }
-    const int RU = KW > 0 ? KW : 4;
+    constexpr int RU = UB;
     for (int tb = 0; tb < ntok; tb += RU) {
 #pragma unroll
         for (int u = 0; u < RU; ++u) {
@@ -486,9 +537,9 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
                     const float2 o = u2f2(R.o[sl][threadIdx.x]);
                     uu[0] = o;
                     if constexpr (KW > 0) {
-                        w[u] = o;
+                        w[KW - 1 + u] = o;
                         float2 g[3];
-                        conv_ring<KW, KS>(tw, w, u, g);
+                        conv_blk<KW, KS>(tw, w, u, g);
                         uu[1] = g[0];
                         uu[2] = g[1];
                         uu[3] = g[2];
@@ -542,6 +593,7 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
                 }
             }
         }
+        if constexpr (KW > 0) ring_shift<KW>(w);
     }
     cpa_wait<0>();
     __syncthreads();
@@ -586,7 +638,8 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
                                                    uint16_t* __restrict__ d_out,
                                                    float* __restrict__ cpart) {
     constexpr int HL = KW > 0 ? KW - 1 : 0;   // tokens after the run whose du the run needs
-    constexpr int RU = KW > 0 ? KW : 4;
+    constexpr int RU = UB;
+    constexpr int NR = KW > 0 ? KW + UB - 1 : 1;   // block ring slots
     extern __shared__ __align__(16) unsigned char smu[];
     ARing<KM>& R = *reinterpret_cast<ARing<KM>*>(smu);
     const int k = (KS == 2) ? KM : d.k, C = d.C;
@@ -652,13 +705,14 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
     };
 #pragma unroll
     for (int q = 0; q < PD - 1; ++q) issue(q, q);
-    float2 tw[3][KW > 0 ? KW : 1], w[KW > 0 ? KW : 1], pend[KW > 0 ? KW : 1];
+    // pend: the block ring of pending outputs, slot KW - 1 + u - i <-> output tb + u - i
+    float2 tw[3][KW > 0 ? KW : 1], w[NR], pend[NR];
     float2 acc[3][KW > 0 ? KW : 1];
     if constexpr (KW > 0) {
         taps_reg<KW, KS>(d, cw, c, act, tw);
-        ring_init<KW>(d, cw, out, c, act, t0, pos0, w);
+        ring_init_b<KW>(d, cw, out, c, act, t0, pos0, w);
 #pragma unroll
-        for (int s = 0; s < KW; ++s) pend[s] = f2z();
+        for (int s = 0; s < NR; ++s) pend[s] = f2z();
 #pragma unroll
         for (int j = 0; j < 3; ++j)
 #pragma unroll
@@ -668,7 +722,6 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
     float* dhalo_row = (HALO && KW > 0 && cw.dhalo != nullptr && pos0 == 0)
                            ? cw.dhalo + (t0 / d.S) * (d.kapmax - 1) * C + c : nullptr;
     for (int tb = 0; tb < nloop; tb += RU) {
-        const bool first_blk = HALO && (tb == 0) && dhalo_row != nullptr;
 #pragma unroll
         for (int u = 0; u < RU; ++u) {
             const int tt = tb + u;
@@ -702,9 +755,9 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
                             }
                         }
                         if constexpr (KW > 0) {
-                            w[u] = o;
+                            w[KW - 1 + u] = o;
                             float2 g[3];
-                            conv_ring<KW, KS>(tw, w, u, g);
+                            conv_blk<KW, KS>(tw, w, u, g);
                             const float2 uu[4] = {o, g[0], g[1], g[2]};
                             const float4* D4 = reinterpret_cast<const float4*>(Dsh + tt * 16);
 #pragma unroll
@@ -739,7 +792,7 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
                             pxo += kC;
                         }
                     } else if constexpr (KW > 0) {
-                        w[u] = f2z();   // past the sequence end
+                        w[KW - 1 + u] = f2z();   // past the sequence end
                     }
                     if constexpr (KW == 0) {
                         if (tt < n1) {
@@ -754,38 +807,47 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
 #pragma unroll
                                 for (int i = 0; i < KW; ++i) {
                                     if (i >= ntap<KW, KS>(j)) continue;
-                                    const float2 o = w[(u - i + KW) % KW];
+                                    const float2 o = w[KW - 1 + u - i];
                                     acc[j][i] = ffma2(du[1 + j], o, acc[j][i]);
                                 }
                         }
-                        // positions before the sequence start (a call on a later chunk of its
-                        // sequences): in the first block of tokens, slot u held the complete
-                        // gradient of halo position u - KW, whose last term came from token u - 1
-                        if constexpr (HALO) {
-                            if (u >= 1 && first_blk) {
-                                const int r = d.kapmax - 1 + u - KW;
-                                if (r >= 0) *reinterpret_cast<float2*>(dhalo_row + (long long)r * C) = pend[u];
-                            }
-                        }
                         // d_out[t - i] += w_j[i] du_{1+j}[t]
-                        pend[u] = du[0];
+                        pend[KW - 1 + u] = du[0];
 #pragma unroll
                         for (int i = 0; i < KW; ++i) {
 #pragma unroll
                             for (int j = 0; j < 3; ++j) {
                                 if (i >= ntap<KW, KS>(j)) continue;
-                                float2& q = pend[(u - i + KW) % KW];
+                                float2& q = pend[KW - 1 + u - i];
                                 q = ffma2(tw[j][i], du[1 + j], q);
                             }
-                        }
-                        // token tt - (KW - 1) has all its terms (du is zero past the sequence end)
-                        if (tt >= KW - 1) {
-                            st2(pdo, pend[(u + 1) % KW]);
-                            pdo += C;
                         }
                     }
                 }
             }
+        }
+        if constexpr (KW > 0) {
+            // outputs tb + q - (KW - 1), q < UB, have all their terms (du is zero past the
+            // sequence end): stored in order; positions before the run start are the halo rows
+            // of a call on a later chunk of its sequences
+            if (act) {
+#pragma unroll
+                for (int q = 0; q < UB; ++q) {
+                    const int ot = tb + q - (KW - 1);
+                    if (ot >= 0) {
+                        if (ot < n1) {
+                            st2(pdo, pend[q]);
+                            pdo += C;
+                        }
+                    } else if constexpr (HALO) {
+                        const int r = d.kapmax - 1 + ot;
+                        if (dhalo_row != nullptr && r >= 0)
+                            *reinterpret_cast<float2*>(dhalo_row + (long long)r * C) = pend[q];
+                    }
+                }
+            }
+            ring_shift<KW>(w);
+            ring_shift<KW>(pend);
         }
     }
     cpa_wait<0>();
