@@ -23,7 +23,6 @@ constexpr int BM = 128;        // tokens per tile (MMA M)
 constexpr int BK = 64;         // k-elements per stage (128 bytes of bf16 = one swizzle row)
 constexpr int MAXSTAGES = 8;
 constexpr int NTHREADS = 192;  // warp 0 TMA, warp 1 MMA + TMEM, warps 2..5 statistics + epilogue
-constexpr uint64_t WAIT_NS = 4000000000ull;  // give up a wait after ~4 s (default limit)
 // a waiting thread may be suspended up to this long per try (it resumes as soon as the phase
 // completes); fewer polls leave the shared-memory pipe to the TMA writes and the epilogues
 constexpr uint32_t WAIT_HINT_NS = 20000;
