@@ -1,9 +1,11 @@
 // Write-back kernels of the connection op with the causal conv held in registers.
 //
 // Every kernel here walks a run of consecutive tokens for one pair of channels per thread.  The
-// conv taps of the pair and a ring of the last KW values of `out` stay in registers; the token
-// loop is unrolled by KW so the ring positions are compile-time constants, and each out value
-// is loaded once per run instead of once per tap.  Runs never cross a sequence boundary (Sec.
+// conv taps of the pair and a ring of the recent values of `out` stay in registers, indexed by
+// compile-time positions: wb_gram unrolls the token loop by KW over a KW-slot ring; the forward
+// apply and the backward kernels unroll it by 4-token blocks over a ring of KW + 3 slots that
+// moves by 4 after each block (a shorter loop body: the 12-token one overflowed the instruction
+// cache).  Each out value is loaded once per run instead of once per tap.  Runs never cross a sequence boundary (Sec.
 // 3.3.4: the conv restarts with every sequence), so the conv needs no per-tap test.  KS = 1
 // specialises the tap counts to the (4, 8, 12) kernels of the MLP sublayers, so no FMA is spent
 // on zero taps.  Per-token reductions over the channels use a reduce-scatter butterfly inside
@@ -17,6 +19,8 @@
 //   wb_bapp   component gradients du_a consumed on the fly: d_out = du_0 + conv^T(du_1..r)
 //             (emitted KW - 1 tokens late), conv weight-gradient partials, and on the last slot
 //             the mixed active-state gradient H_res^T dXn
+//   wb_fwd8, wb_b8   the same for slots without conv (K = 1), 8 channels per thread; wb_b8 does
+//             the backward reductions and apply in one pass
 #pragma once
 #include "xhc_internal.cuh"
 
@@ -964,242 +968,12 @@ __global__ void __launch_bounds__(WT) k_wb_fwd8(Dims d, int slot, int T, int TB,
     }
 }
 
-// backward reductions: P[j][0] = <dXn_j, out> (and, last slot, Q[j][i] = <dXn_j, x_i>), one
-// partial per W8-channel slice
-template <int KM>
-__global__ void __launch_bounds__(WT, 4) k_wb_bred8(Dims d, int slot, int T, int TB,
-                                                 const uint16_t* __restrict__ out,
-                                                 const uint16_t* __restrict__ dX,
-                                                 const int* __restrict__ I,
-                                                 const float* __restrict__ dxact,
-                                                 const uint16_t* __restrict__ xact, int nslice,
-                                                 float* __restrict__ red) {
-    constexpr int NQ = KM + KM * KM;                  // P[j][0], then Q[j][i]
-    constexpr int NV = NQ <= 32 ? 32 : 96;            // reduce-scatter width (blocks of 32)
-    extern __shared__ __align__(16) unsigned char smu[];
-    int* Ish = reinterpret_cast<int*>(smu);           // [TB][KM]
-    float* wsh = reinterpret_cast<float*>(Ish + TB * KM);   // [TB][WT/32][NV]
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int k = d.k, C = d.C;
-    const bool last = (slot == d.G - 1);
-    const long long t0 = (long long)blockIdx.y * TB;
-    const int ntok = (int)(min((long long)T, t0 + TB) - t0);
-    for (int idx = threadIdx.x; idx < ntok * KM; idx += WT) {
-        const int tt = idx / KM, j = idx - tt * KM;
-        Ish[idx] = (j < k) ? I[(t0 + tt) * k + j] : 0;
-    }
-    __syncthreads();
-    const int c = blockIdx.x * W8 + threadIdx.x * 8;
-    const bool act = c < C;
-    const long long kC = (long long)k * C, NC = (long long)d.N * C;
-    const uint16_t* po = out + t0 * C + c;
-    const uint16_t* px = xact + t0 * kC + c;
-    const uint16_t* pX = dX + t0 * NC + c;
-    const float* pd = dxact + t0 * kC + c;
-    // next token's rows: out, dXn_j (bf16 rows of dX, or fp32 active gradient), x_j (last)
-    uint4 on = make_uint4(0, 0, 0, 0), dn0[KM], dn1[KM], xn[KM];
-    auto load = [&](int tt) {
-#pragma unroll
-        for (int j = 0; j < KM; ++j) {
-            dn0[j] = make_uint4(0, 0, 0, 0);
-            dn1[j] = dn0[j];
-            xn[j] = dn0[j];
-        }
-        on = dn0[0];
-        if (!act || tt >= ntok) return;
-        on = ld16(po);
-#pragma unroll
-        for (int j = 0; j < KM; ++j) {
-            if (j >= k) continue;
-            if (last) {
-                dn0[j] = ld16(pX + (long long)Ish[tt * KM + j] * C);
-                xn[j] = ld16(px + j * (long long)C);
-            } else {
-                dn0[j] = ld16(pd + j * (long long)C);
-                dn1[j] = ld16(pd + j * (long long)C + 4);
-            }
-        }
-    };
-    load(0);
-    for (int tt = 0; tt < ntok; ++tt) {
-        const uint4 oc = on;
-        uint4 d0[KM], d1[KM], xc[KM];
-#pragma unroll
-        for (int j = 0; j < KM; ++j) {
-            d0[j] = dn0[j];
-            d1[j] = dn1[j];
-            xc[j] = xn[j];
-        }
-        po += C;
-        if (last) {
-            px += kC;
-            pX += NC;
-        } else {
-            pd += kC;
-        }
-        load(tt + 1);
-        float o[8], dn[KM][8];
-        unpack8(oc, o);
-#pragma unroll
-        for (int j = 0; j < KM; ++j) {
-            if (last) {
-                unpack8(d0[j], dn[j]);
-            } else {
-                dn[j][0] = __uint_as_float(d0[j].x); dn[j][1] = __uint_as_float(d0[j].y);
-                dn[j][2] = __uint_as_float(d0[j].z); dn[j][3] = __uint_as_float(d0[j].w);
-                dn[j][4] = __uint_as_float(d1[j].x); dn[j][5] = __uint_as_float(d1[j].y);
-                dn[j][6] = __uint_as_float(d1[j].z); dn[j][7] = __uint_as_float(d1[j].w);
-            }
-        }
-        float v[NV];
-#pragma unroll
-        for (int q = 0; q < NV; ++q) v[q] = 0.f;
-#pragma unroll
-        for (int j = 0; j < KM; ++j)
-#pragma unroll
-            for (int q = 0; q < 8; ++q) v[j] = fmaf(dn[j][q], o[q], v[j]);
-        if (last) {
-            float x[KM][8];
-#pragma unroll
-            for (int i = 0; i < KM; ++i) unpack8(xc[i], x[i]);
-#pragma unroll
-            for (int j = 0; j < KM; ++j)
-#pragma unroll
-                for (int i = 0; i < KM; ++i)
-#pragma unroll
-                    for (int q = 0; q < 8; ++q) v[KM + j * KM + i] = fmaf(dn[j][q], x[i][q], v[KM + j * KM + i]);
-        }
-        float tot[NV / 32];
-        wred32<NV / 32>(v, lane, tot);
-        float* dst = wsh + ((size_t)tt * (WT / 32) + warp) * NV;
-#pragma unroll
-        for (int bb = 0; bb < NV / 32; ++bb) dst[bb * 32 + lane] = tot[bb];
-    }
-    __syncthreads();
-    // red layout of the reverse maps: P[j][a] at j*4 + a, Q[j][i] at KM*4 + j*KM + i
-    const int nq = last ? NQ : KM;
-    for (int idx = threadIdx.x; idx < ntok * nq; idx += WT) {
-        const int tt = idx / nq, q = idx - tt * nq;
-        float sm = 0.f;
-#pragma unroll
-        for (int ww = 0; ww < WT / 32; ++ww) sm += wsh[((size_t)tt * (WT / 32) + ww) * NV + q];
-        const int slotq = q < KM ? q * 4 : KM * 4 + (q - KM);
-        red[((t0 + tt) * nslice + blockIdx.x) * NRED + slotq] = sm;
-    }
-}
-
-// backward apply: d_out = sum_j E[j][0] dXn_j; last slot: dX_act_i = sum_j H_res[j][i] dXn_j
-template <int KM>
-__global__ void __launch_bounds__(WT) k_wb_bapp8(Dims d, int slot, int T, int TB,
-                                                 const uint16_t* __restrict__ dX,
-                                                 const int* __restrict__ I,
-                                                 const float* dn_in,  // may alias dxact_out
-                                                 const float* __restrict__ tokmat,
-                                                 float* dxact_out,
-                                                 uint16_t* __restrict__ d_out) {
-    extern __shared__ __align__(16) unsigned char smu[];
-    float* Esh = reinterpret_cast<float*>(smu);        // [TB][KM]
-    float* Hsh = Esh + TB * KM;                        // [TB][KM][KM]
-    int* Ish = reinterpret_cast<int*>(Hsh + TB * KM * KM);
-    const int k = d.k, C = d.C;
-    const bool last = (slot == d.G - 1);
-    const long long t0 = (long long)blockIdx.y * TB;
-    const int ntok = (int)(min((long long)T, t0 + TB) - t0);
-    for (int idx = threadIdx.x; idx < ntok * KM; idx += WT) {
-        const int tt = idx / KM, j = idx - tt * KM;
-        Esh[idx] = (j < k) ? tokmat[(t0 + tt) * TOKMAT + j * 4] : 0.f;
-        Ish[idx] = (last && j < k) ? I[(t0 + tt) * k + j] : 0;
-    }
-    if (last)
-        for (int idx = threadIdx.x; idx < ntok * KM * KM; idx += WT) {
-            const int tt = idx / (KM * KM), q = idx - tt * (KM * KM);
-            const int j = q / KM, i = q - j * KM;
-            Hsh[idx] = (j < k && i < k) ? tokmat[(t0 + tt) * TOKMAT + 48 + j * 8 + i] : 0.f;
-        }
-    __syncthreads();
-    const int c = blockIdx.x * W8 + threadIdx.x * 8;
-    if (c >= C) return;
-    const long long kC = (long long)k * C, NC = (long long)d.N * C;
-    const uint16_t* pX = dX + t0 * NC + c;
-    const float* pd = dn_in + t0 * kC + c;
-    uint4 dn0[KM], dn1[KM];
-    auto load = [&](int tt) {
-#pragma unroll
-        for (int j = 0; j < KM; ++j) {
-            dn0[j] = make_uint4(0, 0, 0, 0);
-            dn1[j] = dn0[j];
-        }
-        if (tt >= ntok) return;
-#pragma unroll
-        for (int j = 0; j < KM; ++j) {
-            if (j >= k) continue;
-            if (last) {
-                dn0[j] = ld16(pX + (long long)Ish[tt * KM + j] * C);
-            } else {
-                dn0[j] = ld16(pd + j * (long long)C);
-                dn1[j] = ld16(pd + j * (long long)C + 4);
-            }
-        }
-    };
-    load(0);
-    for (int tt = 0; tt < ntok; ++tt) {
-        uint4 d0[KM], d1[KM];
-#pragma unroll
-        for (int j = 0; j < KM; ++j) {
-            d0[j] = dn0[j];
-            d1[j] = dn1[j];
-        }
-        if (last) pX += NC;
-        else pd += kC;
-        load(tt + 1);
-        const long long t = t0 + tt;
-        float dn[KM][8];
-#pragma unroll
-        for (int j = 0; j < KM; ++j) {
-            if (last) {
-                unpack8(d0[j], dn[j]);
-            } else {
-                dn[j][0] = __uint_as_float(d0[j].x); dn[j][1] = __uint_as_float(d0[j].y);
-                dn[j][2] = __uint_as_float(d0[j].z); dn[j][3] = __uint_as_float(d0[j].w);
-                dn[j][4] = __uint_as_float(d1[j].x); dn[j][5] = __uint_as_float(d1[j].y);
-                dn[j][6] = __uint_as_float(d1[j].z); dn[j][7] = __uint_as_float(d1[j].w);
-            }
-        }
-        float g[8];
-#pragma unroll
-        for (int q = 0; q < 8; ++q) g[q] = 0.f;
-#pragma unroll
-        for (int j = 0; j < KM; ++j) {
-            const float e = Esh[tt * KM + j];
-#pragma unroll
-            for (int q = 0; q < 8; ++q) g[q] = fmaf(e, dn[j][q], g[q]);
-        }
-        *reinterpret_cast<uint4*>(d_out + t * C + c) = pack8(g);
-        if (last) {
-#pragma unroll
-            for (int i = 0; i < KM; ++i) {
-                if (i >= k) continue;
-                float v[8];
-#pragma unroll
-                for (int q = 0; q < 8; ++q) {
-                    float a = 0.f;
-#pragma unroll
-                    for (int j = 0; j < KM; ++j) a = fmaf(Hsh[(tt * KM + j) * KM + i], dn[j][q], a);
-                    v[q] = a;
-                }
-                float4* dst = reinterpret_cast<float4*>(dxact_out + t * kC + (long long)i * C + c);
-                dst[0] = make_float4(v[0], v[1], v[2], v[3]);
-                dst[1] = make_float4(v[4], v[5], v[6], v[7]);
-            }
-        }
-    }
-}
-
 // Backward of a slot without conv (K = 1) in one pass: the apply coefficients of such a slot
 // are forward quantities (E[j][0] = p_j H_post[j], and on the last slot the forward H_res), so
 // the reductions P[j][0] = <dXn_j, out> (last slot: Q[j][i] = <dXn_j, x_i>) and the apply
 // d_out = sum_j E[j][0] dXn_j (last slot: dX_act_i = sum_j H_res[j][i] dXn_j) read dXn once.
-// Partial sums per W8-channel slice in the layout of k_wb_bred8.
+// Partial sums per W8-channel slice: P[j][0] at j*4, Q[j][i] at KM*4 + j*KM + i (the layout
+// bwd_coef reads).
 template <int KM>
 __global__ void __launch_bounds__(WT, 4) k_wb_b8(Dims d, int slot, int T, int TB,
                                               const uint16_t* __restrict__ out,

@@ -32,16 +32,6 @@ cudaError_t bapp_halo(const Dims& d, int slot, int T, const uint16_t* out, ConvP
     }
 }
 
-template <int KM>
-cudaError_t bapp8_kw(const Dims& d, int slot, int T, const uint16_t* dX, const int* I, const float* dn_in,
-                     const float* tokmat, float* dxact_out, uint16_t* d_out, cudaStream_t st) {
-    const int TB = 32;
-    const size_t sm = (size_t)TB * (KM + KM * KM + KM) * 4;
-    dim3 grid((d.C + W8 - 1) / W8, (T + TB - 1) / TB);
-    k_wb_bapp8<KM><<<grid, WT, sm, st>>>(d, slot, T, TB, dX, I, dn_in, tokmat, dxact_out, d_out); note_launch();
-    return cudaGetLastError();
-}
-
 }  // namespace
 
 cudaError_t launch_wb_bapp(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
@@ -54,11 +44,11 @@ cudaError_t launch_wb_bapp(const Dims& d, int slot, int T, const uint16_t* out, 
         if (d.k <= 4) return bapp_halo<4>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st);
         return bapp_halo<8>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st);
     }
+    // a slot without conv takes the one-pass backward (launch_wb_b8), not this kernel
+    if (!conv) return cudaErrorInvalidValue;
     if (d.k <= 4) {
-        if (!conv) return bapp8_kw<4>(d, slot, T, dX, I, dn_in, tokmat, dxact_out, d_out, st);
         XHC_KW_DISPATCH(d, wb_fast(d), (bapp_kw<4, KWC, KSC>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st)));
     }
-    if (!conv) return bapp8_kw<8>(d, slot, T, dX, I, dn_in, tokmat, dxact_out, d_out, st);
     XHC_KW_DISPATCH(d, false, (bapp_kw<8, KWC, KSC>(d, slot, T, out, cw, dX, I, dn_in, tokmat, dxact_out, d_out, cpart, nslice, st)));
 }
 

@@ -20,20 +20,6 @@ cudaError_t bred_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtr
 }
 
 template <int KM>
-cudaError_t bred8_kw(const Dims& d, int slot, int T, const uint16_t* out, const uint16_t* dX, const int* I,
-                     const float* dxact, const uint16_t* xact, int nslice, float* red, cudaStream_t st) {
-    constexpr int NQ = KM + KM * KM;
-    constexpr int NV = NQ <= 32 ? 32 : 96;
-    const int TB = 32;
-    const size_t sm = (size_t)TB * KM * 4 + (size_t)TB * (WT / 32) * NV * 4;
-    cudaError_t e = smem_attr((const void*)k_wb_bred8<KM>, sm);
-    if (e != cudaSuccess) return e;
-    dim3 grid((d.C + W8 - 1) / W8, (T + TB - 1) / TB);
-    k_wb_bred8<KM><<<grid, WT, sm, st>>>(d, slot, T, TB, out, dX, I, dxact, xact, nslice, red); note_launch();
-    return cudaGetLastError();
-}
-
-template <int KM>
 cudaError_t b8_kw(const Dims& d, int slot, int T, const uint16_t* out, const uint16_t* dX, const int* I,
                   const float* p, const float* hpost, const float* hres, const float* dxact,
                   float* dxact_out, const uint16_t* xact, int nslice, float* red, uint16_t* d_out,
@@ -62,10 +48,8 @@ cudaError_t launch_wb_bred(const Dims& d, int slot, int T, const uint16_t* out, 
                            const uint16_t* xact, int nslice, float* red, cudaStream_t st) {
     const bool conv = d.K[slot] > 1;
     const bool last = (slot == d.G - 1);
-    if (!conv) {
-        if (d.k <= 4) return bred8_kw<4>(d, slot, T, out, dX, I, dxact, xact, nslice, red, st);
-        return bred8_kw<8>(d, slot, T, out, dX, I, dxact, xact, nslice, red, st);
-    }
+    // a slot without conv takes the one-pass backward (launch_wb_b8), not this kernel
+    if (!conv) return cudaErrorInvalidValue;
 #define XHC_BRED(KM_, NV_, FAST_)                                                                   \
     do {                                                                                            \
         XHC_KW_DISPATCH(d, FAST_, (bred_kw<KM_, KWC, NV_, KSC>(d, slot, T, out, cw, dX, I, dxact, xact, nslice, red, st))); \
