@@ -80,7 +80,7 @@ def kernel_model(cfg, T):
     row = T * C * b16
     kw = max(cfg.conv_k) if cfg.conv_k else 0
     kw = 0 if kw == 0 else (4 if kw <= 4 else 8 if kw <= 8 else 12 if kw <= 12 else 16)
-    tb = (240 // kw) * kw if kw else 0
+    tb = 296 if kw else 0  # tokens per run of the backward apply (bapp_run)
     runs = (T // S) * -(-S // tb) + -(-(T % S) // tb) if kw else 0
     cpart = runs * sum(cfg.conv_k) * C * f32
     # forward

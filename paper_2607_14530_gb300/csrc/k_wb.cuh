@@ -1166,7 +1166,9 @@ inline long long n_runs(const Dims& d, int T, int TB, bool conv) {
 }
 
 // tokens per run of the backward apply (longer runs amortise the KW - 1 recomputed tokens)
-inline int bapp_run(int KW) { return KW > 0 ? run_len(KW, 240) : 64; }
+// tokens per run of the backward apply (with a conv: any length works with the block ring; 296
+// measured best at S = 4096, C = 4096 among 240 / 256 / 296 — fewer, fuller waves of CTAs)
+inline int bapp_run(int KW) { return KW > 0 ? 296 : 64; }
 
 inline cudaError_t smem_attr(const void* fn, size_t bytes) {
     if (bytes <= 48 * 1024) return cudaSuccess;

@@ -4,7 +4,7 @@ The xHC-Flash-4sub group N=16 k=4 m=2 C=4096 runs on T=32768 tokens (8 sequences
 the inputs bench.py draws (same generators, same seed), through the same Group calls.  The fp64
 oracle cannot run the whole step, so it is checked on windows of L tokens it can compute on its
 own: at the start of a sequence, in the middle of one (across a 128-token tile boundary), across
-the boundaries of the write-back kernels' token runs (60 / 96 / 240 tokens), and the last tokens
+the boundaries of the write-back kernels' token runs (32 / 60 / 64 / 128 / 296 tokens), and the last tokens
 of the last sequence (the last tile).  In the full-state projection every token tile is cut by a
 stream-K segment boundary (about 860 of its 1024 k-blocks per CTA), so every window covers those
 too.
@@ -39,9 +39,10 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 L = 40           # compared tokens per window
 SEED = 1234      # bench.py's seed on rank 0
 # (sequence, first token inside the sequence): start; middle across a 128-token tile boundary
-# (2048); across a boundary of every write-back run length (480 = 8 x 60 = 5 x 96 = 2 x 240); the
-# last L tokens of T
-WINDOWS = [(0, 0), (2, 2030), (5, 470), (7, 4096 - L)]
+# (2048); across a boundary of every write-back run length (888 = 3 x 296 for the backward apply,
+# 896 = 7 x 128 = 14 x 64 = 28 x 32 for the forward apply, the backward reductions and the
+# conv-free kernels, 900 = 15 x 60 for the Gram kernel); the last L tokens of T
+WINDOWS = [(0, 0), (2, 2030), (5, 870), (7, 4096 - L)]
 
 
 def _workload():
