@@ -63,6 +63,9 @@ __device__ __forceinline__ void cpa4(void* dst, const void* src) {
 __device__ __forceinline__ void cpa8(void* dst, const void* src) {
     asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(s_u32(dst)), "l"(src) : "memory");
 }
+__device__ __forceinline__ void cpa16(void* dst, const void* src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(s_u32(dst)), "l"(src) : "memory");
+}
 __device__ __forceinline__ void cpa_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 template <int N>
 __device__ __forceinline__ void cpa_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
@@ -604,6 +607,166 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
     for (int idx = threadIdx.x; idx < ntok * nv; idx += WT) {
         const int tt = idx / nv, q = idx - tt * nv;
         if (KW == 0 && NV == 16 && (q & 3) != 0) continue;  // entries without terms (K = 1)
+        float sm = 0.f;
+#pragma unroll
+        for (int ww = 0; ww < WT / 32; ++ww) sm += wsh[((size_t)tt * (WT / 32) + ww) * NVP + q];
+        red[((t0 + tt) * nslice + slice) * NRED + q] = sm;
+    }
+}
+
+// The same reductions with two channel pairs per thread (4 consecutive channels, WSL2 channels
+// per CTA): a token's warp reduction then covers 128 channels instead of 64, halving its cost
+// per channel, and the loads are 8 / 16 bytes wide.  For the (4, 8, 12) tap set with k = KM
+// and C a multiple of WSL2 (every thread in range).
+constexpr int WSL2 = 4 * WT;
+
+template <int KM>
+struct BRing2 {
+    uint2 o[PD][WT];
+    uint2 x[PD][KM][WT];
+    uint4 dn[PD][KM][WT];
+};
+
+template <int KM, int NV>
+__global__ void __launch_bounds__(WT, 2) k_wb_bred2(Dims d, int slot, int T, int TB,
+                                                    const uint16_t* __restrict__ out, ConvPtrs cw,
+                                                    const uint16_t* __restrict__ dX,
+                                                    const int* __restrict__ I,
+                                                    const float* __restrict__ dxact,
+                                                    const uint16_t* __restrict__ xact, int nslice,
+                                                    float* __restrict__ red) {
+    constexpr int KW = 12, KS = 2;
+    static_assert(NV == 16 || NV % 32 == 0, "reduction width");
+    constexpr int NVP = NV < 32 ? 16 : NV;
+    extern __shared__ __align__(16) unsigned char smu[];
+    BRing2<KM>& R = *reinterpret_cast<BRing2<KM>*>(smu);
+    int* Ish = reinterpret_cast<int*>(smu + sizeof(BRing2<KM>));         // [TB][KM]
+    float* wsh = reinterpret_cast<float*>(Ish + TB * KM);                 // [TB][WT/32][NVP]
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int slice = blockIdx.x, C = d.C, k = KM;
+    const bool last = (slot == d.G - 1);
+    const int nv = last ? KM * 4 + KM * KM : KM * 4;
+    const int c = slice * WSL2 + 4 * threadIdx.x;
+    long long t0, t1, send;
+    int pos0;
+    run_bounds<KW>(d, T, TB, t0, t1, send, pos0);
+    const int ntok = (int)(t1 - t0);
+    for (int q = threadIdx.x; q < ntok * KM; q += WT) {
+        const int tt = q / KM, j = q - tt * KM;
+        Ish[q] = I[(t0 + tt) * k + j];
+    }
+    __syncthreads();
+    const uint16_t* po = out + t0 * C + c;
+    const uint16_t* px = xact + t0 * k * C + c;
+    const uint16_t* pX = dX + t0 * d.N * C + c;
+    const float* pd = dxact + t0 * k * C + c;
+    const long long kC = (long long)k * C, NC = (long long)d.N * C;
+    auto issue = [&](int sl, int tn) {
+        if (tn < ntok) {
+            cpa8(&R.o[sl][threadIdx.x], po);
+#pragma unroll
+            for (int j = 0; j < KM; ++j) {
+                if (last) {
+                    cpa8(&R.x[sl][j][threadIdx.x], px + (long long)j * C);
+                    cpa8(&R.dn[sl][j][threadIdx.x], pX + (long long)Ish[tn * KM + j] * C);
+                } else {
+                    cpa16(&R.dn[sl][j][threadIdx.x], pd + (long long)j * C);
+                }
+            }
+        }
+        po += C;
+        if (last) {
+            px += kC;
+            pX += NC;
+        } else {
+            pd += kC;
+        }
+        cpa_commit();
+    };
+#pragma unroll
+    for (int q = 0; q < PD - 1; ++q) issue(q, q);
+    float2 tw[2][3][KW], w[2][KW + UB - 1];
+#pragma unroll
+    for (int p = 0; p < 2; ++p) {
+        taps_reg<KW, KS>(d, cw, c + 2 * p, true, tw[p]);
+        ring_init_b<KW>(d, cw, out, c + 2 * p, true, t0, pos0, w[p]);
+    }
+    for (int tb = 0; tb < ntok; tb += UB) {
+#pragma unroll
+        for (int u = 0; u < UB; ++u) {
+            const int tt = tb + u;
+            if (tt < ntok) {
+                const int sl = u % PD;
+                issue((u + PD - 1) % PD, tt + PD - 1);
+                cpa_wait<PD - 1>();
+                float2 uu[2][4], dn[2][KM], x[2][KM];
+                const uint2 orow = R.o[sl][threadIdx.x];
+#pragma unroll
+                for (int p = 0; p < 2; ++p) {
+                    const float2 o = u2f2(p == 0 ? orow.x : orow.y);
+                    w[p][KW - 1 + u] = o;
+                    float2 g[3];
+                    conv_blk<KW, KS>(tw[p], w[p], u, g);
+                    uu[p][0] = o;
+                    uu[p][1] = g[0];
+                    uu[p][2] = g[1];
+                    uu[p][3] = g[2];
+                }
+#pragma unroll
+                for (int j = 0; j < KM; ++j) {
+                    const uint4 r = R.dn[sl][j][threadIdx.x];
+                    if (last) {
+                        const uint2 rb = *reinterpret_cast<const uint2*>(&r);
+                        dn[0][j] = u2f2(rb.x);
+                        dn[1][j] = u2f2(rb.y);
+                        const uint2 xr = R.x[sl][j][threadIdx.x];
+                        x[0][j] = u2f2(xr.x);
+                        x[1][j] = u2f2(xr.y);
+                    } else {
+                        dn[0][j] = make_float2(__uint_as_float(r.x), __uint_as_float(r.y));
+                        dn[1][j] = make_float2(__uint_as_float(r.z), __uint_as_float(r.w));
+                        x[0][j] = x[1][j] = f2z();
+                    }
+                }
+                float v[NVP];
+#pragma unroll
+                for (int q = 0; q < NVP; ++q) v[q] = 0.f;
+#pragma unroll
+                for (int j = 0; j < KM; ++j)
+#pragma unroll
+                    for (int a = 0; a < 4; ++a)
+                        if (j * 4 + a < NVP)
+                            v[j * 4 + a] = fmaf(dn[1][j].y, uu[1][a].y,
+                                                fmaf(dn[1][j].x, uu[1][a].x, dot2(dn[0][j], uu[0][a])));
+                if constexpr (NVP >= KM * 4 + KM * KM) {
+                    if (last) {
+#pragma unroll
+                        for (int j = 0; j < KM; ++j)
+#pragma unroll
+                            for (int i = 0; i < KM; ++i)
+                                v[KM * 4 + j * KM + i] = fmaf(dn[1][j].y, x[1][i].y,
+                                                              fmaf(dn[1][j].x, x[1][i].x, dot2(dn[0][j], x[0][i])));
+                    }
+                }
+                float* dst = wsh + ((size_t)tt * (WT / 32) + warp) * NVP;
+                if constexpr (NV == 16) {
+                    const float tot = WRed<16, 16>::run(v, lane);
+                    if ((lane & 1) == 0) dst[lane >> 1] = tot;
+                } else {
+                    float tot[NV / 32];
+                    wred32<NV / 32>(v, lane, tot);
+#pragma unroll
+                    for (int bb = 0; bb < NV / 32; ++bb) dst[bb * 32 + lane] = tot[bb];
+                }
+            }
+        }
+#pragma unroll
+        for (int p = 0; p < 2; ++p) ring_shift<KW>(w[p]);
+    }
+    cpa_wait<0>();
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < ntok * nv; idx += WT) {
+        const int tt = idx / nv, q = idx - tt * nv;
         float sm = 0.f;
 #pragma unroll
         for (int ww = 0; ww < WT / 32; ++ww) sm += wsh[((size_t)tt * (WT / 32) + ww) * NVP + q];

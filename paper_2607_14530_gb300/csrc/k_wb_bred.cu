@@ -19,6 +19,23 @@ cudaError_t bred_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtr
     return cudaGetLastError();
 }
 
+template <int KM, int NV>
+cudaError_t bred2_kw(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw, const uint16_t* dX,
+                     const int* I, const float* dxact, const uint16_t* xact, int nslice, float* red,
+                     cudaStream_t st) {
+    constexpr int NVP = NV < 32 ? 16 : NV;
+    const int TB = 64;
+    const size_t sm = sizeof(BRing2<KM>) + (size_t)TB * KM * 4 + (size_t)TB * (WT / 32) * NVP * sizeof(float);
+    cudaError_t e = smem_attr((const void*)k_wb_bred2<KM, NV>, sm);
+    if (e != cudaSuccess) return e;
+    dim3 grid(d.C / WSL2, (unsigned)n_runs(d, T, TB, true));
+    k_wb_bred2<KM, NV><<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, dX, I, dxact, xact, nslice, red); note_launch();
+    return cudaGetLastError();
+}
+
+// the two-pair reductions: the (4, 8, 12) taps, k = 4, C a multiple of WSL2
+bool bred2_ok(const Dims& d) { return paper_kaps(d) && d.k == 4 && d.C % WSL2 == 0; }
+
 template <int KM>
 cudaError_t b8_kw(const Dims& d, int slot, int T, const uint16_t* out, const uint16_t* dX, const int* I,
                   const float* p, const float* hpost, const float* hres, const float* dxact,
@@ -40,7 +57,8 @@ cudaError_t b8_kw(const Dims& d, int slot, int T, const uint16_t* out, const uin
 
 // slices (partial sums per token) of the backward reductions of a slot
 int wb_bred_slices(const Dims& d, int slot) {
-    return d.K[slot] > 1 ? wb_nslice(d.C) : (d.C + W8 - 1) / W8;
+    if (d.K[slot] == 1) return (d.C + W8 - 1) / W8;
+    return bred2_ok(d) ? d.C / WSL2 : wb_nslice(d.C);
 }
 
 cudaError_t launch_wb_bred(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
@@ -50,6 +68,10 @@ cudaError_t launch_wb_bred(const Dims& d, int slot, int T, const uint16_t* out, 
     const bool last = (slot == d.G - 1);
     // a slot without conv takes the one-pass backward (launch_wb_b8), not this kernel
     if (!conv) return cudaErrorInvalidValue;
+    if (bred2_ok(d)) {
+        if (last) return bred2_kw<4, 32>(d, slot, T, out, cw, dX, I, dxact, xact, nslice, red, st);
+        return bred2_kw<4, 16>(d, slot, T, out, cw, dX, I, dxact, xact, nslice, red, st);
+    }
 #define XHC_BRED(KM_, NV_, FAST_)                                                                   \
     do {                                                                                            \
         XHC_KW_DISPATCH(d, FAST_, (bred_kw<KM_, KWC, NV_, KSC>(d, slot, T, out, cw, dX, I, dxact, xact, nslice, red, st))); \

@@ -42,6 +42,8 @@ CASES = {
     # N = 32: 160 full-state projection columns (router + 4 pre-maps), above the tensor-core
     # full-state dX's single k-block pair
     "flash4_N32_C256": (Config.flash(32, 4, 2, 256, 4, seq_len=128), 256, {}),
+    # C a multiple of 512: the MLP slots' reductions with two channel pairs per thread
+    "flash4_N8k4_C512": (Config.flash(8, 4, 2, 512, 4, seq_len=160), 320, {}),
     # attention-side temporal augmentation (App. "Additional Ablation Studies")
     "flash4_attn_tfa": (Config.flash(16, 4, 2, 256, 4, attn_tfa=True, seq_len=128), 512, {}),
     "flash2_attn_tfa": (Config.flash(16, 4, 2, 256, 2, attn_tfa=True, seq_len=128), 256, {}),

@@ -30,7 +30,8 @@ def _with_seq(cfg: Config, S: int) -> Config:
 @pytest.mark.parametrize("cfg,B,S1,S2", [
     (Config.full(16, 4, 2, 256, True), 3, 5, 7),            # S1 < R = 11: zero halo rows
     (Config.flash(16, 4, 2, 256, 4), 2, 140, 120),         # chunks longer than a token tile
-], ids=["fullM_S5+7", "flash4_S140+120"])
+    (Config.flash(8, 4, 2, 512, 4), 2, 70, 66),            # C = 512: two channel pairs per thread
+], ids=["fullM_S5+7", "flash4_S140+120", "flash4_C512_S70+66"])
 def test_two_chunks_with_halo_equal_the_unsplit_sequences(cfg, B, S1, S2):
     S = S1 + S2
     T = B * S
