@@ -650,10 +650,11 @@ xhc_status post_fwd_impl(const xhc_handle* h, int slot, int64_t T, const xhc_par
     const Dims& d = c.d;
     ConvPtrs cw = conv_of(d, P, slot);
     if (d.K[slot] > 1) cw.halo = halo;
+    const int gsl = wb_gram_slices(d);
     if (d.K[slot] > 1 && d.gs)
-        XHC_K("wb_gram", c.st, launch_wb_gram(d, slot, c.T, out, cw, c.L.nslice, c.W<float>(c.L.red), c.st));
+        XHC_K("wb_gram", c.st, launch_wb_gram(d, slot, c.T, out, cw, gsl, c.W<float>(c.L.red), c.st));
     const bool last = (slot == d.G - 1);
-    XHC_K("wb_coef", c.st, launch_wb_coef(d, slot, c.T, c.W<float>(c.L.red), c.L.nslice, c.S<float>(c.L.p),
+    XHC_K("wb_coef", c.st, launch_wb_coef(d, slot, c.T, c.W<float>(c.L.red), gsl, c.S<float>(c.L.p),
                                           c.S<float>(c.L.hpost[slot]),
                                           (d.K[slot] > 1 && d.gs) ? c.S<double>(c.L.gram[slot]) : nullptr,
                                           c.W<float>(c.L.tokmat), c.st));

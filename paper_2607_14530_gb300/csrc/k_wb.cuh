@@ -309,6 +309,90 @@ __global__ void __launch_bounds__(WT) k_wb_gram(Dims d, int slot, int T, int TB,
     }
 }
 
+// The Gram matrix with two channel pairs per thread (4 consecutive channels, WSL2 channels per
+// CTA) and the 4-token block ring: a token's warp reduction covers 128 channels.  For the
+// (4, 8, 12) tap set and C a multiple of 4 WT.
+constexpr int WSL2 = 4 * WT;
+
+__global__ void __launch_bounds__(WT, 2) k_wb_gram2(Dims d, int slot, int T, int TB,
+                                                    const uint16_t* __restrict__ out, ConvPtrs cw,
+                                                    int nslice, float* __restrict__ red) {
+    constexpr int KW = 12, KS = 2;
+    extern __shared__ float wsh[];  // [TB][WT/32][16]
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int slice = blockIdx.x, C = d.C;
+    const int c = slice * WSL2 + 4 * threadIdx.x;
+    long long t0, t1, send;
+    int pos0;
+    run_bounds<KW>(d, T, TB, t0, t1, send, pos0);
+    const int n1 = (int)(t1 - t0);
+    const int K = d.K[slot];
+    const int nq = K * (K + 1) / 2;
+    float2 tw[2][3][KW], w[2][KW + UB - 1];
+#pragma unroll
+    for (int p = 0; p < 2; ++p) {
+        taps_reg<KW, KS>(d, cw, c + 2 * p, true, tw[p]);
+        ring_init_b<KW>(d, cw, out, c + 2 * p, true, t0, pos0, w[p]);
+    }
+    const uint16_t* po = out + t0 * C + c;
+    // the out values of the next block of UB tokens are loaded while this block is processed
+    uint2 ob[UB];
+#pragma unroll
+    for (int u = 0; u < UB; ++u)
+        ob[u] = (u < n1) ? *reinterpret_cast<const uint2*>(po + (long long)u * C) : make_uint2(0u, 0u);
+    for (int tb = 0; tb < n1; tb += UB) {
+        uint2 on[UB];
+#pragma unroll
+        for (int u = 0; u < UB; ++u) {
+            const int tn = tb + UB + u;
+            on[u] = (tn < n1) ? *reinterpret_cast<const uint2*>(po + (long long)tn * C) : make_uint2(0u, 0u);
+        }
+#pragma unroll
+        for (int u = 0; u < UB; ++u) {
+            const int tt = tb + u;
+            if (tt < n1) {
+                float2 uu[2][4];
+#pragma unroll
+                for (int p = 0; p < 2; ++p) {
+                    const float2 o = u2f2(p == 0 ? ob[u].x : ob[u].y);
+                    w[p][KW - 1 + u] = o;
+                    float2 g[3];
+                    conv_blk<KW, KS>(tw[p], w[p], u, g);
+                    uu[p][0] = o;
+                    uu[p][1] = g[0];
+                    uu[p][2] = g[1];
+                    uu[p][3] = g[2];
+                }
+                float v[16];
+                int q = 0;
+#pragma unroll
+                for (int a = 0; a < 4; ++a)
+#pragma unroll
+                    for (int b = 0; b <= a; ++b)
+                        v[q++] = (a < K) ? fmaf(uu[1][a].y, uu[1][b].y,
+                                                fmaf(uu[1][a].x, uu[1][b].x, dot2(uu[0][a], uu[0][b])))
+                                         : 0.f;
+#pragma unroll
+                for (int r = 10; r < 16; ++r) v[r] = 0.f;
+                const float tot = WRed<16, 16>::run(v, lane);
+                if ((lane & 1) == 0) wsh[(tt * (WT / 32) + warp) * 16 + (lane >> 1)] = tot;
+            }
+        }
+#pragma unroll
+        for (int p = 0; p < 2; ++p) ring_shift<KW>(w[p]);
+#pragma unroll
+        for (int u = 0; u < UB; ++u) ob[u] = on[u];
+    }
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < n1 * nq; idx += WT) {
+        const int tt = idx / nq, q = idx - tt * nq;
+        float s = 0.f;
+#pragma unroll
+        for (int ww = 0; ww < WT / 32; ++ww) s += wsh[(tt * (WT / 32) + ww) * 16 + q];
+        red[((t0 + tt) * nslice + slice) * NRED + q] = s;
+    }
+}
+
 // ---------------------------------------------------------------------------------------------
 // wb_fwd: per-token coefficients E[j][a], H_res and I in shared memory; each thread prefetches
 // the out value and the k active values of its channel pair PD - 1 tokens ahead with cp.async.
@@ -618,7 +702,6 @@ __global__ void __launch_bounds__(WT) k_wb_bred(Dims d, int slot, int T, int TB,
 // per CTA): a token's warp reduction then covers 128 channels instead of 64, halving its cost
 // per channel, and the loads are 8 / 16 bytes wide.  For the (4, 8, 12) tap set with k = KM
 // and C a multiple of WSL2 (every thread in range).
-constexpr int WSL2 = 4 * WT;
 
 template <int KM>
 struct BRing2 {

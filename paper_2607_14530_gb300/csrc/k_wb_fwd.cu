@@ -96,8 +96,21 @@ int wb_conv_runs(const Dims& d, int64_t T) {
     return (int)n_runs(d, (int)T, bapp_run(KW), true);
 }
 
+// the two-pair Gram kernel: the (4, 8, 12) taps and C a multiple of WSL2
+static bool gram2_ok(const Dims& d) { return paper_kaps(d) && d.C % WSL2 == 0; }
+
+// partial-sum slices per token of the Gram kernel (read back by wb_coef)
+int wb_gram_slices(const Dims& d) { return gram2_ok(d) ? d.C / WSL2 : wb_nslice(d.C); }
+
 cudaError_t launch_wb_gram(const Dims& d, int slot, int T, const uint16_t* out, ConvPtrs cw,
                            int nslice, float* red, cudaStream_t st) {
+    if (gram2_ok(d)) {
+        const int TB = 64;
+        const size_t sm = (size_t)TB * (WT / 32) * 16 * sizeof(float);
+        dim3 grid(d.C / WSL2, (unsigned)n_runs(d, T, TB, true));
+        k_wb_gram2<<<grid, WT, sm, st>>>(d, slot, T, TB, out, cw, nslice, red); note_launch();
+        return cudaGetLastError();
+    }
     XHC_KW_DISPATCH(d, d.C % WSL == 0, (gram_kw<KWC, KSC>(d, slot, T, out, cw, nslice, red, st)));
 }
 

@@ -282,6 +282,7 @@ cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, 
                          const int* I, const float* dxact, const float* scal, int scal_ld,
                          uint16_t* dX, int* err, cudaStream_t st);
 int wb_nslice(int C);
+int wb_gram_slices(const Dims& d);  // partial-sum slices of wb_gram (and wb_coef)
 int wb_conv_runs(const Dims& d, int64_t T);
 int wb_bred_slices(const Dims& d, int slot);  // partial-sum slices of wb_bred (and bwd_coef)  // runs (conv weight-gradient partials) of wb_bapp
 // decode (one token per sequence, conv history in a per-sequence ring of max(kappa) - 1 rows)
