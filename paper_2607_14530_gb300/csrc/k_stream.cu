@@ -309,85 +309,100 @@ cudaError_t launch_dinput_act(const Dims& d, int slot, int T, int add_dx, const 
 // ---------------------------------------------------------------------------------------------
 // full_dots: for the non-active streams i, dH_pre[t][q][i] = <x_i, d_input_q> (Eq. dense_read
 // reversed; the dense-read gradient itself, dX[t][i] += sum_q H_pre[t][q][i] d_input_q, is added
-// by the full-state dX kernel).  One CTA per token with one warp per non-active stream (there are
-// N - k of them on every token: the k active streams are distinct); the token's G d_input rows
-// are staged in shared memory while each warp's first X reads are in flight.
+// by the full-state dX kernel).  One CTA per token with one warp per two non-active streams
+// (there are N - k of them on every token: the k active streams are distinct); the token's G
+// d_input rows are staged in shared memory while each warp's first X reads are in flight, and
+// each chunk read back from shared memory serves the warp's two X rows.
 
-__global__ void __launch_bounds__(1024) k_full_dots(Dims d, int T, const uint16_t* __restrict__ X,
-                                                    const uint16_t* __restrict__ dinput,
-                                                    const int* __restrict__ I,
-                                                    float* __restrict__ dhpre) {
+__global__ void __launch_bounds__(512) k_full_dots(Dims d, int T, const uint16_t* __restrict__ X,
+                                                   const uint16_t* __restrict__ dinput,
+                                                   const int* __restrict__ I,
+                                                   float* __restrict__ dhpre) {
     extern __shared__ __align__(16) uint16_t din[];   // [G][C]
     const int t = blockIdx.x, C = d.C, G = d.G;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    // this warp's stream: the warp-th stream that is not active on token t
+    // this warp's streams: the (2 warp)-th and (2 warp + 1)-th streams not active on token t
+    // (each d_input chunk read from shared memory serves two X rows)
     uint32_t act = 0u;
     for (int q = 0; q < d.k; ++q) act |= 1u << I[(int64_t)t * d.k + q];
-    int i = -1;
+    int is[2] = {-1, -1};
     for (int s = 0, cnt = 0; s < d.N; ++s)
         if (!(act & (1u << s))) {
-            if (cnt == warp) {
-                i = s;
-                break;
-            }
+            if (cnt == 2 * warp) is[0] = s;
+            if (cnt == 2 * warp + 1) is[1] = s;
             ++cnt;
         }
     if (!d.dense) {
         // sparse-read ablation: the non-active streams are not read, so their dH_pre is zero
-        if (i >= 0 && lane == 0)
-            for (int q = 0; q < G; ++q) dhpre[((int64_t)t * G + q) * d.N + i] = 0.f;
+        if (lane == 0)
+            for (int h = 0; h < 2; ++h)
+                if (is[h] >= 0)
+                    for (int q = 0; q < G; ++q) dhpre[((int64_t)t * G + q) * d.N + is[h]] = 0.f;
         return;
     }
-    const int64_t row = ((int64_t)t * d.N + (i < 0 ? 0 : i)) * C;
-    // the first 4 chunks per lane, read before the staging barrier
-    uint4 xr[4];
+    int64_t row[2];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-        const int c8 = lane + 32 * u;
-        if (i >= 0 && c8 < C / 8) xr[u] = __ldg(reinterpret_cast<const uint4*>(X + row + c8 * 8));
-    }
+    for (int h = 0; h < 2; ++h) row[h] = ((int64_t)t * d.N + (is[h] < 0 ? 0 : is[h])) * C;
+    // the first 4 chunks per lane and stream, read before the staging barrier
+    uint4 xr[2][4];
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int c8 = lane + 32 * u;
+            xr[h][u] = make_uint4(0u, 0u, 0u, 0u);
+            if (is[h] >= 0 && c8 < C / 8) xr[h][u] = __ldg(reinterpret_cast<const uint4*>(X + row[h] + c8 * 8));
+        }
     for (int idx = threadIdx.x; idx < G * C / 8; idx += blockDim.x) {
         const int q = idx / (C / 8), c8 = idx - q * (C / 8);
         reinterpret_cast<uint4*>(din)[idx] =
             *reinterpret_cast<const uint4*>(dinput + ((int64_t)q * T + t) * C + c8 * 8);
     }
     __syncthreads();
-    if (i < 0) return;
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    if (is[0] < 0) return;
+    float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
     for (int c0 = lane; c0 < C / 8; c0 += 128) {
         if (c0 != lane) {
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int c8 = c0 + 32 * u;
-                if (c8 < C / 8) xr[u] = __ldg(reinterpret_cast<const uint4*>(X + row + c8 * 8));
-            }
+            for (int h = 0; h < 2; ++h)
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int c8 = c0 + 32 * u;
+                    if (is[h] >= 0 && c8 < C / 8) xr[h][u] = __ldg(reinterpret_cast<const uint4*>(X + row[h] + c8 * 8));
+                }
         }
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
             const int c8 = c0 + 32 * u;
             if (c8 >= C / 8) continue;
-            float x[8];
-            unpack8(xr[u], x);
+            float x0[8], x1[8];
+            unpack8(xr[0][u], x0);
+            unpack8(xr[1][u], x1);
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 if (q >= G) continue;
                 float g[8];
                 unpack8(reinterpret_cast<const uint4*>(din + q * C)[c8], g);
 #pragma unroll
-                for (int e = 0; e < 8; ++e) acc[q] = fmaf(x[e], g[e], acc[q]);
+                for (int e = 0; e < 8; ++e) {
+                    acc[0][q] = fmaf(x0[e], g[e], acc[0][q]);
+                    acc[1][q] = fmaf(x1[e], g[e], acc[1][q]);
+                }
             }
         }
     }
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        const float v = warp_sum(acc[q]);
-        if (lane == 0 && q < G) dhpre[((int64_t)t * G + q) * d.N + i] = v;
-    }
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float v = warp_sum(acc[h][q]);
+            if (lane == 0 && q < G && is[h] >= 0) dhpre[((int64_t)t * G + q) * d.N + is[h]] = v;
+        }
 }
 
 cudaError_t launch_full_dots(const Dims& d, int T, const uint16_t* X, const uint16_t* dinput,
                              const int* I, float* dhpre, cudaStream_t st) {
-    const int nw = d.N - d.k;   // non-active streams per token
+    const int nw = (d.N - d.k + 1) / 2;   // warps per token: two non-active streams each
     if (nw <= 0) return cudaSuccess;
     const size_t sm = (size_t)d.G * d.C * 2;
     if (sm > 48 * 1024) {
