@@ -314,6 +314,7 @@ cudaError_t launch_dinput_act(const Dims& d, int slot, int T, int add_dx, const 
 // d_input rows are staged in shared memory while each warp's first X reads are in flight, and
 // each chunk read back from shared memory serves the warp's two X rows.
 
+template <int NS>
 __global__ void __launch_bounds__(512) k_full_dots(Dims d, int T, const uint16_t* __restrict__ X,
                                                    const uint16_t* __restrict__ dinput,
                                                    const int* __restrict__ I,
@@ -321,32 +322,35 @@ __global__ void __launch_bounds__(512) k_full_dots(Dims d, int T, const uint16_t
     extern __shared__ __align__(16) uint16_t din[];   // [G][C]
     const int t = blockIdx.x, C = d.C, G = d.G;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    // this warp's streams: the (2 warp)-th and (2 warp + 1)-th streams not active on token t
-    // (each d_input chunk read from shared memory serves two X rows)
+    // this warp's streams: the (NS warp + h)-th streams not active on token t, h < NS (each
+    // d_input chunk read from shared memory serves NS X rows)
     uint32_t act = 0u;
     for (int q = 0; q < d.k; ++q) act |= 1u << I[(int64_t)t * d.k + q];
-    int is[2] = {-1, -1};
+    int is[NS];
+#pragma unroll
+    for (int h = 0; h < NS; ++h) is[h] = -1;
     for (int s = 0, cnt = 0; s < d.N; ++s)
         if (!(act & (1u << s))) {
-            if (cnt == 2 * warp) is[0] = s;
-            if (cnt == 2 * warp + 1) is[1] = s;
+#pragma unroll
+            for (int h = 0; h < NS; ++h)
+                if (cnt == NS * warp + h) is[h] = s;
             ++cnt;
         }
     if (!d.dense) {
         // sparse-read ablation: the non-active streams are not read, so their dH_pre is zero
         if (lane == 0)
-            for (int h = 0; h < 2; ++h)
+            for (int h = 0; h < NS; ++h)
                 if (is[h] >= 0)
                     for (int q = 0; q < G; ++q) dhpre[((int64_t)t * G + q) * d.N + is[h]] = 0.f;
         return;
     }
-    int64_t row[2];
+    int64_t row[NS];
 #pragma unroll
-    for (int h = 0; h < 2; ++h) row[h] = ((int64_t)t * d.N + (is[h] < 0 ? 0 : is[h])) * C;
+    for (int h = 0; h < NS; ++h) row[h] = ((int64_t)t * d.N + (is[h] < 0 ? 0 : is[h])) * C;
     // the first 4 chunks per lane and stream, read before the staging barrier
-    uint4 xr[2][4];
+    uint4 xr[NS][4];
 #pragma unroll
-    for (int h = 0; h < 2; ++h)
+    for (int h = 0; h < NS; ++h)
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
             const int c8 = lane + 32 * u;
@@ -360,11 +364,15 @@ __global__ void __launch_bounds__(512) k_full_dots(Dims d, int T, const uint16_t
     }
     __syncthreads();
     if (is[0] < 0) return;
-    float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+    float acc[NS][4];
+#pragma unroll
+    for (int h = 0; h < NS; ++h)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) acc[h][q] = 0.f;
     for (int c0 = lane; c0 < C / 8; c0 += 128) {
         if (c0 != lane) {
 #pragma unroll
-            for (int h = 0; h < 2; ++h)
+            for (int h = 0; h < NS; ++h)
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     const int c8 = c0 + 32 * u;
@@ -375,24 +383,23 @@ __global__ void __launch_bounds__(512) k_full_dots(Dims d, int T, const uint16_t
         for (int u = 0; u < 4; ++u) {
             const int c8 = c0 + 32 * u;
             if (c8 >= C / 8) continue;
-            float x0[8], x1[8];
-            unpack8(xr[0][u], x0);
-            unpack8(xr[1][u], x1);
+            float xs[NS][8];
+#pragma unroll
+            for (int h = 0; h < NS; ++h) unpack8(xr[h][u], xs[h]);
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 if (q >= G) continue;
                 float g[8];
                 unpack8(reinterpret_cast<const uint4*>(din + q * C)[c8], g);
 #pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    acc[0][q] = fmaf(x0[e], g[e], acc[0][q]);
-                    acc[1][q] = fmaf(x1[e], g[e], acc[1][q]);
-                }
+                for (int h = 0; h < NS; ++h)
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) acc[h][q] = fmaf(xs[h][e], g[e], acc[h][q]);
             }
         }
     }
 #pragma unroll
-    for (int h = 0; h < 2; ++h)
+    for (int h = 0; h < NS; ++h)
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
             const float v = warp_sum(acc[h][q]);
@@ -402,15 +409,16 @@ __global__ void __launch_bounds__(512) k_full_dots(Dims d, int T, const uint16_t
 
 cudaError_t launch_full_dots(const Dims& d, int T, const uint16_t* X, const uint16_t* dinput,
                              const int* I, float* dhpre, cudaStream_t st) {
-    const int nw = (d.N - d.k + 1) / 2;   // warps per token: two non-active streams each
+    constexpr int NS = 2;                       // non-active streams per warp
+    const int nw = (d.N - d.k + NS - 1) / NS;   // warps per token
     if (nw <= 0) return cudaSuccess;
     const size_t sm = (size_t)d.G * d.C * 2;
     if (sm > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute((const void*)k_full_dots, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaError_t e = cudaFuncSetAttribute((const void*)k_full_dots<NS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)sm);
         if (e != cudaSuccess) return e;
     }
-    k_full_dots<<<T, 32 * nw, sm, st>>>(d, T, X, dinput, I, dhpre); note_launch();
+    k_full_dots<NS><<<T, 32 * nw, sm, st>>>(d, T, X, dinput, I, dhpre); note_launch();
     return cudaGetLastError();
 }
 
