@@ -579,6 +579,10 @@ def run_xhc(args, wl_name):
                        "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": ksteps,
                        "pipelined": "copy-in of step i+1 and copy-out of step i overlap step i+1's compute"}
 
+    # inference leg: decode steps of the same group shape (B sequences, one new token each)
+    if not args.no_decode:
+        line["decode"] = decode_leg(cfg, P, args.decode_batch, max(5, args.steps), dev, stream)
+
     if rank == 0 and not args.no_cpu_baseline:
         T_s = args.cpu_tokens
         Xs, os_, dXs, dis, Ps = cpu_sample(cfg, T_s, 0)
@@ -593,6 +597,68 @@ def run_xhc(args, wl_name):
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def decode_leg(cfg, P, B, steps, dev, stream, seed=1234):
+    """Decode steps of one group (one new token for each of B sequences, conv history in rings,
+    positions past 4096), eagerly and replayed as a captured CUDA graph of one step; CUDA events
+    on the launching stream."""
+    import torch
+    from paper_2607_14530_gb300 import synth, xhc
+
+    def timed(fn, k):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(k):
+            fn()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / k
+
+    gd = xhc.Group(type(cfg).flash(cfg.N, cfg.k, cfg.m, cfg.C, cfg.G, seq_len=0) if cfg.G > 1 else cfg)
+    Xd = synth.normal_bf16_on((B, cfg.N, cfg.C), seed + 3, dev)
+    outs_d = [synth.normal_bf16_on((B, cfg.C), seed + 301 + t, dev) for t in range(cfg.G)]
+    saved_d, ws_d = gd.alloc(B, device=dev)
+    rings = gd.alloc_rings(B, device=dev)
+    pos = torch.full((B,), 4096, dtype=torch.int64, device=dev)
+    ins_d = [torch.empty(B, cfg.C, dtype=torch.bfloat16, device=dev) for _ in range(cfg.G)]
+
+    def dstep():
+        gd.forward_decode(P, Xd, outs_d, rings, pos, saved_d, ws_d, inputs=ins_d)
+
+    eager_ms = timed(dstep, steps)
+    n0 = xhc.launch_count()
+    xhc.trace_enable(True)
+    dstep()
+    torch.cuda.synchronize()
+    launches = xhc.launch_count() - n0
+    per = {}
+    for name, t_ms in xhc.trace_records():
+        per[name] = per.get(name, 0.0) + t_ms
+    xhc.trace_enable(False)
+    top = sorted(per.items(), key=lambda kv: -kv[1])[:6]
+    graph_ms = None
+    try:
+        graph = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream()
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):
+            dstep()
+        stream.wait_stream(side)
+        torch.cuda.synchronize()
+        with torch.cuda.graph(graph):
+            dstep()
+        graph_ms = timed(graph.replay, steps)
+    except Exception as e:  # capture not possible on this stack: eager numbers only
+        graph_ms = f"not captured: {type(e).__name__}"
+    return {"batch": B, "launches_per_step": launches, "eager_ms": eager_ms,
+            "top_calls_ms": [[n, round(t, 4)] for n, t in top],
+            "eager_value": B / (eager_ms / 1000.0), "graph_ms": graph_ms,
+            "graph_value": (B / (graph_ms / 1000.0)) if isinstance(graph_ms, float) else None,
+            "unit": "tokens/s", "note": "one group of G sublayers per token"}
 
 
 def run_decode(args, wl_name):
@@ -642,51 +708,10 @@ def run_decode(args, wl_name):
     del saved, ws, X, X0, inputs
     torch.cuda.empty_cache()
 
-    # decode: B sequences, one token each per step
-    B = args.decode_batch
-    gd = xhc.Group(type(cfg).flash(cfg.N, cfg.k, cfg.m, cfg.C, cfg.G, seq_len=0) if cfg.G > 1 else cfg)
-    Xd = synth.normal_bf16_on((B, cfg.N, cfg.C), seed + 3, dev)
-    outs_d = [synth.normal_bf16_on((B, cfg.C), seed + 301 + t, dev) for t in range(cfg.G)]
-    saved_d, ws_d = gd.alloc(B, device=dev)
-    rings = gd.alloc_rings(B, device=dev)
-    pos = torch.full((B,), 4096, dtype=torch.int64, device=dev)
-    ins_d = [torch.empty(B, cfg.C, dtype=torch.bfloat16, device=dev) for _ in range(cfg.G)]
-
-    def dstep():
-        gd.forward_decode(P, Xd, outs_d, rings, pos, saved_d, ws_d, inputs=ins_d)
-
-    eager_ms = timed(dstep, args.steps)
-    n0 = xhc.launch_count()
-    xhc.trace_enable(True)
-    dstep()
-    torch.cuda.synchronize()
-    launches = xhc.launch_count() - n0
-    per = {}
-    for name, t_ms in xhc.trace_records():
-        per[name] = per.get(name, 0.0) + t_ms
-    xhc.trace_enable(False)
-    top = sorted(per.items(), key=lambda kv: -kv[1])[:6]
-    graph_ms = None
-    try:
-        graph = torch.cuda.CUDAGraph()
-        side = torch.cuda.Stream()
-        side.wait_stream(stream)
-        with torch.cuda.stream(side):
-            dstep()
-        stream.wait_stream(side)
-        torch.cuda.synchronize()
-        with torch.cuda.graph(graph):
-            dstep()
-        graph_ms = timed(graph.replay, args.steps)
-    except Exception as e:  # capture not possible on this stack: eager numbers only
-        graph_ms = f"not captured: {type(e).__name__}"
+    dec = decode_leg(cfg, P, args.decode_batch, args.steps, dev, stream, seed)
     line = {"metric": "inference: prefill and decode tokens/s", "unit": "tokens/s",
             "prefill": {"workload": desc, "tokens": T, "ms": pre_ms, "value": T / (pre_ms / 1000.0)},
-            "decode": {"batch": B, "launches_per_step": launches, "eager_ms": eager_ms,
-                       "top_calls_ms": [[n, round(t, 4)] for n, t in top],
-                       "eager_value": B / (eager_ms / 1000.0),
-                       "graph_ms": graph_ms,
-                       "graph_value": (B / (graph_ms / 1000.0)) if isinstance(graph_ms, float) else None},
+            "decode": dec,
             "steps": args.steps, "dtype": "f32", "data": "synthetic"}
     print(json.dumps(line), flush=True)
 
@@ -703,6 +728,7 @@ def main():
     ap.add_argument("--ref-tokens", type=int, default=64)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-decode", action="store_true", help="skip the decode leg of the default line")
     ap.add_argument("--kernels-out", default="")
     ap.add_argument("--mode", default="train", choices=["train", "inference"],
                     help="inference: forward-only prefill and decode legs (a separate line)")

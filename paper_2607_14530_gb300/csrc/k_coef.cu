@@ -372,7 +372,10 @@ __global__ void k_bwd_coef(Dims d, int slot, int T, const float* __restrict__ re
 #pragma unroll
         for (int i = 0; i < KM; ++i) Q[j][i] = 0.f;
     }
+    // loops to MAXCOMP / KM with guards on K / k: compile-time indices, registers only
+#pragma unroll
     for (int a = 0; a < MAXCOMP; ++a)
+#pragma unroll
         for (int b = 0; b < MAXCOMP; ++b) Gm[a][b] = 0.0;
     for (int s = 0; s < nslice; ++s) {
         const float* rp = red + ((int64_t)t * nslice + s) * NRED;
@@ -390,17 +393,24 @@ __global__ void k_bwd_coef(Dims d, int slot, int T, const float* __restrict__ re
         }
     }
     if (gs) {
-        int q = 0;
-        for (int a = 0; a < K; ++a)
-            for (int b = 0; b <= a; ++b) Gm[a][b] = gram[(int64_t)t * NGRAM + q++];
+#pragma unroll
+        for (int a = 0; a < MAXCOMP; ++a)
+#pragma unroll
+            for (int b = 0; b <= a; ++b)
+                if (a < K) Gm[a][b] = gram[(int64_t)t * NGRAM + a * (a + 1) / 2 + b];
     }
-    for (int a = 0; a < K; ++a)
-        for (int b = a + 1; b < K; ++b) Gm[a][b] = Gm[b][a];
+#pragma unroll
+    for (int a = 0; a < MAXCOMP; ++a)
+#pragma unroll
+        for (int b = a + 1; b < MAXCOMP; ++b)
+            if (b < K) Gm[a][b] = Gm[b][a];
     double B[MAXCOMP][MAXCOMP], cc[MAXCOMP][MAXCOMP], vv[MAXCOMP];
     if (gs) {
         gs_coef(Gm, K, (double)d.eps_gs, B, cc, vv);
     } else {
+#pragma unroll
         for (int a = 0; a < MAXCOMP; ++a)
+#pragma unroll
             for (int b = 0; b < MAXCOMP; ++b) B[a][b] = (a == b) ? 1.0 : 0.0;
     }
     float* tm = tokmat + (int64_t)t * TOKMAT;
@@ -408,9 +418,14 @@ __global__ void k_bwd_coef(Dims d, int slot, int T, const float* __restrict__ re
     const float r = rs[t];
     const float* za = zact + (int64_t)t * n;
     const float ap = alpha_post[slot];
-    float dz[KM * MAXCOMP + KM * KM];
+    // the scaled map-logit gradients go straight to dzs (dz * r); sdz = sum_o dz_o zact_o feeds
+    // the RMS coefficient cx
+    float* dzr = dzs + (int64_t)t * n;
+    float sdz = 0.f;
     double dB[MAXCOMP][MAXCOMP];
+#pragma unroll
     for (int a = 0; a < MAXCOMP; ++a)
+#pragma unroll
         for (int b = 0; b < MAXCOMP; ++b) dB[a][b] = 0.0;
     float dap = 0.f;
 #pragma unroll
@@ -418,37 +433,54 @@ __global__ void k_bwd_coef(Dims d, int slot, int T, const float* __restrict__ re
         if (j >= k) continue;
         const float pj = p[(int64_t)t * k + j];
         float dpj = 0.f;
+#pragma unroll
         for (int a = 0; a < 4; ++a) {
             float e = 0.f;
-            if (a < K)
-                for (int q = 0; q < K; ++q) e += hpost[((int64_t)t * k + j) * K + q] * (float)B[q][a];
+            if (a < K) {
+#pragma unroll
+                for (int q = 0; q < MAXCOMP; ++q)
+                    if (q < K) e += hpost[((int64_t)t * k + j) * K + q] * (float)B[q][a];
+            }
             tm[j * 4 + a] = pj * e;
         }
-        for (int q = 0; q < K; ++q) {
+#pragma unroll
+        for (int q = 0; q < MAXCOMP; ++q) {
+            if (q >= K) continue;
             float pb = 0.f;
-            for (int a = 0; a < K; ++a) pb += Pm[j][a] * (float)B[q][a];
+#pragma unroll
+            for (int a = 0; a < MAXCOMP; ++a)
+                if (a < K) pb += Pm[j][a] * (float)B[q][a];
             const float h = hpost[((int64_t)t * k + j) * K + q];
             const float dh = pj * pb;
             dpj += h * pb;
-            for (int a = 0; a < K; ++a) dB[q][a] += (double)(pj * h) * (double)Pm[j][a];
+#pragma unroll
+            for (int a = 0; a < MAXCOMP; ++a)
+                if (a < K) dB[q][a] += (double)(pj * h) * (double)Pm[j][a];
             // H = 2 sigma(y): dy = dH * H * (1 - H / 2)
             const float dy = dh * h * (1.0f - 0.5f * h);
             const int o = j * K + q;
-            dz[o] = ap * dy;
+            const float dzo = ap * dy;
             dap += dy * (za[o] * r);
             tg[o] = dy;
+            sdz += dzo * za[o];
+            dzr[o] = dzo * r;
         }
         dp[(int64_t)t * k + j] += dpj;
     }
     tg[k * K] = dap;
     // D = dG + dG^T (symmetric Gram entries)
+#pragma unroll
     for (int a = 0; a < 4; ++a)
+#pragma unroll
         for (int b = 0; b < 4; ++b) tm[32 + a * 4 + b] = 0.f;
     if (gs) {
         double dG[MAXCOMP][MAXCOMP];
         gs_coef_bwd(Gm, K, B, cc, vv, dB, dG);
-        for (int a = 0; a < K; ++a)
-            for (int b = 0; b < K; ++b) tm[32 + a * 4 + b] = (float)(dG[a][b] + dG[b][a]);
+#pragma unroll
+        for (int a = 0; a < MAXCOMP; ++a)
+#pragma unroll
+            for (int b = 0; b < MAXCOMP; ++b)
+                if (a < K && b < K) tm[32 + a * 4 + b] = (float)(dG[a][b] + dG[b][a]);
     }
     if (last) {
         float M[KM][KM], dH[KM][KM], H[KM][KM], dM[KM][KM];
@@ -470,19 +502,16 @@ __global__ void k_bwd_coef(Dims d, int slot, int T, const float* __restrict__ re
             for (int b = 0; b < KM; ++b) {
                 if (a >= k || b >= k) continue;
                 const int o = k * K + a * k + b;
-                dz[o] = ar * dM[a][b];
+                const float dzo = ar * dM[a][b];
                 dar += dM[a][b] * (za[o] * r);
                 tg[k * K + 1 + a * k + b] = dM[a][b];
                 tm[48 + a * 8 + b] = H[a][b];
+                sdz += dzo * za[o];
+                dzr[o] = dzo * r;
             }
         tg[k * K + 1 + k * k] = dar;
     }
     // active RMS: z_o = r * zraw_o, r = (sum x^2 / kC + eps)^(-1/2)
-    float sdz = 0.f;
-    for (int o = 0; o < n; ++o) {
-        sdz += dz[o] * za[o];
-        dzs[(int64_t)t * n + o] = dz[o] * r;
-    }
     tm[112] = r * r * r / (float)(k * d.C) * sdz;
 }
 

@@ -19,33 +19,49 @@ __global__ void __launch_bounds__(64) k_wb_coef(Dims d, int slot, int T, const f
     if (t >= T) return;
     const int k = d.k, K = d.K[slot];
     const bool gs = (K > 1) && d.gs;
+    // loops to MAXCOMP with guards on K: compile-time indices, the arrays stay in registers
     double B[MAXCOMP][MAXCOMP];
+#pragma unroll
     for (int a = 0; a < MAXCOMP; ++a)
+#pragma unroll
         for (int b = 0; b < MAXCOMP; ++b) B[a][b] = (a == b) ? 1.0 : 0.0;
     if (gs) {
         double Gm[MAXCOMP][MAXCOMP], cc[MAXCOMP][MAXCOMP], vv[MAXCOMP];
+#pragma unroll
         for (int a = 0; a < MAXCOMP; ++a)
+#pragma unroll
             for (int b = 0; b < MAXCOMP; ++b) Gm[a][b] = 0.0;
         for (int sl = 0; sl < nslice; ++sl) {
             const float* rp = red + ((int64_t)t * nslice + sl) * NRED;
-            int q = 0;
-            for (int a = 0; a < K; ++a)
-                for (int b = 0; b <= a; ++b) Gm[a][b] += (double)rp[q++];
+#pragma unroll
+            for (int a = 0; a < MAXCOMP; ++a)
+#pragma unroll
+                for (int b = 0; b <= a; ++b)
+                    if (a < K) Gm[a][b] += (double)rp[a * (a + 1) / 2 + b];
         }
-        int q = 0;
-        for (int a = 0; a < K; ++a)
-            for (int b = 0; b <= a; ++b) gram[(int64_t)t * NGRAM + q++] = Gm[a][b];
-        for (int a = 0; a < K; ++a)
-            for (int b = a + 1; b < K; ++b) Gm[a][b] = Gm[b][a];
+#pragma unroll
+        for (int a = 0; a < MAXCOMP; ++a)
+#pragma unroll
+            for (int b = 0; b <= a; ++b)
+                if (a < K) gram[(int64_t)t * NGRAM + a * (a + 1) / 2 + b] = Gm[a][b];
+#pragma unroll
+        for (int a = 0; a < MAXCOMP; ++a)
+#pragma unroll
+            for (int b = a + 1; b < MAXCOMP; ++b)
+                if (b < K) Gm[a][b] = Gm[b][a];
         gs_coef(Gm, K, (double)d.eps_gs, B, cc, vv);
     }
     float* em = emat + (int64_t)t * TOKMAT;
     for (int j = 0; j < k; ++j) {
         const float pj = p[(int64_t)t * k + j];
+#pragma unroll
         for (int a = 0; a < 4; ++a) {
             float e = 0.f;
-            if (a < K)
-                for (int q = 0; q < K; ++q) e += hpost[((int64_t)t * k + j) * K + q] * (float)B[q][a];
+            if (a < K) {
+#pragma unroll
+                for (int q = 0; q < MAXCOMP; ++q)
+                    if (q < K) e += hpost[((int64_t)t * k + j) * K + q] * (float)B[q][a];
+            }
             em[j * 4 + a] = pj * e;
         }
     }

@@ -189,24 +189,36 @@ __device__ __forceinline__ int seg_of(const WSegs& w, int o) {
 // Gram-Schmidt of Eq. gs expressed on the Gram matrix of u = [out, g_1, ..., g_r]:
 // v_j = sum_a B[j][a] u_a, B unit lower-triangular.  Denominators <v_i, v_i> + eps.
 
+// The loops run to MAXCOMP with guards on K (the same operations in the same order as loops to
+// K), so every array index is a compile-time constant and the arrays stay in registers.
 __device__ inline void gs_coef(const double (&G)[MAXCOMP][MAXCOMP], int K, double eps,
                         double (&B)[MAXCOMP][MAXCOMP], double (&c)[MAXCOMP][MAXCOMP],
                         double (&vv)[MAXCOMP]) {
+#pragma unroll
     for (int j = 0; j < MAXCOMP; ++j)
+#pragma unroll
         for (int a = 0; a < MAXCOMP; ++a) {
             B[j][a] = (j == a) ? 1.0 : 0.0;
             c[j][a] = 0.0;
         }
-    for (int j = 0; j < K; ++j) {
+#pragma unroll
+    for (int j = 0; j < MAXCOMP; ++j) {
+        if (j >= K) break;
+#pragma unroll
         for (int i = 0; i < j; ++i) {
             double num = 0.0;
+#pragma unroll
             for (int a = 0; a <= i; ++a) num += B[i][a] * G[j][a];
             c[j][i] = num / vv[i];
         }
+#pragma unroll
         for (int i = 0; i < j; ++i)
+#pragma unroll
             for (int a = 0; a <= i; ++a) B[j][a] -= c[j][i] * B[i][a];
         double q = 0.0;
+#pragma unroll
         for (int a = 0; a <= j; ++a)
+#pragma unroll
             for (int b = 0; b <= j; ++b) q += B[j][a] * B[j][b] * G[a][b];
         vv[j] = q + eps;
     }
@@ -218,27 +230,37 @@ __device__ inline void gs_coef_bwd(const double (&G)[MAXCOMP][MAXCOMP], int K,
                             const double (&vv)[MAXCOMP], double (&dB)[MAXCOMP][MAXCOMP],
                             double (&dG)[MAXCOMP][MAXCOMP]) {
     double dvv[MAXCOMP] = {0.0, 0.0, 0.0, 0.0};
+#pragma unroll
     for (int a = 0; a < MAXCOMP; ++a)
+#pragma unroll
         for (int b = 0; b < MAXCOMP; ++b) dG[a][b] = 0.0;
-    for (int j = K - 1; j >= 0; --j) {
+#pragma unroll
+    for (int j = MAXCOMP - 1; j >= 0; --j) {
+        if (j >= K) continue;
         // vv[j] = B[j]^T G B[j] + eps
         if (dvv[j] != 0.0) {
+#pragma unroll
             for (int a = 0; a <= j; ++a) {
                 double s = 0.0;
+#pragma unroll
                 for (int b = 0; b <= j; ++b) s += (G[a][b] + G[b][a]) * B[j][b];
                 dB[j][a] += dvv[j] * s;
+#pragma unroll
                 for (int b = 0; b <= j; ++b) dG[a][b] += dvv[j] * B[j][a] * B[j][b];
             }
         }
         // B[j] = e_j - sum_i c[j][i] B[i];  c[j][i] = num / vv[i];  num = sum_a B[i][a] G[j][a]
+#pragma unroll
         for (int i = j - 1; i >= 0; --i) {
             double dc = 0.0;
+#pragma unroll
             for (int a = 0; a <= i; ++a) {
                 dc -= dB[j][a] * B[i][a];
                 dB[i][a] -= c[j][i] * dB[j][a];
             }
             const double dnum = dc / vv[i];
             dvv[i] -= dc * c[j][i] / vv[i];
+#pragma unroll
             for (int a = 0; a <= i; ++a) {
                 dB[i][a] += dnum * G[j][a];
                 dG[j][a] += dnum * B[i][a];
