@@ -847,7 +847,6 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
             for (int hh = 0; hh < 2; ++hh) {
                 const int cg = chalf * 2 + hh;     // column group of 32
                 // 4 passes of 8 rows; lane -> row rr = 8 pass + lane / 4, channels 8 (lane % 4)..
-                // The reads of passes 0-1 are issued before the accumulator is read out.
                 const int cq = (lane & 3) * 8;
                 const int c = ct * DX_BN + cg * 32 + cq;
                 uint4 xr[4], br[4], br2[4], gr[4];
@@ -878,8 +877,12 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
                         }
                     }
                 };
+                // all four passes' reads are issued before the accumulator is awaited and read
+                // out (8 columns at a time, few registers live next to the 64 of the reads)
                 load_pass(0);
                 load_pass(1);
+                load_pass(2);
+                load_pass(3);
                 if (hh == 0) {
                     if (!mbar_wait(smem_u32(&bars[4 + s]), (uint32_t)((n >> 1) & 1), a.wait_ns)) {
                         atomicExch(a.err, 14);
@@ -888,14 +891,12 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
                     }
                     tc_fence_after();
                 }
-                {
-                    float acc[16];
-                    tmem_ld16(tl + (uint32_t)(cg * 32), acc);
 #pragma unroll
-                    for (int e = 0; e < 16; ++e) tileb[lane * 33 + e] = acc[e];
-                    tmem_ld16(tl + (uint32_t)(cg * 32 + 16), acc);
+                for (int q8 = 0; q8 < 4; ++q8) {
+                    float acc[8];
+                    tmem_ld8(tl + (uint32_t)(cg * 32 + q8 * 8), acc);
 #pragma unroll
-                    for (int e = 0; e < 16; ++e) tileb[lane * 33 + 16 + e] = acc[e];
+                    for (int e = 0; e < 8; ++e) tileb[lane * 33 + q8 * 8 + e] = acc[e];
                 }
                 if (hh == 1) {
                     tc_fence_before();
@@ -903,8 +904,6 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
                     if (lane == 0) mbar_arrive(smem_u32(&bars[6 + s]));  // TMEM buffer free
                 }
                 __syncwarp();
-                load_pass(2);
-                load_pass(3);
 #pragma unroll
                 for (int pass = 0; pass < 4; ++pass) {
                     const int rr = pass * 8 + (lane >> 2);
