@@ -716,6 +716,82 @@ def run_decode(args, wl_name):
     print(json.dumps(line), flush=True)
 
 
+def run_stack(args, wl_name):
+    """A stack of L groups through the model glue (stream expansion, L groups of the workload's
+    shape with scalar-gain sublayers, final stream sum; forward and torch.autograd backward),
+    against L bare group calls (forward + backward through the binding) on the same tokens: the
+    glue's overhead.  One JSON line; CUDA events on the current stream."""
+    import torch
+    from torch import nn
+    from paper_2607_14530_gb300 import build, synth, xhc
+    from paper_2607_14530_gb300.model import XhcStack
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    build.build()
+    xhc.lib()
+    desc, cfg, T = workloads()[wl_name]
+    T = args.tokens or 8192
+    L = args.groups
+    seed = 1234
+
+    class Gain(nn.Module):
+        def __init__(self):
+            super().__init__()
+            self.s = nn.Parameter(torch.tensor(0.03125))
+
+        def forward(self, x):
+            return x.float() * self.s
+
+    stack = XhcStack(cfg, L, lambda l, t: Gain(), seed=seed).to(dev)
+    hid = synth.normal_bf16_on((T, cfg.C), seed + 5, dev)
+    dy = synth.normal_bf16_on((T, cfg.C), seed + 6, dev)
+    stream = torch.cuda.current_stream()
+
+    def stack_step():
+        h = hid.detach().requires_grad_(True)
+        y = stack(h)
+        y.backward(dy)
+
+    def timed(fn, k):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(k):
+            fn()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / k
+
+    stack_ms = timed(stack_step, args.steps)
+    # the same work as bare group calls: L x (forward + backward of one group)
+    g = xhc.Group(cfg)
+    P = {n: v.to(dev) for n, v in synth.params(cfg.param_shapes(), seed).items()}
+    G_ = {n: torch.zeros_like(v) for n, v in P.items()}
+    saved, ws = g.alloc(T, device=dev)
+    X = synth.normal_bf16_on((T, cfg.N, cfg.C), seed, dev)
+    outs = [synth.normal_bf16_on((T, cfg.C), seed + 101 + t, dev) for t in range(cfg.G)]
+    dX = synth.normal_bf16_on((T, cfg.N, cfg.C), seed + 7, dev)
+    dins = [synth.normal_bf16_on((T, cfg.C), seed + 211 + t, dev) for t in range(cfg.G)]
+    inputs = [torch.empty(T, cfg.C, dtype=torch.bfloat16, device=dev) for _ in range(cfg.G)]
+    d_outs = [torch.empty(T, cfg.C, dtype=torch.bfloat16, device=dev) for _ in range(cfg.G)]
+
+    def bare_step():
+        for _ in range(L):
+            g.forward(P, X, outs, saved, ws, inputs=inputs)
+            g.backward(P, X, dX, outs, dins, G_, saved, ws, d_outs=d_outs)
+
+    bare_ms = timed(bare_step, args.steps)
+    line = {"metric": "stack of groups through the autograd glue: tokens/s fwd+bwd", "unit": "tokens/s",
+            "workload": f"{L} groups of: {desc}; sublayers: scalar gains", "tokens": T,
+            "stack_ms": stack_ms, "value": T / (stack_ms / 1000.0),
+            "bare_group_calls_ms": bare_ms, "glue_overhead": stack_ms / bare_ms - 1.0,
+            "steps": args.steps, "dtype": "f32", "data": "synthetic"}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -730,8 +806,10 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-decode", action="store_true", help="skip the decode leg of the default line")
     ap.add_argument("--kernels-out", default="")
-    ap.add_argument("--mode", default="train", choices=["train", "inference"],
-                    help="inference: forward-only prefill and decode legs (a separate line)")
+    ap.add_argument("--mode", default="train", choices=["train", "inference", "stack"],
+                    help="inference: forward-only prefill and decode legs; stack: a stack of groups "
+                         "through the autograd glue (separate lines)")
+    ap.add_argument("--groups", type=int, default=4, help="groups of the stack leg")
     ap.add_argument("--decode-batch", type=int, default=256)
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "xhc":
@@ -740,6 +818,8 @@ def main():
         run_reference(args, args.workload)
     elif args.mode == "inference":
         run_decode(args, args.workload)
+    elif args.mode == "stack":
+        run_stack(args, args.workload)
     else:
         run_xhc(args, args.workload)
 
