@@ -318,13 +318,21 @@ xhc_status xhc_route_noalloc(const xhc_handle* h, int64_t T, const xhc_params* P
                              const uint16_t* X, int32_t* I, float* p, float* hpre, void* stream);
 
 /* Tracing, a host-side profiling aid: while enabled, every kernel launch of the library is
- * bracketed by two CUDA events recorded on the caller's stream.  xhc_trace_enable(1) drops the
- * previous records and starts recording; xhc_trace_enable(0) stops.  xhc_trace_record gives the
- * launch's name and device duration in ms; the caller must have synchronised the stream first
- * (otherwise XHC_ERR_CUDA, "not ready").  Not for concurrent use from several host threads. */
+ * bracketed by two CUDA events recorded on the stream it runs on.  xhc_trace_enable(1) drops the
+ * previous records and starts recording; xhc_trace_enable(0) stops.  xhc_trace_only restricts
+ * the recording to the launches of the named kernels (a comma-separated list of the names the
+ * records carry, e.g. "dxa_tc,dinput_act"; NULL or "" records every launch again); it takes
+ * effect for later launches and is kept until the next xhc_trace_only.  xhc_trace_record gives
+ * record i's name and device duration in ms; xhc_trace_span also gives its start in ms after
+ * the start of record 0 (a timeline across the library's streams).  The caller must have
+ * synchronised the streams first (otherwise XHC_ERR_CUDA, "not ready"); i out of range or a
+ * NULL output pointer is XHC_ERR_INVALID_ARG.  Not for concurrent use from several host
+ * threads. */
 xhc_status xhc_trace_enable(int on);
+xhc_status xhc_trace_only(const char* names);
 int xhc_trace_count(void);
 xhc_status xhc_trace_record(int i, const char** name, float* ms);
+xhc_status xhc_trace_span(int i, const char** name, float* start_ms, float* ms);
 
 /* Device error word of a workspace: kernels with bounded waits (the tensor-core kernels) set it
  * to a nonzero code instead of waiting forever, and return; a launch whose wait gave up leaves
@@ -341,9 +349,13 @@ xhc_status xhc_workspace_error(const void* workspace, int* code, int clear);
  *   of slot 0 on the tensor cores) wait, before it issues any copy or MMA, for a release that
  *   nothing triggers, so that every wait of that launch runs out: it sets the workspace's error
  *   word and returns without touching its outputs.  One-shot.
+ * XHC_DEBUG_ONE_STREAM: value != 0 runs the work that later calls put on the library's side
+ *   stream (weight gradients, column sums, dH_pre dots) on the caller's stream instead, in the
+ *   same order; the results are the same.  0 restores the side stream.
  * Returns XHC_ERR_INVALID_ARG for an unknown `what` or a negative limit. */
 #define XHC_DEBUG_WAIT_LIMIT_NS 1
 #define XHC_DEBUG_FORCE_TIMEOUT 2
+#define XHC_DEBUG_ONE_STREAM 3
 xhc_status xhc_debug_set(int what, int64_t value);
 
 /* Number of kernels the library has launched since it was loaded. */

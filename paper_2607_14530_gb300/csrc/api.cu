@@ -5,6 +5,7 @@
 #include <algorithm>
 #include <atomic>
 #include <mutex>
+#include <string>
 #include <vector>
 
 #include "xhc_internal.cuh"
@@ -18,6 +19,7 @@ void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 // ---- test hooks -----------------------------------------------------------------------------
 static std::atomic<unsigned long long> g_wait_ns{0};   // 0: the default limit (~4 s)
 static std::atomic<int> g_force_timeout{0};
+static std::atomic<int> g_one_stream{0};
 uint64_t debug_wait_ns() {
     const unsigned long long v = g_wait_ns.load();
     return v ? (uint64_t)v : 4000000000ull;
@@ -32,6 +34,14 @@ static std::mutex g_tmu;
 static bool g_trace_on = false;
 static std::vector<TraceRec> g_recs;
 static std::vector<cudaEvent_t> g_pool;
+static std::vector<std::string> g_only;   // names recorded while tracing (empty: every launch)
+
+static bool traced(const char* n) {
+    if (g_only.empty()) return true;
+    for (const auto& s : g_only)
+        if (s == n) return true;
+    return false;
+}
 
 static cudaEvent_t take_event() {
     cudaEvent_t e = nullptr;
@@ -51,6 +61,7 @@ struct TraceScope {
     TraceScope(const char* n, cudaStream_t s) : name(n), st(s) {
         if (!g_trace_on) return;
         std::lock_guard<std::mutex> lk(g_tmu);
+        if (!traced(n)) return;
         a = take_event();
         if (a) cudaEventRecord(a, st);
     }
@@ -238,6 +249,23 @@ xhc_status xhc_trace_enable(int on) {
     return XHC_OK;
 }
 
+xhc_status xhc_trace_only(const char* names) {
+    std::lock_guard<std::mutex> lk(g_tmu);
+    g_only.clear();
+    if (!names) return XHC_OK;
+    std::string cur;
+    for (const char* c = names;; ++c) {
+        if (*c == ',' || *c == 0) {
+            if (!cur.empty()) g_only.push_back(cur);
+            cur.clear();
+            if (*c == 0) break;
+        } else if (*c != ' ') {
+            cur.push_back(*c);
+        }
+    }
+    return XHC_OK;
+}
+
 int xhc_trace_count(void) {
     std::lock_guard<std::mutex> lk(g_tmu);
     return (int)g_recs.size();
@@ -252,6 +280,16 @@ xhc_status xhc_trace_record(int i, const char** name, float* ms) {
     return XHC_OK;
 }
 
+xhc_status xhc_trace_span(int i, const char** name, float* start_ms, float* ms) {
+    std::lock_guard<std::mutex> lk(g_tmu);
+    if (i < 0 || i >= (int)g_recs.size() || !name || !start_ms || !ms) return XHC_ERR_INVALID_ARG;
+    *name = g_recs[i].name;
+    cudaError_t e = cudaEventElapsedTime(start_ms, g_recs[0].a, g_recs[i].a);
+    if (e == cudaSuccess) e = cudaEventElapsedTime(ms, g_recs[i].a, g_recs[i].b);
+    if (e != cudaSuccess) return cuda_fail(e, __LINE__);
+    return XHC_OK;
+}
+
 uint64_t xhc_launch_count(void) { return (uint64_t)g_launches.load(); }
 
 xhc_status xhc_debug_set(int what, int64_t value) {
@@ -262,6 +300,9 @@ xhc_status xhc_debug_set(int what, int64_t value) {
             return XHC_OK;
         case XHC_DEBUG_FORCE_TIMEOUT:
             g_force_timeout.store(value ? 1 : 0);
+            return XHC_OK;
+        case XHC_DEBUG_ONE_STREAM:
+            g_one_stream.store(value ? 1 : 0);
             return XHC_OK;
     }
     return XHC_ERR_INVALID_ARG;
@@ -406,6 +447,7 @@ static bool stream_after(cudaStream_t to, cudaStream_t from) {
 
 // a stream forked from `main`: the side stream, or `main` itself
 static cudaStream_t fork_from(cudaStream_t main) {
+    if (g_one_stream.load()) return main;
     cudaStream_t side = side_stream();
     if (!side || !stream_after(side, main)) return main;
     return side;

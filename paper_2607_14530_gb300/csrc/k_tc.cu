@@ -371,14 +371,16 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                     break;
                 }
                 if (!A_MN && a.pstats) {
-                    // row r of the A tile: 128 bytes, 16-byte chunks permuted by the swizzle (the
-                    // sum over the row does not depend on the order)
+                    // row r of the A tile: 128 bytes, logical 16-byte chunk q at position
+                    // q ^ (r % 8) (128-byte swizzle).  Reading the chunks in logical order puts the
+                    // 8 rows of a quarter warp on 8 different bank groups (physical order would put
+                    // all 32 rows of the warp on the same 4 banks: 8-way conflicts)
                     for (int p2 = 0; p2 < KPS; ++p2) {
                         const uint4* row = reinterpret_cast<const uint4*>(smem + (size_t)s * STAGE +
                                                                           p2 * BM * BK * 2 + r * 128);
                         uint4 v[8];
 #pragma unroll
-                        for (int q = 0; q < 8; ++q) v[q] = row[q];
+                        for (int q = 0; q < 8; ++q) v[q] = row[q ^ (r & 7)];
 #pragma unroll
                         for (int q = 0; q < 8; ++q) {
                             const uint32_t w[4] = {v[q].x, v[q].y, v[q].z, v[q].w};

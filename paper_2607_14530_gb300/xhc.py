@@ -94,6 +94,9 @@ def lib() -> ctypes.CDLL:
         L.xhc_trace_count.restype = ctypes.c_int
         L.xhc_trace_record.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_char_p),
                                        ctypes.POINTER(ctypes.c_float)]
+        L.xhc_trace_only.argtypes = [ctypes.c_char_p]
+        L.xhc_trace_span.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_char_p),
+                                     ctypes.POINTER(ctypes.c_float), ctypes.POINTER(ctypes.c_float)]
         L.xhc_launch_count.restype = ctypes.c_uint64
         L.xhc_status_string.argtypes = [ctypes.c_int]
         L.xhc_status_string.restype = ctypes.c_char_p
@@ -114,6 +117,23 @@ def _check(status: int, what: str):
 def trace_enable(on: bool) -> None:
     """Start (clearing old records) or stop recording per-launch CUDA events in the library."""
     _check(lib().xhc_trace_enable(1 if on else 0), "xhc_trace_enable")
+
+
+def trace_only(names=None) -> None:
+    """Record only the launches of these kernel names (an iterable of names; None: every launch)."""
+    arg = None if not names else ",".join(names).encode()
+    _check(lib().xhc_trace_only(arg), "xhc_trace_only")
+
+
+def trace_spans() -> list:
+    """[(kernel name, start ms after the first record's start, device ms)]; synchronise first."""
+    L = lib()
+    out = []
+    for i in range(L.xhc_trace_count()):
+        name, t0, ms = ctypes.c_char_p(), ctypes.c_float(), ctypes.c_float()
+        _check(L.xhc_trace_span(i, ctypes.byref(name), ctypes.byref(t0), ctypes.byref(ms)), "xhc_trace_span")
+        out.append((name.value.decode(), float(t0.value), float(ms.value)))
+    return out
 
 
 def trace_records() -> list:
@@ -137,6 +157,11 @@ def debug_force_timeout() -> None:
     """Make the next tensor-core full-state projection time out before it issues any work (a
     test hook for the bounded-wait abort path; xhc_debug_set)."""
     _check(lib().xhc_debug_set(2, 1), "xhc_debug_set")
+
+
+def debug_one_stream(on: bool) -> None:
+    """Run the library's side-stream work on the caller's stream (same order, same results)."""
+    _check(lib().xhc_debug_set(3, 1 if on else 0), "xhc_debug_set")
 
 
 def launch_count() -> int:
