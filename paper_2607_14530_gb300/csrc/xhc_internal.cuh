@@ -163,8 +163,19 @@ __device__ __forceinline__ void unpack8(const uint4& u, float* f) {
     f[4] = __uint_as_float(u.z << 16); f[5] = __uint_as_float(u.z & 0xffff0000u);
     f[6] = __uint_as_float(u.w << 16); f[7] = __uint_as_float(u.w & 0xffff0000u);
 }
+// two floats to bf16 (round to nearest even) in one conversion: a in the low half, b in the high
 __device__ __forceinline__ uint32_t pack2(float a, float b) {
-    return (uint32_t)f2bf(a) | ((uint32_t)f2bf(b) << 16);
+    const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+    uint32_t r;
+    memcpy(&r, &h, sizeof(r));
+    return r;
+}
+// 8 bf16 as 4 channel pairs (low half first)
+__device__ __forceinline__ void unpack4x2(const uint4& u, float2* f) {
+    f[0] = make_float2(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xffff0000u));
+    f[1] = make_float2(__uint_as_float(u.y << 16), __uint_as_float(u.y & 0xffff0000u));
+    f[2] = make_float2(__uint_as_float(u.z << 16), __uint_as_float(u.z & 0xffff0000u));
+    f[3] = make_float2(__uint_as_float(u.w << 16), __uint_as_float(u.w & 0xffff0000u));
 }
 __device__ __forceinline__ uint4 pack8(const float* f) {
     return make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
