@@ -54,7 +54,7 @@ def workloads():
 
 
 # side-stream kernels forked at the same point as a main-stream kernel and overlapping it
-OVERLAP = {"dxa_tc": ("dinput_act",)}
+OVERLAP = {}
 # side-stream kernels whose event window spans main-chain kernels running beside them (the window
 # is not the kernel's own duration): not candidates for the dominant kernel
 WINDOWED = ("wgrad_tc_full", "wgrad_tc_active")
@@ -127,10 +127,13 @@ def kernel_model(cfg, T):
             add("colsum", T * 16 * f32)
         if Ks[t] > 1:
             add("conv_wgrad_reduce", cpart)
-        # pre-map backward of the slot: dH_pre dots and the d_input copy, then the active-state
-        # gradient update dX_act += dZ W^T + H_pre d_input - cx x_act on the tensor cores
-        add("dinput_act", row + xa + row)
-        add("dxa_tc", 2 * xa32 + xa + row + 3 * T * nact[t] * b16, 2.0 * T * k * C * 3 * nact[t], "hbm")
+        # pre-map backward of the slot on the tensor cores: dX_act += dZ W^T + H_pre d_input
+        # - cx x_act, with the dH_pre dot partials (per 32 channels) and the d_input copy written in
+        # the same pass; then the partials summed per token and active stream
+        dotp = k * (C // 32) * T * f32
+        add("dxa_tc", 2 * xa32 + xa + row + row + dotp + 3 * T * nact[t] * b16,
+            2.0 * T * k * C * 3 * nact[t], "hbm")
+        add("dots_act", dotp + T * k * 4 + T * k * f32)
     if hr:
         add("colsum", N * C * N * f32)
     # dH_pre of the inactive streams: their X rows and the G d_input rows read

@@ -209,6 +209,7 @@ Layout make_layout(const Dims& d, int64_t T) {
     L.red = o; o = al(o + t * L.nslice * NRED * 4);
     L.dxact = o; o = al(o + t * d.k * d.C * 4);
     L.dinput = o; o = al(o + (size_t)d.G * t * d.C * 2);
+    L.dotp = o; o = al(o + (size_t)d.k * (d.C / 32) * t * 4);
     L.dp = o; o = al(o + t * d.k * 4);
     L.dhpre = o; o = al(o + t * d.G * d.N * 4);
     L.tokmat = o; o = al(o + t * TOKMAT * 4);
@@ -936,25 +937,25 @@ xhc_status xhc_pre_bwd(const xhc_handle* h, int slot, int64_t T, const xhc_param
     uint16_t* dinput = c.W<uint16_t>(c.L.dinput);
     const int n = d.nact[slot];
     const bool tc = dxa_tc_ok(T32, d.k, d.C, n);
-    // with the tensor-core update the dH_pre dots and the d_input copy do not touch dX_act: side
-    // stream, overlapping the update
-    const cudaStream_t sa = tc ? fork_from(c.st) : c.st;
-    XHC_K("dinput_act", sa, launch_dinput_act(d, slot, T32, tc ? 0 : 1, d_input, c.xact(slot),
-                             c.S<float>(c.L.hpre), c.S<int>(c.L.I), c.W<float>(c.L.dxact),
-                             c.W<float>(c.L.dhpre), dinput, c.W<float>(c.L.tokmat), sa));
     if (tc) {
-        // post_bwd(slot) left dZ_act of this slot in the workspace
+        // post_bwd(slot) left dZ_act of this slot in the workspace; the update also forms the
+        // dH_pre dots of the active streams (per 32 channels) and copies d_input
         XHC_K("dxa_tc", c.st, launch_dxa_tc(d, slot, T32, c.W<float>(c.L.dz), n, act_segs(d, P, slot),
                                             c.W<uint16_t>(c.L.dz16), c.W<uint16_t>(c.L.w16), d_input,
                                             c.S<float>(c.L.hpre), c.S<int>(c.L.I), c.xact(slot),
                                             c.W<float>(c.L.tokmat), c.W<float>(c.L.dxact),
-                                            c.W<int>(c.L.err), c.st));
+                                            c.W<float>(c.L.dotp), dinput, c.W<int>(c.L.err), c.st));
+        XHC_K("dots_act", c.st, launch_dots_act(d, slot, T32, c.W<float>(c.L.dotp), c.S<int>(c.L.I),
+                                                c.W<float>(c.L.dhpre), c.st));
+    } else {
+        XHC_K("dinput_act", c.st, launch_dinput_act(d, slot, T32, 1, d_input, c.xact(slot),
+                                    c.S<float>(c.L.hpre), c.S<int>(c.L.I), c.W<float>(c.L.dxact),
+                                    c.W<float>(c.L.dhpre), dinput, c.W<float>(c.L.tokmat), c.st));
     }
-    if (slot != 0) return join_into(c.st, sa);
+    if (slot != 0) return XHC_OK;
     if (d.hr)
         XHC_K("colsum", c.st, launch_colsum(P->W_r, d.N * d.C, d.N, d.N, c.W<float>(c.L.wsum), 0,
                                c.W<float>(c.L.colscr), c.st));
-    if (join_into(c.st, sa) != XHC_OK) return XHC_ERR_CUDA;
     XHC_K("full_dots", c.st, launch_full_dots(d, T32, X, dinput, c.S<int>(c.L.I), c.W<float>(c.L.dhpre), c.st));
     XHC_K("full_coef", c.st, launch_full_coef(d, T32, c.W<float>(c.L.dhpre), c.S<float>(c.L.hpre),
                               c.S<float>(c.L.zfull), c.S<float>(c.L.stats), c.W<float>(c.L.wsum),

@@ -717,11 +717,16 @@ struct DxArgs {
     int scal_ld;
     int* err;
     uint64_t wait_ns;     // limit of every bounded wait
+    float* dotp;          // active epilogue: [k][ncg][T] dot partials over 32-channel groups
+    uint16_t* dcopy;      // active epilogue: [G][T][C] copies of d_input (written by slot-0 tiles)
+    int ncg;              // active epilogue: C / 32
 };
 
 // ACT = true (the instantiated form): active-state epilogue, "streams" are the k active slots j:
 //              dX_act[t][j][c] += acc + H_pre[t][slot][I_j] d_input[t][c] - cx_t x_act[t][j][c]
-//              (X = x_act of the slot, scal = the per-token matrices with cx at 112).
+//              (X = x_act of the slot, scal = the per-token matrices with cx at 112); from the
+//              same loads, the dH_pre dot <x_act_j, d_input> of each 32-channel group (dotp) and,
+//              in the j = 0 tiles, the workspace copy of d_input (dcopy).
 // ACT = false: a full-state epilogue over the N streams; not instantiated (the full-state dX is
 // k_dxf_tc, which also adds the dense-read gradient of the non-active rows).
 template <bool ACT>
@@ -893,7 +898,8 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
                 load_pass(2);
                 load_pass(3);
                 if (hh == 0) {
-                    if (!mbar_wait(smem_u32(&bars[4 + s]), (uint32_t)((n >> 1) & 1), a.wait_ns)) {
+                    // one decision per warp (the TMEM reads and the shuffles below are warp-wide)
+                    if (!__all_sync(0xffffffffu, mbar_wait(smem_u32(&bars[4 + s]), (uint32_t)((n >> 1) & 1), a.wait_ns))) {
                         atomicExch(a.err, 14);
                         ok = false;
                         break;
@@ -917,7 +923,8 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
                 for (int pass = 0; pass < 4; ++pass) {
                     const int rr = pass * 8 + (lane >> 2);
                     const int t = tt * BM + quarter * 32 + rr;
-                    if (t >= a.T) continue;
+                    const bool live = t < a.T;    // the same for the 4 lanes of a row
+                    if (!ACT && !live) continue;
                     const float* m = meta + rr * 8;
                     const float* ac = tileb + rr * 33 + cq;
                     float x[8], v[8];
@@ -940,9 +947,22 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
                         o1.y = v[5] + ac[5] + (hq * g[5] - cx * x[5]);
                         o1.z = v[6] + ac[6] + (hq * g[6] - cx * x[6]);
                         o1.w = v[7] + ac[7] + (hq * g[7] - cx * x[7]);
-                        float4* dst = reinterpret_cast<float4*>(a.dxa + ((long long)t * a.k + i) * a.C + c);
-                        dst[0] = o0;
-                        dst[1] = o1;
+                        // dH_pre of stream I_i: <x_act_i, d_input>, this lane's 8 channels, then
+                        // the row's 32 (4 lanes); rows past T hold zeros
+                        float dp = x[0] * g[0];
+#pragma unroll
+                        for (int e = 1; e < 8; ++e) dp = fmaf(x[e], g[e], dp);
+                        if (live) {
+                            float4* dst = reinterpret_cast<float4*>(a.dxa + ((long long)t * a.k + i) * a.C + c);
+                            dst[0] = o0;
+                            dst[1] = o1;
+                            if (i == 0)
+                                *reinterpret_cast<uint4*>(a.dcopy + ((long long)a.slot * a.T + t) * a.C + c) = gr[pass];
+                        }
+                        dp += __shfl_xor_sync(0xffffffffu, dp, 1);
+                        dp += __shfl_xor_sync(0xffffffffu, dp, 2);
+                        if (live && (lane & 3) == 0)
+                            a.dotp[((long long)i * a.ncg + ct * (DX_BN / 32) + cg) * a.T + t] = dp;
                     } else {
                         const int j = __float_as_int(m[0]);
                         const long long off = ((long long)t * a.N + i) * a.C + c;
@@ -1351,7 +1371,7 @@ bool dxa_tc_ok(int T, int k, int C, int nact) {
 cudaError_t launch_dxa_tc(const Dims& d, int slot, int T, const float* dzs, int nact, const WSegs& W,
                           uint16_t* dz3, uint16_t* w3, const uint16_t* d_input, const float* hpre,
                           const int* I, const uint16_t* xact, const float* tokmat, float* dxact,
-                          int* err, cudaStream_t st) {
+                          float* dotp, uint16_t* dcopy, int* err, cudaStream_t st) {
     const int KC = d.k * d.C;
     const int K3 = 3 * nact;
     const int ld = (K3 + 7) / 8 * 8;
@@ -1381,6 +1401,7 @@ cudaError_t launch_dxa_tc(const Dims& d, int slot, int T, const float* dzs, int 
     a.dinput = d_input; a.hpre = hpre; a.I = I; a.dxa = dxact; a.err = err;
     a.wait_ns = debug_wait_ns();
     a.X = xact; a.scal = tokmat; a.scal_ld = TOKMAT;
+    a.dotp = dotp; a.dcopy = dcopy; a.ncg = d.C / 32;
     // one operand stage (the MMA of a tile is short next to its epilogue): the shared memory
     // left over is L1 for the epilogue's in-flight reads
     a.ns = 1;
@@ -1389,6 +1410,34 @@ cudaError_t launch_dxa_tc(const Dims& d, int slot, int T, const float* dzs, int 
     e = cudaFuncSetAttribute((const void*)k_dx_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
     k_dx_tc<true><<<a.P, DX_THREADS, sm, st>>>(ma, mb, a); note_launch();
+    return cudaGetLastError();
+}
+
+namespace {
+// dH_pre[t][slot][I_j] from the dot partials of k_dx_tc<true>: one thread per (j, t), the C / 32
+// groups summed in four interleaved chains combined in a fixed order
+__global__ void k_dots_act(const float* __restrict__ dotp, int T, int k, int ncg, int G, int N, int slot,
+                           const int* __restrict__ I, float* __restrict__ dhpre) {
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)k * T) return;
+    const int j = (int)(idx / T), t = (int)(idx - (long long)j * T);
+    const float* p = dotp + (long long)j * ncg * T + t;
+    float s[4] = {0.f, 0.f, 0.f, 0.f};
+    int g = 0;
+    for (; g + 4 <= ncg; g += 4) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) s[q] += p[(long long)(g + q) * T];
+    }
+    for (; g < ncg; ++g) s[0] += p[(long long)g * T];
+    dhpre[((long long)t * G + slot) * N + I[(long long)t * k + j]] = (s[0] + s[1]) + (s[2] + s[3]);
+}
+}  // namespace
+
+cudaError_t launch_dots_act(const Dims& d, int slot, int T, const float* dotp, const int* I, float* dhpre,
+                            cudaStream_t st) {
+    const long long n = (long long)d.k * T;
+    k_dots_act<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(dotp, T, d.k, d.C / 32, d.G, d.N, slot, I, dhpre);
+    note_launch();
     return cudaGetLastError();
 }
 

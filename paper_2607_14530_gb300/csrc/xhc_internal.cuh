@@ -94,6 +94,7 @@ struct Layout {
     size_t red;             // f32 [T][nslice][NRED]: per-slice reduction partials
     size_t dxact;           // f32 [T][k][C]: active-state gradient
     size_t dinput;          // bf16 [G][T][C]: copies of d_input
+    size_t dotp;            // f32 [k][C/32][T]: <x_act_j, d_input> over 32-channel groups
     size_t dp;              // f32 [T][k]: routing-weight gradient accumulated over slots
     size_t dhpre;           // f32 [T][G][N]
     size_t tokmat;          // f32 [T][TOKMAT]: per-token matrices (E, D, H_res, scalars)
@@ -305,11 +306,16 @@ cudaError_t launch_wgrad_tc(const uint16_t* A, int T, int E, const float* dz, in
 bool dx_tc_ok(int T, int N, int C, int nfull, int G);
 bool dxa_tc_ok(int T, int k, int C, int nact);
 // dX_act += dZ_act W_act^T (three-term bf16 split on the tensor cores) + H_pre[slot][I_j] d_input
-//           - cx x_act (the write-back's own term, cx per token in tokmat)
+//           - cx x_act (the write-back's own term, cx per token in tokmat);
+// in the same pass: dotp[j][g][t] = <x_act_j, d_input> over channels 32 g .. 32 g + 31, and the
+// copy dcopy[slot][t][:] = d_input[t][:]
 cudaError_t launch_dxa_tc(const Dims& d, int slot, int T, const float* dzs, int nact, const WSegs& W,
                           uint16_t* dz3, uint16_t* w3, const uint16_t* d_input, const float* hpre,
                           const int* I, const uint16_t* xact, const float* tokmat, float* dxact,
-                          int* err, cudaStream_t st);
+                          float* dotp, uint16_t* dcopy, int* err, cudaStream_t st);
+// dH_pre[t][slot][I_j] = sum over the C/32 groups g of dotp[j][g][t] (g in order)
+cudaError_t launch_dots_act(const Dims& d, int slot, int T, const float* dotp, const int* I, float* dhpre,
+                            cudaStream_t st);
 cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, uint16_t* dz16,
                          uint16_t* w16, const uint16_t* X, const uint16_t* dinput, const float* hpre,
                          const int* I, const float* dxact, const float* scal, int scal_ld,
