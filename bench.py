@@ -765,7 +765,7 @@ def run_stack(args, wl_name):
             self.s = nn.Parameter(torch.tensor(0.03125))
 
         def forward(self, x):
-            return x.float() * self.s
+            return x * self.s.to(x.dtype)
 
     stack = XhcStack(cfg, L, lambda l, t: Gain(), seed=seed).to(dev)
     hid = synth.normal_bf16_on((T, cfg.C), seed + 5, dev)
@@ -808,10 +808,32 @@ def run_stack(args, wl_name):
             g.backward(P, X, dX, outs, dins, G_, saved, ws, d_outs=d_outs)
 
     bare_ms = timed(bare_step, args.steps)
+    # the parts of a stack step that are neither the library's group calls nor glue: the L x G
+    # sublayers' own forward and backward, and the stream expansion and sum with their backward
+    gains = [Gain().to(dev) for _ in range(L * cfg.G)]
+
+    def sublayer_step():
+        for m in gains:
+            x = hid.detach().requires_grad_(True)
+            m(x).backward(hid)
+
+    sub_ms = timed(sublayer_step, args.steps)
+    gx = stack.groups[0].g
+
+    def expand_sum_step():
+        Xs = gx.stream_expand(hid)
+        gx.stream_sum(Xs)
+        gx.stream_expand(dy)
+        gx.stream_sum(Xs)
+
+    es_ms = timed(expand_sum_step, args.steps)
     line = {"metric": "stack of groups through the autograd glue: tokens/s fwd+bwd", "unit": "tokens/s",
-            "workload": f"{L} groups of: {desc}; sublayers: scalar gains", "tokens": T,
+            "workload": f"{L} groups of: {desc}; sublayers: scalar gains (bf16)", "tokens": T,
             "stack_ms": stack_ms, "value": T / (stack_ms / 1000.0),
-            "bare_group_calls_ms": bare_ms, "glue_overhead": stack_ms / bare_ms - 1.0,
+            "bare_group_calls_ms": bare_ms, "sublayers_ms": sub_ms, "expand_sum_ms": es_ms,
+            "glue_overhead": (stack_ms - sub_ms - es_ms) / bare_ms - 1.0,
+            "note": "glue_overhead: the stack step less the sublayers' own work and the stream "
+                    "expansion / sum, over the bare group calls, minus 1",
             "steps": args.steps, "dtype": "f32", "data": "synthetic"}
     print(json.dumps(line), flush=True)
 

@@ -14,7 +14,10 @@ those steps for autograd; every step of the connection op itself runs in libxhc'
   pre_bwd(t) in reverse slot order.  The residual state is updated in place (xhc.h: the library
   writes the k active rows of X and restores them in the backward), so the state tensor flows
   through the groups of a stack without copies; the library's saved / workspace buffers are kept
-  per group and per token count.
+  per group and per token count.  So does the state gradient: a group's backward updates the
+  gradient it receives in place when that tensor is the one the next group or the stream sum
+  returned (a hook on the state that keeps the gradient it is given must copy it); any other
+  incoming gradient is copied first.
 * ``XhcStack``: expansion, L groups, stream sum.
 """
 from __future__ import annotations
@@ -24,6 +27,13 @@ from torch import nn
 
 from . import synth
 from .xhc import Config, Group
+
+
+def _owned(t: torch.Tensor) -> torch.Tensor:
+    """Mark a state gradient this module created and hands on to autograd (nothing else keeps it):
+    the group whose backward receives it next updates it in place instead of copying it."""
+    t._xhc_owned = True
+    return t
 
 
 class StreamExpand(torch.autograd.Function):
@@ -49,7 +59,7 @@ class StreamSum(torch.autograd.Function):
 
     @staticmethod
     def backward(ctx, dy):
-        return ctx.g.stream_expand(dy.contiguous()), None
+        return _owned(ctx.g.stream_expand(dy.contiguous())), None
 
 
 class _GroupFn(torch.autograd.Function):
@@ -85,7 +95,10 @@ class _GroupFn(torch.autograd.Function):
         saved, ws, leaves, outs = ctx.io
         g, cfg = mod.g, mod.cfg
         T = X.shape[0]
-        dX = dX_out.to(torch.bfloat16).contiguous().clone()
+        if getattr(dX_out, "_xhc_owned", False) and dX_out.dtype == torch.bfloat16 and dX_out.is_contiguous():
+            dX = dX_out   # the next group's (or the stream sum's) own result: updated in place
+        else:
+            dX = dX_out.to(torch.bfloat16).contiguous().clone()
         P = mod.param_dict()
         grads = {n: torch.zeros_like(v) for n, v in P.items()}
         pp, gg = g.params(P), g.params(grads)
@@ -100,7 +113,7 @@ class _GroupFn(torch.autograd.Function):
                 d_in = torch.zeros(T, cfg.C, dtype=torch.bfloat16, device=X.device)
             g.pre_bwd(t, pp, X, d_in.to(torch.bfloat16).contiguous(), dX, gg, saved, ws)
         ctx.io = None
-        return (dX, None) + tuple(grads[n] for n in mod.names)
+        return (_owned(dX), None) + tuple(grads[n] for n in mod.names)
 
 
 class XhcGroup(nn.Module):

@@ -41,6 +41,7 @@ class FakeGroup:
 
     def post_bwd(self, t, P, X, dX, out, d_out, gg, saved, ws):
         self.log.append((self.tag, "post_bwd", t))
+        self.log.append((self.tag, "dX_ptr", dX.data_ptr()))
         a = P[f"W_post.{t}"][0, 0]
         X.copy_((X.float() - a * out.float()[:, None, :]).to(torch.bfloat16))   # restore the entry state
         d_out.copy_((a * dX.float().sum(1)).to(torch.bfloat16))
@@ -83,6 +84,9 @@ def test_group_chain_call_order_and_gradients():
     # order: forward group by group, slot by slot; backward in reverse, sublayer backward between
     fwd = [e for e in log if e[1] in ("pre_fwd", "post_fwd")]
     assert fwd == [(l, k, t) for l in range(2) for t in range(2) for k in ("pre_fwd", "post_fwd")]
+    # the state gradient passes from group 1's backward to group 0's without a copy
+    ptrs = {e[0]: e[2] for e in log if e[1] == "dX_ptr"}
+    assert ptrs[0] == ptrs[1]
     bwd = [e for e in log if e[1] in ("post_bwd", "pre_bwd", "sublayer_bwd")]
     want = []
     for l in (1, 0):
