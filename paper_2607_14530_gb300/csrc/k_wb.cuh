@@ -1126,6 +1126,8 @@ __global__ void __launch_bounds__(WT, 2) k_wb_bapp(Dims d, int slot, int T, int 
 constexpr int W8 = WT * 8;   // channels per CTA
 
 __device__ __forceinline__ uint4 ld16(const void* p) { return __ldg(reinterpret_cast<const uint4*>(p)); }
+__device__ __forceinline__ void l2_prefetch(const void* p) { asm volatile("prefetch.global.L2 [%0];" ::"l"(p)); }
+constexpr int B8_PF = 2;   // L2 prefetch distance of the one-pass attention backward, in tokens
 
 // per-token tables shared by the CTA: E[j][0] (write-back coefficient of out), H_res, I
 template <int KM>
@@ -1221,7 +1223,7 @@ __global__ void __launch_bounds__(WT) k_wb_fwd8(Dims d, int slot, int T, int TB,
 // Partial sums per W8-channel slice: P[j][0] at j*4, Q[j][i] at KM*4 + j*KM + i (the layout
 // bwd_coef reads).
 template <int KM>
-__global__ void __launch_bounds__(WT, 4) k_wb_b8(Dims d, int slot, int T, int TB,
+__global__ void __launch_bounds__(WT, 3) k_wb_b8(Dims d, int slot, int T, int TB,
                                               const uint16_t* __restrict__ out,
                                               const uint16_t* __restrict__ dX,
                                               const int* __restrict__ I,
@@ -1267,7 +1269,27 @@ __global__ void __launch_bounds__(WT, 4) k_wb_b8(Dims d, int slot, int T, int TB
     const float* pd = dxact + t0 * kC + c;
     // next token's rows: out, dXn_j (bf16 rows of dX, or fp32 active gradient), x_j (last)
     uint4 on = make_uint4(0, 0, 0, 0), dn0[KM], dn1[KM], xn[KM];
+    // an L2 prefetch of the rows B8_PF tokens further on, one request per 128-byte line
+    const bool pf32 = (threadIdx.x & 3) == 0, pf16 = (threadIdx.x & 7) == 0;
+    auto prefetch = [&](int tt) {
+        if (B8_PF == 0 || !act || tt >= ntok) return;
+        const long long dt = (long long)B8_PF;
+        if (pf16) l2_prefetch(po + dt * C);
+#pragma unroll
+        for (int j = 0; j < KM; ++j) {
+            if (j >= k) continue;
+            if (last) {
+                if (pf16) {
+                    l2_prefetch(pX + dt * NC + (long long)Ish[tt * KM + j] * C);
+                    l2_prefetch(px + dt * kC + j * (long long)C);
+                }
+            } else if (pf32) {
+                l2_prefetch(pd + dt * kC + j * (long long)C);
+            }
+        }
+    };
     auto load = [&](int tt) {
+        prefetch(tt + B8_PF);
 #pragma unroll
         for (int j = 0; j < KM; ++j) {
             dn0[j] = make_uint4(0, 0, 0, 0);
