@@ -1081,22 +1081,23 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
     const uint32_t tmem = *tmem_slot;
     const int N = a.N;
     const int ndin = N - a.m;   // leading tiles of a block that may read d_input (streams m..N-1)
-    const long long nblk = (a.ntiles > blockIdx.x) ? (a.ntiles - 1 - blockIdx.x) / a.P + 1 : 0;
-    const long long nloc = nblk * N;
+    const int nblk = (a.ntiles > blockIdx.x) ? (int)((a.ntiles - 1 - blockIdx.x) / a.P) + 1 : 0;
+    const int nloc = nblk * N;   // < 2^31: the host checks ntiles * N
     // local tile n: block n / N of this CTA, position p in the block, stream (p + m) mod N
-    auto decode = [&](long long n, int& p, int& tt, int& cb, int& i) {
-        const long long b = n / N;
-        p = (int)(n - b * N);
-        const long long block = blockIdx.x + b * a.P;
-        tt = (int)(block / a.CT);
-        cb = (int)(block - (long long)tt * a.CT);
+    // (32-bit arithmetic: the divisions run per tile in every role)
+    auto decode = [&](int n, int& p, int& tt, int& cb, int& i) {
+        const int b = n / N;
+        p = n - b * N;
+        const int block = (int)blockIdx.x + b * a.P;
+        tt = block / a.CT;
+        cb = block - tt * a.CT;
         i = p + a.m;
         if (i >= N) i -= N;
     };
 
     if (warp == 0) {
         if (lane == 0) {
-            for (long long n = 0; n < nloc; ++n) {
+            for (int n = 0; n < nloc; ++n) {
                 if (*s_abort) break;
                 int p, tt, cb, i;
                 if (DG_PF > 0 && n + DG_PF < nloc) {
@@ -1109,7 +1110,7 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
                         for (int q = 0; q < a.G; ++q) tma_prefetch_2d(&tmG, cb * DG_BN, q * a.T + tt * BM);
                 }
                 decode(n, p, tt, cb, i);
-                const long long blk = n / N;
+                const int blk = n / N;
                 if (p == 0) {
                     if (blk >= 1 && !mbar_wait(smem_u32(&bars[1]), (uint32_t)((blk - 1) & 1), a.wait_ns)) {
                         atomicExch(a.err, 31);
@@ -1159,9 +1160,9 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
     } else if (warp == 1) {
         if (lane == 0) {
             const uint32_t idesc = idesc_bf16(BM, DG_BN);
-            for (long long n = 0; n < nloc; ++n) {
-                const long long blk = n / N;
-                const int p = (int)(n - blk * N);
+            for (int n = 0; n < nloc; ++n) {
+                const int blk = n / N;
+                const int p = n - blk * N;
                 const int s = (int)(n & 1);
                 bool ok = (p != 0) || mbar_wait(smem_u32(&bars[0]), (uint32_t)(blk & 1), a.wait_ns);
                 ok = ok && mbar_wait(smem_u32(&bars[2 + s]), (uint32_t)((n >> 1) & 1), a.wait_ns);
@@ -1204,10 +1205,10 @@ k_dxf_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtens
         int cur_blk = -1;
         uint32_t ib[2] = {0xffffffffu, 0xffffffffu};
         float sa = 0.f, sb = 0.f;
-        for (long long n = grp; n < nloc; n += 2) {
+        for (int n = grp; n < nloc; n += 2) {
             int p, tt, cb, i;
             decode(n, p, tt, cb, i);
-            const long long blk = n / N;
+            const int blk = n / N;
             const bool usesg = p < ndin;
             const int t = tt * BM + r;
             // the dense-read weights of this tile's rows: loads issued first, used after the waits
@@ -1452,7 +1453,8 @@ static size_t dxf_smem(int nfull, int G) {
 // block may use
 bool dx_tc_ok(int T, int N, int C, int nfull, int G) {
     return T >= BM && C % DG_BN == 0 && nfull <= 3 * BK && N >= 2 && G >= 1 && G <= 4 &&
-           dxf_smem(nfull, G) <= 232448;
+           dxf_smem(nfull, G) <= 232448 &&
+           (long long)((T + BM - 1) / BM) * (C / DG_BN) * N < (1LL << 31);   // 32-bit tile indices
 }
 
 cudaError_t launch_dx_tc(const Dims& d, int T, const float* dz, const WSegs& W, uint16_t* dz16,
