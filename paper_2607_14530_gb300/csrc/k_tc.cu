@@ -266,17 +266,21 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                 atomicExch(a.err, 6);
                 s_abort = 1;
             }
-            long long it = 0;
+            // stage s and phase ph of load `it`, tile m and k-block kb of g: advanced step by
+            // step (no division per k-block)
+            int it = 0, s = 0, m = (int)(g0 / a.KB), kb = (int)(g0 % a.KB);
+            uint32_t ph = 0;
             for (long long g = g0; g < g1 && !*(volatile int*)&s_abort; ++g, ++it) {
-                const int s = (int)(it % STAGES);
-                const uint32_t ph = (uint32_t)((it / STAGES) & 1);
+                if (g > g0) {
+                    if (++kb == a.KB) { kb = 0; ++m; }
+                    if (++s == STAGES) { s = 0; ph ^= 1u; }
+                }
                 if (it >= STAGES && !mbar_wait(smem_u32(&bars[STAGES + s]), ph ^ 1, a.wait_ns)) {
                     atomicExch(a.err, 1);
                     s_abort = 1;
                     break;
                 }
                 if (*(volatile int*)&s_abort) break;
-                const int m = (int)(g / a.KB), kb = (int)(g % a.KB);
                 const uint32_t full = smem_u32(&bars[s]);
                 mbar_expect_tx(full, STAGE);
                 unsigned char* st = smem + (size_t)s * STAGE;
@@ -299,7 +303,8 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
         if (lane == 0) {
             const int nb_chunk = a.NB / a.nchunk;
             const uint32_t idesc = idesc_bf16(BM, nb_chunk, A_MN);
-            long long it = 0;
+            int s = 0;          // stage of the next k-block and its phase, advanced per k-block
+            uint32_t ph = 0;
             int seg = 0;
             long long g = g0;
             while (g < g1) {
@@ -313,9 +318,7 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                 }
                 tc_fence_after();
                 bool first = true;
-                for (; g < gend; ++g, ++it) {
-                    const int s = (int)(it % STAGES);
-                    const uint32_t ph = (uint32_t)((it / STAGES) & 1);
+                for (; g < gend; ++g) {
                     if (!mbar_wait(smem_u32(&bars[s]), ph, a.wait_ns)) {
                         atomicExch(a.err, 3);
                         s_abort = 1;
@@ -341,6 +344,7 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                     }
                     first = false;
                     mma_commit(smem_u32(&bars[STAGES + s]));  // stage free once these MMAs finish
+                    if (++s == STAGES) { s = 0; ph ^= 1u; }
                 }
                 if (*(volatile int*)&s_abort) break;
                 mma_commit(smem_u32(&bars[2 * STAGES]));     // accumulator ready
@@ -351,7 +355,8 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
         // ---------------- statistics + epilogue (warps 2..5) ----------------
         const int quarter = warp & 3;           // TMEM lanes this warp may access
         const int r = quarter * 32 + lane;      // tile row = token within the tile
-        long long it = 0;
+        int s = 0;                              // stage of the next k-block and its phase
+        uint32_t ph = 0;
         int seg = 0;
         long long g = g0;
         bool ok = true;
@@ -369,9 +374,7 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
 #pragma unroll
                 for (int e = 0; e < 4; ++e) a1[e] = a2[e] = make_float2(0.f, 0.f);
             }
-            for (; g < gend; ++g, ++it) {
-                const int s = (int)(it % STAGES);
-                const uint32_t ph = (uint32_t)((it / STAGES) & 1);
+            for (; g < gend; ++g) {
                 if (!mbar_wait(smem_u32(&bars[s]), ph, a.wait_ns)) {
                     atomicExch(a.err, 4);
                     ok = false;
@@ -403,6 +406,7 @@ k_proj_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUten
                 }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&bars[STAGES + s]));
+                if (++s == STAGES) { s = 0; ph ^= 1u; }
             }
             if (!ok) break;
             // the segment's slot: index of this CTA among those covering tile m
@@ -762,15 +766,16 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    const long long nloc = (a.ntiles > blockIdx.x) ? (a.ntiles - 1 - blockIdx.x) / a.P + 1 : 0;
+    // 32-bit tile arithmetic (the host keeps ntiles below 2^31): the divisions run per tile
+    const int nloc = (a.ntiles > blockIdx.x) ? (int)((a.ntiles - 1 - blockIdx.x) / a.P) + 1 : 0;
 
     if (warp == 0) {
         if (lane == 0) {
-            for (long long n = 0; n < nloc; ++n) {
-                const long long tile = blockIdx.x + n * a.P;
-                const int i = (int)(tile % a.N);
-                const long long rest = tile / a.N;
-                const int ct = (int)(rest % a.CT), tt = (int)(rest / a.CT);
+            for (int n = 0; n < nloc; ++n) {
+                const int tile = (int)blockIdx.x + n * a.P;
+                const int i = tile % a.N;
+                const int rest = tile / a.N;
+                const int ct = rest % a.CT, tt = rest / a.CT;
                 const int s = (int)(n & nsh);
                 if (n >= NS && !mbar_wait(smem_u32(&bars[2 + s]), (uint32_t)(((n >> nsh) - 1) & 1), a.wait_ns)) {
                     atomicExch(a.err, 11);
@@ -789,7 +794,7 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
     } else if (warp == 1) {
         if (lane == 0) {
             const uint32_t idesc = idesc_bf16(BM, DX_BN);
-            for (long long n = 0; n < nloc; ++n) {
+            for (int n = 0; n < nloc; ++n) {
                 const int s = (int)(n & 1);        // TMEM buffer
                 const int os = (int)(n & nsh);     // operand stage
                 if (!mbar_wait(smem_u32(&bars[os]), (uint32_t)((n >> nsh) & 1), a.wait_ns)) {
@@ -825,11 +830,11 @@ k_dx_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtenso
         const int chalf = (ew & 7) >> 2;           // 64-column half of the tile
         float* tileb = reinterpret_cast<float*>(smem + NS * STAGE + 128) + ew * (32 * 33 + 32 * 8);
         float* meta = tileb + 32 * 33;             // per row: j, h0..h3, sa, sb
-        for (long long n = grp; n < nloc; n += 2) {
-            const long long tile = blockIdx.x + n * a.P;
-            const int i = (int)(tile % a.N);
-            const long long rest = tile / a.N;
-            const int ct = (int)(rest % a.CT), tt = (int)(rest / a.CT);
+        for (int n = grp; n < nloc; n += 2) {
+            const int tile = (int)blockIdx.x + n * a.P;
+            const int i = tile % a.N;
+            const int rest = tile / a.N;
+            const int ct = rest % a.CT, tt = rest / a.CT;
             const int s = (int)(n & 1);
             {
                 // per-row metadata of this lane's row (row-per-lane, matches the TMEM layout)
@@ -1365,8 +1370,8 @@ __global__ void k_pack3(WSegs W, int n, int rows, int ld, int lo_part, uint16_t*
 
 // two operand stages of up to two k-blocks each fit the 227 KB of shared memory
 bool dxa_tc_ok(int T, int k, int C, int nact) {
-    (void)k;
-    return T >= BM && C % DX_BN == 0 && 3 * nact <= 2 * BK;
+    return T >= BM && C % DX_BN == 0 && 3 * nact <= 2 * BK &&
+           (long long)((T + BM - 1) / BM) * (C / DX_BN) * k < (1LL << 31);   // 32-bit tile indices
 }
 
 cudaError_t launch_dxa_tc(const Dims& d, int slot, int T, const float* dzs, int nact, const WSegs& W,
