@@ -1420,29 +1420,35 @@ cudaError_t launch_dxa_tc(const Dims& d, int slot, int T, const float* dzs, int 
 }
 
 namespace {
-// dH_pre[t][slot][I_j] from the dot partials of k_dx_tc<true>: one thread per (j, t), the C / 32
-// groups summed in four interleaved chains combined in a fixed order
-__global__ void k_dots_act(const float* __restrict__ dotp, int T, int k, int ncg, int G, int N, int slot,
-                           const int* __restrict__ I, float* __restrict__ dhpre) {
-    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-    if (idx >= (long long)k * T) return;
-    const int j = (int)(idx / T), t = (int)(idx - (long long)j * T);
-    const float* p = dotp + (long long)j * ncg * T + t;
-    float s[4] = {0.f, 0.f, 0.f, 0.f};
-    int g = 0;
-    for (; g + 4 <= ncg; g += 4) {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) s[q] += p[(long long)(g + q) * T];
+// dH_pre[t][slot][I_j] from the dot partials of k_dx_tc<true>: a block per (32 tokens, j); warp w
+// sums the groups g = w, w + 8, ... of its lane's token (coalesced 128-byte rows), and the eight
+// warp sums are added in warp order (a fixed order: the result does not depend on the schedule)
+__global__ void __launch_bounds__(256) k_dots_act(const float* __restrict__ dotp, int T, int k, int ncg,
+                                                  int G, int N, int slot, const int* __restrict__ I,
+                                                  float* __restrict__ dhpre) {
+    __shared__ float part[8][32];
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    const int j = blockIdx.y, t = blockIdx.x * 32 + lane;
+    float s = 0.f;
+    if (t < T) {
+        const float* p = dotp + (long long)j * ncg * T + t;
+        for (int g = w; g < ncg; g += 8) s += p[(long long)g * T];
     }
-    for (; g < ncg; ++g) s[0] += p[(long long)g * T];
-    dhpre[((long long)t * G + slot) * N + I[(long long)t * k + j]] = (s[0] + s[1]) + (s[2] + s[3]);
+    part[w][lane] = s;
+    __syncthreads();
+    if (w == 0 && t < T) {
+        float v = part[0][lane];
+#pragma unroll
+        for (int q = 1; q < 8; ++q) v += part[q][lane];
+        dhpre[((long long)t * G + slot) * N + I[(long long)t * k + j]] = v;
+    }
 }
 }  // namespace
 
 cudaError_t launch_dots_act(const Dims& d, int slot, int T, const float* dotp, const int* I, float* dhpre,
                             cudaStream_t st) {
-    const long long n = (long long)d.k * T;
-    k_dots_act<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(dotp, T, d.k, d.C / 32, d.G, d.N, slot, I, dhpre);
+    const dim3 grid((unsigned)((T + 31) / 32), (unsigned)d.k);
+    k_dots_act<<<grid, 256, 0, st>>>(dotp, T, d.k, d.C / 32, d.G, d.N, slot, I, dhpre);
     note_launch();
     return cudaGetLastError();
 }
