@@ -54,8 +54,7 @@ __global__ void __launch_bounds__(256) k_rowproj(const uint16_t* __restrict__ A,
             const int kr = k0 + kk;
             float v = 0.f;
             if (o < n && kr < kend) {
-                const int s = seg_of(W, o);
-                v = __ldg(W.ptr[s] + (int64_t)kr * W.width[s] + (o - W.off[s]));
+                v = seg_elem<true>(W, kr, o);
             }
             Ws[kk][o] = v;
         }
@@ -197,8 +196,7 @@ __global__ void __launch_bounds__(256) k_gemm_dzw(const float* __restrict__ dz, 
             const int e = e0 + ee, o = o0 + oo;
             float v = 0.f;
             if (e < E && o < n) {
-                const int s = seg_of(W, o);
-                v = __ldg(W.ptr[s] + (int64_t)e * W.width[s] + (o - W.off[s]));
+                v = seg_elem<true>(W, e, o);
             }
             Wt[oo][ee] = v;
         }
@@ -272,8 +270,7 @@ __global__ void __launch_bounds__(256) k_full_dx(Dims d, int T, const float* __r
             const int e = e0 + ee, o = o0 + oo;
             float v = 0.f;
             if (e < E && o < n) {
-                const int s = seg_of(W, o);
-                v = __ldg(W.ptr[s] + (int64_t)e * W.width[s] + (o - W.off[s]));
+                v = seg_elem<true>(W, e, o);
             }
             Wt[oo][ee] = v;
         }
@@ -414,11 +411,17 @@ __global__ void k_wgrad_reduce(const float* __restrict__ wpart, int splits, int 
     const int e = (int)(idx / n), o = (int)(idx - (int64_t)e * n);
     float s = 0.f;
     for (int q = 0; q < splits; ++q) s += wpart[(int64_t)q * E * n + idx];
-    int sg = 0;
-    for (int q = 1; q < G.n; ++q)
-        if (o >= G.off[q]) sg = q;
-    float* dst = G.ptr[sg] + (int64_t)e * G.width[sg] + (o - G.off[sg]);
-    *dst += s;
+    // the segment of column o, selected with static indices (no local copy of the parameter)
+    float* p = G.ptr[0];
+    int width = G.width[0], off = G.off[0];
+#pragma unroll
+    for (int q = 1; q < MAXSEG; ++q)
+        if (q < G.n && o >= G.off[q]) {
+            p = G.ptr[q];
+            width = G.width[q];
+            off = G.off[q];
+        }
+    p[(int64_t)e * width + (o - off)] += s;
 }
 
 cudaError_t launch_wgrad_reduce(const float* wpart, int splits, int E, int n, const WSegsOut& G,

@@ -209,14 +209,25 @@ __global__ void k_conv_wgrad_reduce(Dims d, const float* __restrict__ cpart, int
     const int idx = blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= d.kapsum * d.C) return;
     const int q = idx / d.C, c = idx - q * d.C;
-    float s = 0.f;
-    for (int tile = 0; tile < ntiles; ++tile) s += cpart[((int64_t)tile * d.kapsum + q) * d.C + c];
-    int j = 0, off = 0;
-    while (q >= off + d.kap[j]) {
-        off += d.kap[j];
-        ++j;
+    // four interleaved partial sums over the runs, added in a fixed order
+    const float* p = cpart + (int64_t)q * d.C + c;
+    const int64_t step = (int64_t)d.kapsum * d.C;
+    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+    int tile = 0;
+    for (; tile + 4 <= ntiles; tile += 4) {
+        s0 += p[(int64_t)tile * step];
+        s1 += p[(int64_t)(tile + 1) * step];
+        s2 += p[(int64_t)(tile + 2) * step];
+        s3 += p[(int64_t)(tile + 3) * step];
     }
-    g.w[j][(q - off) * d.C + c] += s;
+    for (; tile < ntiles; ++tile) s0 += p[(int64_t)tile * step];
+    const float s = (s0 + s1) + (s2 + s3);
+    // the component of row q, selected with static indices (no local copy of the parameters)
+    const int off1 = d.kap[0], off2 = d.kap[0] + d.kap[1];
+    const int j = q >= off2 ? 2 : (q >= off1 ? 1 : 0);
+    const int off = j == 2 ? off2 : (j == 1 ? off1 : 0);
+    float* w = j == 2 ? g.w[2] : (j == 1 ? g.w[1] : g.w[0]);
+    w[(q - off) * d.C + c] += s;
 }
 
 cudaError_t launch_conv_wgrad_reduce(const Dims& d, int slot, const float* cpart, int ntiles,

@@ -474,8 +474,7 @@ __global__ void k_pack_w(WSegs W, int nfull, int NB, int K, uint16_t* __restrict
     const int e = blockIdx.x * blockDim.x + threadIdx.x;
     if (e >= K) return;
     for (int o = 0; o < nfull; ++o) {
-        const int s = seg_of(W, o);
-        const float w = W.ptr[s][(int64_t)e * W.width[s] + (o - W.off[s])];
+        const float w = seg_elem(W, e, o);
         const __nv_bfloat16 h = __float2bfloat16_rn(w);
         const float rem = w - __bfloat162float(h);
         Wpack[(int64_t)o * K + e] = __bfloat16_as_ushort(h);
@@ -1342,10 +1341,7 @@ __global__ void k_pack_rows(WSegs W, int n, int rows, int ld, uint16_t* __restri
     if (idx >= (long long)rows * ld) return;
     const int r = (int)(idx / ld), o = (int)(idx - (long long)r * ld);
     float v = 0.f;
-    if (o < n) {
-        const int s = seg_of(W, o);
-        v = W.ptr[s][(long long)r * W.width[s] + (o - W.off[s])];
-    }
+    if (o < n) v = seg_elem(W, r, o);
     dst[idx] = __bfloat16_as_ushort(__float2bfloat16_rn(v));
 }
 
@@ -1358,8 +1354,7 @@ __global__ void k_pack3(WSegs W, int n, int rows, int ld, int lo_part, uint16_t*
     float v = 0.f;
     if (col < 3 * n) {
         const int part = col / n, o = col - part * n;
-        const int sg = seg_of(W, o);
-        const float w = W.ptr[sg][(long long)r * W.width[sg] + (o - W.off[sg])];
+        const float w = seg_elem(W, r, o);
         const float hi = __bfloat162float(__float2bfloat16_rn(w));
         v = (part == lo_part) ? (w - hi) : hi;
     }

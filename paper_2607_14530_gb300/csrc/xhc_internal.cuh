@@ -196,6 +196,21 @@ __device__ __forceinline__ int seg_of(const WSegs& w, int o) {
         if (q < w.n && o >= w.off[q]) s = q;
     return s;
 }
+// W[r][o] of the segmented weight (the segment of column o): the segment's fields are selected
+// with static indices, so the kernel parameter is not copied to local memory for a dynamic index
+template <bool RO = false>
+__device__ __forceinline__ float seg_elem(const WSegs& w, long long r, int o) {
+    const float* p = w.ptr[0];
+    int width = w.width[0], off = w.off[0];
+#pragma unroll
+    for (int q = 1; q < MAXSEG; ++q)
+        if (q < w.n && o >= w.off[q]) {
+            p = w.ptr[q];
+            width = w.width[q];
+            off = w.off[q];
+        }
+    return RO ? __ldg(p + r * width + (o - off)) : p[r * width + (o - off)];
+}
 
 // ---------------------------------------------------------------------------------------------
 // Gram-Schmidt of Eq. gs expressed on the Gram matrix of u = [out, g_1, ..., g_r]:
