@@ -33,7 +33,11 @@ __device__ __forceinline__ void dec_components(const Dims& d, int slot, int t, i
     if (d.K[slot] <= 1) return;
     const int r0 = (int)(pos % R);                             // ring row of position pos
     const uint16_t* rt = ring + (long long)t * R * C + c;
-    for (int j = 0; j < d.nconv; ++j) {
+    // the component loop runs to its maximum of 3 with a guard, so that cw.w[j] and d.kap[j]
+    // are static indices (a dynamic index copies the parameter structs to local memory)
+#pragma unroll
+    for (int j = 0; j < 3; ++j) {
+        if (j >= d.nconv) break;
         float2 g = make_float2(0.f, 0.f);
         for (int i = 0; i < d.kap[j]; ++i) {
             if (pos - i < 0) break;                            // before the sequence start: zero
