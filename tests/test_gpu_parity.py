@@ -24,7 +24,7 @@ from xhc_cases import (Guarded, alpha_term_scales, ambiguity_masks, assert_alpha
 pytestmark = pytest.mark.gpu
 
 CASES = {
-    # BASELINE config 1 shapes: N=16, k=4, C=256, T=512
+    # the small flash4 shapes: N=16, k=4, C=256, T=512
     "fullA_N16k4_C256": (Config.full(16, 4, 2, 256, False, seq_len=512), 512, {}),
     "fullM_N16k4_C256": (Config.full(16, 4, 2, 256, True, seq_len=128), 512, {}),
     "flash2_N16k4_C256": (Config.flash(16, 4, 2, 256, 2, seq_len=256), 512, {}),
