@@ -164,3 +164,24 @@ def test_debug_hook_argument_checks(L):
     assert L.xhc_debug_set(99, 0) == INVALID
     assert L.xhc_debug_set(1, 0) == OK
     assert L.xhc_debug_set(2, 0) == OK
+    assert L.xhc_debug_set(3, 1) == OK    # side-stream work on the caller's stream
+    assert L.xhc_debug_set(3, 0) == OK
+
+
+def test_trace_filter_and_records_on_host(L):
+    """The trace filter parses its name list on the host; with nothing recorded, every record
+    index is out of range (no CUDA call is made)."""
+    name, ms, t0 = ctypes.c_char_p(), ctypes.c_float(), ctypes.c_float()
+    try:
+        assert L.xhc_trace_only(b" dxa_tc, read,,dots_act ") == OK
+        assert L.xhc_trace_only(b"") == OK
+        assert L.xhc_trace_only(None) == OK
+        assert L.xhc_trace_enable(1) == OK       # drops the previous records
+        assert L.xhc_trace_count() == 0
+        assert L.xhc_trace_record(0, ctypes.byref(name), ctypes.byref(ms)) == INVALID
+        assert L.xhc_trace_span(0, ctypes.byref(name), ctypes.byref(t0), ctypes.byref(ms)) == INVALID
+        assert L.xhc_trace_span(-1, ctypes.byref(name), ctypes.byref(t0), ctypes.byref(ms)) == INVALID
+        assert L.xhc_trace_span(0, None, None, None) == INVALID
+    finally:
+        L.xhc_trace_enable(0)
+        L.xhc_trace_only(None)
