@@ -16,8 +16,8 @@ those steps for autograd; every step of the connection op itself runs in libxhc'
   through the groups of a stack without copies; the library's saved / workspace buffers are kept
   per group and per token count.  So does the state gradient: a group's backward updates the
   gradient it receives in place when that tensor is the one the next group or the stream sum
-  returned (a hook on the state that keeps the gradient it is given must copy it); any other
-  incoming gradient is copied first.
+  returned and no hook or retain_grad watches the state; any other incoming gradient is copied
+  first.
 * ``XhcStack``: expansion, L groups, stream sum.
 """
 from __future__ import annotations
@@ -95,8 +95,14 @@ class _GroupFn(torch.autograd.Function):
         saved, ws, leaves, outs = ctx.io
         g, cfg = mod.g, mod.cfg
         T = X.shape[0]
-        if getattr(dX_out, "_xhc_owned", False) and dX_out.dtype == torch.bfloat16 and dX_out.is_contiguous():
-            dX = dX_out   # the next group's (or the stream sum's) own result: updated in place
+        # the incoming gradient is updated in place only when it is the next group's (or the
+        # stream sum's) own result and nothing else can hold it: a hook or retain_grad on the
+        # state (they follow the state tensor through the groups' in-place updates) receives
+        # that same tensor, so then it is copied first
+        state_watched = ctx.X.retains_grad or bool(ctx.X._backward_hooks)
+        if (getattr(dX_out, "_xhc_owned", False) and not state_watched and dX_out.dtype == torch.bfloat16
+                and dX_out.is_contiguous()):
+            dX = dX_out
         else:
             dX = dX_out.to(torch.bfloat16).contiguous().clone()
         P = mod.param_dict()

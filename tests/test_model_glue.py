@@ -110,3 +110,30 @@ def test_group_chain_call_order_and_gradients():
         for t in range(2):
             assert torch.allclose(grp.sublayers[t].s.grad, s[l][t].grad, rtol=2e-2), (l, t)
             assert torch.allclose(getattr(grp, f"W_post_{t}").grad[0, 0], a[l][t].grad, rtol=2e-2), (l, t)
+
+
+def test_state_gradient_seen_by_a_hook_is_not_overwritten():
+    """A hook that keeps the state gradient it is given (no copy), and retain_grad on the state,
+    see the gradient as it arrived: the in-place update of the groups' backward works on a copy
+    whenever the state is watched."""
+    cfg = Config.flash(4, 2, 1, 8, 2, seq_len=3)
+    log = []
+    stack = M.XhcStack(cfg, 2, lambda l, t: Scale(0.5 if t == 0 else 2.0, log, (l, t)))
+    for l, grp in enumerate(stack.groups):
+        grp.g = FakeGroup(cfg, log, l)
+    T = 6
+    g = torch.Generator().manual_seed(1)
+    h = torch.randn(T, cfg.C, generator=g).to(torch.bfloat16).requires_grad_(True)
+    dy = torch.randn(T, cfg.C, generator=g)
+    X = M.StreamExpand.apply(h, stack.groups[0].g)
+    for grp in stack.groups:
+        X = grp(X)
+    kept = []
+    X.register_hook(lambda gr: kept.append(gr))
+    X.retain_grad()
+    y = M.StreamSum.apply(X, stack.groups[0].g)
+    (y.float() * dy).sum().backward()
+    # the gradient of the final state is the stream sum's backward: dy on every stream
+    want = dy.to(torch.bfloat16)[:, None, :].expand(T, cfg.N, cfg.C)
+    assert torch.equal(kept[0], want)
+    assert torch.equal(X.grad, want)
