@@ -142,10 +142,14 @@ class XhcGroup(nn.Module):
         return {n: getattr(self, n.replace(".", "_")).detach().contiguous() for n in self.names}
 
     def buffers(self, T: int, device):
+        """(saved, workspace) for one forward call: a fresh `saved` (it carries this call's
+        forward state to its backward, so two forwards in flight, e.g. two micro-batches before
+        one backward, must not share it; the caching allocator makes it cheap) and the workspace
+        kept per token count (scratch, reusable between the phases of calls)."""
         key = (T, str(device))
         if key not in self._bufs:
-            self._bufs[key] = self.g.alloc(T, device=device)
-        return self._bufs[key]
+            self._bufs[key] = self.g.alloc_workspace(T, device=device)
+        return self.g.alloc_saved(T, device=device), self._bufs[key]
 
     def forward(self, X):
         return _GroupFn.apply(X, self, *[getattr(self, n.replace(".", "_")) for n in self.names])

@@ -336,11 +336,20 @@ class Group:
                         for t in range(G)]
         return out
 
-    def alloc(self, T: int, device="cuda"):
-        """(saved, workspace) uint8 CUDA tensors of the sizes the library asks for."""
+    def alloc_saved(self, T: int, device="cuda"):
+        """A `saved` buffer: one per forward whose backward is still to come."""
+        return torch.empty(self.saved_bytes(T), dtype=torch.uint8, device=device)
+
+    def alloc_workspace(self, T: int, device="cuda"):
+        """A `workspace` buffer (scratch, reusable between the phases of groups), error word zeroed."""
         ws = torch.empty(self.workspace_bytes(T), dtype=torch.uint8, device=device)
         ws[:256].zero_()  # device error word
-        return (torch.empty(self.saved_bytes(T), dtype=torch.uint8, device=device), ws)
+        return ws
+
+    def alloc(self, T: int, device="cuda"):
+        """(saved, workspace) uint8 CUDA tensors of the sizes the library asks for."""
+        ws = self.alloc_workspace(T, device)
+        return (self.alloc_saved(T, device), ws)
 
     def device_error(self, ws, clear: bool = False) -> int:
         """The workspace's device error word (nonzero: a bounded wait gave up).  Synchronous."""

@@ -21,8 +21,11 @@ class FakeGroup:
     def params(self, P):
         return P
 
-    def alloc(self, T, device="cpu"):
-        return None, None
+    def alloc_saved(self, T, device="cpu"):
+        return {"T": T}           # a distinct object per forward call
+
+    def alloc_workspace(self, T, device="cpu"):
+        return None
 
     def stream_expand(self, h, X=None):
         return h[:, None, :].expand(h.shape[0], self.cfg.N, h.shape[1]).contiguous()
@@ -137,3 +140,52 @@ def test_state_gradient_seen_by_a_hook_is_not_overwritten():
     want = dy.to(torch.bfloat16)[:, None, :].expand(T, cfg.N, cfg.C)
     assert torch.equal(kept[0], want)
     assert torch.equal(X.grad, want)
+
+
+class FakeGroupSaved(FakeGroup):
+    """As FakeGroup, but the backward takes the sublayer output from `saved` (what the forward
+    left there), as the library's backward takes its forward state."""
+
+    def post_fwd(self, t, P, X, out, saved, ws):
+        saved[("out", t)] = out.clone()
+        super().post_fwd(t, P, X, out, saved, ws)
+
+    def post_bwd(self, t, P, X, dX, out, d_out, gg, saved, ws):
+        super().post_bwd(t, P, X, dX, saved[("out", t)], d_out, gg, saved, ws)
+
+
+def _stack_with(cfg, fake, log):
+    stack = M.XhcStack(cfg, 2, lambda l, t: Scale(0.5 if t == 0 else 2.0, log, (l, t)))
+    for l, grp in enumerate(stack.groups):
+        grp.g = fake(cfg, log, l)
+        with torch.no_grad():
+            for t in range(cfg.G):
+                getattr(grp, f"W_post_{t}")[0, 0] = 0.25 * (1 + l + t)
+    return stack
+
+
+def test_two_forwards_before_one_backward():
+    """Two micro-batches through the same stack before one backward: each forward has its own
+    `saved`, so the gradients equal the sum of the two micro-batches run one at a time."""
+    cfg = Config.flash(4, 2, 1, 8, 2, seq_len=3)
+    T = 6
+    g = torch.Generator().manual_seed(2)
+    hs = [torch.randn(T, cfg.C, generator=g).to(torch.bfloat16) for _ in range(2)]
+    dys = [torch.randn(T, cfg.C, generator=g) for _ in range(2)]
+
+    both = _stack_with(cfg, FakeGroupSaved, [])
+    xs = [h.clone().requires_grad_(True) for h in hs]
+    ys = [both(x) for x in xs]
+    sum((y.float() * dy).sum() for y, dy in zip(ys, dys)).backward()
+
+    one = _stack_with(cfg, FakeGroupSaved, [])
+    for i in range(2):
+        x = hs[i].clone().requires_grad_(True)
+        (one(x).float() * dys[i]).sum().backward()
+        assert torch.allclose(x.grad.float(), xs[i].grad.float())
+    for (n1, p1), (n2, p2) in zip(both.named_parameters(), one.named_parameters()):
+        assert n1 == n2
+        if p1.grad is None:
+            assert p2.grad is None, n1
+        else:
+            assert torch.allclose(p1.grad, p2.grad, rtol=1e-5, atol=1e-6), n1
