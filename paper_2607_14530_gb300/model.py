@@ -146,13 +146,38 @@ class XhcGroup(nn.Module):
         forward state to its backward, so two forwards in flight, e.g. two micro-batches before
         one backward, must not share it; the caching allocator makes it cheap) and the workspace
         kept per token count (scratch, reusable between the phases of calls)."""
+        return self.g.alloc_saved(T, device=device), self.buffers_workspace(T, device)
+
+    def buffers_workspace(self, T: int, device):
         key = (T, str(device))
         if key not in self._bufs:
             self._bufs[key] = self.g.alloc_workspace(T, device=device)
-        return self.g.alloc_saved(T, device=device), self._bufs[key]
+        return self._bufs[key]
 
     def forward(self, X):
+        if not torch.is_grad_enabled():
+            return self._forward_inference(X)
         return _GroupFn.apply(X, self, *[getattr(self, n.replace(".", "_")) for n in self.names])
+
+    def _forward_inference(self, X):
+        """The forward without autograd (grad mode off: prefill or evaluation): the same calls,
+        the sublayers run without recording a graph, and `saved` is scratch kept per token count
+        (no backward will read it)."""
+        g, cfg = self.g, self.cfg
+        T = X.shape[0]
+        key = ("scratch", T, str(X.device))
+        if key not in self._bufs:
+            self._bufs[key] = g.alloc_saved(T, device=X.device)
+        saved, ws = self._bufs[key], self.buffers_workspace(T, X.device)
+        pp = g.params(self.param_dict())
+        for t in range(cfg.G):
+            inp = torch.empty(T, cfg.C, dtype=torch.bfloat16, device=X.device)
+            g.pre_fwd(t, pp, X, inp, saved, ws)
+            out = self.sublayers[t](inp)
+            if out.shape != (T, cfg.C):
+                raise ValueError(f"sublayer {t} must return [T, C], got {tuple(out.shape)}")
+            g.post_fwd(t, pp, X, out.to(torch.bfloat16).contiguous(), saved, ws)
+        return X
 
 
 class XhcStack(nn.Module):

@@ -170,3 +170,17 @@ def test_stack_matches_the_composed_oracle(cfg):
         for t in range(cfg.G):
             r = _rel(grp.sublayers[t].s.grad, ref["Ss"][l][t].grad)
             assert r <= 1e-2, (l, t, r)
+
+
+@pytest.mark.parametrize("cfg", [Config.flash(8, 4, 2, 128, 4, seq_len=64)], ids=["flash4"])
+def test_stack_without_grad_equals_the_grad_forward(cfg):
+    """With grad mode off (prefill / evaluation) the stack runs the same library calls without
+    autograd: its output is bit-identical to the grad-mode forward's."""
+    stack = XhcStack(cfg, L, lambda l, t: Scale(scales(l, t)), seed=13).cuda()
+    h = synth.normal_bf16((T, cfg.C), 18, std=0.5).cuda()
+    y1 = stack(h.clone().requires_grad_(True))
+    with torch.no_grad():
+        y2 = stack(h.clone())
+    torch.cuda.synchronize()
+    assert y2.grad_fn is None
+    assert torch.equal(y1.detach(), y2)

@@ -64,7 +64,8 @@ class Scale(nn.Module):
     def forward(self, x):
         self.log.append((self.tag, "sublayer", 0))
         y = x.float() * self.s
-        y.register_hook(lambda g: self.log.append((self.tag, "sublayer_bwd", 0)))
+        if y.requires_grad:
+            y.register_hook(lambda g: self.log.append((self.tag, "sublayer_bwd", 0)))
         return y
 
 
@@ -189,3 +190,22 @@ def test_two_forwards_before_one_backward():
             assert p2.grad is None, n1
         else:
             assert torch.allclose(p1.grad, p2.grad, rtol=1e-5, atol=1e-6), n1
+
+
+def test_forward_without_grad_records_nothing():
+    """With grad mode off the stack runs the same calls without autograd: the output equals the
+    grad-mode forward's, and no sublayer graph is recorded."""
+    cfg = Config.flash(4, 2, 1, 8, 2, seq_len=3)
+    T = 6
+    g = torch.Generator().manual_seed(3)
+    h = torch.randn(T, cfg.C, generator=g).to(torch.bfloat16)
+    log1, log2 = [], []
+    s1 = _stack_with(cfg, FakeGroupSaved, log1)
+    s2 = _stack_with(cfg, FakeGroupSaved, log2)
+    y1 = s1(h.clone().requires_grad_(True))
+    with torch.no_grad():
+        y2 = s2(h.clone())
+    assert torch.equal(y1.detach(), y2)
+    assert y2.grad_fn is None and not y2.requires_grad
+    calls = [e for e in log2 if e[1] in ("pre_fwd", "post_fwd", "sublayer")]
+    assert calls == [e for e in log1 if e[1] in ("pre_fwd", "post_fwd", "sublayer")]
