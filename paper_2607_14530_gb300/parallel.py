@@ -67,16 +67,17 @@ def allreduce_grads(grads: dict, group=None) -> dict:
     """Sum every parameter gradient over the ranks, in place (the gradients are sums over
     tokens; each rank holds the sum over its own tokens).  One flat buffer per dtype, so a group's
     gradients take one collective."""
-    names = sorted(grads)
-    if not names:
-        return grads
-    flat = torch.cat([grads[n].reshape(-1) for n in names])
-    dist.all_reduce(flat, op=dist.ReduceOp.SUM, group=group)
-    off = 0
-    for n in names:
-        k = grads[n].numel()
-        grads[n].copy_(flat[off:off + k].view_as(grads[n]))
-        off += k
+    by_dtype = {}
+    for n in sorted(grads):
+        by_dtype.setdefault(grads[n].dtype, []).append(n)
+    for names in by_dtype.values():
+        flat = torch.cat([grads[n].reshape(-1) for n in names])
+        dist.all_reduce(flat, op=dist.ReduceOp.SUM, group=group)
+        off = 0
+        for n in names:
+            k = grads[n].numel()
+            grads[n].copy_(flat[off:off + k].view_as(grads[n]))
+            off += k
     return grads
 
 

@@ -128,3 +128,30 @@ def test_data_parallel_gradient_allreduce_equals_one_rank(tmp_path):
         res = torch.load(os.path.join(tmp_path, f"dp{rank}.pt"))
         for n in dP:
             assert torch.allclose(res[n], dP[n], atol=1e-11, rtol=1e-12), (rank, n)
+
+
+def _mixed_rank(rank, world, port, out_dir):
+    sys.path.insert(0, ROOT)
+    from paper_2607_14530_gb300 import parallel
+    dist.init_process_group("gloo", init_method=f"tcp://127.0.0.1:{port}", rank=rank, world_size=world)
+    try:
+        g = {"a": torch.full((3,), 1.0 + rank, dtype=torch.float32),
+             "b": torch.full((2, 2), 0.5 * (rank + 1), dtype=F64),
+             "c": torch.arange(4, dtype=torch.float32) * (rank + 1)}
+        parallel.allreduce_grads(g)
+        torch.save(g, os.path.join(out_dir, f"mx{rank}.pt"))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_gradient_allreduce_keeps_each_dtype(tmp_path):
+    """Gradients of different dtypes are summed in one collective per dtype and keep their dtype
+    (one concatenated buffer would promote them)."""
+    world = 2
+    mp.start_processes(_mixed_rank, args=(world, _free_port(), str(tmp_path)), nprocs=world, join=True,
+                       start_method="spawn")
+    for rank in range(world):
+        g = torch.load(os.path.join(tmp_path, f"mx{rank}.pt"))
+        assert g["a"].dtype == torch.float32 and torch.equal(g["a"], torch.full((3,), 3.0))
+        assert g["b"].dtype == F64 and torch.equal(g["b"], torch.full((2, 2), 1.5, dtype=F64))
+        assert torch.equal(g["c"], torch.arange(4, dtype=torch.float32) * 3)
